@@ -1,0 +1,356 @@
+#!/usr/bin/env python
+"""Benchmark of the WaveZip condensation pass on GB300.
+
+Metric: video frames condensed per second per GB300 (the whole pass: query
+pooling, relevance, visual change, WTA, budgets, WSM operator and the fused
+condensation GEMM) on the 256-frame 27x27x3584 bf16 workload (~1.3 GB of
+tokens, larger than L2, so no L2 flush is needed between steps), with the
+achieved HBM bandwidth of the dominant kernel against the measured peak.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun every rank condenses its own independent video (replicas, weak
+scaling); the time is the max over ranks.  `--impl reference` times the CPU
+oracle on a bounded sample of the same workload instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "video frames/sec condensed per GB300 (and GB/s vs ~8 TB/s HBM roofline)"
+UNIT = "frames/s"
+WORKLOAD = "video256_27x27_bf16"
+KERNELS = ("query_pool", "relevance", "frame_stats", "temporal", "spatial", "condense")
+KERNEL_SOURCES = {"query_pool": "relevance.cu", "relevance": "relevance.cu", "frame_stats": "relevance.cu",
+                  "temporal": "temporal.cu", "spatial": "spatial.cu", "condense": "condense_tc.cu"}
+CPU_SAMPLE_FRAMES = 48          # oracle sample for the cpu_baseline leg (~10-30 s on one core)
+REF_SAMPLE_FRAMES = 16          # oracle sample per step of the reference arm
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--config", default=WORKLOAD)
+    p.add_argument("--path", default="auto", choices=["auto", "tensor", "simt"])
+    p.add_argument("--e2e-steps", type=int, default=5)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def config_dict(spec, name):
+    return {"workload": name, "T": spec.T, "H": spec.H, "W": spec.W, "D": spec.D, "Lq": spec.Lq,
+            "ratio": spec.ratio, "features_dtype": spec.dtype, "seed": spec.seed,
+            "feature_bytes": spec.T * spec.H * spec.W * spec.D * (2 if spec.dtype == "bf16" else 4),
+            "l2": "inputs larger than L2 (no flush needed)", "parallelism": "replicas"}
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def source_hash(fname):
+    with open(os.path.join(ROOT, "paper_2607_23265_gb300", "csrc", fname), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def recorded_traffic(kernel):
+    """dram bytes per launch from the committed ncu summary, if the kernel's
+    source is unchanged since the capture; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f).get(kernel)
+    except (OSError, ValueError):
+        return None
+    if not rec or rec.get("source_sha256_16") != source_hash(KERNEL_SOURCES[kernel]):
+        return None
+    return rec.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.rows = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-i", str(gpu_index), "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 9:
+                self.rows.append(parts)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.3)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in self.rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in self.rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.rows)}
+
+
+def cpu_baseline(spec, frames):
+    """Time the oracle, as it stands, on one host core: a `frames`-frame video
+    drawn with the same recipe.  Runs in a fresh interpreter pinned to one BLAS
+    thread."""
+    code = (
+        "import json,sys,time; sys.path.insert(0, %r)\n"
+        "import workload as wl, oracle as O\n"
+        "s = wl.VideoSpec(T=%d, H=%d, W=%d, D=%d, dtype=%r, Lq=%d, ratio=%r, ar=%r, cuts=%d, seed=%d)\n"
+        "X, Q, _ = wl.make_video(s)\n"
+        "x, q = X.double().numpy(), Q.double().numpy()\n"
+        "t = time.perf_counter(); O.condense(x, q, s.ratio); dt = time.perf_counter() - t\n"
+        "print(json.dumps({'seconds': dt, 'frames': s.T}))\n"
+    ) % (ROOT, frames, spec.H, spec.W, spec.D, spec.dtype, spec.Lq, spec.ratio, spec.ar,
+         max(1, spec.cuts * frames // spec.T), spec.seed)
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    res = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=900)
+    if res.returncode != 0:
+        return {"value": None, "unit": UNIT, "cores": 1, "kind": "oracle", "error": res.stderr[-400:]}
+    r = json.loads(res.stdout.strip().splitlines()[-1])
+    return {"value": r["frames"] / r["seconds"], "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"first {frames} frames of the workload recipe ({spec.H}x{spec.W}x{spec.D} "
+                      f"{spec.dtype}, Lq={spec.Lq}, ratio={spec.ratio}) condensed by the fp64 oracle",
+            "seconds": r["seconds"]}
+
+
+def run_reference(args, spec, world, rank):
+    """The oracle, timed on the host cores, on a bounded sample per step."""
+    if rank != 0:
+        return
+    os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")
+    import oracle as O
+    import workload as wl
+    frames = REF_SAMPLE_FRAMES
+    s = wl.VideoSpec(**{**spec.__dict__, "T": frames, "cuts": max(1, spec.cuts * frames // spec.T)})
+    X, Q, _ = wl.make_video(s)
+    x, q = X.double().numpy(), Q.double().numpy()
+    for _ in range(args.warmup):
+        O.condense(x, q, s.ratio)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        O.condense(x, q, s.ratio)
+    dt = time.perf_counter() - t0
+    value = frames * args.steps / dt
+    sample = f"{frames}-frame video per step ({spec.H}x{spec.W}x{spec.D} {spec.dtype}, same recipe), fp64 oracle"
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_dict(spec, args.config),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def algorithmic_bytes(spec, budgets, B, K_pad):
+    """Bytes each kernel must move per launch (one video)."""
+    esz = 2 if spec.dtype == "bf16" else 4
+    N, D, T = spec.H * spec.W, spec.D, spec.T
+    active = int((budgets > 0).sum())
+    return {
+        "relevance": T * N * D * esz + T * N * 4,
+        "condense": active * N * D * esz + B * D * esz + B * K_pad * 4,
+        "spatial": B * K_pad * 4 + active * N * 4,
+        "frame_stats": None, "query_pool": None, "temporal": None,
+    }
+
+
+def run_ours(args, spec, world, rank, local):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2607_23265_gb300.build as build
+    build.build()
+    import paper_2607_23265_gb300.wavezip as wz
+    import workload as wl
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    rspec = wl.VideoSpec(**{**spec.__dict__, "seed": spec.seed + 7919 * rank})
+    X, Q, _ = wl.make_video(rspec, device=dev)
+    T, H, W, D = X.shape
+    B = wz.wz_budget_size(T, H, W, spec.ratio)
+    K_pad = (H * W + 31) // 32 * 32
+    ws = torch.empty((wz.wz_condense_workspace_size(T, H, W, D, wz._dtype_code(X), spec.ratio),),
+                     dtype=torch.uint8, device=dev)
+    status = torch.zeros((1,), dtype=torch.int32, device=dev)
+    tokens = torch.empty((B, D), dtype=X.dtype, device=dev)
+    index = torch.empty((B, 3), dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(events=None):
+        return wz.wz_condense_ex(X, Q, spec.ratio, workspace=ws, out_tokens=tokens, out_index=index,
+                                 device_status=status, path=args.path, kernel_events=events)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    evs = []
+    for _ in range(args.steps):
+        row = [torch.cuda.Event(enable_timing=True) for _ in range(2 * len(KERNELS))]
+        for e in row:
+            e.record(stream)
+        evs.append(row)
+    for _ in range(max(3, args.warmup)):
+        res = step()
+    barrier()
+    gpu_index = os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")[local] \
+        if os.environ.get("CUDA_VISIBLE_DEVICES") else str(local)
+    sampler = ClockSampler(gpu_index)
+    time.sleep(0.4)
+    barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for k in range(args.steps):
+        res = step(evs[k])
+    t1.record(stream)
+    barrier()
+    clocks = sampler.stop()
+    ms = t0.elapsed_time(t1) / args.steps
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    kern_ms = {name: statistics.mean(evs[k][2 * j].elapsed_time(evs[k][2 * j + 1]) for k in range(args.steps))
+               for j, name in enumerate(KERNELS)}
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())}: a bounded wait timed out")
+    budgets = res["budgets"].cpu()
+
+    # end to end through the public API: pinned host buffers in, results out
+    Xh = X.cpu().pin_memory()
+    Qh = Q.cpu().pin_memory()
+    Xd, Qd = torch.empty_like(X), torch.empty_like(Q)
+    tok_h = torch.empty((B, D), dtype=X.dtype).pin_memory()
+    idx_h = torch.empty((B, 3), dtype=torch.int32).pin_memory()
+
+    def e2e_step():
+        Xd.copy_(Xh, non_blocking=True)
+        Qd.copy_(Qh, non_blocking=True)
+        r = wz.wz_condense_ex(Xd, Qd, spec.ratio, workspace=ws, out_tokens=tokens, out_index=index,
+                              device_status=status, path=args.path)
+        tok_h.copy_(r["tokens"], non_blocking=True)
+        idx_h.copy_(r["index"], non_blocking=True)
+
+    e2e_step()
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1) / args.e2e_steps
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+
+    if rank == 0:
+        peak, peak_kind = measured_peak()
+        ab = algorithmic_bytes(spec, budgets, B, K_pad)
+        dominant = max(KERNELS, key=lambda k: kern_ms[k])
+        kern = {}
+        for k in KERNELS:
+            entry = {"ms": round(kern_ms[k], 5), "share": round(kern_ms[k] / sum(kern_ms.values()), 4)}
+            if ab.get(k):
+                entry["gb_s"] = round(ab[k] / (kern_ms[k] * 1e-3) / 1e9, 1)
+            kern[k] = entry
+        bytes_dom = ab.get(dominant)
+        achieved = bytes_dom / (kern_ms[dominant] * 1e-3) / 1e9 if bytes_dom else None
+        frames = T * world
+        out = {
+            "metric": METRIC, "value": frames / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic", "config": config_dict(spec, args.config),
+            "tokens_out_per_s": B * world / (ms * 1e-3),
+            "roofline": {"bound": "hbm", "kernel": dominant, "achieved": achieved, "peak": peak,
+                         "unit": "GB/s", "frac": achieved / peak if achieved else None,
+                         "traffic": recorded_traffic(dominant), "peak_source": peak_kind,
+                         "frac_of_8000": achieved / 8000.0 if achieved else None},
+            "kernels": kern,
+            "active_frames": int((budgets > 0).sum()), "budget_B": B,
+            "e2e": {"value": frames / (e2e_ms * 1e-3), "unit": UNIT,
+                    "h2d_bytes_per_step": X.numel() * X.element_size() + Q.numel() * Q.element_size(),
+                    "d2h_bytes_per_step": tokens.numel() * tokens.element_size() + index.numel() * 4},
+            "clocks": clocks,
+            "gpu_launches": len(KERNELS) * args.steps,
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            out["cpu_baseline"] = cpu_baseline(spec, CPU_SAMPLE_FRAMES)
+        print(json.dumps(out))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    world, rank, local = dist_setup()
+    import workload as wl
+    spec = wl.CONFIGS[args.config]
+    if args.impl == "reference":
+        run_reference(args, spec, world, rank)
+    else:
+        run_ours(args, spec, world, rank, local)
+
+
+if __name__ == "__main__":
+    main()

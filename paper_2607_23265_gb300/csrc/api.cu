@@ -1,0 +1,557 @@
+// C ABI of the WaveZip library: argument checks, workspace layout and the
+// launch sequence of the condensation pass (Section 3.2).
+//
+//   query_pool -> relevance_pass -> frame_stats -> temporal -> spatial ->
+//   condense (tensor cores or CUDA cores)
+//
+// All launches go to the caller's stream; nothing synchronises the host.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <vector>
+
+#include "wz_internal.cuh"
+
+namespace wz {
+
+size_t spatial_smem_bytes(const Ctx &c);
+bool tensor_path_available();
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+// Sub-buffer offsets of one call's workspace.
+struct Layout {
+    size_t qbar32, qbar64, qnorm, vpar, a, part, trip, fr, tmp, list, n, off, hw, prod,
+        units, ucount, status, Wop, total;
+};
+
+struct Shape {
+    int V, T, H, W, D, N, dtype, F, hp, wp, K_pad, DC, n_ct, max_units_v;
+    int64_t rows_total;
+};
+
+Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
+    Layout L{};
+    size_t o = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = o;
+        o = align_up(o + bytes);
+        return at;
+    };
+    const size_t VT = (size_t)s.V * s.T;
+    L.qbar32 = take((size_t)s.V * s.D * 4);
+    L.qbar64 = take((size_t)s.V * s.D * 8);
+    L.qnorm = take((size_t)s.V * 8);
+    L.vpar = take((size_t)s.V * sizeof(VideoPar));
+    L.a = with_a ? take(VT * s.N * 4) : 0;
+    L.part = take(((size_t)kG1Max + VT) * s.D * 4);
+    L.trip = take(VT * s.DC * 3 * 8);
+    L.fr = take(VT * 4 * 8);
+    L.tmp = take(VT * 4 * 8);
+    L.list = take(VT * 2 * 4);
+    L.n = take(VT * 4);
+    L.off = take(VT * 4);
+    L.hw = take(VT * 2 * 4);
+    L.prod = take((size_t)s.V * 4);
+    L.units = take((size_t)s.V * s.max_units_v * 16);
+    L.ucount = take((size_t)s.V * 4);
+    L.status = take(16);
+    L.Wop = with_operator ? take((size_t)s.rows_total * s.K_pad * 4) : 0;
+    L.total = o;
+    return L;
+}
+
+bool valid_ratio(float r) { return std::isfinite(r) && r > 0.f && r <= 1.f; }
+
+int64_t budget(int T, int N, float ratio) {
+    const double x = (double)ratio * (double)T * (double)N;   // exact: 24 + 12 + 12 bits
+    return (int64_t)std::floor(x + 0.5);
+}
+
+int check_sizes(int V, int T, int H, int W, int D, int dtype) {
+    if (V < 1 || T < 1 || H < 1 || W < 1 || D < 1) return WZ_ERR_INVALID_ARG;
+    if (dtype != WZ_DTYPE_BF16 && dtype != WZ_DTYPE_F32) return WZ_ERR_INVALID_ARG;
+    if (D % 8 != 0) return WZ_ERR_UNSUPPORTED;
+    if (V > WZ_MAX_VIDEOS || T > WZ_MAX_T || H > WZ_MAX_HW || W > WZ_MAX_HW || D > WZ_MAX_D)
+        return WZ_ERR_UNSUPPORTED;
+    return WZ_OK;
+}
+
+Shape make_shape(int V, int T, int H, int W, int D, int dtype, int F, const int64_t *B) {
+    Shape s{};
+    s.V = V; s.T = T; s.H = H; s.W = W; s.D = D; s.N = H * W; s.dtype = dtype; s.F = F;
+    s.hp = (H + F - 1) / 2;
+    s.wp = (W + F - 1) / 2;
+    s.K_pad = (s.N + 31) / 32 * 32;
+    s.DC = (D + kStatsChunk - 1) / kStatsChunk;
+    s.n_ct = (D + kTileC - 1) / kTileC;
+    int64_t rows = 0, bmax = 0;
+    for (int v = 0; v < V; ++v) {
+        rows += B ? B[v] : 0;
+        bmax = std::max<int64_t>(bmax, B ? B[v] : 0);
+    }
+    s.rows_total = rows;
+    s.max_units_v = (int)((T + (bmax + kColBlock - 1) / kColBlock) * s.n_ct);
+    return s;
+}
+
+struct Common {
+    float lambda, tau;
+    int wta_wavelet, wsm_wavelet, mode, path;
+};
+
+int check_common(const Common &m, int dtype) {
+    if (!std::isfinite(m.lambda) || m.lambda < 0.f || !std::isfinite(m.tau)) return WZ_ERR_INVALID_ARG;
+    if (m.wta_wavelet != WZ_WAVELET_HAAR) return m.wta_wavelet >= 1 && m.wta_wavelet <= 10
+                                                      ? WZ_ERR_UNSUPPORTED : WZ_ERR_INVALID_ARG;
+    if (m.wsm_wavelet < 1 || m.wsm_wavelet > 10) return WZ_ERR_INVALID_ARG;
+    if (m.mode < WZ_MODE_SYMMETRIC || m.mode > WZ_MODE_PERIODIC) return WZ_ERR_INVALID_ARG;
+    if (m.path < WZ_PATH_AUTO || m.path > WZ_PATH_SIMT) return WZ_ERR_INVALID_ARG;
+    if (m.path == WZ_PATH_TENSOR && dtype != WZ_DTYPE_BF16) return WZ_ERR_UNSUPPORTED;
+    return WZ_OK;
+}
+
+int resolve_path(int path, int dtype) {
+    if (path != WZ_PATH_AUTO) return path;
+    return (dtype == WZ_DTYPE_BF16 && tensor_path_available()) ? WZ_PATH_TENSOR : WZ_PATH_SIMT;
+}
+
+void set_filters(Ctx &c, int p) {
+    double dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
+    daubechies(p, dl, dh, rl, rh);
+    c.F = 2 * p;
+    for (int k = 0; k < kMaxTaps; ++k) {
+        c.dec_lo[k] = k < c.F ? (float)dl[k] : 0.f;
+        c.dec_hi[k] = k < c.F ? (float)dh[k] : 0.f;
+        c.rec_lo[k] = k < c.F ? (float)rl[k] : 0.f;
+        c.rec_hi[k] = k < c.F ? (float)rh[k] : 0.f;
+    }
+}
+
+void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
+    c.V = s.V; c.T = s.T; c.H = s.H; c.W = s.W; c.D = s.D; c.N = s.N; c.dtype = s.dtype;
+    c.hp = s.hp; c.wp = s.wp; c.K_pad = s.K_pad; c.DC = s.DC; c.n_ct = s.n_ct;
+    c.max_units_v = s.max_units_v; c.rows_total = s.rows_total;
+    c.qbar32 = reinterpret_cast<float *>(ws + L.qbar32);
+    c.qbar64 = reinterpret_cast<double *>(ws + L.qbar64);
+    c.qnorm = reinterpret_cast<double *>(ws + L.qnorm);
+    c.vpar = reinterpret_cast<VideoPar *>(ws + L.vpar);
+    if (L.a) c.a = reinterpret_cast<float *>(ws + L.a);
+    c.part = reinterpret_cast<float *>(ws + L.part);
+    c.trip = reinterpret_cast<double *>(ws + L.trip);
+    c.fr = reinterpret_cast<double *>(ws + L.fr);
+    c.tmp = reinterpret_cast<double *>(ws + L.tmp);
+    c.list = reinterpret_cast<int *>(ws + L.list);
+    c.n = reinterpret_cast<int *>(ws + L.n);
+    c.off = reinterpret_cast<int *>(ws + L.off);
+    c.hw = reinterpret_cast<int *>(ws + L.hw);
+    c.prod = reinterpret_cast<int *>(ws + L.prod);
+    c.units = reinterpret_cast<int4 *>(ws + L.units);
+    c.ucount = reinterpret_cast<int *>(ws + L.ucount);
+    c.status = reinterpret_cast<int *>(ws + L.status);
+    if (L.Wop) c.Wop = ws + L.Wop;
+}
+
+// Scratch either from the caller or from the stream-ordered allocator.
+struct Scratch {
+    char *ptr = nullptr;
+    bool owned = false;
+    cudaStream_t stream = nullptr;
+    int acquire(void *given, size_t given_bytes, size_t need, cudaStream_t s) {
+        stream = s;
+        if (given) {
+            if (!aligned(given, kAlign)) return WZ_ERR_INVALID_ARG;
+            if (given_bytes < need) return WZ_ERR_WORKSPACE;
+            ptr = static_cast<char *>(given);
+            return WZ_OK;
+        }
+        void *p = nullptr;
+        if (cudaMallocAsync(&p, need, s) != cudaSuccess) {
+            cudaGetLastError();
+            return WZ_ERR_NO_MEMORY;
+        }
+        ptr = static_cast<char *>(p);
+        owned = true;
+        return WZ_OK;
+    }
+    ~Scratch() {
+        if (owned) cudaFreeAsync(ptr, stream);
+    }
+};
+
+#define WZ_CUDA(call)                        \
+    do {                                     \
+        if ((call) != cudaSuccess) {         \
+            cudaGetLastError();              \
+            return WZ_ERR_CUDA;              \
+        }                                    \
+    } while (0)
+
+struct CondenseRequest {
+    int V, T, H, W, D, dtype;
+    const void *features, *queries;
+    std::vector<int> Lq;
+    std::vector<float> ratio;
+    Common m;
+    void *out_tokens;
+    int32_t *out_index, *out_budgets, *out_count, *device_status;
+    float *out_relevance;
+    void *workspace;
+    size_t workspace_bytes;
+    void *const *events;
+    cudaStream_t stream;
+};
+
+int validate(const CondenseRequest &r, std::vector<int64_t> &B, int64_t &rows) {
+    int st = check_sizes(r.V, r.T, r.H, r.W, r.D, r.dtype);
+    if (st != WZ_OK) return st;
+    st = check_common(r.m, r.dtype);
+    if (st != WZ_OK) return st;
+    if (!r.features || !r.queries) return WZ_ERR_INVALID_ARG;
+    if (!aligned(r.features, 16) || !aligned(r.queries, 16)) return WZ_ERR_INVALID_ARG;
+    B.assign(r.V, 0);
+    rows = 0;
+    int64_t qrows = 0;
+    for (int v = 0; v < r.V; ++v) {
+        if (r.Lq[v] < 1 || !valid_ratio(r.ratio[v])) return WZ_ERR_INVALID_ARG;
+        B[v] = budget(r.T, r.H * r.W, r.ratio[v]);
+        rows += B[v];
+        qrows += r.Lq[v];
+    }
+    if (rows > (int64_t)INT32_MAX || qrows > (int64_t)INT32_MAX) return WZ_ERR_UNSUPPORTED;
+    if (rows > 0) {
+        if (!r.out_tokens || !r.out_index) return WZ_ERR_INVALID_ARG;
+        if (!aligned(r.out_tokens, 16) || !aligned(r.out_index, 4)) return WZ_ERR_INVALID_ARG;
+    }
+    return WZ_OK;
+}
+
+int run_condense(const CondenseRequest &r) {
+    std::vector<int64_t> B;
+    int64_t rows = 0;
+    int st = validate(r, B, rows);
+    if (st != WZ_OK) return st;
+    Ctx c{};
+    c.lambda = r.m.lambda;
+    c.tau = r.m.tau;
+    c.mode = r.m.mode;
+    c.path = resolve_path(r.m.path, r.dtype);
+    set_filters(c, r.m.wsm_wavelet);
+    const Shape s = make_shape(r.V, r.T, r.H, r.W, r.D, r.dtype, c.F, B.data());
+    const Layout L = make_layout(s, true, true);
+    Scratch ws;
+    st = ws.acquire(r.workspace, r.workspace_bytes, L.total, r.stream);
+    if (st != WZ_OK) return st;
+    bind(c, s, L, ws.ptr);
+    c.X = r.features;
+    c.Q = r.queries;
+    c.out = r.out_tokens;
+    c.out_index = r.out_index;
+    c.out_budgets = r.out_budgets;
+    c.out_count = r.out_count;
+    c.out_rel = r.out_relevance;
+    if (r.device_status) c.status = r.device_status;
+    else WZ_CUDA(cudaMemsetAsync(c.status, 0, sizeof(int), r.stream));
+    c.G1 = relevance_grid(c);
+    if (c.G1 < 1) {
+        cudaGetLastError();
+        return WZ_ERR_CUDA;
+    }
+    const int64_t total = (int64_t)s.V * s.T * s.N;
+    c.L1 = (total + c.G1 - 1) / c.G1;
+    std::vector<VideoPar> par(r.V);
+    int qrow = 0;
+    int64_t row0 = 0;
+    for (int v = 0; v < r.V; ++v) {
+        par[v].q_row0 = qrow;
+        par[v].Lq = r.Lq[v];
+        par[v].B = (int)B[v];
+        par[v].row0 = (int)row0;
+        qrow += r.Lq[v];
+        row0 += B[v];
+    }
+    auto mark = [&](int k) -> cudaError_t {
+        return r.events ? cudaEventRecord((cudaEvent_t)r.events[k], r.stream) : cudaSuccess;
+    };
+    WZ_CUDA(mark(2 * WZ_KERNEL_QUERY_POOL));
+    WZ_CUDA(launch_query_pool(c, par.data(), r.stream));
+    WZ_CUDA(mark(2 * WZ_KERNEL_QUERY_POOL + 1));
+    WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE));
+    WZ_CUDA(launch_relevance_pass(c, r.stream));
+    WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE + 1));
+    WZ_CUDA(mark(2 * WZ_KERNEL_FRAME_STATS));
+    WZ_CUDA(launch_frame_stats(c, r.stream));
+    WZ_CUDA(mark(2 * WZ_KERNEL_FRAME_STATS + 1));
+    WZ_CUDA(mark(2 * WZ_KERNEL_TEMPORAL));
+    WZ_CUDA(launch_temporal(c, r.stream));
+    WZ_CUDA(mark(2 * WZ_KERNEL_TEMPORAL + 1));
+    WZ_CUDA(mark(2 * WZ_KERNEL_SPATIAL));
+    WZ_CUDA(launch_spatial(c, r.stream));
+    WZ_CUDA(mark(2 * WZ_KERNEL_SPATIAL + 1));
+    WZ_CUDA(mark(2 * WZ_KERNEL_CONDENSE));
+    if (rows > 0) {
+        if (c.path == WZ_PATH_TENSOR) WZ_CUDA(launch_condense_tc(c, r.stream));
+        else WZ_CUDA(launch_condense_simt(c, r.stream));
+    }
+    WZ_CUDA(mark(2 * WZ_KERNEL_CONDENSE + 1));
+    return WZ_OK;
+}
+
+size_t condense_ws(int V, int T, int H, int W, int D, int dtype, const float *ratio) {
+    if (check_sizes(V, T, H, W, D, dtype) != WZ_OK || !ratio) return 0;
+    std::vector<int64_t> B(V);
+    for (int v = 0; v < V; ++v) {
+        if (!valid_ratio(ratio[v])) return 0;
+        B[v] = budget(T, H * W, ratio[v]);
+    }
+    const Shape s = make_shape(V, T, H, W, D, dtype, 2, B.data());
+    return make_layout(s, true, true).total;
+}
+
+}  // namespace
+}  // namespace wz
+
+using namespace wz;
+
+extern "C" {
+
+int64_t wz_budget_size(int T, int H, int W, float ratio) {
+    if (T < 1 || H < 1 || W < 1 || !valid_ratio(ratio)) return -1;
+    return budget(T, H * W, ratio);
+}
+
+void wz_condense_args_init(wz_condense_args *a) {
+    if (!a) return;
+    std::memset(a, 0, sizeof(*a));
+    a->dtype = WZ_DTYPE_BF16;
+    a->lambda = 1.5f;
+    a->tau = 0.f;
+    a->wta_wavelet = WZ_WAVELET_HAAR;
+    a->wsm_wavelet = WZ_WAVELET_DB4;
+    a->mode = WZ_MODE_SYMMETRIC;
+    a->path = WZ_PATH_AUTO;
+}
+
+void wz_batch_args_init(wz_batch_args *a) {
+    if (!a) return;
+    std::memset(a, 0, sizeof(*a));
+    a->dtype = WZ_DTYPE_BF16;
+    a->lambda = 1.5f;
+    a->tau = 0.f;
+    a->wta_wavelet = WZ_WAVELET_HAAR;
+    a->wsm_wavelet = WZ_WAVELET_DB4;
+    a->mode = WZ_MODE_SYMMETRIC;
+    a->path = WZ_PATH_AUTO;
+}
+
+size_t wz_condense_workspace_size(int T, int H, int W, int D, int dtype, float ratio) {
+    return condense_ws(1, T, H, W, D, dtype, &ratio);
+}
+
+int wz_condense_ex(const wz_condense_args *a) {
+    if (!a) return WZ_ERR_INVALID_ARG;
+    CondenseRequest r;
+    r.V = 1; r.T = a->T; r.H = a->H; r.W = a->W; r.D = a->D; r.dtype = a->dtype;
+    r.features = a->features;
+    r.queries = a->query;
+    r.Lq.assign(1, a->Lq);
+    r.ratio.assign(1, a->ratio);
+    r.m = Common{a->lambda, a->tau, a->wta_wavelet, a->wsm_wavelet, a->mode, a->path};
+    r.out_tokens = a->out_tokens;
+    r.out_index = a->out_index;
+    r.out_budgets = a->out_budgets;
+    r.out_count = a->out_count;
+    r.out_relevance = a->out_relevance;
+    r.device_status = a->device_status;
+    r.workspace = a->workspace;
+    r.workspace_bytes = a->workspace_bytes;
+    r.events = a->kernel_events;
+    r.stream = (cudaStream_t)a->stream;
+    return run_condense(r);
+}
+
+int wz_condense(const void *features, int T, int H, int W, int D, const void *query, int Lq,
+                float ratio, void *out_tokens, int32_t *out_index, wz_stream_t stream) {
+    wz_condense_args a;
+    wz_condense_args_init(&a);
+    a.features = features;
+    a.T = T; a.H = H; a.W = W; a.D = D;
+    a.query = query;
+    a.Lq = Lq;
+    a.ratio = ratio;
+    a.out_tokens = out_tokens;
+    a.out_index = out_index;
+    a.stream = stream;
+    return wz_condense_ex(&a);
+}
+
+int64_t wz_batch_rows(int V, int T, int H, int W, const float *ratio, int64_t *row_offsets) {
+    if (V < 1 || T < 1 || H < 1 || W < 1 || !ratio) return -1;
+    int64_t rows = 0;
+    for (int v = 0; v < V; ++v) {
+        if (!valid_ratio(ratio[v])) return -1;
+        if (row_offsets) row_offsets[v] = rows;
+        rows += budget(T, H * W, ratio[v]);
+    }
+    if (row_offsets) row_offsets[V] = rows;
+    return rows;
+}
+
+size_t wz_batch_workspace_size(int V, int T, int H, int W, int D, int dtype, const float *ratio) {
+    return condense_ws(V, T, H, W, D, dtype, ratio);
+}
+
+int wz_condense_batch(const wz_batch_args *a) {
+    if (!a || !a->Lq || !a->ratio) return WZ_ERR_INVALID_ARG;
+    if (a->V < 1 || a->V > WZ_MAX_VIDEOS) return a->V < 1 ? WZ_ERR_INVALID_ARG : WZ_ERR_UNSUPPORTED;
+    CondenseRequest r;
+    r.V = a->V; r.T = a->T; r.H = a->H; r.W = a->W; r.D = a->D; r.dtype = a->dtype;
+    r.features = a->features;
+    r.queries = a->queries;
+    r.Lq.assign(a->Lq, a->Lq + a->V);
+    r.ratio.assign(a->ratio, a->ratio + a->V);
+    r.m = Common{a->lambda, a->tau, a->wta_wavelet, a->wsm_wavelet, a->mode, a->path};
+    r.out_tokens = a->out_tokens;
+    r.out_index = a->out_index;
+    r.out_budgets = a->out_budgets;
+    r.out_count = a->out_count;
+    r.out_relevance = a->out_relevance;
+    r.device_status = a->device_status;
+    r.workspace = a->workspace;
+    r.workspace_bytes = a->workspace_bytes;
+    r.events = a->kernel_events;
+    r.stream = (cudaStream_t)a->stream;
+    if (a->row_offsets && wz_batch_rows(a->V, a->T, a->H, a->W, a->ratio, a->row_offsets) < 0)
+        return WZ_ERR_INVALID_ARG;
+    return run_condense(r);
+}
+
+size_t wz_relevance_workspace_size(int T, int H, int W, int D) {
+    if (check_sizes(1, T, H, W, D, WZ_DTYPE_BF16) != WZ_OK) return 0;
+    const Shape s = make_shape(1, T, H, W, D, WZ_DTYPE_BF16, 2, nullptr);
+    return make_layout(s, false, false).total;
+}
+
+int wz_relevance(const void *features, int T, int H, int W, int D, int dtype, const void *query,
+                 int Lq, float *token_scores, float *frame_scores, float *frame_mean,
+                 void *workspace, size_t workspace_bytes, wz_stream_t stream) {
+    int st = check_sizes(1, T, H, W, D, dtype);
+    if (st != WZ_OK) return st;
+    if (!features || !query || !token_scores || !frame_scores || Lq < 1) return WZ_ERR_INVALID_ARG;
+    if (!aligned(features, 16) || !aligned(query, 16) || !aligned(token_scores, 4) ||
+        !aligned(frame_scores, 4) || (frame_mean && !aligned(frame_mean, 4)))
+        return WZ_ERR_INVALID_ARG;
+    const Shape s = make_shape(1, T, H, W, D, dtype, 2, nullptr);
+    const Layout L = make_layout(s, false, false);
+    Scratch ws;
+    st = ws.acquire(workspace, workspace_bytes, L.total, (cudaStream_t)stream);
+    if (st != WZ_OK) return st;
+    Ctx c{};
+    bind(c, s, L, ws.ptr);
+    c.X = features;
+    c.Q = query;
+    c.a = token_scores;
+    c.frame_scores = frame_scores;
+    c.frame_mean = frame_mean;
+    c.G1 = relevance_grid(c);
+    if (c.G1 < 1) {
+        cudaGetLastError();
+        return WZ_ERR_CUDA;
+    }
+    c.L1 = ((int64_t)T * s.N + c.G1 - 1) / c.G1;
+    VideoPar par{0, Lq, 0, 0};
+    const cudaStream_t cs = (cudaStream_t)stream;
+    WZ_CUDA(launch_query_pool(c, &par, cs));
+    WZ_CUDA(launch_relevance_pass(c, cs));
+    WZ_CUDA(launch_frame_stats(c, cs));
+    WZ_CUDA(launch_relevance_finalize(c, cs));
+    return WZ_OK;
+}
+
+int wz_dwt_len(int n, int wavelet) {
+    if (n < 1 || wavelet < 1 || wavelet > 10) return -1;
+    return (n + 2 * wavelet - 1) / 2;
+}
+
+int wz_wavelet_filters(int wavelet, double *dec_lo, double *dec_hi, double *rec_lo, double *rec_hi) {
+    if (wavelet < 1 || wavelet > 10) return WZ_ERR_INVALID_ARG;
+    return daubechies(wavelet, dec_lo, dec_hi, rec_lo, rec_hi) ? WZ_OK : WZ_ERR_INVALID_ARG;
+}
+
+static void float_taps(int p, float *dl, float *dh, float *rl, float *rh) {
+    double a[kMaxTaps], b[kMaxTaps], c[kMaxTaps], d[kMaxTaps];
+    daubechies(p, a, b, c, d);
+    for (int k = 0; k < 2 * p; ++k) {
+        dl[k] = (float)a[k];
+        dh[k] = (float)b[k];
+        rl[k] = (float)c[k];
+        rh[k] = (float)d[k];
+    }
+}
+
+int wz_dwt1d(const float *x, int rows, int L, int wavelet, int mode, float *cA, float *cD,
+             wz_stream_t stream) {
+    if (rows < 0 || L < 1 || wavelet < 1 || wavelet > 10 || mode < 0 || mode > 2) return WZ_ERR_INVALID_ARG;
+    if (rows > 0 && (!x || !cA || !cD)) return WZ_ERR_INVALID_ARG;
+    float dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
+    float_taps(wavelet, dl, dh, rl, rh);
+    WZ_CUDA(launch_dwt1d(x, rows, L, 2 * wavelet, mode, dl, dh, cA, cD, (cudaStream_t)stream));
+    return WZ_OK;
+}
+
+int wz_idwt1d(const float *cA, const float *cD, int rows, int L, int wavelet, float *x,
+              wz_stream_t stream) {
+    if (rows < 0 || L < 1 || wavelet < 1 || wavelet > 10) return WZ_ERR_INVALID_ARG;
+    if (rows > 0 && (!x || !cA || !cD)) return WZ_ERR_INVALID_ARG;
+    float dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
+    float_taps(wavelet, dl, dh, rl, rh);
+    WZ_CUDA(launch_idwt1d(cA, cD, rows, L, 2 * wavelet, rl, rh, x, (cudaStream_t)stream));
+    return WZ_OK;
+}
+
+int wz_dwt2d(const void *features, int T, int H, int W, int D, int dtype, int wavelet, int mode,
+             float *LL, float *LH, float *HL, float *HH, wz_stream_t stream) {
+    if (T < 1 || H < 1 || W < 1 || D < 1 || wavelet < 1 || wavelet > 10 || mode < 0 || mode > 2)
+        return WZ_ERR_INVALID_ARG;
+    if (dtype != WZ_DTYPE_BF16 && dtype != WZ_DTYPE_F32) return WZ_ERR_INVALID_ARG;
+    if (H > WZ_MAX_HW || W > WZ_MAX_HW || T > 65535) return WZ_ERR_UNSUPPORTED;
+    if (!features || !LL || !LH || !HL || !HH) return WZ_ERR_INVALID_ARG;
+    float dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
+    float_taps(wavelet, dl, dh, rl, rh);
+    WZ_CUDA(launch_dwt2d(features, dtype, T, H, W, D, 2 * wavelet, mode, dl, dh, LL, LH, HL, HH,
+                         (cudaStream_t)stream));
+    return WZ_OK;
+}
+
+int wz_idwt2d(const float *LL, const float *LH, const float *HL, const float *HH, int T, int H, int W,
+              int D, int wavelet, float *out, wz_stream_t stream) {
+    if (T < 1 || H < 1 || W < 1 || D < 1 || wavelet < 1 || wavelet > 10) return WZ_ERR_INVALID_ARG;
+    if (H > WZ_MAX_HW || W > WZ_MAX_HW || T > 65535) return WZ_ERR_UNSUPPORTED;
+    if (!out || !LL || !LH || !HL || !HH) return WZ_ERR_INVALID_ARG;
+    float dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
+    float_taps(wavelet, dl, dh, rl, rh);
+    WZ_CUDA(launch_idwt2d(LL, LH, HL, HH, T, H, W, D, 2 * wavelet, rl, rh, out, (cudaStream_t)stream));
+    return WZ_OK;
+}
+
+const char *wz_status_string(int status) {
+    switch (status) {
+        case WZ_OK: return "ok";
+        case WZ_ERR_INVALID_ARG: return "invalid argument";
+        case WZ_ERR_UNSUPPORTED: return "unsupported by this build";
+        case WZ_ERR_CUDA: return "CUDA error";
+        case WZ_ERR_NO_MEMORY: return "workspace allocation failed";
+        case WZ_ERR_WORKSPACE: return "workspace too small";
+        default: return "unknown status";
+    }
+}
+
+int wz_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,341 @@
+// Temporal tail of the condensation pass, one CTA per video, in fp64:
+//
+//   r_t       cos(v_bar_t, u_q)                       Section 3.2.1
+//   delta_t   1 - cos(v_bar_t, v_bar_{t-1}), clamped  Eq. 7
+//   gamma_t   min-max of delta over the video         Section 3.2.2
+//   M         {1} u {t : delta_t >= tau}              Section 3.2.2 (frame filter)
+//   r~        Haar DWT of r_M, detail * pair-mean of gamma, inverse DWT   Eq. 8-10
+//   n_m       largest-remainder apportionment of B over max(r~, 0),
+//             capped at N with re-apportionment       Eq. 5, Eq. 15
+//   offsets   exclusive prefix of n over frames       Eq. 18 (temporal order)
+//   (h, w)    condensation grid of each frame         Eq. 16
+//   units     the tensor-core work list of the frame  (this library)
+//
+// Every reduction runs in a fixed order for a fixed block size, so results
+// do not depend on scheduling.
+#include <cmath>
+
+#include "wz_internal.cuh"
+
+namespace wz {
+
+constexpr int kTemporalThreads = 1024;
+
+// Exclusive scan of one int per thread over the block; returns the prefix and
+// writes the block total to *total.
+__device__ int block_excl_scan(int x, int *ws, int *total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nw = blockDim.x >> 5;
+    int incl = x;
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    __syncthreads();
+    if (lane == 31) ws[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int w = lane < nw ? ws[lane] : 0;
+        int wi = w;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += y;
+        }
+        if (lane < nw) ws[32 + lane] = wi - w;
+        if (lane == nw - 1) ws[64] = wi;
+    }
+    __syncthreads();
+    const int r = ws[32 + warp] + incl - x;
+    *total = ws[64];
+    __syncthreads();
+    return r;
+}
+
+// Frames per thread for the scans (T <= 4096 with 1024 threads).
+constexpr int kPerThread = WZ_MAX_T / kTemporalThreads;
+
+__device__ __forceinline__ int grid_h(int n, int H, int W) {
+    if (n <= 0) return 0;
+    long long h = (long long)ceil(sqrt((double)n * H / W));
+    if (h < 1) h = 1;
+    while (h * h * W < (long long)n * H) ++h;
+    while (h > 1 && (h - 1) * (h - 1) * W >= (long long)n * H) --h;
+    return (int)(h < H ? h : H);
+}
+
+__global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
+    __shared__ double dscr[64];
+    __shared__ long long lscr[32];
+    __shared__ int iscr[72];
+    const int v = blockIdx.x;
+    const int T = c.T;
+    const int64_t base = (int64_t)v * T;
+    const VideoPar vp = c.vpar[v];
+    const double qn = c.qnorm[v];
+    double *fr = c.fr + base * 4;          // r, delta, gamma, r~
+    double *ff = c.tmp + base * 4;         // |v|^2, <v, v_prev>, weight, frac
+    int *lst = c.list + 2 * base;          // retained frames, then their budgets
+
+    // r_t and the norms (sums of the frame-stats chunks in a fixed order)
+    for (int t = threadIdx.x; t < T; t += blockDim.x) {
+        const double *tr = c.trip + (size_t)(base + t) * c.DC * 3;
+        double dq = 0.0, vv = 0.0, vp_ = 0.0;
+        for (int k = 0; k < c.DC; ++k) {
+            dq += tr[3 * k + 0];
+            vv += tr[3 * k + 1];
+            vp_ += tr[3 * k + 2];
+        }
+        fr[4 * t + 0] = (vv > 0.0 && qn > 0.0) ? dq / (sqrt(vv) * qn) : 0.0;
+        ff[4 * t + 0] = vv;
+        ff[4 * t + 1] = vp_;
+    }
+    __syncthreads();
+    // delta_t (Eq. 7) and its range
+    double lo = INFINITY, hi = -INFINITY;
+    for (int t = threadIdx.x; t < T; t += blockDim.x) {
+        double d = 0.0;
+        if (t > 0) {
+            const double den = sqrt(ff[4 * t] * ff[4 * (t - 1)]);
+            const double cs = den > 0.0 ? ff[4 * t + 1] / den : 0.0;
+            d = fmin(2.0, fmax(0.0, 1.0 - cs));
+        }
+        fr[4 * t + 1] = d;
+        lo = fmin(lo, d);
+        hi = fmax(hi, d);
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        lo = fmin(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+        hi = fmax(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    __syncthreads();
+    if ((threadIdx.x & 31) == 0) {
+        dscr[threadIdx.x >> 5] = lo;
+        dscr[32 + (threadIdx.x >> 5)] = hi;
+    }
+    __syncthreads();
+    lo = INFINITY;
+    hi = -INFINITY;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+        lo = fmin(lo, dscr[w]);
+        hi = fmax(hi, dscr[32 + w]);
+    }
+    __syncthreads();
+    // gamma_t and the retained set (frame 1 always kept)
+    const double tau = (double)c.tau;
+    int keep[kPerThread];
+    int cnt = 0;
+    const int t0 = threadIdx.x * kPerThread;
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k) {
+        const int t = t0 + k;
+        keep[k] = 0;
+        if (t < T) {
+            const double d = fr[4 * t + 1];
+            fr[4 * t + 2] = hi > lo ? (d - lo) / (hi - lo) : 0.0;
+            fr[4 * t + 3] = NAN;
+            keep[k] = (t == 0 || d >= tau) ? 1 : 0;
+            cnt += keep[k];
+        }
+    }
+    int L = 0;
+    int pos = block_excl_scan(cnt, iscr, &L);
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k)
+        if (keep[k]) lst[pos++] = t0 + k;
+    __syncthreads();
+
+    // WTA: Haar DWT of r over the retained sequence, detail gated by the
+    // pair mean of gamma, inverse DWT (Eq. 8-10).  Odd L: the last sample
+    // pairs with its mirror image, so its detail is 0.
+    const double s2 = 0.70710678118654752440;
+    for (int k = threadIdx.x; 2 * k < L; k += blockDim.x) {
+        const int i0 = 2 * k, i1 = min(2 * k + 1, L - 1);
+        const int a0 = lst[i0], a1 = lst[i1];
+        const double r0 = fr[4 * a0], r1 = fr[4 * a1];
+        const double A = s2 * r0 + s2 * r1;
+        const double Dd = s2 * r0 - s2 * r1;
+        const double g = 0.5 * (fr[4 * a0 + 2] + fr[4 * a1 + 2]);
+        const double Dt = g * Dd;
+        fr[4 * a0 + 3] = s2 * A + s2 * Dt;
+        if (i1 != i0) fr[4 * a1 + 3] = s2 * A - s2 * Dt;
+    }
+    __syncthreads();
+
+    // Budgets (Eq. 5, Eq. 15): weights max(r~, 0); uniform if none positive.
+    const int N = c.N;
+    const int B = vp.B;
+    int anypos = 0;
+    for (int m = threadIdx.x; m < L; m += blockDim.x) {
+        const double w = fmax(fr[4 * lst[m] + 3], 0.0);
+        ff[4 * lst[m] + 2] = w;
+        anypos |= (w > 0.0);
+    }
+    anypos = __syncthreads_or(anypos);
+    int *nb = lst + T;                     // budget of retained frame m; -1 while active
+    for (int m = threadIdx.x; m < L; m += blockDim.x) {
+        nb[m] = -1;                        // -1: still active
+        if (!anypos) ff[4 * lst[m] + 2] = 1.0;
+    }
+    __syncthreads();
+    if ((long long)L * N <= (long long)B) {
+        for (int m = threadIdx.x; m < L; m += blockDim.x) nb[m] = N;
+    } else {
+        long long remaining = B;
+        for (int round = 0; round <= L; ++round) {
+            // candidates: active frames with positive weight, else all active
+            double sp = 0.0;
+            int npos = 0;
+            for (int m = threadIdx.x; m < L; m += blockDim.x)
+                if (nb[m] < 0 && ff[4 * lst[m] + 2] > 0.0) {
+                    sp += ff[4 * lst[m] + 2];
+                    npos = 1;
+                }
+            npos = __syncthreads_or(npos);
+            const bool uniform = (npos == 0);
+            double S = 0.0;
+            if (uniform) {
+                int na = 0;
+                for (int m = threadIdx.x; m < L; m += blockDim.x) na += (nb[m] < 0);
+                S = (double)block_sum_ll(na, lscr);
+            } else {
+                S = block_sum(sp, dscr);
+            }
+            int ncap = 0;
+            for (int m = threadIdx.x; m < L; m += blockDim.x) {
+                if (nb[m] >= 0) continue;
+                const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
+                if (!uniform && !(w > 0.0)) continue;
+                const double q = (double)remaining * w / S;
+                if (q > (double)N) ncap += 1;
+            }
+            ncap = (int)block_sum_ll(ncap, lscr);
+            if (ncap > 0) {
+                for (int m = threadIdx.x; m < L; m += blockDim.x) {
+                    if (nb[m] >= 0) continue;
+                    const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
+                    if (!uniform && !(w > 0.0)) continue;
+                    if ((double)remaining * w / S > (double)N) nb[m] = N;
+                }
+                remaining -= (long long)N * ncap;
+                __syncthreads();
+                continue;
+            }
+            // largest remainder among the candidates
+            long long fsum = 0;
+            for (int m = threadIdx.x; m < L; m += blockDim.x) {
+                const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
+                const bool cand = nb[m] < 0 && (uniform || w > 0.0);
+                double frac = -1.0;
+                if (cand) {
+                    const double q = (double)remaining * w / S;
+                    const double fl = floor(q);
+                    frac = q - fl;
+                    fsum += (long long)fl;
+                }
+                ff[4 * lst[m] + 3] = frac;
+            }
+            const long long R = remaining - block_sum_ll(fsum, lscr);
+            __syncthreads();
+            for (int m = threadIdx.x; m < L; m += blockDim.x) {
+                const double fm = ff[4 * lst[m] + 3];
+                if (fm < 0.0) continue;
+                long long rank = 0;
+                for (int k = 0; k < L; ++k) {
+                    const double fk = ff[4 * lst[k] + 3];
+                    rank += (fk > fm || (fk == fm && k < m)) ? 1 : 0;
+                }
+                const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
+                const long long fl = (long long)floor((double)remaining * w / S);
+                nb[m] = (int)(fl + (rank < R ? 1 : 0));
+            }
+            __syncthreads();
+            break;
+        }
+        for (int m = threadIdx.x; m < L; m += blockDim.x)
+            if (nb[m] < 0) nb[m] = 0;
+    }
+    __syncthreads();
+    // scatter to frames, offsets, grids
+    for (int t = threadIdx.x; t < T; t += blockDim.x) c.n[base + t] = 0;
+    __syncthreads();
+    for (int m = threadIdx.x; m < L; m += blockDim.x) c.n[base + lst[m]] = nb[m];
+    __syncthreads();
+    int nloc[kPerThread];
+    int sum = 0;
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k) {
+        const int t = t0 + k;
+        nloc[k] = t < T ? c.n[base + t] : 0;
+        sum += nloc[k];
+    }
+    int produced = 0;
+    int o = block_excl_scan(sum, iscr, &produced);
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k) {
+        const int t = t0 + k;
+        if (t < T) {
+            c.off[base + t] = vp.row0 + o;
+            const int h = grid_h(nloc[k], c.H, c.W);
+            c.hw[2 * (base + t)] = h;
+            c.hw[2 * (base + t) + 1] = h > 0 ? (nloc[k] + h - 1) / h : 0;
+            if (c.out_budgets) c.out_budgets[base + t] = nloc[k];
+            if (c.out_rel) {
+                float *orl = c.out_rel + (base + t) * 4;
+                orl[0] = (float)fr[4 * t];
+                orl[1] = (float)fr[4 * t + 1];
+                orl[2] = (float)fr[4 * t + 2];
+                orl[3] = (float)fr[4 * t + 3];
+            }
+        }
+        o += nloc[k];
+    }
+    if (threadIdx.x == 0) {
+        c.prod[v] = produced;
+        if (c.out_count) c.out_count[v] = produced;
+    }
+    // tensor-core units: per frame, column blocks of <= 256 tokens; per
+    // block, groups of CG 128-channel tiles with CG * round16(nc) <= 256.
+    if (c.path == WZ_PATH_TENSOR) {
+        int ucnt[kPerThread];
+        int us = 0;
+#pragma unroll
+        for (int k = 0; k < kPerThread; ++k) {
+            ucnt[k] = 0;
+            for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
+                const int nc = min(kColBlock, nloc[k] - j0);
+                const int ncp = (nc + 15) / 16 * 16;
+                const int cg = max(1, min(4, kColBlock / ncp));
+                ucnt[k] += (c.n_ct + cg - 1) / cg;
+            }
+            us += ucnt[k];
+        }
+        int total = 0;
+        int u = block_excl_scan(us, iscr, &total);
+        int4 *units = c.units + (size_t)v * c.max_units_v;
+#pragma unroll
+        for (int k = 0; k < kPerThread; ++k) {
+            const int t = t0 + k;
+            for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
+                const int nc = min(kColBlock, nloc[k] - j0);
+                const int ncp = (nc + 15) / 16 * 16;
+                const int cg = max(1, min(4, kColBlock / ncp));
+                for (int ct = 0; ct < c.n_ct; ct += cg) {
+                    const int g = min(cg, c.n_ct - ct);
+                    if (u < c.max_units_v) units[u] = make_int4((int)(base + t), j0, ct, nc | (g << 16));
+                    ++u;
+                }
+            }
+        }
+        if (threadIdx.x == 0) {
+            c.ucount[v] = min(total, c.max_units_v);
+            if (total > c.max_units_v) atomicOr(c.status, 2);
+        }
+    }
+}
+
+cudaError_t launch_temporal(const Ctx &c, cudaStream_t s) {
+    temporal_kernel<<<c.V, kTemporalThreads, 0, s>>>(c);
+    return cudaGetLastError();
+}
+
+}  // namespace wz

@@ -1,0 +1,186 @@
+// Internal declarations of the WaveZip CUDA library (not part of the C ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/wavezip.h"
+
+namespace wz {
+
+constexpr int kMaxTaps = 20;          // Daubechies order <= 10
+constexpr int kG1Max = 2048;          // relevance-pass CTAs (upper bound)
+constexpr int kStatsChunk = 256;      // channels per frame-stats block
+constexpr int kColBlock = 256;        // output tokens per tensor-core unit
+constexpr int kTileC = 128;           // channels per tensor-core M tile
+
+// Per-video parameters written to the workspace by the query-pool kernel.
+struct VideoPar {
+    int q_row0;    // first query row of the video
+    int Lq;        // query rows
+    int B;         // global budget of the video
+    int row0;      // first output row of the video
+};
+
+// Everything a kernel of one call needs: sizes, inputs, workspace views,
+// outputs and scalar parameters.  Passed by value.
+struct Ctx {
+    int V, T, H, W, D, N;
+    int dtype;            // WZ_DTYPE_*
+    int hp, wp;           // WSM subband sizes
+    int K_pad;            // N rounded up to 32 (row length of the operator)
+    int G1;               // relevance CTAs actually launched
+    int DC;               // frame-stats blocks per frame
+    int n_ct;             // 128-channel tiles
+    int max_units_v;      // unit-list capacity per video
+    int F;                // WSM filter taps
+    int64_t L1;           // tokens per relevance CTA
+    int64_t rows_total;   // sum of budgets over videos (operator rows)
+
+    const void *X;
+    const void *Q;
+
+    float *qbar32;        // [V][D]
+    double *qbar64;       // [V][D]
+    double *qnorm;        // [V]
+    VideoPar *vpar;       // [V]
+    float *a;             // [V*T][N] token saliency
+    float *part;          // [G1 + V*T][D] column-sum partials
+    double *trip;         // [V*T][DC][3] (v.q, v.v, v.v_prev)
+    double *fr;           // [V*T][4] (r, delta, gamma, r~)
+    double *tmp;          // [V*T][4] temporal-kernel scratch
+    int *list;            // [V][2T] retained frames and their budgets
+    int *n;               // [V*T] budgets
+    int *off;             // [V*T] global output row of the frame's first token
+    int *hw;              // [V*T][2] condensation grid
+    int *prod;            // [V] produced rows
+    int4 *units;          // [V][max_units_v] tensor-core work units
+    int *ucount;          // [V]
+    void *Wop;            // operator rows: bf16 hi [rows][K_pad] then lo, or f32
+    int *status;          // device status word (bounded waits)
+
+    void *out;            // [rows][D] dtype
+    int *out_index;       // [rows][3]
+    int *out_budgets;     // [V*T] or null
+    int *out_count;       // [V] or null
+    float *out_rel;       // [V*T][4] or null
+    float *frame_mean;    // [V*T][D] or null (relevance entry point)
+    float *frame_scores;  // [V*T] or null (relevance entry point)
+
+    float lambda, tau;
+    int mode;             // WZ_MODE_*
+    int path;             // resolved WZ_PATH_TENSOR or WZ_PATH_SIMT
+    float dec_lo[kMaxTaps], dec_hi[kMaxTaps], rec_lo[kMaxTaps], rec_hi[kMaxTaps];
+};
+
+// ---- device helpers -------------------------------------------------------
+
+__device__ __forceinline__ int ext_index(int i, int n, int mode) {
+    if (i >= 0 && i < n) return i;
+    if (mode == WZ_MODE_ZERO) return -1;
+    if (mode == WZ_MODE_PERIODIC) {
+        int k = i % n;
+        return k < 0 ? k + n : k;
+    }
+    int p = 2 * n;
+    int k = i % p;
+    if (k < 0) k += p;
+    return k < n ? k : p - 1 - k;
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+template <typename T> struct VecOf;
+template <> struct VecOf<__nv_bfloat16> { static constexpr int kElems = 8; };
+template <> struct VecOf<float> { static constexpr int kElems = 4; };
+
+// Unpack a 16-byte vector into floats.
+__device__ __forceinline__ void unpack(const uint4 &v, float (&f)[8], __nv_bfloat16 *) {
+    f[0] = bf16_lo(v.x); f[1] = bf16_hi(v.x);
+    f[2] = bf16_lo(v.y); f[3] = bf16_hi(v.y);
+    f[4] = bf16_lo(v.z); f[5] = bf16_hi(v.z);
+    f[6] = bf16_lo(v.w); f[7] = bf16_hi(v.w);
+}
+__device__ __forceinline__ void unpack(const uint4 &v, float (&f)[4], float *) {
+    f[0] = __uint_as_float(v.x); f[1] = __uint_as_float(v.y);
+    f[2] = __uint_as_float(v.z); f[3] = __uint_as_float(v.w);
+}
+
+__device__ __forceinline__ uint4 ldg_stream(const uint4 *p) {
+    uint4 r;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(p));
+    return r;
+}
+
+template <typename T>
+__device__ __forceinline__ float load_scalar(const T *p);
+template <> __device__ __forceinline__ float load_scalar<float>(const float *p) { return *p; }
+template <> __device__ __forceinline__ float load_scalar<__nv_bfloat16>(const __nv_bfloat16 *p) {
+    return __bfloat162float(*p);
+}
+
+template <typename T>
+__device__ __forceinline__ T from_float(float v);
+template <> __device__ __forceinline__ float from_float<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(float v) {
+    return __float2bfloat16_rn(v);
+}
+
+// Block-wide sum of a double in a fixed order (deterministic for a fixed
+// block size).  `scratch` holds >= 32 doubles; all threads receive the sum.
+__device__ __forceinline__ double block_sum(double v, double *scratch) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nw = (blockDim.x + 31) >> 5;
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) scratch[warp] = v;
+    __syncthreads();
+    double s = 0.0;
+    for (int w = 0; w < nw; ++w) s += scratch[w];
+    __syncthreads();
+    return s;
+}
+
+__device__ __forceinline__ long long block_sum_ll(long long v, long long *scratch) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nw = (blockDim.x + 31) >> 5;
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) scratch[warp] = v;
+    __syncthreads();
+    long long s = 0;
+    for (int w = 0; w < nw; ++w) s += scratch[w];
+    __syncthreads();
+    return s;
+}
+
+// ---- launchers (one per kernel family) -------------------------------------
+
+cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s);
+cudaError_t launch_relevance_pass(const Ctx &c, cudaStream_t s);
+cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s);
+cudaError_t launch_relevance_finalize(const Ctx &c, cudaStream_t s);
+cudaError_t launch_temporal(const Ctx &c, cudaStream_t s);
+cudaError_t launch_spatial(const Ctx &c, cudaStream_t s);
+cudaError_t launch_condense_simt(const Ctx &c, cudaStream_t s);
+cudaError_t launch_condense_tc(const Ctx &c, cudaStream_t s);
+int relevance_grid(const Ctx &c);   // CTAs for the relevance pass on this device
+
+cudaError_t launch_dwt1d(const float *x, int rows, int L, int F, int mode, const float *dlo,
+                         const float *dhi, float *cA, float *cD, cudaStream_t s);
+cudaError_t launch_idwt1d(const float *cA, const float *cD, int rows, int L, int F,
+                          const float *rlo, const float *rhi, float *x, cudaStream_t s);
+cudaError_t launch_dwt2d(const void *X, int dtype, int T, int H, int W, int D, int F, int mode,
+                         const float *dlo, const float *dhi, float *LL, float *LH, float *HL,
+                         float *HH, cudaStream_t s);
+cudaError_t launch_idwt2d(const float *LL, const float *LH, const float *HL, const float *HH,
+                          int T, int H, int W, int D, int F, const float *rlo, const float *rhi,
+                          float *out, cudaStream_t s);
+
+// Host: Daubechies filter bank of order p (2p taps); false if p is out of range.
+bool daubechies(int p, double *dec_lo, double *dec_hi, double *rec_lo, double *rec_hi);
+
+}  // namespace wz

@@ -1,0 +1,333 @@
+"""Python binding of the WaveZip C ABI (include/wavezip.h).
+
+Argument marshalling only: every function allocates its outputs as torch
+tensors on the inputs' device, passes raw device pointers and the current
+CUDA stream to the library, and raises WaveZipError on a nonzero status.  All
+computation happens in the CUDA kernels of libwavezip.so; there is no other
+implementation to fall back to, and importing fails if the library is absent.
+"""
+
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libwavezip.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_NO_MEMORY, ERR_WORKSPACE = 0, -1, -2, -3, -4, -5
+DTYPE_BF16, DTYPE_F32 = 0, 1
+MODE_SYMMETRIC, MODE_ZERO, MODE_PERIODIC = 0, 1, 2
+PATH_AUTO, PATH_TENSOR, PATH_SIMT = 0, 1, 2
+MODES = {"symmetric": MODE_SYMMETRIC, "zero": MODE_ZERO, "periodic": MODE_PERIODIC}
+PATHS = {"auto": PATH_AUTO, "tensor": PATH_TENSOR, "simt": PATH_SIMT}
+
+
+class WaveZipError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+class CondenseArgs(C.Structure):
+    _fields_ = [
+        ("features", C.c_void_p), ("T", C.c_int), ("H", C.c_int), ("W", C.c_int), ("D", C.c_int),
+        ("dtype", C.c_int), ("query", C.c_void_p), ("Lq", C.c_int), ("ratio", C.c_float),
+        ("lam", C.c_float), ("tau", C.c_float), ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int),
+        ("mode", C.c_int), ("path", C.c_int), ("out_tokens", C.c_void_p), ("out_index", C.c_void_p),
+        ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
+        ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
+        ("kernel_events", C.POINTER(C.c_void_p)), ("stream", C.c_void_p),
+    ]
+
+
+class BatchArgs(C.Structure):
+    _fields_ = [
+        ("V", C.c_int), ("features", C.c_void_p), ("T", C.c_int), ("H", C.c_int), ("W", C.c_int),
+        ("D", C.c_int), ("dtype", C.c_int), ("queries", C.c_void_p), ("Lq", C.POINTER(C.c_int32)),
+        ("ratio", C.POINTER(C.c_float)), ("lam", C.c_float), ("tau", C.c_float),
+        ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int), ("mode", C.c_int), ("path", C.c_int),
+        ("out_tokens", C.c_void_p), ("out_index", C.c_void_p), ("row_offsets", C.POINTER(C.c_int64)),
+        ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
+        ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
+        ("kernel_events", C.POINTER(C.c_void_p)), ("stream", C.c_void_p),
+    ]
+
+NUM_KERNELS = 6
+KERNEL_NAMES = ("query_pool", "relevance", "frame_stats", "temporal", "spatial", "condense")
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2607_23265_gb300.build` "
+                          "(the WaveZip path has no non-CUDA implementation)")
+    lib = C.CDLL(LIB_PATH)
+    vp, i, f, sz, i64 = C.c_void_p, C.c_int, C.c_float, C.c_size_t, C.c_int64
+    sig = {
+        "wz_budget_size": (i64, [i, i, i, f]),
+        "wz_condense": (i, [vp, i, i, i, i, vp, i, f, vp, vp, vp]),
+        "wz_condense_args_init": (None, [C.POINTER(CondenseArgs)]),
+        "wz_condense_workspace_size": (sz, [i, i, i, i, i, f]),
+        "wz_condense_ex": (i, [C.POINTER(CondenseArgs)]),
+        "wz_batch_args_init": (None, [C.POINTER(BatchArgs)]),
+        "wz_batch_rows": (i64, [i, i, i, i, C.POINTER(C.c_float), C.POINTER(C.c_int64)]),
+        "wz_batch_workspace_size": (sz, [i, i, i, i, i, i, C.POINTER(C.c_float)]),
+        "wz_condense_batch": (i, [C.POINTER(BatchArgs)]),
+        "wz_relevance": (i, [vp, i, i, i, i, i, vp, i, vp, vp, vp, vp, sz, vp]),
+        "wz_relevance_workspace_size": (sz, [i, i, i, i]),
+        "wz_dwt_len": (i, [i, i]),
+        "wz_wavelet_filters": (i, [i] + [C.POINTER(C.c_double)] * 4),
+        "wz_dwt1d": (i, [vp, i, i, i, i, vp, vp, vp]),
+        "wz_idwt1d": (i, [vp, vp, i, i, i, vp, vp]),
+        "wz_dwt2d": (i, [vp, i, i, i, i, i, i, i, vp, vp, vp, vp, vp]),
+        "wz_idwt2d": (i, [vp, vp, vp, vp, i, i, i, i, i, vp, vp]),
+        "wz_status_string": (C.c_char_p, [i]),
+        "wz_version": (i, []),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+_lib = _load()
+
+
+def status_string(status: int) -> str:
+    return _lib.wz_status_string(int(status)).decode()
+
+
+def _check(status: int, where: str):
+    if status != OK:
+        raise WaveZipError(status, where)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return DTYPE_BF16
+    if t.dtype == torch.float32:
+        return DTYPE_F32
+    raise TypeError(f"features must be bfloat16 or float32, got {t.dtype}")
+
+
+def _stream(stream, device) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream(device)
+    return int(stream.cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _cuda_contig(t: torch.Tensor, name: str) -> torch.Tensor:
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    return t.contiguous()
+
+
+# --------------------------------------------------------------------------
+# Condensation
+# --------------------------------------------------------------------------
+
+def wz_budget_size(T: int, H: int, W: int, ratio: float) -> int:
+    return int(_lib.wz_budget_size(T, H, W, ratio))
+
+
+def wz_condense_workspace_size(T, H, W, D, dtype=DTYPE_BF16, ratio=0.1) -> int:
+    return int(_lib.wz_condense_workspace_size(T, H, W, D, dtype, ratio))
+
+
+def wz_condense(features: torch.Tensor, query: torch.Tensor, ratio: float, stream=None):
+    """wz_condense: bf16 [T,H,W,D] features, [Lq,D] query -> (tokens [B,D], index [B,3])."""
+    features = _cuda_contig(features, "features")
+    query = _cuda_contig(query, "query")
+    T, H, W, D = features.shape
+    B = wz_budget_size(T, H, W, ratio)
+    if B < 0:
+        raise WaveZipError(ERR_INVALID_ARG, "wz_condense")
+    tokens = torch.empty((B, D), dtype=features.dtype, device=features.device)
+    index = torch.empty((B, 3), dtype=torch.int32, device=features.device)
+    st = _lib.wz_condense(features.data_ptr(), T, H, W, D, query.data_ptr(), query.shape[0], ratio,
+                          tokens.data_ptr(), index.data_ptr(), _stream(stream, features.device))
+    _check(st, "wz_condense")
+    return tokens, index
+
+
+def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *, lam: float = 1.5,
+                   tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
+                   workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
+                   device_status: torch.Tensor | None = None, kernel_events=None, stream=None):
+    """wz_condense_ex.  Returns a dict with tokens, index, budgets, count and relevance.
+
+    kernel_events: optional list of 2*NUM_KERNELS recorded torch.cuda.Event
+    objects; event 2k / 2k+1 is recorded right before / after kernel k."""
+    features = _cuda_contig(features, "features")
+    query = _cuda_contig(query, "query")
+    T, H, W, D = features.shape
+    dev = features.device
+    B = wz_budget_size(T, H, W, ratio)
+    if B < 0:
+        raise WaveZipError(ERR_INVALID_ARG, "wz_condense_ex")
+    tokens = out_tokens if out_tokens is not None else torch.empty((B, D), dtype=features.dtype, device=dev)
+    index = out_index if out_index is not None else torch.empty((B, 3), dtype=torch.int32, device=dev)
+    budgets = torch.empty((T,), dtype=torch.int32, device=dev)
+    count = torch.empty((1,), dtype=torch.int32, device=dev)
+    rel = torch.empty((T, 4), dtype=torch.float32, device=dev)
+    a = CondenseArgs()
+    _lib.wz_condense_args_init(C.byref(a))
+    a.features, a.T, a.H, a.W, a.D = features.data_ptr(), T, H, W, D
+    a.dtype = _dtype_code(features)
+    a.query, a.Lq, a.ratio = query.data_ptr(), query.shape[0], ratio
+    a.lam, a.tau, a.wsm_wavelet = lam, tau, wsm_wavelet
+    a.mode = MODES[mode] if isinstance(mode, str) else int(mode)
+    a.path = PATHS[path] if isinstance(path, str) else int(path)
+    a.out_tokens, a.out_index = tokens.data_ptr(), index.data_ptr()
+    a.out_budgets, a.out_count, a.out_relevance = budgets.data_ptr(), count.data_ptr(), rel.data_ptr()
+    if workspace is not None:
+        a.workspace, a.workspace_bytes = workspace.data_ptr(), workspace.numel() * workspace.element_size()
+    a.device_status = _ptr(device_status)
+    if kernel_events is not None:
+        handles = (C.c_void_p * (2 * NUM_KERNELS))(*[e.cuda_event for e in kernel_events])
+        a.kernel_events = handles
+    a.stream = _stream(stream, dev)
+    _check(_lib.wz_condense_ex(C.byref(a)), "wz_condense_ex")
+    return {"tokens": tokens, "index": index, "budgets": budgets, "count": count, "relevance": rel}
+
+
+def wz_batch_rows(V, T, H, W, ratios):
+    r = (C.c_float * V)(*ratios)
+    offs = (C.c_int64 * (V + 1))()
+    rows = _lib.wz_batch_rows(V, T, H, W, r, offs)
+    if rows < 0:
+        raise WaveZipError(ERR_INVALID_ARG, "wz_batch_rows")
+    return int(rows), [int(o) for o in offs]
+
+
+def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios, *, lam: float = 1.5,
+                      tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
+                      workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
+                      stream=None):
+    """wz_condense_batch: features [V,T,H,W,D], queries [sum Lq, D]."""
+    features = _cuda_contig(features, "features")
+    queries = _cuda_contig(queries, "queries")
+    V, T, H, W, D = features.shape
+    dev = features.device
+    rows, offs = wz_batch_rows(V, T, H, W, ratios)
+    tokens = out_tokens if out_tokens is not None else torch.empty((rows, D), dtype=features.dtype, device=dev)
+    index = out_index if out_index is not None else torch.empty((rows, 3), dtype=torch.int32, device=dev)
+    budgets = torch.empty((V, T), dtype=torch.int32, device=dev)
+    count = torch.empty((V,), dtype=torch.int32, device=dev)
+    rel = torch.empty((V, T, 4), dtype=torch.float32, device=dev)
+    lq = (C.c_int32 * V)(*[int(x) for x in Lq])
+    rt = (C.c_float * V)(*[float(x) for x in ratios])
+    ro = (C.c_int64 * (V + 1))()
+    a = BatchArgs()
+    _lib.wz_batch_args_init(C.byref(a))
+    a.V, a.features, a.T, a.H, a.W, a.D = V, features.data_ptr(), T, H, W, D
+    a.dtype = _dtype_code(features)
+    a.queries, a.Lq, a.ratio = queries.data_ptr(), lq, rt
+    a.lam, a.tau, a.wsm_wavelet = lam, tau, wsm_wavelet
+    a.mode = MODES[mode] if isinstance(mode, str) else int(mode)
+    a.path = PATHS[path] if isinstance(path, str) else int(path)
+    a.out_tokens, a.out_index, a.row_offsets = tokens.data_ptr(), index.data_ptr(), ro
+    a.out_budgets, a.out_count, a.out_relevance = budgets.data_ptr(), count.data_ptr(), rel.data_ptr()
+    if workspace is not None:
+        a.workspace, a.workspace_bytes = workspace.data_ptr(), workspace.numel() * workspace.element_size()
+    a.stream = _stream(stream, dev)
+    _check(_lib.wz_condense_batch(C.byref(a)), "wz_condense_batch")
+    return {"tokens": tokens, "index": index, "budgets": budgets, "count": count, "relevance": rel,
+            "row_offsets": [int(ro[v]) for v in range(V + 1)]}
+
+
+def wz_batch_workspace_size(V, T, H, W, D, dtype, ratios) -> int:
+    rt = (C.c_float * V)(*[float(x) for x in ratios])
+    return int(_lib.wz_batch_workspace_size(V, T, H, W, D, dtype, rt))
+
+
+# --------------------------------------------------------------------------
+# Relevance and DWT
+# --------------------------------------------------------------------------
+
+def wz_relevance(features: torch.Tensor, query: torch.Tensor, *, frame_mean: bool = False,
+                 workspace: torch.Tensor | None = None, stream=None):
+    """(token_scores [T,H*W], frame_scores [T], frame_mean [T,D] or None)."""
+    features = _cuda_contig(features, "features")
+    query = _cuda_contig(query, "query")
+    T, H, W, D = features.shape
+    dev = features.device
+    ts = torch.empty((T, H * W), dtype=torch.float32, device=dev)
+    fs = torch.empty((T,), dtype=torch.float32, device=dev)
+    fm = torch.empty((T, D), dtype=torch.float32, device=dev) if frame_mean else None
+    wsp, wsb = (workspace.data_ptr(), workspace.numel() * workspace.element_size()) if workspace is not None else (None, 0)
+    st = _lib.wz_relevance(features.data_ptr(), T, H, W, D, _dtype_code(features), query.data_ptr(),
+                           query.shape[0], ts.data_ptr(), fs.data_ptr(), _ptr(fm), wsp, wsb,
+                           _stream(stream, dev))
+    _check(st, "wz_relevance")
+    return ts, fs, fm
+
+
+def wz_relevance_workspace_size(T, H, W, D) -> int:
+    return int(_lib.wz_relevance_workspace_size(T, H, W, D))
+
+
+def wz_dwt_len(n: int, wavelet: int = 4) -> int:
+    return int(_lib.wz_dwt_len(n, wavelet))
+
+
+def wz_wavelet_filters(wavelet: int = 4):
+    F = 2 * wavelet
+    bufs = [(C.c_double * F)() for _ in range(4)]
+    _check(_lib.wz_wavelet_filters(wavelet, *bufs), "wz_wavelet_filters")
+    return {k: [float(x) for x in b] for k, b in zip(("dec_lo", "dec_hi", "rec_lo", "rec_hi"), bufs)}
+
+
+def wz_dwt1d(x: torch.Tensor, wavelet: int = 4, mode="symmetric", stream=None):
+    x = _cuda_contig(x, "x").float()
+    rows, L = x.shape
+    Lo = wz_dwt_len(L, wavelet)
+    cA = torch.empty((rows, Lo), dtype=torch.float32, device=x.device)
+    cD = torch.empty_like(cA)
+    st = _lib.wz_dwt1d(x.data_ptr(), rows, L, wavelet, MODES[mode] if isinstance(mode, str) else mode,
+                       cA.data_ptr(), cD.data_ptr(), _stream(stream, x.device))
+    _check(st, "wz_dwt1d")
+    return cA, cD
+
+
+def wz_idwt1d(cA: torch.Tensor, cD: torch.Tensor, L: int, wavelet: int = 4, stream=None):
+    cA = _cuda_contig(cA, "cA").float()
+    cD = _cuda_contig(cD, "cD").float()
+    x = torch.empty((cA.shape[0], L), dtype=torch.float32, device=cA.device)
+    st = _lib.wz_idwt1d(cA.data_ptr(), cD.data_ptr(), cA.shape[0], L, wavelet, x.data_ptr(),
+                        _stream(stream, cA.device))
+    _check(st, "wz_idwt1d")
+    return x
+
+
+def wz_dwt2d(features: torch.Tensor, wavelet: int = 4, mode="symmetric", stream=None):
+    features = _cuda_contig(features, "features")
+    T, H, W, D = features.shape
+    hp, wp = wz_dwt_len(H, wavelet), wz_dwt_len(W, wavelet)
+    bands = [torch.empty((T, hp, wp, D), dtype=torch.float32, device=features.device) for _ in range(4)]
+    st = _lib.wz_dwt2d(features.data_ptr(), T, H, W, D, _dtype_code(features), wavelet,
+                       MODES[mode] if isinstance(mode, str) else mode, *[b.data_ptr() for b in bands],
+                       _stream(stream, features.device))
+    _check(st, "wz_dwt2d")
+    return tuple(bands)
+
+
+def wz_idwt2d(LL, LH, HL, HH, H: int, W: int, wavelet: int = 4, stream=None):
+    bands = [_cuda_contig(b, "band").float() for b in (LL, LH, HL, HH)]
+    T, _, _, D = bands[0].shape
+    out = torch.empty((T, H, W, D), dtype=torch.float32, device=bands[0].device)
+    st = _lib.wz_idwt2d(*[b.data_ptr() for b in bands], T, H, W, D, wavelet, out.data_ptr(),
+                        _stream(stream, bands[0].device))
+    _check(st, "wz_idwt2d")
+    return out
+
+
+def wz_version() -> int:
+    return int(_lib.wz_version())
