@@ -1,11 +1,325 @@
-// Condensed tokens Z_m = W_m X_m on the tcgen05 tensor cores (placeholder
-// until the tensor-core kernel lands; the CUDA-core path serves meanwhile).
+// Condensed tokens Z_m = W_m X_m on the 5th-generation tensor cores
+// (tcgen05.mma, TMA, tensor memory) -- the fused WSM + bilinear + pack step
+// (Eq. 11-14, 16, 18) as one streaming pass over the features.
+//
+// Orientation: the MMA computes D[c][j] = sum_k X_m[k][c] * W_m[j][k] with
+//   A = X tile, M = 128 channels, K = 16 tokens, MN-major (channels
+//       contiguous, exactly as the features lie in HBM), loaded by TMA with
+//       128-byte swizzle, box 64 channels x 32 tokens x 1 frame;
+//   B = W tile, N = n (the frame's condensed tokens, <= 256 per unit, padded
+//       to 16), K-major, loaded by TMA with 64-byte swizzle;
+//   D = fp32 accumulators in tensor memory, 128 lanes x N columns per
+//       128-channel tile.
+// W_m is fp32 split into bf16 hi + lo (two MMAs into one accumulator), so the
+// product keeps ~16 bits of W while X (exact in bf16) streams once.
+//
+// A unit of work is (frame, <= 256 output tokens, CG <= 4 channel tiles) with
+// CG * N <= 256 accumulator columns; two accumulator buffers let the
+// epilogue of one unit overlap the main loop of the next.  One CTA per SM,
+// persistent over the unit list:
+//   warp 0     TMA producer (one thread), 5-stage shared-memory ring
+//   warp 1     TMEM allocation and the MMA issuer (one thread)
+//   warps 2-5  epilogue: tcgen05.ld -> bf16 -> packed output rows
+// Every mbarrier wait is bounded; on a timeout the kernel records a status
+// bit, drains what it issued, frees tensor memory and exits.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "wz_internal.cuh"
+#include "wz_ptx.cuh"
 
 namespace wz {
 
-bool tensor_path_available() { return false; }
+namespace {
 
-cudaError_t launch_condense_tc(const Ctx &, cudaStream_t) { return cudaErrorNotSupported; }
+constexpr int kKC = 32;                    // tokens per K chunk (two K=16 MMA steps)
+constexpr int kStages = 5;
+constexpr int kStageBytes = 40 * 1024;     // >= CG*8 KB (X) + 2*N*64 B (W hi, lo)
+constexpr int kThreads = 192;
+constexpr int kTmemCols = 512;
+constexpr int kAccCols = 256;
+constexpr uint64_t kTimeoutNs = 2000000000ull;
+
+struct TcShared {
+    uint64_t full[kStages];
+    uint64_t empty[kStages];
+    uint64_t tfull[2];
+    uint64_t tempty[2];
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort;
+    int vprefix[WZ_MAX_VIDEOS + 1];
+};
+
+constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + sizeof(TcShared);
+
+struct Unit {
+    int f, j0, ct0, nc, cg;
+};
+
+__device__ __forceinline__ Unit decode_unit(const Ctx &c, const int *vprefix, int u) {
+    int lo = 0, hi = c.V - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (vprefix[mid] <= u) lo = mid;
+        else hi = mid - 1;
+    }
+    const int4 q = c.units[(size_t)lo * c.max_units_v + (u - vprefix[lo])];
+    Unit r;
+    r.f = q.x;
+    r.j0 = q.y;
+    r.ct0 = q.z;
+    r.nc = q.w & 0xffff;
+    r.cg = q.w >> 16;
+    return r;
+}
+
+__device__ __forceinline__ void fail(const Ctx &c, volatile int *abort_flag, int code) {
+    *abort_flag = 1;
+    atomicOr(c.status, code);
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(kThreads, 1)
+condense_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmWhi,
+                   const __grid_constant__ CUtensorMap tmWlo, Ctx c) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    TcShared *S = reinterpret_cast<TcShared *>(ring + (size_t)kStages * kStageBytes);
+    volatile int *abort_flag = &S->abort;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            ptx::mbar_init(&S->full[s], 1);
+            ptx::mbar_init(&S->empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            ptx::mbar_init(&S->tfull[b], 1);
+            ptx::mbar_init(&S->tempty[b], 4);
+        }
+        ptx::mbar_init(&S->drain, 1);
+        S->abort = 0;
+        int acc = 0;
+        for (int v = 0; v < c.V; ++v) {
+            S->vprefix[v] = acc;
+            acc += c.ucount[v];
+        }
+        S->vprefix[c.V] = acc;
+        ptx::fence_barrier_init();
+        ptx::fence_proxy_async_smem();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(&S->tmem_base, kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    if (warp == 0 && lane == 0) {
+        ptx::prefetch_tmap(&tmX);
+        ptx::prefetch_tmap(&tmWhi);
+        ptx::prefetch_tmap(&tmWlo);
+    }
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = S->tmem_base;
+    const int n_units = S->vprefix[c.V];
+    const int KC = c.K_pad / kKC;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer ----------------
+        const uint64_t pol_x = ptx::policy_evict_first();
+        const uint64_t pol_w = ptx::policy_evict_last();
+        int stage = 0;
+        uint32_t phase = 0;
+        int issued_parity[kStages];
+        for (int s = 0; s < kStages; ++s) issued_parity[s] = -1;
+        for (int u = blockIdx.x; u < n_units && !*abort_flag; u += gridDim.x) {
+            const Unit un = decode_unit(c, S->vprefix, u);
+            const int ncp = (un.nc + 15) & ~15;
+            const int row0 = c.off[un.f] + un.j0;
+            const uint32_t bytes = (uint32_t)un.cg * 8192u + 2u * (uint32_t)ncp * 64u;
+            bool ok = true;
+            for (int kc = 0; kc < KC; ++kc) {
+                if (!ptx::mbar_wait(&S->empty[stage], phase ^ 1u, kTimeoutNs)) {
+                    fail(c, abort_flag, 1);
+                    ok = false;
+                    break;
+                }
+                uint8_t *st = ring + (size_t)stage * kStageBytes;
+                ptx::mbar_arrive_expect_tx(&S->full[stage], bytes);
+                for (int ct = 0; ct < un.cg; ++ct)
+                    for (int h = 0; h < 2; ++h)
+                        ptx::tma_load_3d(st + ct * 8192 + h * 4096, &tmX, &S->full[stage],
+                                         (un.ct0 + ct) * kTileC + h * 64, kc * kKC, un.f, pol_x);
+                uint8_t *wh = st + un.cg * 8192;
+                for (int r = 0; r < ncp; r += 16) {
+                    ptx::tma_load_2d(wh + r * 64, &tmWhi, &S->full[stage], kc * kKC, row0 + r, pol_w);
+                    ptx::tma_load_2d(wh + ncp * 64 + r * 64, &tmWlo, &S->full[stage], kc * kKC, row0 + r, pol_w);
+                }
+                issued_parity[stage] = (int)phase;
+                if (++stage == kStages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok) break;
+        }
+        // let every copy this thread issued land before the CTA can exit
+        for (int s = 0; s < kStages; ++s)
+            if (issued_parity[s] >= 0) ptx::mbar_wait(&S->full[s], (uint32_t)issued_parity[s], kTimeoutNs);
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer ----------------
+        int stage = 0;
+        uint32_t phase = 0;
+        int it = 0;
+        for (int u = blockIdx.x; u < n_units && !*abort_flag; u += gridDim.x, ++it) {
+            const Unit un = decode_unit(c, S->vprefix, u);
+            const int ncp = (un.nc + 15) & ~15;
+            const int b = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1);
+            if (!ptx::mbar_wait(&S->tempty[b], (use & 1u) ^ 1u, kTimeoutNs)) {
+                fail(c, abort_flag, 2);
+                break;
+            }
+            ptx::tc_fence_after();
+            const uint32_t idesc = ptx::idesc_bf16(128, ncp, true, false);
+            const uint32_t dbase = tmem + (uint32_t)(b * kAccCols);
+            bool ok = true;
+            for (int kc = 0; kc < KC; ++kc) {
+                if (!ptx::mbar_wait(&S->full[stage], phase, kTimeoutNs)) {
+                    fail(c, abort_flag, 4);
+                    ok = false;
+                    break;
+                }
+                ptx::tc_fence_after();
+                const uint32_t st = ptx::smem_u32(ring + (size_t)stage * kStageBytes);
+                const uint32_t wh = st + (uint32_t)un.cg * 8192u;
+                const uint32_t wl = wh + (uint32_t)ncp * 64u;
+#pragma unroll
+                for (int s = 0; s < 2; ++s) {
+                    const uint64_t bh = ptx::smem_desc(wh + s * 32, 16, 512, 4);
+                    const uint64_t bl = ptx::smem_desc(wl + s * 32, 16, 512, 4);
+                    for (int ct = 0; ct < un.cg; ++ct) {
+                        const uint64_t a = ptx::smem_desc(st + ct * 8192 + s * 2048, 4096, 1024, 2);
+                        const uint32_t d = dbase + (uint32_t)(ct * ncp);
+                        ptx::mma_bf16(d, a, bh, idesc, (kc | s) ? 1u : 0u);
+                        ptx::mma_bf16(d, a, bl, idesc, 1u);
+                    }
+                }
+                ptx::mma_commit(&S->empty[stage]);
+                if (++stage == kStages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok) break;
+            ptx::mma_commit(&S->tfull[b]);
+        }
+        // every MMA issued by this thread completes before tensor memory is freed
+        ptx::mma_commit(&S->drain);
+        ptx::mbar_wait(&S->drain, 0, kTimeoutNs);
+    } else if (warp >= 2) {
+        // ---------------- epilogue ----------------
+        const int q = warp & 3;                          // TMEM lane quadrant of this warp
+        __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(c.out);
+        int it = 0;
+        for (int u = blockIdx.x; u < n_units && !*abort_flag; u += gridDim.x, ++it) {
+            const Unit un = decode_unit(c, S->vprefix, u);
+            const int ncp = (un.nc + 15) & ~15;
+            const int b = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1);
+            if (!ptx::mbar_wait(&S->tfull[b], use & 1u, kTimeoutNs)) {
+                fail(c, abort_flag, 8);
+                break;
+            }
+            ptx::tc_fence_after();
+            const size_t row0 = (size_t)c.off[un.f] + un.j0;
+            for (int ct = 0; ct < un.cg; ++ct) {
+                const int ch = (un.ct0 + ct) * kTileC + q * 32 + lane;
+                for (int j0 = 0; j0 < ncp; j0 += 16) {
+                    uint32_t r[16];
+                    ptx::tmem_ld_32x32b_x16(tmem + ((uint32_t)(q * 32) << 16) +
+                                                (uint32_t)(b * kAccCols + ct * ncp + j0), r);
+                    ptx::tmem_ld_wait();
+                    if (ch < c.D) {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            if (j0 + j < un.nc)
+                                out[(row0 + j0 + j) * (size_t)c.D + ch] = __float2bfloat16_rn(__uint_as_float(r[j]));
+                    }
+                }
+            }
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&S->tempty[b]);
+        }
+    }
+    __syncthreads();
+    if (warp == 1) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+}  // namespace
+
+bool tensor_path_available() { return true; }
+
+cudaError_t launch_condense_tc(const Ctx &c, cudaStream_t s) {
+    auto enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    if (c.dtype != WZ_DTYPE_BF16 || c.rows_total < 1) return cudaErrorInvalidValue;
+    CUtensorMap tmX, tmWhi, tmWlo;
+    {
+        cuuint64_t dims[3] = {(cuuint64_t)c.D, (cuuint64_t)c.N, (cuuint64_t)c.V * c.T};
+        cuuint64_t strides[2] = {(cuuint64_t)c.D * 2, (cuuint64_t)c.N * c.D * 2};
+        cuuint32_t box[3] = {64, (cuuint32_t)kKC, 1};
+        cuuint32_t es[3] = {1, 1, 1};
+        if (enc(&tmX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(c.X), dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    __nv_bfloat16 *whi = static_cast<__nv_bfloat16 *>(c.Wop);
+    __nv_bfloat16 *wlo = whi + (size_t)c.rows_total * c.K_pad;
+    {
+        cuuint64_t dims[2] = {(cuuint64_t)c.K_pad, (cuuint64_t)c.rows_total};
+        cuuint64_t strides[1] = {(cuuint64_t)c.K_pad * 2};
+        cuuint32_t box[2] = {(cuuint32_t)kKC, 16};
+        cuuint32_t es[2] = {1, 1};
+        if (enc(&tmWhi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, whi, dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+        if (enc(&tmWlo, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, wlo, dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(condense_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    condense_tc_kernel<<<sms, kThreads, kSmemBytes, s>>>(tmX, tmWhi, tmWlo, c);
+    return cudaGetLastError();
+}
 
 }  // namespace wz
