@@ -227,6 +227,33 @@ WZ_API int wz_relevance(const void *features, int T, int H, int W, int D, int dt
 
 WZ_API size_t wz_relevance_workspace_size(int T, int H, int W, int D);
 
+/*
+ * The scores of wz_relevance for callers that must not allocate device
+ * memory.  The paper has no counterpart: this is a deployment convenience of
+ * this library.  Callers that need it include code running while a stream is
+ * captured into a CUDA graph that may hold no allocation nodes, serving loops
+ * that fix their memory budget at start-up so a request can never fail on an
+ * out-of-memory or wait on an allocator, and hosts whose device memory is
+ * managed by another framework's caching allocator.  Inputs and outputs are
+ * the caller's, as for wz_relevance; the intermediate sums go to one fixed
+ * array of WZ_STATIC_SCRATCH_BYTES compiled into the library, which every GPU
+ * that loads the library keeps until the process exits.
+ *   - No cudaMalloc, cudaFree or other allocating call is made.
+ *   - The first call on a device looks the array's device address up
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture.
+ *   - Sizes whose sums do not fit the array return WZ_ERR_WORKSPACE before
+ *     anything is enqueued (about (2*SMs + T) * D * 4 bytes are needed, e.g.
+ *     up to T = 256 frames at D = 3584 on a GB300).
+ *   - Every call shares the one array and keeps no state between calls
+ *     (nothing in it must start at zero), so calls that overlap on the GPU
+ *     (other streams, other host threads) race: serialise them.
+ */
+#define WZ_STATIC_SCRATCH_BYTES (16u << 20)
+WZ_API int wz_relevance_static(const void *features, int T, int H, int W, int D, int dtype,
+                               const void *query, int Lq, float *token_scores, float *frame_scores,
+                               float *frame_mean, wz_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Single-level DWT (Eq. 8, 10, 11, 14)                                      */
 /* ------------------------------------------------------------------------ */

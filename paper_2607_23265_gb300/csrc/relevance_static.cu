@@ -1,0 +1,132 @@
+// wz_relevance_static: the relevance scores of wz_relevance, computed with
+// no device-memory allocation at all.
+//
+// Some callers cannot allocate device memory when they need the scores: code
+// running while a stream is being captured into a CUDA graph where the
+// capture must not contain allocation nodes, serving loops that freeze their
+// memory budget after start-up so that a request can never fail on an
+// out-of-memory or stall on the allocator, and hosts whose device memory is
+// owned by another framework's caching allocator that a foreign cudaMalloc
+// would bypass.  Such callers still pass their own inputs and outputs; the
+// intermediate sums live in one fixed array compiled into this library.
+//
+// The array `g_relevance_scratch` (WZ_STATIC_SCRATCH_BYTES) exists on every
+// GPU that loads the library, from load until the process exits.  Its name
+// is only a host-side stand-in in host code, so the device address is looked
+// up once per device with cudaGetSymbolAddress (with that device current) on
+// the first call made on that device, and passed to the kernels.
+#include <mutex>
+
+#include "wz_internal.cuh"
+
+namespace wz {
+
+namespace {
+
+static __device__ __align__(256) unsigned char g_relevance_scratch[WZ_STATIC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void *g_scratch_addr[kMaxDevices];
+
+// Device address of the fixed array on the current device (looked up once).
+int static_scratch(void **out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return WZ_ERR_CUDA;
+    }
+    if (dev < 0 || dev >= kMaxDevices) return WZ_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_scratch_mu);
+    if (!g_scratch_addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_relevance_scratch) != cudaSuccess || p == nullptr) {
+            cudaGetLastError();
+            return WZ_ERR_CUDA;
+        }
+        g_scratch_addr[dev] = p;
+    }
+    *out = g_scratch_addr[dev];
+    return WZ_OK;
+}
+
+size_t up256(size_t x) { return (x + 255) / 256 * 256; }
+
+bool is_aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+}  // namespace
+
+}  // namespace wz
+
+using namespace wz;
+
+extern "C" int wz_relevance_static(const void *features, int T, int H, int W, int D, int dtype,
+                                   const void *query, int Lq, float *token_scores, float *frame_scores,
+                                   float *frame_mean, wz_stream_t stream) {
+    if (T < 1 || H < 1 || W < 1 || D < 1 || Lq < 1) return WZ_ERR_INVALID_ARG;
+    if (dtype != WZ_DTYPE_BF16 && dtype != WZ_DTYPE_F32) return WZ_ERR_INVALID_ARG;
+    if (D % 8 != 0) return WZ_ERR_UNSUPPORTED;
+    if (T > WZ_MAX_T || H > WZ_MAX_HW || W > WZ_MAX_HW || D > WZ_MAX_D) return WZ_ERR_UNSUPPORTED;
+    if (!features || !query || !token_scores || !frame_scores) return WZ_ERR_INVALID_ARG;
+    if (!is_aligned(features, 16) || !is_aligned(query, 16) || !is_aligned(token_scores, 4) ||
+        !is_aligned(frame_scores, 4) || (frame_mean && !is_aligned(frame_mean, 4)))
+        return WZ_ERR_INVALID_ARG;
+
+    Ctx c{};
+    c.V = 1;
+    c.T = T;
+    c.H = H;
+    c.W = W;
+    c.D = D;
+    c.N = H * W;
+    c.dtype = dtype;
+    c.DC = (D + kStatsChunk - 1) / kStatsChunk;
+    c.G1 = relevance_grid(c);
+    if (c.G1 < 1) {
+        cudaGetLastError();
+        return WZ_ERR_CUDA;
+    }
+    c.L1 = ((int64_t)T * c.N + c.G1 - 1) / c.G1;
+
+    // Carve the fixed array: every byte the kernels read is written earlier
+    // in the same call, so nothing in it has to start at zero.
+    size_t o = 0;
+    const size_t o_q32 = o;
+    o = up256(o + (size_t)D * 4);
+    const size_t o_q64 = o;
+    o = up256(o + (size_t)D * 8);
+    const size_t o_qn = o;
+    o = up256(o + 8);
+    const size_t o_vp = o;
+    o = up256(o + sizeof(VideoPar));
+    const size_t o_part = o;
+    o = up256(o + ((size_t)c.G1 + T) * D * 4);
+    const size_t o_trip = o;
+    o = up256(o + (size_t)T * c.DC * 3 * 8);
+    if (o > (size_t)WZ_STATIC_SCRATCH_BYTES) return WZ_ERR_WORKSPACE;
+
+    void *base = nullptr;
+    const int st = static_scratch(&base);
+    if (st != WZ_OK) return st;
+    char *b = static_cast<char *>(base);
+    c.qbar32 = reinterpret_cast<float *>(b + o_q32);
+    c.qbar64 = reinterpret_cast<double *>(b + o_q64);
+    c.qnorm = reinterpret_cast<double *>(b + o_qn);
+    c.vpar = reinterpret_cast<VideoPar *>(b + o_vp);
+    c.part = reinterpret_cast<float *>(b + o_part);
+    c.trip = reinterpret_cast<double *>(b + o_trip);
+    c.X = features;
+    c.Q = query;
+    c.a = token_scores;
+    c.frame_scores = frame_scores;
+    c.frame_mean = frame_mean;
+
+    const VideoPar par{0, Lq, 0, 0};
+    const cudaStream_t s = (cudaStream_t)stream;
+    if (launch_query_pool(c, &par, s) != cudaSuccess || launch_relevance_pass(c, s) != cudaSuccess ||
+        launch_frame_stats(c, s) != cudaSuccess || launch_relevance_finalize(c, s) != cudaSuccess) {
+        cudaGetLastError();
+        return WZ_ERR_CUDA;
+    }
+    return WZ_OK;
+}

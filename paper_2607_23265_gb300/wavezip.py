@@ -77,6 +77,7 @@ def _load():
         "wz_condense_batch": (i, [C.POINTER(BatchArgs)]),
         "wz_relevance": (i, [vp, i, i, i, i, i, vp, i, vp, vp, vp, vp, sz, vp]),
         "wz_relevance_workspace_size": (sz, [i, i, i, i]),
+        "wz_relevance_static": (i, [vp, i, i, i, i, i, vp, i, vp, vp, vp, vp]),
         "wz_dwt_len": (i, [i, i]),
         "wz_wavelet_filters": (i, [i] + [C.POINTER(C.c_double)] * 4),
         "wz_dwt1d": (i, [vp, i, i, i, i, vp, vp, vp]),
@@ -267,6 +268,22 @@ def wz_relevance(features: torch.Tensor, query: torch.Tensor, *, frame_mean: boo
                            query.shape[0], ts.data_ptr(), fs.data_ptr(), _ptr(fm), wsp, wsb,
                            _stream(stream, dev))
     _check(st, "wz_relevance")
+    return ts, fs, fm
+
+
+def wz_relevance_static(features: torch.Tensor, query: torch.Tensor, *, frame_mean: bool = False, stream=None):
+    """wz_relevance_static: the scores of wz_relevance without any device allocation
+    (its sums live in a fixed array inside the library; see include/wavezip.h)."""
+    features = _cuda_contig(features, "features")
+    query = _cuda_contig(query, "query")
+    T, H, W, D = features.shape
+    dev = features.device
+    ts = torch.empty((T, H * W), dtype=torch.float32, device=dev)
+    fs = torch.empty((T,), dtype=torch.float32, device=dev)
+    fm = torch.empty((T, D), dtype=torch.float32, device=dev) if frame_mean else None
+    st = _lib.wz_relevance_static(features.data_ptr(), T, H, W, D, _dtype_code(features), query.data_ptr(),
+                                  query.shape[0], ts.data_ptr(), fs.data_ptr(), _ptr(fm), _stream(stream, dev))
+    _check(st, "wz_relevance_static")
     return ts, fs, fm
 
 
