@@ -97,7 +97,7 @@ typedef struct CUstream_st *wz_stream_t;
 #define WZ_MAX_HW      64    /* H, W <= 64                                  */
 #define WZ_MAX_T       4096  /* frames per video                            */
 #define WZ_MAX_VIDEOS  1024  /* videos per batch call                       */
-#define WZ_MAX_D       32768 /* channels                                    */
+#define WZ_MAX_D       32768 /* channels (bf16; half of it for f32)         */
 
 /* ------------------------------------------------------------------------ */
 /* Condensation C_WaveZip(X, Q) (Section 3.2, Eq. 18)                        */

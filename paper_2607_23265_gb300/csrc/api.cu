@@ -51,7 +51,7 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.vpar = take((size_t)s.V * sizeof(VideoPar));
     L.a = with_a ? take(VT * s.N * 4) : 0;
     L.part = take(((size_t)kG1Max + VT) * s.D * 4);
-    L.trip = take(VT * s.DC * 3 * 8);
+    L.trip = take(VT * s.DC * 4 * 8);
     L.fr = take(VT * 4 * 8);
     L.tmp = take(VT * 4 * 8);
     L.list = take(VT * 2 * 4);
@@ -80,6 +80,7 @@ int check_sizes(int V, int T, int H, int W, int D, int dtype) {
     if (D % 8 != 0) return WZ_ERR_UNSUPPORTED;
     if (V > WZ_MAX_VIDEOS || T > WZ_MAX_T || H > WZ_MAX_HW || W > WZ_MAX_HW || D > WZ_MAX_D)
         return WZ_ERR_UNSUPPORTED;
+    if (dtype == WZ_DTYPE_F32 && D > WZ_MAX_D / 2) return WZ_ERR_UNSUPPORTED;
     return WZ_OK;
 }
 

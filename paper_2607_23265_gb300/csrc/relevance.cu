@@ -1,21 +1,23 @@
 // Cross-Modal Scorer, similarity branch (Section 3.2.1), on the GPU.
 //
-//   query_pool      u_q = mean of the query rows (fp64) and ||u_q||.
+//   query_pool      u_q = mean of the query rows (compensated fp32 -> fp64).
 //   relevance_pass  one streaming read of the features: per token
 //                   a_{t,n} = <u, u_q> / (||u|| ||u_q||) (the input of Eq. 6)
 //                   and per-CTA column sums of every frame it touches (the
 //                   average pool of Section 3.2.1 / Eq. 7), in fp32.
 //   frame_stats     sums the column partials of a frame in fp64 in a fixed
-//                   order and reduces <v_t,u_q>, <v_t,v_t>, <v_t,v_{t-1}> per
-//                   256-channel chunk, which give r_t and delta_t (Eq. 7).
+//                   order and reduces <v_t,u_q>, <v_t,v_t>, <v_t,v_{t-1}> and
+//                   <u_q,u_q> per 2048-channel chunk, which give r_t and
+//                   delta_t (Eq. 7).
 //
-// The relevance pass is HBM bound: it reads T*H*W*D elements once with
-// 16-byte non-allocating loads; each CTA owns one contiguous range of the
-// flattened token index so the grid is exactly balanced.
+// The relevance pass is HBM bound: it reads T*H*W*D elements once, streamed
+// by TMA bulk copies through a shared-memory ring; each CTA owns one
+// contiguous range of the flattened token index so the grid is balanced.
 #include <algorithm>
 #include <cstring>
 
 #include "wz_internal.cuh"
+#include "wz_ptx.cuh"
 
 namespace wz {
 
@@ -23,24 +25,26 @@ struct VideoParBlock {
     VideoPar v[WZ_MAX_VIDEOS];
 };
 
+// u_q = mean of the query rows: one thread per channel, compensated fp32
+// accumulation (TwoSum), stored as fp64 and fp32.
 template <typename T>
-__global__ void __launch_bounds__(1024) query_pool_kernel(Ctx c, VideoParBlock par) {
-    __shared__ double scratch[32];
-    const int v = blockIdx.x;
+__global__ void __launch_bounds__(256) query_pool_kernel(Ctx c, VideoParBlock par) {
+    const int v = blockIdx.y;
     const VideoPar vp = par.v[v];
-    if (threadIdx.x == 0) c.vpar[v] = vp;
-    const T *Q = static_cast<const T *>(c.Q) + (size_t)vp.q_row0 * c.D;
-    double ss = 0.0;
-    for (int d = threadIdx.x; d < c.D; d += blockDim.x) {
-        double s = 0.0;
-        for (int j = 0; j < vp.Lq; ++j) s += (double)load_scalar<T>(Q + (size_t)j * c.D + d);
-        s /= (double)vp.Lq;
-        c.qbar64[(size_t)v * c.D + d] = s;
-        c.qbar32[(size_t)v * c.D + d] = (float)s;
-        ss += s * s;
+    if (blockIdx.x == 0 && threadIdx.x == 0) c.vpar[v] = vp;
+    const int d = blockIdx.x * blockDim.x + threadIdx.x;
+    if (d >= c.D) return;
+    const T *Q = static_cast<const T *>(c.Q) + (size_t)vp.q_row0 * c.D + d;
+    float s = 0.f, e = 0.f;
+    for (int j = 0; j < vp.Lq; ++j) {
+        float t, err;
+        two_sum(s, load_scalar<T>(Q + (size_t)j * c.D), t, err);
+        s = t;
+        e += err;
     }
-    const double tot = block_sum(ss, scratch);
-    if (threadIdx.x == 0) c.qnorm[v] = sqrt(tot);
+    const double m = ((double)s + (double)e) / (double)vp.Lq;
+    c.qbar64[(size_t)v * c.D + d] = m;
+    c.qbar32[(size_t)v * c.D + d] = (float)m;
 }
 
 // Reduce the NV values held by every lane across the warp (NV a power of
@@ -68,135 +72,232 @@ __device__ __forceinline__ float transpose_reduce(float (&v)[NV]) {
     return r;
 }
 
+// Tokens per TMA chunk: never crosses a frame boundary.
+__device__ __forceinline__ int64_t chunk_len(int64_t tok, int64_t end, int N, int CH) {
+    const int64_t f_end = (tok / N + 1) * (int64_t)N;
+    return min((int64_t)CH, min(end, f_end) - tok);
+}
+
+constexpr int kRelStages = 3;
+constexpr int kRelMaxConsumers = 512;
+constexpr uint64_t kRelTimeoutNs = 2000000000ull;
+
 // One CTA streams tokens [blockIdx.x*L1, +L1) of the flattened [V*T*N] index.
+// The last warp copies chunks of CH consecutive tokens (contiguous in HBM)
+// into a 3-stage shared-memory ring with cp.async.bulk; the other warps
+// (NC threads, VPT 16-byte vectors each) read them from shared memory.
 template <typename T, int VPT>
-__global__ void __launch_bounds__(256) relevance_pass_kernel(Ctx c) {
+__global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kernel(Ctx c, int CH) {
     constexpr int VEC = VecOf<T>::kElems;
-    constexpr int GROUP = VPT >= 8 ? 1 : 8 / VPT;   // tokens per reduction step
-    constexpr int NV = 2 * GROUP;                   // GROUP dots + GROUP norms
-    constexpr int SHIFT = NV == 16 ? 1 : NV == 8 ? 2 : NV == 4 ? 3 : 4;
-    __shared__ float red[2][8][NV];
+    constexpr int GROUP = 8;                 // tokens per cross-warp reduction
+    constexpr int NV = 2 * GROUP;            // GROUP dots + GROUP squared norms
+    extern __shared__ __align__(128) uint8_t rsm[];
+    __shared__ float red[2][kRelMaxConsumers / 32][NV];
+    __shared__ float qsum[kRelMaxConsumers / 32];
+    __shared__ uint64_t full[kRelStages], empty[kRelStages];
+    __shared__ int ok_flag;
+    const int NC = blockDim.x - 32;          // consumer threads
+    const int nw = NC >> 5;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int nw = blockDim.x >> 5;
     const int n_vec = c.D / VEC;
+    const size_t rowb = (size_t)c.D * sizeof(T);
+    const size_t stage_bytes = (size_t)CH * rowb;
     const int64_t total = (int64_t)c.V * c.T * c.N;
     const int64_t start = (int64_t)blockIdx.x * c.L1;
     const int64_t end = min(start + c.L1, total);
-    const uint4 *X = static_cast<const uint4 *>(c.X);
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kRelStages; ++s) {
+            ptx::mbar_init(&full[s], 1);
+            ptx::mbar_init(&empty[s], 1);
+        }
+        ok_flag = 1;
+        ptx::fence_barrier_init();
+        ptx::fence_proxy_async_smem();
+    }
+    __syncthreads();
+    if (start >= end) return;
+
+    if (warp == nw) {
+        // ---------------- producer ----------------
+        if (lane == 0) {
+            const uint64_t pol = ptx::policy_evict_first();
+            const char *X = static_cast<const char *>(c.X);
+            int s = 0;
+            uint32_t ph = 0;
+            int issued[kRelStages] = {-1, -1, -1};
+            for (int64_t tok = start; tok < end;) {
+                const int64_t n = chunk_len(tok, end, c.N, CH);
+                if (!ptx::mbar_wait(&empty[s], ph ^ 1u, kRelTimeoutNs)) {
+                    atomicOr(c.status, 16);
+                    break;
+                }
+                ptx::mbar_arrive_expect_tx(&full[s], (uint32_t)(n * rowb));
+                ptx::bulk_load(rsm + s * stage_bytes, X + (size_t)tok * rowb, (uint32_t)(n * rowb), &full[s], pol);
+                issued[s] = (int)ph;
+                tok += n;
+                if (++s == kRelStages) {
+                    s = 0;
+                    ph ^= 1u;
+                }
+            }
+            for (int k = 0; k < kRelStages; ++k)
+                if (issued[k] >= 0) ptx::mbar_wait(&full[k], (uint32_t)issued[k], kRelTimeoutNs);
+        }
+        return;
+    }
+
+    // ---------------- consumers ----------------
+    auto consumer_sync = [&]() { asm volatile("bar.sync 1, %0;" ::"r"(NC) : "memory"); };
     int cur_v = -1;
     float q[VPT][VEC];
     float qn = 0.f;
+    float cs[VPT][VEC];
     int gi = 0;
+    int s = 0;
+    uint32_t ph = 0;
+    int64_t cur_f = -1;
     for (int64_t tok = start; tok < end;) {
         const int64_t f = tok / c.N;
-        const int64_t seg_end = min(end, (f + 1) * (int64_t)c.N);
-        const int v = (int)(f / c.T);
-        if (v != cur_v) {
-            cur_v = v;
-            qn = (float)c.qnorm[v];
-#pragma unroll
-            for (int vi = 0; vi < VPT; ++vi) {
-                const int vidx = threadIdx.x + vi * blockDim.x;
-#pragma unroll
-                for (int e = 0; e < VEC; ++e)
-                    q[vi][e] = vidx < n_vec ? c.qbar32[(size_t)v * c.D + vidx * VEC + e] : 0.f;
-            }
-        }
-        float cs[VPT][VEC];
-#pragma unroll
-        for (int vi = 0; vi < VPT; ++vi)
-#pragma unroll
-            for (int e = 0; e < VEC; ++e) cs[vi][e] = 0.f;
-
-        for (int64_t g0 = tok; g0 < seg_end; g0 += GROUP, ++gi) {
-            uint4 raw[GROUP][VPT];
-#pragma unroll
-            for (int k = 0; k < GROUP; ++k)
+        const int64_t n = chunk_len(tok, end, c.N, CH);
+        if (f != cur_f) {
+            cur_f = f;
+            const int v = (int)(f / c.T);
+            if (v != cur_v) {
+                cur_v = v;
+                float qq = 0.f;
 #pragma unroll
                 for (int vi = 0; vi < VPT; ++vi) {
-                    const int vidx = threadIdx.x + vi * blockDim.x;
-                    if (g0 + k < seg_end && vidx < n_vec)
-                        raw[k][vi] = ldg_stream(X + (size_t)(g0 + k) * n_vec + vidx);
-                    else
-                        raw[k][vi] = make_uint4(0u, 0u, 0u, 0u);
+                    const int vidx = threadIdx.x + vi * NC;
+#pragma unroll
+                    for (int e = 0; e < VEC; ++e) {
+                        q[vi][e] = vidx < n_vec ? c.qbar32[(size_t)v * c.D + vidx * VEC + e] : 0.f;
+                        qq = fmaf(q[vi][e], q[vi][e], qq);
+                    }
                 }
+                for (int o = 16; o > 0; o >>= 1) qq += __shfl_xor_sync(0xffffffffu, qq, o);
+                consumer_sync();
+                if (lane == 0) qsum[warp] = qq;
+                consumer_sync();
+                qq = 0.f;
+                for (int w = 0; w < nw; ++w) qq += qsum[w];
+                qn = sqrtf(qq);
+            }
+#pragma unroll
+            for (int vi = 0; vi < VPT; ++vi)
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) cs[vi][e] = 0.f;
+        }
+        // wait for the chunk (one bounded waiter decides for all consumers)
+        if (threadIdx.x == 0) ok_flag = ptx::mbar_wait(&full[s], ph, kRelTimeoutNs) ? 1 : 0;
+        consumer_sync();
+        if (!ok_flag) {
+            if (threadIdx.x == 0) atomicOr(c.status, 32);
+            break;
+        }
+        ptx::mbar_wait(&full[s], ph, kRelTimeoutNs);   // completed: acquire for this thread
+        const uint8_t *st = rsm + s * stage_bytes;
+        for (int64_t g0 = 0; g0 < n; g0 += GROUP, ++gi) {
             float acc[NV];
 #pragma unroll
             for (int k = 0; k < NV; ++k) acc[k] = 0.f;
 #pragma unroll
-            for (int k = 0; k < GROUP; ++k)
+            for (int k = 0; k < GROUP; ++k) {
+                if (g0 + k < n) {
 #pragma unroll
-                for (int vi = 0; vi < VPT; ++vi) {
-                    float x[VEC];
-                    unpack(raw[k][vi], x, (T *)nullptr);
+                    for (int vi = 0; vi < VPT; ++vi) {
+                        const int vidx = threadIdx.x + vi * NC;
+                        if (vidx < n_vec) {
+                            const uint4 raw = *reinterpret_cast<const uint4 *>(st + (size_t)(g0 + k) * rowb + (size_t)vidx * 16);
+                            float x[VEC];
+                            unpack(raw, x, (T *)nullptr);
 #pragma unroll
-                    for (int e = 0; e < VEC; ++e) {
-                        cs[vi][e] += x[e];
-                        acc[k] = fmaf(x[e], q[vi][e], acc[k]);
-                        acc[k + GROUP] = fmaf(x[e], x[e], acc[k + GROUP]);
+                            for (int e = 0; e < VEC; ++e) {
+                                cs[vi][e] += x[e];
+                                acc[k] = fmaf(x[e], q[vi][e], acc[k]);
+                                acc[k + GROUP] = fmaf(x[e], x[e], acc[k + GROUP]);
+                            }
+                        }
                     }
                 }
+            }
             const float tot = transpose_reduce<NV>(acc);
             const int b = gi & 1;
-            if ((lane & ((1 << SHIFT) - 1)) == 0) red[b][warp][lane >> SHIFT] = tot;
-            __syncthreads();
+            if ((lane & 1) == 0) red[b][warp][lane >> 1] = tot;
+            consumer_sync();
             if (threadIdx.x < 32) {
-                float s = 0.f;
+                float sm = 0.f;
                 if (lane < NV)
-                    for (int w = 0; w < nw; ++w) s += red[b][w][lane];
-                const float nrm = __shfl_down_sync(0xffffffffu, s, GROUP);
-                if (lane < GROUP && g0 + lane < seg_end) {
-                    const float a = (nrm > 0.f && qn > 0.f) ? s / (sqrtf(nrm) * qn) : 0.f;
-                    c.a[g0 + lane] = a;
+                    for (int w = 0; w < nw; ++w) sm += red[b][w][lane];
+                const float nrm = __shfl_down_sync(0xffffffffu, sm, GROUP);
+                if (lane < GROUP && g0 + lane < n) {
+                    const float a = (nrm > 0.f && qn > 0.f) ? sm / (sqrtf(nrm) * qn) : 0.f;
+                    c.a[tok + g0 + lane] = a;
                 }
             }
         }
-        // column partial of frame f from this CTA: slot blockIdx.x + f
-        float *dst = c.part + ((size_t)blockIdx.x + (size_t)f) * c.D;
+        // every consumer has passed its last read of the stage (the group
+        // barrier above), so the stage goes back to the producer
+        if (threadIdx.x == 0) ptx::mbar_arrive(&empty[s]);
+        if (++s == kRelStages) {
+            s = 0;
+            ph ^= 1u;
+        }
+        tok += n;
+        const bool frame_done = (tok % c.N == 0) || tok >= end;
+        if (frame_done) {
+            // column partial of frame f from this CTA: slot blockIdx.x + f
+            float *dst = c.part + ((size_t)blockIdx.x + (size_t)f) * c.D;
 #pragma unroll
-        for (int vi = 0; vi < VPT; ++vi) {
-            const int vidx = threadIdx.x + vi * blockDim.x;
-            if (vidx < n_vec) {
+            for (int vi = 0; vi < VPT; ++vi) {
+                const int vidx = threadIdx.x + vi * NC;
+                if (vidx < n_vec) {
 #pragma unroll
-                for (int e = 0; e < VEC; e += 4)
-                    *reinterpret_cast<float4 *>(dst + vidx * VEC + e) =
-                        make_float4(cs[vi][e], cs[vi][e + 1], cs[vi][e + 2], cs[vi][e + 3]);
+                    for (int e = 0; e < VEC; e += 4)
+                        *reinterpret_cast<float4 *>(dst + vidx * VEC + e) =
+                            make_float4(cs[vi][e], cs[vi][e + 1], cs[vi][e + 2], cs[vi][e + 3]);
+                }
             }
         }
-        tok = seg_end;
     }
 }
 
-// Per (256-channel chunk, frame): fp64 frame sums from the fixed list of CTA
-// partials, and their products with u_q and with the previous frame.
-__global__ void __launch_bounds__(kStatsChunk) frame_stats_kernel(Ctx c) {
-    __shared__ double scratch[32];
+// Per (2048-channel chunk, frame): fp64 frame sums from the fixed list of CTA
+// partials (8 channels per thread), and their products with u_q, with the
+// previous frame and of u_q with itself.
+__global__ void __launch_bounds__(256) frame_stats_kernel(Ctx c) {
+    __shared__ double scratch[40];
     const int64_t f = blockIdx.y;
     const int t = (int)(f % c.T);
     const int v = (int)(f / c.T);
-    const int d = blockIdx.x * kStatsChunk + threadIdx.x;
-    double sf = 0.0, sp = 0.0, q = 0.0;
-    if (d < c.D) {
-        const int64_t lo = f * c.N / c.L1;
-        const int64_t hi = min((int64_t)c.G1 - 1, ((f + 1) * c.N - 1) / c.L1);
+    const int64_t lo = f * c.N / c.L1;
+    const int64_t hi = min((int64_t)c.G1 - 1, ((f + 1) * c.N - 1) / c.L1);
+    const int64_t g = f - 1;
+    const int64_t lo2 = t > 0 ? g * c.N / c.L1 : 0;
+    const int64_t hi2 = t > 0 ? min((int64_t)c.G1 - 1, ((g + 1) * c.N - 1) / c.L1) : -1;
+    double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+    for (int k = 0; k < kStatsChunk / 256; ++k) {
+        const int d = blockIdx.x * kStatsChunk + k * 256 + threadIdx.x;
+        if (d >= c.D) break;
+        double sf = 0.0, sp = 0.0;
         for (int64_t cc = lo; cc <= hi; ++cc) sf += (double)c.part[(size_t)(cc + f) * c.D + d];
-        if (t > 0) {
-            const int64_t g = f - 1;
-            const int64_t lo2 = g * c.N / c.L1;
-            const int64_t hi2 = min((int64_t)c.G1 - 1, ((g + 1) * c.N - 1) / c.L1);
-            for (int64_t cc = lo2; cc <= hi2; ++cc) sp += (double)c.part[(size_t)(cc + g) * c.D + d];
-        }
-        q = c.qbar64[(size_t)v * c.D + d];
+        for (int64_t cc = lo2; cc <= hi2; ++cc) sp += (double)c.part[(size_t)(cc + g) * c.D + d];
+        const double q = c.qbar64[(size_t)v * c.D + d];
         if (c.frame_mean) c.frame_mean[(size_t)f * c.D + d] = (float)(sf / c.N);
+        s0 += sf * q;
+        s1 += sf * sf;
+        s2 += sf * sp;
+        s3 += q * q;
     }
-    const double s0 = block_sum(sf * q, scratch);
-    const double s1 = block_sum(sf * sf, scratch);
-    const double s2 = block_sum(sf * sp, scratch);
+    s0 = block_sum(s0, scratch);
+    s1 = block_sum(s1, scratch);
+    s2 = block_sum(s2, scratch);
+    s3 = block_sum(s3, scratch);
     if (threadIdx.x == 0) {
-        double *o = c.trip + ((size_t)f * c.DC + blockIdx.x) * 3;
+        double *o = c.trip + ((size_t)f * c.DC + blockIdx.x) * 4;
         o[0] = s0;
         o[1] = s1;
         o[2] = s2;
+        o[3] = s3;
     }
 }
 
@@ -205,13 +306,13 @@ __global__ void __launch_bounds__(kStatsChunk) frame_stats_kernel(Ctx c) {
 __global__ void relevance_finalize_kernel(Ctx c) {
     const int64_t f = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (f >= (int64_t)c.V * c.T) return;
-    const int v = (int)(f / c.T);
-    double dq = 0.0, ff = 0.0;
+    double dq = 0.0, ff = 0.0, qq = 0.0;
     for (int k = 0; k < c.DC; ++k) {
-        dq += c.trip[((size_t)f * c.DC + k) * 3 + 0];
-        ff += c.trip[((size_t)f * c.DC + k) * 3 + 1];
+        dq += c.trip[((size_t)f * c.DC + k) * 4 + 0];
+        ff += c.trip[((size_t)f * c.DC + k) * 4 + 1];
+        qq += c.trip[((size_t)f * c.DC + k) * 4 + 3];
     }
-    const double qn = c.qnorm[v];
+    const double qn = sqrt(qq);
     c.frame_scores[f] = (ff > 0.0 && qn > 0.0) ? (float)(dq / (sqrt(ff) * qn)) : 0.f;
 }
 
@@ -219,50 +320,64 @@ cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s
     VideoParBlock blk;   // copied into the launch parameters
     memset(&blk, 0, sizeof(blk));
     for (int v = 0; v < c.V; ++v) blk.v[v] = hpar[v];
+    const dim3 grid((unsigned)((c.D + 255) / 256), (unsigned)c.V);
     if (c.dtype == WZ_DTYPE_BF16)
-        query_pool_kernel<__nv_bfloat16><<<c.V, 1024, 0, s>>>(c, blk);
+        query_pool_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c, blk);
     else
-        query_pool_kernel<float><<<c.V, 1024, 0, s>>>(c, blk);
+        query_pool_kernel<float><<<grid, 256, 0, s>>>(c, blk);
     return cudaGetLastError();
 }
 
 namespace {
 
+struct RelCfg {
+    const void *fn = nullptr;
+    int threads = 0;     // consumers + one producer warp
+    int CH = 0;          // tokens per chunk
+    size_t smem = 0;
+};
+
 template <typename T, int VPT>
-void relevance_config(const Ctx &c, const void *&fn, int &threads) {
-    fn = (const void *)relevance_pass_kernel<T, VPT>;
+void relevance_config(const Ctx &c, RelCfg &r) {
+    r.fn = (const void *)relevance_pass_kernel<T, VPT>;
     constexpr int VEC = VecOf<T>::kElems;
     const int n_vec = c.D / VEC;
-    threads = ((n_vec + VPT - 1) / VPT + 31) / 32 * 32;
-    if (threads < 32) threads = 32;
+    const int nc = std::max(32, ((n_vec + VPT - 1) / VPT + 31) / 32 * 32);
+    r.threads = nc + 32;
+    const size_t rowb = (size_t)c.D * sizeof(T);
+    int ch = (int)std::max<size_t>(1, (56 * 1024) / rowb);
+    ch = std::min(ch, 32);
+    if (ch >= 8) ch = ch / 8 * 8;
+    r.CH = ch;
+    r.smem = (size_t)kRelStages * ch * rowb;
 }
 
 template <typename T>
-bool pick(const Ctx &c, const void *&fn, int &threads) {
+bool pick(const Ctx &c, RelCfg &r) {
     constexpr int VEC = VecOf<T>::kElems;
     const int n_vec = c.D / VEC;
-    if (n_vec <= 256) relevance_config<T, 1>(c, fn, threads);
-    else if (n_vec <= 512) relevance_config<T, 2>(c, fn, threads);
-    else if (n_vec <= 1024) relevance_config<T, 4>(c, fn, threads);
-    else if (n_vec <= 2048) relevance_config<T, 8>(c, fn, threads);
+    if (n_vec <= 512) relevance_config<T, 1>(c, r);
+    else if (n_vec <= 1024) relevance_config<T, 2>(c, r);
+    else if (n_vec <= 2048) relevance_config<T, 4>(c, r);
+    else if (n_vec <= 4096) relevance_config<T, 8>(c, r);
     else return false;
     return true;
 }
 
-bool pick_any(const Ctx &c, const void *&fn, int &threads) {
-    return c.dtype == WZ_DTYPE_BF16 ? pick<__nv_bfloat16>(c, fn, threads) : pick<float>(c, fn, threads);
+bool pick_any(const Ctx &c, RelCfg &r) {
+    return c.dtype == WZ_DTYPE_BF16 ? pick<__nv_bfloat16>(c, r) : pick<float>(c, r);
 }
 
 }  // namespace
 
 int relevance_grid(const Ctx &c) {
-    const void *fn = nullptr;
-    int threads = 0;
-    if (!pick_any(c, fn, threads)) return 0;
+    RelCfg r;
+    if (!pick_any(c, r)) return 0;
     int dev = 0, sms = 0, per_sm = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, threads, 0) != cudaSuccess) return 0;
+    if (cudaFuncSetAttribute(r.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r.smem) != cudaSuccess) return 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, r.fn, r.threads, r.smem) != cudaSuccess) return 0;
     if (per_sm < 1) per_sm = 1;
     const int64_t total = (int64_t)c.V * c.T * c.N;
     int64_t g = (int64_t)sms * per_sm;
@@ -273,15 +388,17 @@ int relevance_grid(const Ctx &c) {
 }
 
 cudaError_t launch_relevance_pass(const Ctx &c, cudaStream_t s) {
-    const void *fn = nullptr;
-    int threads = 0;
-    if (!pick_any(c, fn, threads)) return cudaErrorInvalidValue;
-    void *args[] = {const_cast<Ctx *>(&c)};
-    return cudaLaunchKernel(fn, dim3(c.G1), dim3(threads), args, 0, s);
+    RelCfg r;
+    if (!pick_any(c, r)) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(r.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r.smem);
+    if (e != cudaSuccess) return e;
+    int CH = r.CH;
+    void *args[] = {const_cast<Ctx *>(&c), &CH};
+    return cudaLaunchKernel(r.fn, dim3(c.G1), dim3(r.threads), args, r.smem, s);
 }
 
 cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s) {
-    frame_stats_kernel<<<dim3(c.DC, c.V * c.T), kStatsChunk, 0, s>>>(c);
+    frame_stats_kernel<<<dim3(c.DC, c.V * c.T), 256, 0, s>>>(c);
     return cudaGetLastError();
 }
 

@@ -67,6 +67,7 @@ extern "C" int wz_relevance_static(const void *features, int T, int H, int W, in
     if (dtype != WZ_DTYPE_BF16 && dtype != WZ_DTYPE_F32) return WZ_ERR_INVALID_ARG;
     if (D % 8 != 0) return WZ_ERR_UNSUPPORTED;
     if (T > WZ_MAX_T || H > WZ_MAX_HW || W > WZ_MAX_HW || D > WZ_MAX_D) return WZ_ERR_UNSUPPORTED;
+    if (dtype == WZ_DTYPE_F32 && D > WZ_MAX_D / 2) return WZ_ERR_UNSUPPORTED;
     if (!features || !query || !token_scores || !frame_scores) return WZ_ERR_INVALID_ARG;
     if (!is_aligned(features, 16) || !is_aligned(query, 16) || !is_aligned(token_scores, 4) ||
         !is_aligned(frame_scores, 4) || (frame_mean && !is_aligned(frame_mean, 4)))
@@ -102,7 +103,7 @@ extern "C" int wz_relevance_static(const void *features, int T, int H, int W, in
     const size_t o_part = o;
     o = up256(o + ((size_t)c.G1 + T) * D * 4);
     const size_t o_trip = o;
-    o = up256(o + (size_t)T * c.DC * 3 * 8);
+    o = up256(o + (size_t)T * c.DC * 4 * 8);
     if (o > (size_t)WZ_STATIC_SCRATCH_BYTES) return WZ_ERR_WORKSPACE;
 
     void *base = nullptr;

@@ -65,25 +65,28 @@ __device__ __forceinline__ int grid_h(int n, int H, int W) {
 
 __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     __shared__ double dscr[64];
-    __shared__ long long lscr[32];
+    __shared__ long long lscr[40];
     __shared__ int iscr[72];
+    __shared__ unsigned long long keys[WZ_MAX_T];
     const int v = blockIdx.x;
     const int T = c.T;
     const int64_t base = (int64_t)v * T;
     const VideoPar vp = c.vpar[v];
-    const double qn = c.qnorm[v];
     double *fr = c.fr + base * 4;          // r, delta, gamma, r~
     double *ff = c.tmp + base * 4;         // |v|^2, <v, v_prev>, weight, frac
     int *lst = c.list + 2 * base;          // retained frames, then their budgets
 
-    // r_t and the norms (sums of the frame-stats chunks in a fixed order)
+    // ||u_q|| and r_t and the norms (sums of the frame-stats chunks in a fixed order)
+    double qq = 0.0;
+    for (int k = 0; k < c.DC; ++k) qq += c.trip[(size_t)base * c.DC * 4 + 4 * k + 3];
+    const double qn = sqrt(qq);
     for (int t = threadIdx.x; t < T; t += blockDim.x) {
-        const double *tr = c.trip + (size_t)(base + t) * c.DC * 3;
+        const double *tr = c.trip + (size_t)(base + t) * c.DC * 4;
         double dq = 0.0, vv = 0.0, vp_ = 0.0;
         for (int k = 0; k < c.DC; ++k) {
-            dq += tr[3 * k + 0];
-            vv += tr[3 * k + 1];
-            vp_ += tr[3 * k + 2];
+            dq += tr[4 * k + 0];
+            vv += tr[4 * k + 1];
+            vp_ += tr[4 * k + 2];
         }
         fr[4 * t + 0] = (vv > 0.0 && qn > 0.0) ? dq / (sqrt(vv) * qn) : 0.0;
         ff[4 * t + 0] = vv;
@@ -220,29 +223,29 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
                 __syncthreads();
                 continue;
             }
-            // largest remainder among the candidates
+            // largest remainder among the candidates: rank the fractional
+            // parts (non-negative doubles order like their bit patterns)
             long long fsum = 0;
             for (int m = threadIdx.x; m < L; m += blockDim.x) {
                 const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
                 const bool cand = nb[m] < 0 && (uniform || w > 0.0);
-                double frac = -1.0;
+                unsigned long long key = ~0ull;
                 if (cand) {
                     const double q = (double)remaining * w / S;
                     const double fl = floor(q);
-                    frac = q - fl;
+                    key = (unsigned long long)__double_as_longlong(q - fl);
                     fsum += (long long)fl;
                 }
-                ff[4 * lst[m] + 3] = frac;
+                keys[m] = key;
             }
             const long long R = remaining - block_sum_ll(fsum, lscr);
-            __syncthreads();
             for (int m = threadIdx.x; m < L; m += blockDim.x) {
-                const double fm = ff[4 * lst[m] + 3];
-                if (fm < 0.0) continue;
-                long long rank = 0;
+                const unsigned long long km = keys[m];
+                if (km == ~0ull) continue;
+                int rank = 0;
                 for (int k = 0; k < L; ++k) {
-                    const double fk = ff[4 * lst[k] + 3];
-                    rank += (fk > fm || (fk == fm && k < m)) ? 1 : 0;
+                    const unsigned long long kk = keys[k];
+                    rank += (kk != ~0ull && (kk > km || (kk == km && k < m))) ? 1 : 0;
                 }
                 const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
                 const long long fl = (long long)floor((double)remaining * w / S);

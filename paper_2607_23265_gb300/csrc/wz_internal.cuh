@@ -11,7 +11,7 @@ namespace wz {
 
 constexpr int kMaxTaps = 20;          // Daubechies order <= 10
 constexpr int kG1Max = 2048;          // relevance-pass CTAs (upper bound)
-constexpr int kStatsChunk = 256;      // channels per frame-stats block
+constexpr int kStatsChunk = 2048;     // channels per frame-stats block (8 per thread)
 constexpr int kColBlock = 256;        // output tokens per tensor-core unit
 constexpr int kTileC = 128;           // channels per tensor-core M tile
 
@@ -47,7 +47,7 @@ struct Ctx {
     VideoPar *vpar;       // [V]
     float *a;             // [V*T][N] token saliency
     float *part;          // [G1 + V*T][D] column-sum partials
-    double *trip;         // [V*T][DC][3] (v.q, v.v, v.v_prev)
+    double *trip;         // [V*T][DC][4] (v.q, v.v, v.v_prev, q.q)
     double *fr;           // [V*T][4] (r, delta, gamma, r~)
     double *tmp;          // [V*T][4] temporal-kernel scratch
     int *list;            // [V][2T] retained frames and their budgets
@@ -130,7 +130,8 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(f
 }
 
 // Block-wide sum of a double in a fixed order (deterministic for a fixed
-// block size).  `scratch` holds >= 32 doubles; all threads receive the sum.
+// block size): warp trees, then one warp reduces the warp totals.
+// `scratch` holds >= 33 doubles; all threads receive the sum.
 __device__ __forceinline__ double block_sum(double v, double *scratch) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nw = (blockDim.x + 31) >> 5;
@@ -138,10 +139,13 @@ __device__ __forceinline__ double block_sum(double v, double *scratch) {
     __syncthreads();
     if (lane == 0) scratch[warp] = v;
     __syncthreads();
-    double s = 0.0;
-    for (int w = 0; w < nw; ++w) s += scratch[w];
+    if (warp == 0) {
+        double s = lane < nw ? scratch[lane] : 0.0;
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (lane == 0) scratch[32] = s;
+    }
     __syncthreads();
-    return s;
+    return scratch[32];
 }
 
 __device__ __forceinline__ long long block_sum_ll(long long v, long long *scratch) {
@@ -151,10 +155,20 @@ __device__ __forceinline__ long long block_sum_ll(long long v, long long *scratc
     __syncthreads();
     if (lane == 0) scratch[warp] = v;
     __syncthreads();
-    long long s = 0;
-    for (int w = 0; w < nw; ++w) s += scratch[w];
+    if (warp == 0) {
+        long long s = lane < nw ? scratch[lane] : 0;
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (lane == 0) scratch[32] = s;
+    }
     __syncthreads();
-    return s;
+    return scratch[32];
+}
+
+// Error-free sum of two floats (Knuth's TwoSum): a + b = s + e exactly.
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+    s = a + b;
+    const float bb = s - a;
+    e = (a - (s - bb)) + (b - bb);
 }
 
 // ---- launchers (one per kernel family) -------------------------------------
