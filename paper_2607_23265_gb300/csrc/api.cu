@@ -27,13 +27,13 @@ bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
 // Sub-buffer offsets of one call's workspace.
 struct Layout {
-    size_t qbar32, qbar64, qnorm, vpar, a, part, trip, fr, tmp, list, n, off, hw, prod,
+    size_t qbar32, qbar64, qnorm, vpar, a, part, trip, fr, tmp, list, n, off, woff, hw, prod,
         units, ucount, status, Wop, total;
 };
 
 struct Shape {
     int V, T, H, W, D, N, dtype, F, hp, wp, K_pad, DC, n_ct, max_units_v;
-    int64_t rows_total;
+    int64_t rows_total, w_rows;
 };
 
 Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
@@ -57,12 +57,13 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.list = take(VT * 2 * 4);
     L.n = take(VT * 4);
     L.off = take(VT * 4);
+    L.woff = take(VT * 4);
     L.hw = take(VT * 2 * 4);
     L.prod = take((size_t)s.V * 4);
     L.units = take((size_t)s.V * s.max_units_v * 16);
     L.ucount = take((size_t)s.V * 4);
     L.status = take(16);
-    L.Wop = with_operator ? take((size_t)s.rows_total * s.K_pad * 4) : 0;
+    L.Wop = with_operator ? take((size_t)std::max<int64_t>(s.rows_total, s.w_rows) * s.K_pad * 4) : 0;
     L.total = o;
     return L;
 }
@@ -84,6 +85,10 @@ int check_sizes(int V, int T, int H, int W, int D, int dtype) {
     return WZ_OK;
 }
 
+// Tensor-core operator rows reserved for one video: every frame's block
+// starts on a multiple of 16, so round16(B) + 16 T rows always suffice.
+int64_t video_w_rows(int64_t B, int T) { return (B + 15) / 16 * 16 + (int64_t)16 * T; }
+
 Shape make_shape(int V, int T, int H, int W, int D, int dtype, int F, const int64_t *B) {
     Shape s{};
     s.V = V; s.T = T; s.H = H; s.W = W; s.D = D; s.N = H * W; s.dtype = dtype; s.F = F;
@@ -92,12 +97,15 @@ Shape make_shape(int V, int T, int H, int W, int D, int dtype, int F, const int6
     s.K_pad = (s.N + 31) / 32 * 32;
     s.DC = (D + kStatsChunk - 1) / kStatsChunk;
     s.n_ct = (D + kTileC - 1) / kTileC;
-    int64_t rows = 0, bmax = 0;
+    int64_t rows = 0, bmax = 0, wrows = 0;
     for (int v = 0; v < V; ++v) {
-        rows += B ? B[v] : 0;
-        bmax = std::max<int64_t>(bmax, B ? B[v] : 0);
+        const int64_t b = B ? B[v] : 0;
+        rows += b;
+        wrows += video_w_rows(b, T);
+        bmax = std::max<int64_t>(bmax, b);
     }
     s.rows_total = rows;
+    s.w_rows = wrows;
     s.max_units_v = (int)((T + (bmax + kColBlock - 1) / kColBlock) * s.n_ct);
     return s;
 }
@@ -138,7 +146,7 @@ void set_filters(Ctx &c, int p) {
 void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.V = s.V; c.T = s.T; c.H = s.H; c.W = s.W; c.D = s.D; c.N = s.N; c.dtype = s.dtype;
     c.hp = s.hp; c.wp = s.wp; c.K_pad = s.K_pad; c.DC = s.DC; c.n_ct = s.n_ct;
-    c.max_units_v = s.max_units_v; c.rows_total = s.rows_total;
+    c.max_units_v = s.max_units_v; c.rows_total = s.rows_total; c.w_rows = s.w_rows;
     c.qbar32 = reinterpret_cast<float *>(ws + L.qbar32);
     c.qbar64 = reinterpret_cast<double *>(ws + L.qbar64);
     c.qnorm = reinterpret_cast<double *>(ws + L.qnorm);
@@ -151,6 +159,7 @@ void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.list = reinterpret_cast<int *>(ws + L.list);
     c.n = reinterpret_cast<int *>(ws + L.n);
     c.off = reinterpret_cast<int *>(ws + L.off);
+    c.woff = reinterpret_cast<int *>(ws + L.woff);
     c.hw = reinterpret_cast<int *>(ws + L.hw);
     c.prod = reinterpret_cast<int *>(ws + L.prod);
     c.units = reinterpret_cast<int4 *>(ws + L.units);
@@ -225,7 +234,7 @@ int validate(const CondenseRequest &r, std::vector<int64_t> &B, int64_t &rows) {
         rows += B[v];
         qrows += r.Lq[v];
     }
-    if (rows > (int64_t)INT32_MAX || qrows > (int64_t)INT32_MAX) return WZ_ERR_UNSUPPORTED;
+    if (rows + (int64_t)16 * r.V * r.T > (int64_t)INT32_MAX || qrows > (int64_t)INT32_MAX) return WZ_ERR_UNSUPPORTED;
     if (rows > 0) {
         if (!r.out_tokens || !r.out_index) return WZ_ERR_INVALID_ARG;
         if (!aligned(r.out_tokens, 16) || !aligned(r.out_index, 4)) return WZ_ERR_INVALID_ARG;
@@ -268,14 +277,16 @@ int run_condense(const CondenseRequest &r) {
     c.L1 = (total + c.G1 - 1) / c.G1;
     std::vector<VideoPar> par(r.V);
     int qrow = 0;
-    int64_t row0 = 0;
+    int64_t row0 = 0, wrow0 = 0;
     for (int v = 0; v < r.V; ++v) {
         par[v].q_row0 = qrow;
         par[v].Lq = r.Lq[v];
         par[v].B = (int)B[v];
         par[v].row0 = (int)row0;
+        par[v].w_row0 = (int)wrow0;
         qrow += r.Lq[v];
         row0 += B[v];
+        wrow0 += video_w_rows(B[v], r.T);
     }
     auto mark = [&](int k) -> cudaError_t {
         return r.events ? cudaEventRecord((cudaEvent_t)r.events[k], r.stream) : cudaSuccess;
@@ -466,7 +477,7 @@ int wz_relevance(const void *features, int T, int H, int W, int D, int dtype, co
         return WZ_ERR_CUDA;
     }
     c.L1 = ((int64_t)T * s.N + c.G1 - 1) / c.G1;
-    VideoPar par{0, Lq, 0, 0};
+    VideoPar par{0, Lq, 0, 0, 0};
     const cudaStream_t cs = (cudaStream_t)stream;
     WZ_CUDA(launch_query_pool(c, &par, cs));
     WZ_CUDA(launch_relevance_pass(c, cs));

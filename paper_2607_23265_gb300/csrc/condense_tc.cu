@@ -7,7 +7,8 @@
 //       contiguous, exactly as the features lie in HBM), loaded by TMA with
 //       128-byte swizzle, box 64 channels x 32 tokens x 1 frame;
 //   B = W tile, N = n (the frame's condensed tokens, <= 256 per unit, padded
-//       to 16), K-major, loaded by TMA with 64-byte swizzle;
+//       to 16), K-major 8x8 core matrices without swizzle, stored in HBM in
+//       exactly that order (tile_index) so one bulk copy moves a stage;
 //   D = fp32 accumulators in tensor memory, 128 lanes x N columns per
 //       128-channel tile.
 // W_m is fp32 split into bf16 hi + lo (two MMAs into one accumulator), so the
@@ -24,6 +25,8 @@
 // bit, drains what it issued, frees tensor memory and exits.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+
+#include <cstring>
 
 #include "wz_internal.cuh"
 #include "wz_ptx.cuh"
@@ -52,6 +55,15 @@ struct TcShared {
 };
 
 constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + sizeof(TcShared);
+
+// Feature tensor maps: a 4D view [frames][D/64][N][64] whose box covers all
+// 2*CG 64-channel blocks of a stage in one copy (one map per CG), and the 3D
+// view [frames][N][D] for D not a multiple of 64 (two copies per tile).
+struct TcMaps {
+    CUtensorMap x3;
+    CUtensorMap x4[4];
+    int use4;
+};
 
 struct Unit {
     int f, j0, ct0, nc, cg;
@@ -82,8 +94,7 @@ __device__ __forceinline__ void fail(const Ctx &c, volatile int *abort_flag, int
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads, 1)
-condense_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmWhi,
-                   const __grid_constant__ CUtensorMap tmWlo, Ctx c) {
+condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     TcShared *S = reinterpret_cast<TcShared *>(ring + (size_t)kStages * kStageBytes);
@@ -115,9 +126,10 @@ condense_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constan
         ptx::tmem_relinquish();
     }
     if (warp == 0 && lane == 0) {
-        ptx::prefetch_tmap(&tmX);
-        ptx::prefetch_tmap(&tmWhi);
-        ptx::prefetch_tmap(&tmWlo);
+        if (maps.use4)
+            for (int g = 0; g < 4; ++g) ptx::prefetch_tmap(&maps.x4[g]);
+        else
+            ptx::prefetch_tmap(&maps.x3);
     }
     __syncthreads();
     ptx::tc_fence_after();
@@ -129,6 +141,9 @@ condense_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constan
         // ---------------- TMA producer ----------------
         const uint64_t pol_x = ptx::policy_evict_first();
         const uint64_t pol_w = ptx::policy_evict_last();
+        const char *whi = static_cast<const char *>(c.Wop);
+        const char *wlo = whi + (size_t)c.w_rows * c.K_pad * 2;
+        const size_t groups = (size_t)(c.w_rows >> 3);
         int stage = 0;
         uint32_t phase = 0;
         int issued_parity[kStages];
@@ -136,7 +151,7 @@ condense_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constan
         for (int u = blockIdx.x; u < n_units && !*abort_flag; u += gridDim.x) {
             const Unit un = decode_unit(c, S->vprefix, u);
             const int ncp = (un.nc + 15) & ~15;
-            const int row0 = c.off[un.f] + un.j0;
+            const int64_t wrow0 = (int64_t)c.woff[un.f] + un.j0;     // multiple of 16
             const uint32_t bytes = (uint32_t)un.cg * 8192u + 2u * (uint32_t)ncp * 64u;
             bool ok = true;
             for (int kc = 0; kc < KC; ++kc) {
@@ -147,15 +162,18 @@ condense_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constan
                 }
                 uint8_t *st = ring + (size_t)stage * kStageBytes;
                 ptx::mbar_arrive_expect_tx(&S->full[stage], bytes);
-                for (int ct = 0; ct < un.cg; ++ct)
-                    for (int h = 0; h < 2; ++h)
-                        ptx::tma_load_3d(st + ct * 8192 + h * 4096, &tmX, &S->full[stage],
-                                         (un.ct0 + ct) * kTileC + h * 64, kc * kKC, un.f, pol_x);
-                uint8_t *wh = st + un.cg * 8192;
-                for (int r = 0; r < ncp; r += 16) {
-                    ptx::tma_load_2d(wh + r * 64, &tmWhi, &S->full[stage], kc * kKC, row0 + r, pol_w);
-                    ptx::tma_load_2d(wh + ncp * 64 + r * 64, &tmWlo, &S->full[stage], kc * kKC, row0 + r, pol_w);
+                if (maps.use4) {
+                    ptx::tma_load_4d(st, &maps.x4[un.cg - 1], &S->full[stage], 0, kc * kKC, 2 * un.ct0, un.f, pol_x);
+                } else {
+                    for (int ct = 0; ct < un.cg; ++ct)
+                        for (int h = 0; h < 2; ++h)
+                            ptx::tma_load_3d(st + ct * 8192 + h * 4096, &maps.x3, &S->full[stage],
+                                             (un.ct0 + ct) * kTileC + h * 64, kc * kKC, un.f, pol_x);
                 }
+                uint8_t *wh = st + un.cg * 8192;
+                const size_t toff = ((size_t)kc * groups + (size_t)(wrow0 >> 3)) * 512;
+                ptx::bulk_load(wh, whi + toff, (uint32_t)ncp * 64u, &S->full[stage], pol_w);
+                ptx::bulk_load(wh + ncp * 64, wlo + toff, (uint32_t)ncp * 64u, &S->full[stage], pol_w);
                 issued_parity[stage] = (int)phase;
                 if (++stage == kStages) {
                     stage = 0;
@@ -197,8 +215,9 @@ condense_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constan
                 const uint32_t wl = wh + (uint32_t)ncp * 64u;
 #pragma unroll
                 for (int s = 0; s < 2; ++s) {
-                    const uint64_t bh = ptx::smem_desc(wh + s * 32, 16, 512, 4);
-                    const uint64_t bl = ptx::smem_desc(wl + s * 32, 16, 512, 4);
+                    // no swizzle: core matrices 128 B apart along K, 8-row groups 512 B apart
+                    const uint64_t bh = ptx::smem_desc(wh + s * 256, 128, 512, 0);
+                    const uint64_t bl = ptx::smem_desc(wl + s * 256, 128, 512, 0);
                     for (int ct = 0; ct < un.cg; ++ct) {
                         const uint64_t a = ptx::smem_desc(st + ct * 8192 + s * 2048, 4096, 1024, 2);
                         const uint32_t d = dbase + (uint32_t)(ct * ncp);
@@ -284,32 +303,33 @@ cudaError_t launch_condense_tc(const Ctx &c, cudaStream_t s) {
     auto enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
     if (c.dtype != WZ_DTYPE_BF16 || c.rows_total < 1) return cudaErrorInvalidValue;
-    CUtensorMap tmX, tmWhi, tmWlo;
+    TcMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    void *X = const_cast<void *>(c.X);
+    const cuuint64_t frames = (cuuint64_t)c.V * c.T;
     {
-        cuuint64_t dims[3] = {(cuuint64_t)c.D, (cuuint64_t)c.N, (cuuint64_t)c.V * c.T};
+        cuuint64_t dims[3] = {(cuuint64_t)c.D, (cuuint64_t)c.N, frames};
         cuuint64_t strides[2] = {(cuuint64_t)c.D * 2, (cuuint64_t)c.N * c.D * 2};
         cuuint32_t box[3] = {64, (cuuint32_t)kKC, 1};
         cuuint32_t es[3] = {1, 1, 1};
-        if (enc(&tmX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(c.X), dims, strides, box, es,
+        if (enc(&maps.x3, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, X, dims, strides, box, es,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
-    __nv_bfloat16 *whi = static_cast<__nv_bfloat16 *>(c.Wop);
-    __nv_bfloat16 *wlo = whi + (size_t)c.rows_total * c.K_pad;
-    {
-        cuuint64_t dims[2] = {(cuuint64_t)c.K_pad, (cuuint64_t)c.rows_total};
-        cuuint64_t strides[1] = {(cuuint64_t)c.K_pad * 2};
-        cuuint32_t box[2] = {(cuuint32_t)kKC, 16};
-        cuuint32_t es[2] = {1, 1};
-        if (enc(&tmWhi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, whi, dims, strides, box, es,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-            return cudaErrorInvalidValue;
-        if (enc(&tmWlo, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, wlo, dims, strides, box, es,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-            return cudaErrorInvalidValue;
+    maps.use4 = 0;
+    if (c.D % 64 == 0) {
+        cuuint64_t dims[4] = {64, (cuuint64_t)c.N, (cuuint64_t)(c.D / 64), frames};
+        cuuint64_t strides[3] = {(cuuint64_t)c.D * 2, 128, (cuuint64_t)c.N * c.D * 2};
+        cuuint32_t es[4] = {1, 1, 1, 1};
+        bool ok = true;
+        for (int g = 0; g < 4 && ok; ++g) {
+            cuuint32_t box[4] = {64, (cuuint32_t)kKC, (cuuint32_t)(2 * (g + 1)), 1};
+            ok = enc(&maps.x4[g], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, X, dims, strides, box, es,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+        }
+        maps.use4 = ok ? 1 : 0;
     }
     int dev = 0, sms = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -318,7 +338,7 @@ cudaError_t launch_condense_tc(const Ctx &c, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(condense_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess) return e;
-    condense_tc_kernel<<<sms, kThreads, kSmemBytes, s>>>(tmX, tmWhi, tmWlo, c);
+    condense_tc_kernel<<<sms, kThreads, kSmemBytes, s>>>(maps, c);
     return cudaGetLastError();
 }
 

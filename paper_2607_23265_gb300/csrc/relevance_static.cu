@@ -122,7 +122,7 @@ extern "C" int wz_relevance_static(const void *features, int T, int H, int W, in
     c.frame_scores = frame_scores;
     c.frame_mean = frame_mean;
 
-    const VideoPar par{0, Lq, 0, 0};
+    const VideoPar par{0, Lq, 0, 0, 0};
     const cudaStream_t s = (cudaStream_t)stream;
     if (launch_query_pool(c, &par, s) != cudaSuccess || launch_relevance_pass(c, s) != cudaSuccess ||
         launch_frame_stats(c, s) != cudaSuccess || launch_relevance_finalize(c, s) != cudaSuccess) {

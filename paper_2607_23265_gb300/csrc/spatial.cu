@@ -196,10 +196,11 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
     __syncthreads();
     // operator rows of this grid row: p = pi*w + q, q < w, p < n
     const int nq = min(w, n - pi * w);
-    const int64_t row0 = (int64_t)c.off[f] + (int64_t)pi * w;
+    const int64_t row0 = (int64_t)c.off[f] + (int64_t)pi * w;      // output row
     const bool bf = c.path == WZ_PATH_TENSOR;
+    const int64_t wrow0 = bf ? (int64_t)c.woff[f] + (int64_t)pi * w : row0;   // operator row
     __nv_bfloat16 *Whi = static_cast<__nv_bfloat16 *>(c.Wop);
-    __nv_bfloat16 *Wlo = Whi + (size_t)c.rows_total * c.K_pad;
+    __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * c.K_pad;
     float *W32 = static_cast<float *>(c.Wop);
     for (int item = tid; item < nq * W; item += blockDim.x) {
         const int q = item / W, j = item % W;
@@ -215,25 +216,25 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
 #pragma unroll
             for (int b = 0; b < WPMAX; ++b)
                 if (b < wp) s += Yl[b * H + i] * qa_l[b] + Yh[b * H + i] * qa_h[b];
-            const size_t k = rbase + (size_t)i * W + j;
             if (bf) {
+                const size_t k = tile_index(wrow0 + q, i * W + j, c.w_rows);
                 const __nv_bfloat16 hb = __float2bfloat16_rn(s);
                 Whi[k] = hb;
                 Wlo[k] = __float2bfloat16_rn(s - __bfloat162float(hb));
             } else {
-                W32[k] = s;
+                W32[rbase + (size_t)i * W + j] = s;
             }
         }
     }
     // zero the K padding of these rows, and the index map rows
     const int padw = c.K_pad - N;
     for (int k = tid; k < nq * padw; k += blockDim.x) {
-        const size_t idx = (size_t)(row0 + k / padw) * c.K_pad + N + (k % padw);
         if (bf) {
+            const size_t idx = tile_index(wrow0 + k / padw, N + (k % padw), c.w_rows);
             Whi[idx] = __float2bfloat16_rn(0.f);
             Wlo[idx] = __float2bfloat16_rn(0.f);
         } else {
-            W32[idx] = 0.f;
+            W32[(size_t)(row0 + k / padw) * c.K_pad + N + (k % padw)] = 0.f;
         }
     }
     const int t = (int)(f % c.T);

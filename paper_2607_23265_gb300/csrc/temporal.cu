@@ -296,6 +296,18 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         c.prod[v] = produced;
         if (c.out_count) c.out_count[v] = produced;
     }
+    // first tensor-core operator row of each frame: budgets padded to 16
+    int s16 = 0;
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k) s16 += (nloc[k] + 15) & ~15;
+    int wtot = 0;
+    int wo = block_excl_scan(s16, iscr, &wtot);
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k) {
+        const int t = t0 + k;
+        if (t < T) c.woff[base + t] = vp.w_row0 + wo;
+        wo += (nloc[k] + 15) & ~15;
+    }
     // tensor-core units: per frame, column blocks of <= 256 tokens; per
     // block, groups of CG 128-channel tiles with CG * round16(nc) <= 256.
     if (c.path == WZ_PATH_TENSOR) {

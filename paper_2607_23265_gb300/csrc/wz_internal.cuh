@@ -21,6 +21,7 @@ struct VideoPar {
     int Lq;        // query rows
     int B;         // global budget of the video
     int row0;      // first output row of the video
+    int w_row0;    // first tensor-core operator row of the video (multiple of 16)
 };
 
 // Everything a kernel of one call needs: sizes, inputs, workspace views,
@@ -36,7 +37,8 @@ struct Ctx {
     int max_units_v;      // unit-list capacity per video
     int F;                // WSM filter taps
     int64_t L1;           // tokens per relevance CTA
-    int64_t rows_total;   // sum of budgets over videos (operator rows)
+    int64_t rows_total;   // sum of budgets over videos (output rows)
+    int64_t w_rows;       // operator rows of the tensor-core layout (frames padded to 16)
 
     const void *X;
     const void *Q;
@@ -53,11 +55,13 @@ struct Ctx {
     int *list;            // [V][2T] retained frames and their budgets
     int *n;               // [V*T] budgets
     int *off;             // [V*T] global output row of the frame's first token
+    int *woff;            // [V*T] first tensor-core operator row of the frame
     int *hw;              // [V*T][2] condensation grid
     int *prod;            // [V] produced rows
     int4 *units;          // [V][max_units_v] tensor-core work units
     int *ucount;          // [V]
-    void *Wop;            // operator rows: bf16 hi [rows][K_pad] then lo, or f32
+    void *Wop;            // operator: tensor path bf16 hi then lo in the tiled
+                          // layout of tile_index(), CUDA-core path f32 [rows][K_pad]
     int *status;          // device status word (bounded waits)
 
     void *out;            // [rows][D] dtype
@@ -169,6 +173,17 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     s = a + b;
     const float bb = s - a;
     e = (a - (s - bb)) + (b - bb);
+}
+
+// Element index of operator entry (row r, column k) in the tensor-core
+// layout: 8 x 8 core matrices (8 rows of 8 bf16 = 16 bytes), ordered by
+// 32-column K chunk, then 8-row group, then the four 8-column quarters of the
+// chunk.  The rows [r0, r0 + n) of one K chunk (r0, n multiples of 8) are
+// therefore one contiguous block that a single bulk copy moves into shared
+// memory, where it is the canonical no-swizzle K-major operand of tcgen05.mma.
+__host__ __device__ __forceinline__ size_t tile_index(int64_t r, int k, int64_t w_rows) {
+    return ((((size_t)(k >> 5) * (size_t)(w_rows >> 3) + (size_t)(r >> 3)) * 4 + ((k >> 3) & 3)) * 64) +
+           (size_t)(r & 7) * 8 + (size_t)(k & 7);
 }
 
 // ---- launchers (one per kernel family) -------------------------------------
