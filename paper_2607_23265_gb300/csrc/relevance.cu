@@ -25,26 +25,42 @@ struct VideoParBlock {
     VideoPar v[WZ_MAX_VIDEOS];
 };
 
-// u_q = mean of the query rows: one thread per channel, compensated fp32
-// accumulation (TwoSum), stored as fp64 and fp32.
+// u_q = mean of the query rows: a block covers 32 channels with 8 row
+// slices; compensated fp32 sums (TwoSum) per slice, combined in a fixed
+// order, stored as fp64 and fp32.
 template <typename T>
 __global__ void __launch_bounds__(256) query_pool_kernel(Ctx c, VideoParBlock par) {
+    __shared__ float ps[8][32], pe[8][32];
     const int v = blockIdx.y;
     const VideoPar vp = par.v[v];
     if (blockIdx.x == 0 && threadIdx.x == 0) c.vpar[v] = vp;
-    const int d = blockIdx.x * blockDim.x + threadIdx.x;
-    if (d >= c.D) return;
-    const T *Q = static_cast<const T *>(c.Q) + (size_t)vp.q_row0 * c.D + d;
+    const int cl = threadIdx.x & 31, slice = threadIdx.x >> 5;
+    const int d = blockIdx.x * 32 + cl;
     float s = 0.f, e = 0.f;
-    for (int j = 0; j < vp.Lq; ++j) {
-        float t, err;
-        two_sum(s, load_scalar<T>(Q + (size_t)j * c.D), t, err);
-        s = t;
-        e += err;
+    if (d < c.D) {
+        const T *Q = static_cast<const T *>(c.Q) + (size_t)vp.q_row0 * c.D + d;
+        for (int j = slice; j < vp.Lq; j += 8) {
+            float t, err;
+            two_sum(s, load_scalar<T>(Q + (size_t)j * c.D), t, err);
+            s = t;
+            e += err;
+        }
     }
-    const double m = ((double)s + (double)e) / (double)vp.Lq;
-    c.qbar64[(size_t)v * c.D + d] = m;
-    c.qbar32[(size_t)v * c.D + d] = (float)m;
+    ps[slice][cl] = s;
+    pe[slice][cl] = e;
+    __syncthreads();
+    if (slice == 0 && d < c.D) {
+        float S = 0.f, E = 0.f;
+        for (int k = 0; k < 8; ++k) {
+            float t, err;
+            two_sum(S, ps[k][cl], t, err);
+            S = t;
+            E += err + pe[k][cl];
+        }
+        const double m = ((double)S + (double)E) / (double)vp.Lq;
+        c.qbar64[(size_t)v * c.D + d] = m;
+        c.qbar32[(size_t)v * c.D + d] = (float)m;
+    }
 }
 
 // Reduce the NV values held by every lane across the warp (NV a power of
@@ -274,20 +290,22 @@ __global__ void __launch_bounds__(256) frame_stats_kernel(Ctx c) {
     const int64_t g = f - 1;
     const int64_t lo2 = t > 0 ? g * c.N / c.L1 : 0;
     const int64_t hi2 = t > 0 ? min((int64_t)c.G1 - 1, ((g + 1) * c.N - 1) / c.L1) : -1;
-    double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+    // fp32 products summed over this thread's 8 channels, fp64 across threads
+    float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f;
     for (int k = 0; k < kStatsChunk / 256; ++k) {
         const int d = blockIdx.x * kStatsChunk + k * 256 + threadIdx.x;
         if (d >= c.D) break;
-        double sf = 0.0, sp = 0.0;
-        for (int64_t cc = lo; cc <= hi; ++cc) sf += (double)c.part[(size_t)(cc + f) * c.D + d];
-        for (int64_t cc = lo2; cc <= hi2; ++cc) sp += (double)c.part[(size_t)(cc + g) * c.D + d];
-        const double q = c.qbar64[(size_t)v * c.D + d];
-        if (c.frame_mean) c.frame_mean[(size_t)f * c.D + d] = (float)(sf / c.N);
-        s0 += sf * q;
-        s1 += sf * sf;
-        s2 += sf * sp;
-        s3 += q * q;
+        float sf = 0.f, sp = 0.f;
+        for (int64_t cc = lo; cc <= hi; ++cc) sf += c.part[(size_t)(cc + f) * c.D + d];
+        for (int64_t cc = lo2; cc <= hi2; ++cc) sp += c.part[(size_t)(cc + g) * c.D + d];
+        const float q = c.qbar32[(size_t)v * c.D + d];
+        if (c.frame_mean) c.frame_mean[(size_t)f * c.D + d] = sf / (float)c.N;
+        p0 = fmaf(sf, q, p0);
+        p1 = fmaf(sf, sf, p1);
+        p2 = fmaf(sf, sp, p2);
+        p3 = fmaf(q, q, p3);
     }
+    double s0 = p0, s1 = p1, s2 = p2, s3 = p3;
     s0 = block_sum(s0, scratch);
     s1 = block_sum(s1, scratch);
     s2 = block_sum(s2, scratch);
@@ -320,7 +338,7 @@ cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s
     VideoParBlock blk;   // copied into the launch parameters
     memset(&blk, 0, sizeof(blk));
     for (int v = 0; v < c.V; ++v) blk.v[v] = hpar[v];
-    const dim3 grid((unsigned)((c.D + 255) / 256), (unsigned)c.V);
+    const dim3 grid((unsigned)((c.D + 31) / 32), (unsigned)c.V);
     if (c.dtype == WZ_DTYPE_BF16)
         query_pool_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c, blk);
     else

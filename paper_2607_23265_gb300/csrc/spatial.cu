@@ -14,7 +14,9 @@
 //   Y_v[b,i]         = sum_u sum_a P_u[p,a] A_u[a,i] g_uv[a,b].
 //
 // One CTA per (frame, grid row p) builds the w_m rows of W_m for that grid
-// row in fp32 from tables in shared memory, writes them as bf16 hi/lo pairs
+// row in fp32 from tables in shared memory (each thread owns one output
+// token q and input column j and sums only over the few b where A'_v[b, j]
+// is nonzero), writes them as bf16 hi/lo pairs
 // (tensor-core path) or fp32 (CUDA-core path), writes the index map rows,
 // and trailing CTAs fill rows that cannot be produced with -1 / zeros.
 #include <cmath>
@@ -27,25 +29,34 @@ constexpr int kSpatialThreads = 256;
 constexpr int kTailBlocks = 64;
 
 struct SpatialSmem {
-    int N, hp, wp, H, W;
+    int N, hp, wp, H, W, HP4;
     // float offsets
-    int M, G, AHl, AHh, AWl, AWh, PAl, PAh, Yl, Yh, Ql, Qh, red, total;
+    int M, G, AHl, AHh, AWl, AWh, PAl, PAh, Yl, Yh, Ql, Qh, red, blo, bhi, total;
+    // Every table starts on a 16-byte boundary (float4 reads of Y).
     __host__ __device__ void init(int H_, int W_, int hp_, int wp_) {
         H = H_; W = W_; hp = hp_; wp = wp_; N = H * W;
+        HP4 = (H + 3) & ~3;
         int o = 0;
-        M = o; o += N;
-        G = o; o += hp * wp;
-        AHl = o; o += hp * H;
-        AHh = o; o += hp * H;
-        AWl = o; o += wp * W;
-        AWh = o; o += wp * W;
-        PAl = o; o += hp * H;
-        PAh = o; o += hp * H;
-        Yl = o; o += wp * H;
-        Yh = o; o += wp * H;
-        Ql = o; o += W * wp;
-        Qh = o; o += W * wp;
-        red = o; o += 64;
+        auto take = [&](int n) {
+            const int at = o;
+            o = (o + n + 3) & ~3;
+            return at;
+        };
+        M = take(N);
+        G = take(hp * wp);
+        AHl = take(hp * H);
+        AHh = take(hp * H);
+        AWl = take(wp * W);
+        AWh = take(wp * W);
+        PAl = take(hp * H);
+        PAh = take(hp * H);
+        Yl = take(wp * HP4);
+        Yh = take(wp * HP4);
+        Ql = take(W * wp);
+        Qh = take(W * wp);
+        red = take(64);
+        blo = take(W);
+        bhi = take(W);
         total = o;
     }
 };
@@ -66,7 +77,7 @@ __device__ __forceinline__ void bilinear_src(int i, int in, int out, int &y0, in
     l = (float)(s - f);
 }
 
-template <int WPMAX>
+template <int HMAX>
 __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
     extern __shared__ float sm[];
     const int tid = threadIdx.x;
@@ -100,6 +111,8 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
     float *AHl = sm + L.AHl, *AHh = sm + L.AHh, *AWl = sm + L.AWl, *AWh = sm + L.AWh;
     float *PAl = sm + L.PAl, *PAh = sm + L.PAh, *Yl = sm + L.Yl, *Yh = sm + L.Yh;
     float *Ql = sm + L.Ql, *Qh = sm + L.Qh, *red = sm + L.red;
+    int *blo = reinterpret_cast<int *>(sm + L.blo), *bhi = reinterpret_cast<int *>(sm + L.bhi);
+    const int HP4 = L.HP4;
 
     // saliency map M (Eq. 6): per-frame min-max of a_{t,n}
     const float *a = c.a + f * N;
@@ -179,16 +192,29 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
         Ql[k] = (1.f - lx) * synth(c.rec_lo, F, x0, b) + lx * synth(c.rec_lo, F, x1, b);
         Qh[k] = (1.f - lx) * synth(c.rec_hi, F, x0, b) + lx * synth(c.rec_hi, F, x1, b);
     }
+    // support of the width analysis: rows b of A' that reach column j
+    for (int j = tid; j < W; j += blockDim.x) {
+        int lo_b = wp, hi_b = -1;
+        for (int b = 0; b < wp; ++b)
+            if (AWl[b * W + j] != 0.f || AWh[b * W + j] != 0.f) {
+                lo_b = min(lo_b, b);
+                hi_b = max(hi_b, b);
+            }
+        blo[j] = lo_b;
+        bhi[j] = hi_b;
+    }
     __syncthreads();
-    // Y_v[b][i]
-    for (int k = tid; k < wp * H; k += blockDim.x) {
-        const int b = k / H, i = k % H;
+    // Y_v[b][i], rows padded to a multiple of 4 with zeros
+    for (int k = tid; k < wp * HP4; k += blockDim.x) {
+        const int b = k / HP4, i = k % HP4;
         float yl = 0.f, yh = 0.f;
-        for (int ai = 0; ai < hp; ++ai) {
-            const float g = G[ai * wp + b];
-            const float pl = PAl[ai * H + i], ph = PAh[ai * H + i];
-            yl += pl + ph * g;
-            yh += (pl + ph) * g;
+        if (i < H) {
+            for (int ai = 0; ai < hp; ++ai) {
+                const float g = G[ai * wp + b];
+                const float pl = PAl[ai * H + i], ph = PAh[ai * H + i];
+                yl += pl + ph * g;
+                yh += (pl + ph) * g;
+            }
         }
         Yl[k] = yl;
         Yh[k] = yh;
@@ -202,27 +228,42 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
     __nv_bfloat16 *Whi = static_cast<__nv_bfloat16 *>(c.Wop);
     __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * c.K_pad;
     float *W32 = static_cast<float *>(c.Wop);
+    // one thread per (output q, input column j): all H rows i in registers,
+    // summed over the support of column j only
     for (int item = tid; item < nq * W; item += blockDim.x) {
         const int q = item / W, j = item % W;
-        float qa_l[WPMAX], qa_h[WPMAX];
+        float acc[HMAX];
 #pragma unroll
-        for (int b = 0; b < WPMAX; ++b) {
-            qa_l[b] = b < wp ? Ql[q * wp + b] * AWl[b * W + j] : 0.f;
-            qa_h[b] = b < wp ? Qh[q * wp + b] * AWh[b * W + j] : 0.f;
+        for (int i = 0; i < HMAX; ++i) acc[i] = 0.f;
+        for (int b = blo[j]; b <= bhi[j]; ++b) {
+            const float ql = Ql[q * wp + b] * AWl[b * W + j];
+            const float qh = Qh[q * wp + b] * AWh[b * W + j];
+            const float4 *yl = reinterpret_cast<const float4 *>(Yl + b * HP4);
+            const float4 *yh = reinterpret_cast<const float4 *>(Yh + b * HP4);
+#pragma unroll
+            for (int i4 = 0; i4 < HMAX / 4; ++i4) {
+                if (4 * i4 < H) {
+                    const float4 a = yl[i4], d = yh[i4];
+                    acc[4 * i4 + 0] = fmaf(a.x, ql, fmaf(d.x, qh, acc[4 * i4 + 0]));
+                    acc[4 * i4 + 1] = fmaf(a.y, ql, fmaf(d.y, qh, acc[4 * i4 + 1]));
+                    acc[4 * i4 + 2] = fmaf(a.z, ql, fmaf(d.z, qh, acc[4 * i4 + 2]));
+                    acc[4 * i4 + 3] = fmaf(a.w, ql, fmaf(d.w, qh, acc[4 * i4 + 3]));
+                }
+            }
         }
         const size_t rbase = (size_t)(row0 + q) * c.K_pad;
-        for (int i = 0; i < H; ++i) {
-            float s = 0.f;
 #pragma unroll
-            for (int b = 0; b < WPMAX; ++b)
-                if (b < wp) s += Yl[b * H + i] * qa_l[b] + Yh[b * H + i] * qa_h[b];
-            if (bf) {
-                const size_t k = tile_index(wrow0 + q, i * W + j, c.w_rows);
-                const __nv_bfloat16 hb = __float2bfloat16_rn(s);
-                Whi[k] = hb;
-                Wlo[k] = __float2bfloat16_rn(s - __bfloat162float(hb));
-            } else {
-                W32[rbase + (size_t)i * W + j] = s;
+        for (int i = 0; i < HMAX; ++i) {
+            if (i < H) {
+                const float s = acc[i];
+                if (bf) {
+                    const size_t k = tile_index(wrow0 + q, i * W + j, c.w_rows);
+                    const __nv_bfloat16 hb = __float2bfloat16_rn(s);
+                    Whi[k] = hb;
+                    Wlo[k] = __float2bfloat16_rn(s - __bfloat162float(hb));
+                } else {
+                    W32[rbase + (size_t)i * W + j] = s;
+                }
             }
         }
     }
@@ -253,13 +294,15 @@ size_t spatial_smem_bytes(const Ctx &c) {
 }
 
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
+    SpatialSmem L;
+    L.init(c.H, c.W, c.hp, c.wp);
+    if ((L.Yl & 3) != 0 || (L.Yh & 3) != 0) return cudaErrorMisalignedAddress;
     const size_t smem = spatial_smem_bytes(c);
     const unsigned blocks = (unsigned)((int64_t)c.V * c.T * c.H + kTailBlocks);
     const void *fn;
-    if (c.wp <= 12) fn = (const void *)spatial_kernel<12>;
-    else if (c.wp <= 20) fn = (const void *)spatial_kernel<20>;
-    else if (c.wp <= 36) fn = (const void *)spatial_kernel<36>;
-    else if (c.wp <= 44) fn = (const void *)spatial_kernel<44>;
+    if (c.H <= 16) fn = (const void *)spatial_kernel<16>;
+    else if (c.H <= 32) fn = (const void *)spatial_kernel<32>;
+    else if (c.H <= 64) fn = (const void *)spatial_kernel<64>;
     else return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
