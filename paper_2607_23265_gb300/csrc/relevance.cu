@@ -164,10 +164,11 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
 
     // ---------------- consumers ----------------
     auto consumer_sync = [&]() { asm volatile("bar.sync 1, %0;" ::"r"(NC) : "memory"); };
+    constexpr int NP = VEC / 2;                  // packed pairs per 16-byte vector
     int cur_v = -1;
-    float q[VPT][VEC];
+    f2_t q[VPT][NP];
     float qn = 0.f;
-    float cs[VPT][VEC];
+    f2_t cs[VPT][NP];
     int gi = 0;
     int s = 0;
     uint32_t ph = 0;
@@ -185,9 +186,11 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
                 for (int vi = 0; vi < VPT; ++vi) {
                     const int vidx = threadIdx.x + vi * NC;
 #pragma unroll
-                    for (int e = 0; e < VEC; ++e) {
-                        q[vi][e] = vidx < n_vec ? c.qbar32[(size_t)v * c.D + vidx * VEC + e] : 0.f;
-                        qq = fmaf(q[vi][e], q[vi][e], qq);
+                    for (int e = 0; e < NP; ++e) {
+                        const float q0 = vidx < n_vec ? c.qbar32[(size_t)v * c.D + vidx * VEC + 2 * e] : 0.f;
+                        const float q1 = vidx < n_vec ? c.qbar32[(size_t)v * c.D + vidx * VEC + 2 * e + 1] : 0.f;
+                        q[vi][e] = pack2(q0, q1);
+                        qq = fmaf(q0, q0, fmaf(q1, q1, qq));
                     }
                 }
                 for (int o = 16; o > 0; o >>= 1) qq += __shfl_xor_sync(0xffffffffu, qq, o);
@@ -201,7 +204,7 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
 #pragma unroll
             for (int vi = 0; vi < VPT; ++vi)
 #pragma unroll
-                for (int e = 0; e < VEC; ++e) cs[vi][e] = 0.f;
+                for (int e = 0; e < NP; ++e) cs[vi][e] = 0ull;
         }
         // wait for the chunk (one bounded waiter decides for all consumers)
         if (threadIdx.x == 0) ok_flag = ptx::mbar_wait(&full[s], ph, kRelTimeoutNs) ? 1 : 0;
@@ -211,30 +214,36 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
             break;
         }
         ptx::mbar_wait(&full[s], ph, kRelTimeoutNs);   // completed: acquire for this thread
-        const uint8_t *st = rsm + s * stage_bytes;
-        for (int64_t g0 = 0; g0 < n; g0 += GROUP, ++gi) {
+        const uint32_t st32 = ptx::smem_u32(rsm) + (uint32_t)(s * stage_bytes);
+        const uint32_t rowb32 = (uint32_t)rowb;
+        const int nt = (int)n;
+        for (int g0 = 0; g0 < nt; g0 += GROUP, ++gi) {
             float acc[NV];
-#pragma unroll
-            for (int k = 0; k < NV; ++k) acc[k] = 0.f;
+            const bool full_group = nt - g0 >= GROUP;
 #pragma unroll
             for (int k = 0; k < GROUP; ++k) {
-                if (g0 + k < n) {
+                f2_t dd = 0ull, nn = 0ull;
+                if (full_group || g0 + k < nt) {
+                    const uint32_t row = st32 + (uint32_t)(g0 + k) * rowb32;
 #pragma unroll
                     for (int vi = 0; vi < VPT; ++vi) {
                         const int vidx = threadIdx.x + vi * NC;
                         if (vidx < n_vec) {
-                            const uint4 raw = *reinterpret_cast<const uint4 *>(st + (size_t)(g0 + k) * rowb + (size_t)vidx * 16);
-                            float x[VEC];
-                            unpack(raw, x, (T *)nullptr);
+                            const uint4 raw = ptx::lds128(row + (uint32_t)vidx * 16u);
+                            f2_t x[NP];
+                            unpack_pairs(raw, x, (T *)nullptr);
 #pragma unroll
-                            for (int e = 0; e < VEC; ++e) {
-                                cs[vi][e] += x[e];
-                                acc[k] = fmaf(x[e], q[vi][e], acc[k]);
-                                acc[k + GROUP] = fmaf(x[e], x[e], acc[k + GROUP]);
+                            for (int e = 0; e < NP; ++e) {
+                                cs[vi][e] = add2(cs[vi][e], x[e]);
+                                dd = fma2(x[e], q[vi][e], dd);
+                                nn = fma2(x[e], x[e], nn);
                             }
                         }
                     }
                 }
+                const float2 d2 = unpack2(dd), n2 = unpack2(nn);
+                acc[k] = d2.x + d2.y;
+                acc[k + GROUP] = n2.x + n2.y;
             }
             const float tot = transpose_reduce<NV>(acc);
             const int b = gi & 1;
@@ -245,7 +254,7 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
                 if (lane < NV)
                     for (int w = 0; w < nw; ++w) sm += red[b][w][lane];
                 const float nrm = __shfl_down_sync(0xffffffffu, sm, GROUP);
-                if (lane < GROUP && g0 + lane < n) {
+                if (lane < GROUP && g0 + lane < nt) {
                     const float a = (nrm > 0.f && qn > 0.f) ? sm / (sqrtf(nrm) * qn) : 0.f;
                     c.a[tok + g0 + lane] = a;
                 }
@@ -268,9 +277,10 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
                 const int vidx = threadIdx.x + vi * NC;
                 if (vidx < n_vec) {
 #pragma unroll
-                    for (int e = 0; e < VEC; e += 4)
-                        *reinterpret_cast<float4 *>(dst + vidx * VEC + e) =
-                            make_float4(cs[vi][e], cs[vi][e + 1], cs[vi][e + 2], cs[vi][e + 3]);
+                    for (int e = 0; e < NP; e += 2) {
+                        const float2 a = unpack2(cs[vi][e]), b = unpack2(cs[vi][e + 1]);
+                        *reinterpret_cast<float4 *>(dst + vidx * VEC + 2 * e) = make_float4(a.x, a.y, b.x, b.y);
+                    }
                 }
             }
         }

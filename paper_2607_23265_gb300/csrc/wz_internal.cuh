@@ -168,6 +168,46 @@ __device__ __forceinline__ long long block_sum_ll(long long v, long long *scratc
     return scratch[32];
 }
 
+// ---- packed fp32 pairs (f32x2 instructions of sm_100-class GPUs) ----------
+
+typedef unsigned long long f2_t;
+
+__device__ __forceinline__ f2_t pack2(float lo, float hi) {
+    f2_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ float2 unpack2(f2_t v) {
+    float2 r;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
+    return r;
+}
+
+__device__ __forceinline__ f2_t fma2(f2_t a, f2_t b, f2_t c) {
+    f2_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+
+__device__ __forceinline__ f2_t add2(f2_t a, f2_t b) {
+    f2_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+
+// A 16-byte vector as VEC/2 packed pairs of consecutive elements.
+__device__ __forceinline__ void unpack_pairs(const uint4 &v, f2_t (&p)[4], __nv_bfloat16 *) {
+    p[0] = pack2(bf16_lo(v.x), bf16_hi(v.x));
+    p[1] = pack2(bf16_lo(v.y), bf16_hi(v.y));
+    p[2] = pack2(bf16_lo(v.z), bf16_hi(v.z));
+    p[3] = pack2(bf16_lo(v.w), bf16_hi(v.w));
+}
+__device__ __forceinline__ void unpack_pairs(const uint4 &v, f2_t (&p)[2], float *) {
+    p[0] = pack2(__uint_as_float(v.x), __uint_as_float(v.y));
+    p[1] = pack2(__uint_as_float(v.z), __uint_as_float(v.w));
+}
+
 // Error-free sum of two floats (Knuth's TwoSum): a + b = s + e exactly.
 __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     s = a + b;
