@@ -27,12 +27,12 @@ bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
 // Sub-buffer offsets of one call's workspace.
 struct Layout {
-    size_t qbar32, qbar64, qnorm, vpar, a, part, trip, fr, tmp, list, n, off, woff, hw, prod,
+    size_t qbar32, qbar64, vpar, a, part, fr, tmp, list, n, off, woff, hw, prod,
         units, ucount, status, Wop, total;
 };
 
 struct Shape {
-    int V, T, H, W, D, N, dtype, F, hp, wp, K_pad, DC, n_ct, max_units_v;
+    int V, T, H, W, D, N, dtype, F, hp, wp, K_pad, n_ct, max_units_v;
     int64_t rows_total, w_rows;
 };
 
@@ -47,11 +47,9 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     const size_t VT = (size_t)s.V * s.T;
     L.qbar32 = take((size_t)s.V * s.D * 4);
     L.qbar64 = take((size_t)s.V * s.D * 8);
-    L.qnorm = take((size_t)s.V * 8);
     L.vpar = take((size_t)s.V * sizeof(VideoPar));
     L.a = with_a ? take(VT * s.N * 4) : 0;
     L.part = take(((size_t)kG1Max + VT) * s.D * 4);
-    L.trip = take(VT * s.DC * 4 * 8);
     L.fr = take(VT * 4 * 8);
     L.tmp = take(VT * 4 * 8);
     L.list = take(VT * 2 * 4);
@@ -95,7 +93,6 @@ Shape make_shape(int V, int T, int H, int W, int D, int dtype, int F, const int6
     s.hp = (H + F - 1) / 2;
     s.wp = (W + F - 1) / 2;
     s.K_pad = (s.N + 31) / 32 * 32;
-    s.DC = (D + kStatsChunk - 1) / kStatsChunk;
     s.n_ct = (D + kTileC - 1) / kTileC;
     int64_t rows = 0, bmax = 0, wrows = 0;
     for (int v = 0; v < V; ++v) {
@@ -145,15 +142,13 @@ void set_filters(Ctx &c, int p) {
 
 void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.V = s.V; c.T = s.T; c.H = s.H; c.W = s.W; c.D = s.D; c.N = s.N; c.dtype = s.dtype;
-    c.hp = s.hp; c.wp = s.wp; c.K_pad = s.K_pad; c.DC = s.DC; c.n_ct = s.n_ct;
+    c.hp = s.hp; c.wp = s.wp; c.K_pad = s.K_pad; c.n_ct = s.n_ct;
     c.max_units_v = s.max_units_v; c.rows_total = s.rows_total; c.w_rows = s.w_rows;
     c.qbar32 = reinterpret_cast<float *>(ws + L.qbar32);
     c.qbar64 = reinterpret_cast<double *>(ws + L.qbar64);
-    c.qnorm = reinterpret_cast<double *>(ws + L.qnorm);
     c.vpar = reinterpret_cast<VideoPar *>(ws + L.vpar);
     if (L.a) c.a = reinterpret_cast<float *>(ws + L.a);
     c.part = reinterpret_cast<float *>(ws + L.part);
-    c.trip = reinterpret_cast<double *>(ws + L.trip);
     c.fr = reinterpret_cast<double *>(ws + L.fr);
     c.tmp = reinterpret_cast<double *>(ws + L.tmp);
     c.list = reinterpret_cast<int *>(ws + L.list);
@@ -450,6 +445,7 @@ size_t wz_relevance_workspace_size(int T, int H, int W, int D) {
     return make_layout(s, false, false).total;
 }
 
+
 int wz_relevance(const void *features, int T, int H, int W, int D, int dtype, const void *query,
                  int Lq, float *token_scores, float *frame_scores, float *frame_mean,
                  void *workspace, size_t workspace_bytes, wz_stream_t stream) {
@@ -482,7 +478,6 @@ int wz_relevance(const void *features, int T, int H, int W, int D, int dtype, co
     WZ_CUDA(launch_query_pool(c, &par, cs));
     WZ_CUDA(launch_relevance_pass(c, cs));
     WZ_CUDA(launch_frame_stats(c, cs));
-    WZ_CUDA(launch_relevance_finalize(c, cs));
     return WZ_OK;
 }
 

@@ -5,10 +5,10 @@
 //                   a_{t,n} = <u, u_q> / (||u|| ||u_q||) (the input of Eq. 6)
 //                   and per-CTA column sums of every frame it touches (the
 //                   average pool of Section 3.2.1 / Eq. 7), in fp32.
-//   frame_stats     sums the column partials of a frame in fp64 in a fixed
-//                   order and reduces <v_t,u_q>, <v_t,v_t>, <v_t,v_{t-1}> and
-//                   <u_q,u_q> per 2048-channel chunk, which give r_t and
-//                   delta_t (Eq. 7).
+//   frame_stats     one block per frame sums the column partials of the frame
+//                   in a fixed order and forms r_t and delta_t (Eq. 7) from
+//                   <v_t,u_q>, <v_t,v_t>, <v_t,v_{t-1}>, <v_{t-1},v_{t-1}>
+//                   and <u_q,u_q>, reduced in fp64.
 //
 // The relevance pass is HBM bound: it reads T*H*W*D elements once, streamed
 // by TMA bulk copies through a shared-memory ring; each CTA owns one
@@ -101,17 +101,22 @@ constexpr uint64_t kRelTimeoutNs = 2000000000ull;
 // One CTA streams tokens [blockIdx.x*L1, +L1) of the flattened [V*T*N] index.
 // The last warp copies chunks of CH consecutive tokens (contiguous in HBM)
 // into a 3-stage shared-memory ring with cp.async.bulk; the other warps
-// (NC threads, VPT 16-byte vectors each) read them from shared memory.
+// (NC threads, VPT 16-byte vectors each) read them from shared memory.  Each
+// consumer warp waits for a chunk itself and hands it back itself; per-token
+// partial dots and norms go to a shared window that all consumers reduce
+// together once per <= 64 tokens, so block barriers are rare.
 template <typename T, int VPT>
 __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kernel(Ctx c, int CH) {
     constexpr int VEC = VecOf<T>::kElems;
-    constexpr int GROUP = 8;                 // tokens per cross-warp reduction
+    constexpr int GROUP = 8;                 // tokens per warp transpose-reduction
     constexpr int NV = 2 * GROUP;            // GROUP dots + GROUP squared norms
+    constexpr int WIN = 64;                  // tokens per cross-warp reduction
+    constexpr int NWMAX = kRelMaxConsumers / 32;
     extern __shared__ __align__(128) uint8_t rsm[];
-    __shared__ float red[2][kRelMaxConsumers / 32][NV];
-    __shared__ float qsum[kRelMaxConsumers / 32];
+    __shared__ float wpart[2][NWMAX][2][WIN];
+    __shared__ float qsum[NWMAX];
     __shared__ uint64_t full[kRelStages], empty[kRelStages];
-    __shared__ int ok_flag;
+    __shared__ volatile int abort_flag;
     const int NC = blockDim.x - 32;          // consumer threads
     const int nw = NC >> 5;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -124,9 +129,9 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
     if (threadIdx.x == 0) {
         for (int s = 0; s < kRelStages; ++s) {
             ptx::mbar_init(&full[s], 1);
-            ptx::mbar_init(&empty[s], 1);
+            ptx::mbar_init(&empty[s], (uint32_t)nw);
         }
-        ok_flag = 1;
+        abort_flag = 0;
         ptx::fence_barrier_init();
         ptx::fence_proxy_async_smem();
     }
@@ -141,10 +146,11 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
             int s = 0;
             uint32_t ph = 0;
             int issued[kRelStages] = {-1, -1, -1};
-            for (int64_t tok = start; tok < end;) {
+            for (int64_t tok = start; tok < end && !abort_flag;) {
                 const int64_t n = chunk_len(tok, end, c.N, CH);
                 if (!ptx::mbar_wait(&empty[s], ph ^ 1u, kRelTimeoutNs)) {
                     atomicOr(c.status, 16);
+                    abort_flag = 1;
                     break;
                 }
                 ptx::mbar_arrive_expect_tx(&full[s], (uint32_t)(n * rowb));
@@ -165,14 +171,17 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
     // ---------------- consumers ----------------
     auto consumer_sync = [&]() { asm volatile("bar.sync 1, %0;" ::"r"(NC) : "memory"); };
     constexpr int NP = VEC / 2;                  // packed pairs per 16-byte vector
+    constexpr int SHIFT = 1;                     // lane l holds reduced value l >> 1
     int cur_v = -1;
     f2_t q[VPT][NP];
     float qn = 0.f;
     f2_t cs[VPT][NP];
-    int gi = 0;
     int s = 0;
     uint32_t ph = 0;
     int64_t cur_f = -1;
+    bool dead = false;
+    int buf = 0, wcount = 0;
+    int64_t wbase = start;
     for (int64_t tok = start; tok < end;) {
         const int64_t f = tok / c.N;
         const int64_t n = chunk_len(tok, end, c.N, CH);
@@ -206,70 +215,68 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
 #pragma unroll
                 for (int e = 0; e < NP; ++e) cs[vi][e] = 0ull;
         }
-        // wait for the chunk (one bounded waiter decides for all consumers)
-        if (threadIdx.x == 0) ok_flag = ptx::mbar_wait(&full[s], ph, kRelTimeoutNs) ? 1 : 0;
-        consumer_sync();
-        if (!ok_flag) {
-            if (threadIdx.x == 0) atomicOr(c.status, 32);
-            break;
+        // this warp waits for the chunk itself (bounded)
+        int ok = 1;
+        if (lane == 0 && !dead) ok = ptx::mbar_wait(&full[s], ph, kRelTimeoutNs) ? 1 : 0;
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok && !dead) {
+            dead = true;
+            if (lane == 0) {
+                abort_flag = 1;
+                atomicOr(c.status, 32);
+            }
         }
-        ptx::mbar_wait(&full[s], ph, kRelTimeoutNs);   // completed: acquire for this thread
-        const uint32_t st32 = ptx::smem_u32(rsm) + (uint32_t)(s * stage_bytes);
-        const uint32_t rowb32 = (uint32_t)rowb;
         const int nt = (int)n;
-        for (int g0 = 0; g0 < nt; g0 += GROUP, ++gi) {
-            float acc[NV];
-            const bool full_group = nt - g0 >= GROUP;
+        if (!dead) {
+            ptx::mbar_wait(&full[s], ph, kRelTimeoutNs);   // completed: acquire for this thread
+            const uint32_t st32 = ptx::smem_u32(rsm) + (uint32_t)(s * stage_bytes);
+            const uint32_t rowb32 = (uint32_t)rowb;
+            for (int g0 = 0; g0 < nt; g0 += GROUP) {
+                float acc[NV];
+                const bool full_group = nt - g0 >= GROUP;
 #pragma unroll
-            for (int k = 0; k < GROUP; ++k) {
-                f2_t dd = 0ull, nn = 0ull;
-                if (full_group || g0 + k < nt) {
-                    const uint32_t row = st32 + (uint32_t)(g0 + k) * rowb32;
+                for (int k = 0; k < GROUP; ++k) {
+                    f2_t dd = 0ull, nn = 0ull;
+                    if (full_group || g0 + k < nt) {
+                        const uint32_t row = st32 + (uint32_t)(g0 + k) * rowb32;
 #pragma unroll
-                    for (int vi = 0; vi < VPT; ++vi) {
-                        const int vidx = threadIdx.x + vi * NC;
-                        if (vidx < n_vec) {
-                            const uint4 raw = ptx::lds128(row + (uint32_t)vidx * 16u);
-                            f2_t x[NP];
-                            unpack_pairs(raw, x, (T *)nullptr);
+                        for (int vi = 0; vi < VPT; ++vi) {
+                            const int vidx = threadIdx.x + vi * NC;
+                            if (vidx < n_vec) {
+                                const uint4 raw = ptx::lds128(row + (uint32_t)vidx * 16u);
+                                f2_t x[NP];
+                                unpack_pairs(raw, x, (T *)nullptr);
 #pragma unroll
-                            for (int e = 0; e < NP; ++e) {
-                                cs[vi][e] = add2(cs[vi][e], x[e]);
-                                dd = fma2(x[e], q[vi][e], dd);
-                                nn = fma2(x[e], x[e], nn);
+                                for (int e = 0; e < NP; ++e) {
+                                    cs[vi][e] = add2(cs[vi][e], x[e]);
+                                    dd = fma2(x[e], q[vi][e], dd);
+                                    nn = fma2(x[e], x[e], nn);
+                                }
                             }
                         }
                     }
+                    const float2 d2 = unpack2(dd), n2 = unpack2(nn);
+                    acc[k] = d2.x + d2.y;
+                    acc[k + GROUP] = n2.x + n2.y;
                 }
-                const float2 d2 = unpack2(dd), n2 = unpack2(nn);
-                acc[k] = d2.x + d2.y;
-                acc[k + GROUP] = n2.x + n2.y;
-            }
-            const float tot = transpose_reduce<NV>(acc);
-            const int b = gi & 1;
-            if ((lane & 1) == 0) red[b][warp][lane >> 1] = tot;
-            consumer_sync();
-            if (threadIdx.x < 32) {
-                float sm = 0.f;
-                if (lane < NV)
-                    for (int w = 0; w < nw; ++w) sm += red[b][w][lane];
-                const float nrm = __shfl_down_sync(0xffffffffu, sm, GROUP);
-                if (lane < GROUP && g0 + lane < nt) {
-                    const float a = (nrm > 0.f && qn > 0.f) ? sm / (sqrtf(nrm) * qn) : 0.f;
-                    c.a[tok + g0 + lane] = a;
-                }
+                const float tot = transpose_reduce<NV>(acc);
+                const int idx = lane >> SHIFT;              // value held by this lane
+                const int kk = idx & (GROUP - 1);
+                if ((lane & 1) == 0 && g0 + kk < nt)
+                    wpart[buf][warp][idx >> 3][wcount + g0 + kk] = tot;
             }
         }
-        // every consumer has passed its last read of the stage (the group
-        // barrier above), so the stage goes back to the producer
-        if (threadIdx.x == 0) ptx::mbar_arrive(&empty[s]);
+        // hand the stage back once this warp's reads are done
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&empty[s]);
         if (++s == kRelStages) {
             s = 0;
             ph ^= 1u;
         }
         tok += n;
+        wcount += nt;
         const bool frame_done = (tok % c.N == 0) || tok >= end;
-        if (frame_done) {
+        if (frame_done && !dead) {
             // column partial of frame f from this CTA: slot blockIdx.x + f
             float *dst = c.part + ((size_t)blockIdx.x + (size_t)f) * c.D;
 #pragma unroll
@@ -284,15 +291,34 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
                 }
             }
         }
+        // reduce the window across warps: when it is full, at the end of the
+        // range, and before a new video changes u_q
+        const bool new_video = tok < end && (tok / c.N) / c.T != cur_v;
+        if (tok >= end || wcount + CH > WIN || new_video) {
+            consumer_sync();
+            if (abort_flag) break;
+            for (int t = threadIdx.x; t < wcount; t += NC) {
+                float dot = 0.f, nrm = 0.f;
+                for (int w = 0; w < nw; ++w) {
+                    dot += wpart[buf][w][0][t];
+                    nrm += wpart[buf][w][1][t];
+                }
+                c.a[wbase + t] = (nrm > 0.f && qn > 0.f) ? dot / (sqrtf(nrm) * qn) : 0.f;
+            }
+            buf ^= 1;
+            wbase = tok;
+            wcount = 0;
+        }
     }
 }
 
-// Per (2048-channel chunk, frame): fp64 frame sums from the fixed list of CTA
-// partials (8 channels per thread), and their products with u_q, with the
-// previous frame and of u_q with itself.
-__global__ void __launch_bounds__(256) frame_stats_kernel(Ctx c) {
+// One block per frame: the frame sums (fixed list of CTA partials) for all
+// channels, fp32 products summed over each thread's channels, fp64 across
+// threads, then r_t = cos(v_bar_t, u_q) and delta_t = 1 - cos(v_bar_t,
+// v_bar_{t-1}) clamped to [0, 2] (Eq. 7) in fp64.
+__global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     __shared__ double scratch[40];
-    const int64_t f = blockIdx.y;
+    const int64_t f = blockIdx.x;
     const int t = (int)(f % c.T);
     const int v = (int)(f / c.T);
     const int64_t lo = f * c.N / c.L1;
@@ -300,11 +326,8 @@ __global__ void __launch_bounds__(256) frame_stats_kernel(Ctx c) {
     const int64_t g = f - 1;
     const int64_t lo2 = t > 0 ? g * c.N / c.L1 : 0;
     const int64_t hi2 = t > 0 ? min((int64_t)c.G1 - 1, ((g + 1) * c.N - 1) / c.L1) : -1;
-    // fp32 products summed over this thread's 8 channels, fp64 across threads
-    float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f;
-    for (int k = 0; k < kStatsChunk / 256; ++k) {
-        const int d = blockIdx.x * kStatsChunk + k * 256 + threadIdx.x;
-        if (d >= c.D) break;
+    float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f, p4 = 0.f;
+    for (int d = threadIdx.x; d < c.D; d += blockDim.x) {
         float sf = 0.f, sp = 0.f;
         for (int64_t cc = lo; cc <= hi; ++cc) sf += c.part[(size_t)(cc + f) * c.D + d];
         for (int64_t cc = lo2; cc <= hi2; ++cc) sp += c.part[(size_t)(cc + g) * c.D + d];
@@ -314,34 +337,26 @@ __global__ void __launch_bounds__(256) frame_stats_kernel(Ctx c) {
         p1 = fmaf(sf, sf, p1);
         p2 = fmaf(sf, sp, p2);
         p3 = fmaf(q, q, p3);
+        p4 = fmaf(sp, sp, p4);
     }
-    double s0 = p0, s1 = p1, s2 = p2, s3 = p3;
-    s0 = block_sum(s0, scratch);
-    s1 = block_sum(s1, scratch);
-    s2 = block_sum(s2, scratch);
-    s3 = block_sum(s3, scratch);
+    const double vq = block_sum((double)p0, scratch);
+    const double vv = block_sum((double)p1, scratch);
+    const double vp = block_sum((double)p2, scratch);
+    const double qq = block_sum((double)p3, scratch);
+    const double pp = block_sum((double)p4, scratch);
     if (threadIdx.x == 0) {
-        double *o = c.trip + ((size_t)f * c.DC + blockIdx.x) * 4;
-        o[0] = s0;
-        o[1] = s1;
-        o[2] = s2;
-        o[3] = s3;
+        const double qn = sqrt(qq);
+        const double r = (vv > 0.0 && qn > 0.0) ? vq / (sqrt(vv) * qn) : 0.0;
+        double d = 0.0;
+        if (t > 0) {
+            const double den = sqrt(vv * pp);
+            const double cs = den > 0.0 ? vp / den : 0.0;
+            d = fmin(2.0, fmax(0.0, 1.0 - cs));
+        }
+        c.fr[4 * f + 0] = r;
+        c.fr[4 * f + 1] = d;
+        if (c.frame_scores) c.frame_scores[f] = (float)r;
     }
-}
-
-// r_t only (the relevance entry point); the condensation pass does this in
-// the temporal kernel.
-__global__ void relevance_finalize_kernel(Ctx c) {
-    const int64_t f = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (f >= (int64_t)c.V * c.T) return;
-    double dq = 0.0, ff = 0.0, qq = 0.0;
-    for (int k = 0; k < c.DC; ++k) {
-        dq += c.trip[((size_t)f * c.DC + k) * 4 + 0];
-        ff += c.trip[((size_t)f * c.DC + k) * 4 + 1];
-        qq += c.trip[((size_t)f * c.DC + k) * 4 + 3];
-    }
-    const double qn = sqrt(qq);
-    c.frame_scores[f] = (ff > 0.0 && qn > 0.0) ? (float)(dq / (sqrt(ff) * qn)) : 0.f;
 }
 
 cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s) {
@@ -426,13 +441,7 @@ cudaError_t launch_relevance_pass(const Ctx &c, cudaStream_t s) {
 }
 
 cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s) {
-    frame_stats_kernel<<<dim3(c.DC, c.V * c.T), 256, 0, s>>>(c);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_relevance_finalize(const Ctx &c, cudaStream_t s) {
-    const int n = c.V * c.T;
-    relevance_finalize_kernel<<<(n + 255) / 256, 256, 0, s>>>(c);
+    frame_stats_kernel<<<c.V * c.T, 512, 0, s>>>(c);
     return cudaGetLastError();
 }
 

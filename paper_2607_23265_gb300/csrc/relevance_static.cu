@@ -81,7 +81,6 @@ extern "C" int wz_relevance_static(const void *features, int T, int H, int W, in
     c.D = D;
     c.N = H * W;
     c.dtype = dtype;
-    c.DC = (D + kStatsChunk - 1) / kStatsChunk;
     c.G1 = relevance_grid(c);
     if (c.G1 < 1) {
         cudaGetLastError();
@@ -96,14 +95,12 @@ extern "C" int wz_relevance_static(const void *features, int T, int H, int W, in
     o = up256(o + (size_t)D * 4);
     const size_t o_q64 = o;
     o = up256(o + (size_t)D * 8);
-    const size_t o_qn = o;
-    o = up256(o + 8);
     const size_t o_vp = o;
     o = up256(o + sizeof(VideoPar));
     const size_t o_part = o;
     o = up256(o + ((size_t)c.G1 + T) * D * 4);
-    const size_t o_trip = o;
-    o = up256(o + (size_t)T * c.DC * 4 * 8);
+    const size_t o_fr = o;
+    o = up256(o + (size_t)T * 4 * 8);
     if (o > (size_t)WZ_STATIC_SCRATCH_BYTES) return WZ_ERR_WORKSPACE;
 
     void *base = nullptr;
@@ -112,10 +109,9 @@ extern "C" int wz_relevance_static(const void *features, int T, int H, int W, in
     char *b = static_cast<char *>(base);
     c.qbar32 = reinterpret_cast<float *>(b + o_q32);
     c.qbar64 = reinterpret_cast<double *>(b + o_q64);
-    c.qnorm = reinterpret_cast<double *>(b + o_qn);
     c.vpar = reinterpret_cast<VideoPar *>(b + o_vp);
     c.part = reinterpret_cast<float *>(b + o_part);
-    c.trip = reinterpret_cast<double *>(b + o_trip);
+    c.fr = reinterpret_cast<double *>(b + o_fr);
     c.X = features;
     c.Q = query;
     c.a = token_scores;
@@ -125,7 +121,7 @@ extern "C" int wz_relevance_static(const void *features, int T, int H, int W, in
     const VideoPar par{0, Lq, 0, 0, 0};
     const cudaStream_t s = (cudaStream_t)stream;
     if (launch_query_pool(c, &par, s) != cudaSuccess || launch_relevance_pass(c, s) != cudaSuccess ||
-        launch_frame_stats(c, s) != cudaSuccess || launch_relevance_finalize(c, s) != cudaSuccess) {
+        launch_frame_stats(c, s) != cudaSuccess) {
         cudaGetLastError();
         return WZ_ERR_CUDA;
     }

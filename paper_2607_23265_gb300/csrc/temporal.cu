@@ -1,8 +1,7 @@
 // Temporal tail of the condensation pass, one CTA per video, in fp64:
 //
-//   r_t       cos(v_bar_t, u_q)                       Section 3.2.1
-//   delta_t   1 - cos(v_bar_t, v_bar_{t-1}), clamped  Eq. 7
 //   gamma_t   min-max of delta over the video         Section 3.2.2
+//             (r_t and delta_t, Eq. 7, come from frame_stats)
 //   M         {1} u {t : delta_t >= tau}              Section 3.2.2 (frame filter)
 //   r~        Haar DWT of r_M, detail * pair-mean of gamma, inverse DWT   Eq. 8-10
 //   n_m       largest-remainder apportionment of B over max(r~, 0),
@@ -19,7 +18,7 @@
 
 namespace wz {
 
-constexpr int kTemporalThreads = 1024;
+constexpr int kTemporalThreads = 256;
 
 // Exclusive scan of one int per thread over the block; returns the prefix and
 // writes the block total to *total.
@@ -51,7 +50,7 @@ __device__ int block_excl_scan(int x, int *ws, int *total) {
     return r;
 }
 
-// Frames per thread for the scans (T <= 4096 with 1024 threads).
+// Frames per thread for the scans (T <= 4096 with 256 threads).
 constexpr int kPerThread = WZ_MAX_T / kTemporalThreads;
 
 __device__ __forceinline__ int grid_h(int n, int H, int W) {
@@ -76,33 +75,10 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     double *ff = c.tmp + base * 4;         // |v|^2, <v, v_prev>, weight, frac
     int *lst = c.list + 2 * base;          // retained frames, then their budgets
 
-    // ||u_q|| and r_t and the norms (sums of the frame-stats chunks in a fixed order)
-    double qq = 0.0;
-    for (int k = 0; k < c.DC; ++k) qq += c.trip[(size_t)base * c.DC * 4 + 4 * k + 3];
-    const double qn = sqrt(qq);
-    for (int t = threadIdx.x; t < T; t += blockDim.x) {
-        const double *tr = c.trip + (size_t)(base + t) * c.DC * 4;
-        double dq = 0.0, vv = 0.0, vp_ = 0.0;
-        for (int k = 0; k < c.DC; ++k) {
-            dq += tr[4 * k + 0];
-            vv += tr[4 * k + 1];
-            vp_ += tr[4 * k + 2];
-        }
-        fr[4 * t + 0] = (vv > 0.0 && qn > 0.0) ? dq / (sqrt(vv) * qn) : 0.0;
-        ff[4 * t + 0] = vv;
-        ff[4 * t + 1] = vp_;
-    }
-    __syncthreads();
-    // delta_t (Eq. 7) and its range
+    // r_t and delta_t come from frame_stats; the range of delta (Eq. 7)
     double lo = INFINITY, hi = -INFINITY;
     for (int t = threadIdx.x; t < T; t += blockDim.x) {
-        double d = 0.0;
-        if (t > 0) {
-            const double den = sqrt(ff[4 * t] * ff[4 * (t - 1)]);
-            const double cs = den > 0.0 ? ff[4 * t + 1] / den : 0.0;
-            d = fmin(2.0, fmax(0.0, 1.0 - cs));
-        }
-        fr[4 * t + 1] = d;
+        const double d = fr[4 * t + 1];
         lo = fmin(lo, d);
         hi = fmax(hi, d);
     }
@@ -110,7 +86,6 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         lo = fmin(lo, __shfl_xor_sync(0xffffffffu, lo, o));
         hi = fmax(hi, __shfl_xor_sync(0xffffffffu, hi, o));
     }
-    __syncthreads();
     if ((threadIdx.x & 31) == 0) {
         dscr[threadIdx.x >> 5] = lo;
         dscr[32 + (threadIdx.x >> 5)] = hi;
@@ -125,14 +100,16 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     __syncthreads();
     // gamma_t and the retained set (frame 1 always kept)
     const double tau = (double)c.tau;
+    // each thread owns `per` consecutive frames (per <= kPerThread)
+    const int per = (T + (int)blockDim.x - 1) / (int)blockDim.x;
     int keep[kPerThread];
     int cnt = 0;
-    const int t0 = threadIdx.x * kPerThread;
+    const int t0 = threadIdx.x * per;
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
         keep[k] = 0;
-        if (t < T) {
+        if (k < per && t < T) {
             const double d = fr[4 * t + 1];
             fr[4 * t + 2] = hi > lo ? (d - lo) / (hi - lo) : 0.0;
             fr[4 * t + 3] = NAN;
@@ -144,7 +121,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     int pos = block_excl_scan(cnt, iscr, &L);
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k)
-        if (keep[k]) lst[pos++] = t0 + k;
+        if (k < per && keep[k]) lst[pos++] = t0 + k;
     __syncthreads();
 
     // WTA: Haar DWT of r over the retained sequence, detail gated by the
@@ -268,7 +245,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
-        nloc[k] = t < T ? c.n[base + t] : 0;
+        nloc[k] = (k < per && t < T) ? c.n[base + t] : 0;
         sum += nloc[k];
     }
     int produced = 0;
@@ -276,7 +253,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
-        if (t < T) {
+        if (k < per && t < T) {
             c.off[base + t] = vp.row0 + o;
             const int h = grid_h(nloc[k], c.H, c.W);
             c.hw[2 * (base + t)] = h;
@@ -305,7 +282,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
-        if (t < T) c.woff[base + t] = vp.w_row0 + wo;
+        if (k < per && t < T) c.woff[base + t] = vp.w_row0 + wo;
         wo += (nloc[k] + 15) & ~15;
     }
     // tensor-core units: per frame, column blocks of <= 256 tokens; per

@@ -11,7 +11,6 @@ namespace wz {
 
 constexpr int kMaxTaps = 20;          // Daubechies order <= 10
 constexpr int kG1Max = 2048;          // relevance-pass CTAs (upper bound)
-constexpr int kStatsChunk = 2048;     // channels per frame-stats block (8 per thread)
 constexpr int kColBlock = 256;        // output tokens per tensor-core unit
 constexpr int kTileC = 128;           // channels per tensor-core M tile
 
@@ -32,7 +31,6 @@ struct Ctx {
     int hp, wp;           // WSM subband sizes
     int K_pad;            // N rounded up to 32 (row length of the operator)
     int G1;               // relevance CTAs actually launched
-    int DC;               // frame-stats blocks per frame
     int n_ct;             // 128-channel tiles
     int max_units_v;      // unit-list capacity per video
     int F;                // WSM filter taps
@@ -45,12 +43,10 @@ struct Ctx {
 
     float *qbar32;        // [V][D]
     double *qbar64;       // [V][D]
-    double *qnorm;        // [V]
     VideoPar *vpar;       // [V]
     float *a;             // [V*T][N] token saliency
     float *part;          // [G1 + V*T][D] column-sum partials
-    double *trip;         // [V*T][DC][4] (v.q, v.v, v.v_prev, q.q)
-    double *fr;           // [V*T][4] (r, delta, gamma, r~)
+    double *fr;           // [V*T][4] (r, delta, gamma, r~); r, delta from frame_stats
     double *tmp;          // [V*T][4] temporal-kernel scratch
     int *list;            // [V][2T] retained frames and their budgets
     int *n;               // [V*T] budgets
@@ -231,7 +227,6 @@ __host__ __device__ __forceinline__ size_t tile_index(int64_t r, int k, int64_t 
 cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s);
 cudaError_t launch_relevance_pass(const Ctx &c, cudaStream_t s);
 cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s);
-cudaError_t launch_relevance_finalize(const Ctx &c, cudaStream_t s);
 cudaError_t launch_temporal(const Ctx &c, cudaStream_t s);
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s);
 cudaError_t launch_condense_simt(const Ctx &c, cudaStream_t s);
