@@ -14,9 +14,14 @@
 // W_m is fp32 split into bf16 hi + lo (two MMAs into one accumulator), so the
 // product keeps ~16 bits of W while X (exact in bf16) streams once.
 //
-// A unit of work is (frame, <= 256 output tokens, CG <= 4 channel tiles) with
-// CG * N <= 256 accumulator columns; two accumulator buffers let the
-// epilogue of one unit overlap the main loop of the next.  One CTA per SM,
+// A unit of work is (frame, <= 256 output tokens, CG <= 4 channel tiles).
+// The cost of an MMA instruction hardly depends on N, so for N <= 128 the hi
+// and lo operator halves (adjacent in shared memory) form one MMA of N = 2N
+// whose accumulator holds the hi and lo products side by side; for larger N
+// hi and lo are two MMAs into the same accumulator.  Every unit fits one of
+// two 256-column accumulator buffers, so the epilogue of a unit overlaps the
+// main loop of the next.  The epilogue transposes each warp's 32 channels x
+// 32 tokens through shared memory and writes 16-byte rows.  One CTA per SM,
 // persistent over the unit list:
 //   warp 0     TMA producer (one thread), 5-stage shared-memory ring
 //   warp 1     TMEM allocation and the MMA issuer (one thread)
@@ -39,8 +44,8 @@ constexpr int kKC = 32;                    // tokens per K chunk (two K=16 MMA s
 constexpr int kStages = 5;
 constexpr int kStageBytes = 40 * 1024;     // >= CG*8 KB (X) + 2*N*64 B (W hi, lo)
 constexpr int kThreads = 192;
-constexpr int kTmemCols = 512;
-constexpr int kAccCols = 256;
+constexpr int kAccCols = 256;             // one of the two accumulator buffers
+constexpr int kBufs = 2;
 constexpr uint64_t kTimeoutNs = 2000000000ull;
 
 struct TcShared {
@@ -54,7 +59,11 @@ struct TcShared {
     int vprefix[WZ_MAX_VIDEOS + 1];
 };
 
-constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + sizeof(TcShared);
+constexpr int kEpiWarps = 4;
+constexpr int kEpiBytes = 32 * 32 * 2;     // one warp's 32 channels x 32 tokens, bf16
+constexpr size_t kSharedBytes = (sizeof(TcShared) + 127) / 128 * 128;   // epilogue tiles start 128-B aligned
+constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + kSharedBytes + kEpiWarps * kEpiBytes;
+static_assert(kSmemBytes <= 227 * 1024, "shared memory of the condensation CTA");
 
 // Feature tensor maps: a 4D view [frames][D/64][N][64] whose box covers all
 // 2*CG 64-channel blocks of a stage in one copy (one map per CG), and the 3D
@@ -122,7 +131,7 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
         ptx::fence_proxy_async_smem();
     }
     if (warp == 1) {
-        ptx::tmem_alloc(&S->tmem_base, kTmemCols);
+        ptx::tmem_alloc(&S->tmem_base, kAccCols * kBufs);
         ptx::tmem_relinquish();
     }
     if (warp == 0 && lane == 0) {
@@ -193,14 +202,16 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
         for (int u = blockIdx.x; u < n_units && !*abort_flag; u += gridDim.x, ++it) {
             const Unit un = decode_unit(c, S->vprefix, u);
             const int ncp = (un.nc + 15) & ~15;
-            const int b = it & 1;
-            const uint32_t use = (uint32_t)(it >> 1);
+            const bool fused = ncp <= 128;             // hi|lo as one MMA of N = 2*ncp
+            const int tcols = fused ? 2 * ncp : ncp;   // accumulator columns per tile
+            const int b = it % kBufs;
+            const uint32_t use = (uint32_t)(it / kBufs);
             if (!ptx::mbar_wait(&S->tempty[b], (use & 1u) ^ 1u, kTimeoutNs)) {
                 fail(c, abort_flag, 2);
                 break;
             }
             ptx::tc_fence_after();
-            const uint32_t idesc = ptx::idesc_bf16(128, ncp, true, false);
+            const uint32_t idesc = ptx::idesc_bf16(128, fused ? 2 * ncp : ncp, true, false);
             const uint32_t dbase = tmem + (uint32_t)(b * kAccCols);
             bool ok = true;
             for (int kc = 0; kc < KC; ++kc) {
@@ -210,19 +221,23 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
                     break;
                 }
                 ptx::tc_fence_after();
+                // descriptors are built once per stage; the start-address field
+                // is the low 14 bits, so per-MMA operands are constant offsets
                 const uint32_t st = ptx::smem_u32(ring + (size_t)stage * kStageBytes);
                 const uint32_t wh = st + (uint32_t)un.cg * 8192u;
-                const uint32_t wl = wh + (uint32_t)ncp * 64u;
+                const uint64_t a0 = ptx::smem_desc(st, 4096, 1024, 2);
+                const uint64_t bh0 = ptx::smem_desc(wh, 128, 512, 0);       // no swizzle
+                const uint64_t bl0 = bh0 + (uint64_t)((ncp * 64) >> 4);
 #pragma unroll
                 for (int s = 0; s < 2; ++s) {
-                    // no swizzle: core matrices 128 B apart along K, 8-row groups 512 B apart
-                    const uint64_t bh = ptx::smem_desc(wh + s * 256, 128, 512, 0);
-                    const uint64_t bl = ptx::smem_desc(wl + s * 256, 128, 512, 0);
+                    const uint64_t bh = bh0 + (uint64_t)(s * (256 >> 4));
+                    const uint64_t bl = bl0 + (uint64_t)(s * (256 >> 4));
+                    const uint32_t acc = (kc | s) ? 1u : 0u;
                     for (int ct = 0; ct < un.cg; ++ct) {
-                        const uint64_t a = ptx::smem_desc(st + ct * 8192 + s * 2048, 4096, 1024, 2);
-                        const uint32_t d = dbase + (uint32_t)(ct * ncp);
-                        ptx::mma_bf16(d, a, bh, idesc, (kc | s) ? 1u : 0u);
-                        ptx::mma_bf16(d, a, bl, idesc, 1u);
+                        const uint64_t a = a0 + (uint64_t)((ct * 8192 + s * 2048) >> 4);
+                        const uint32_t d = dbase + (uint32_t)(ct * tcols);
+                        ptx::mma_bf16(d, a, bh, idesc, acc);
+                        if (!fused) ptx::mma_bf16(d, a, bl, idesc, 1u);
                     }
                 }
                 ptx::mma_commit(&S->empty[stage]);
@@ -240,31 +255,72 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
     } else if (warp >= 2) {
         // ---------------- epilogue ----------------
         const int q = warp & 3;                          // TMEM lane quadrant of this warp
-        __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(c.out);
+        uint8_t *tr = reinterpret_cast<uint8_t *>(S) + kSharedBytes + (size_t)(warp - 2) * kEpiBytes;
+        const uint32_t tr32 = ptx::smem_u32(tr);
+        char *out = static_cast<char *>(c.out);
+        const size_t rowb = (size_t)c.D * 2;
         int it = 0;
         for (int u = blockIdx.x; u < n_units && !*abort_flag; u += gridDim.x, ++it) {
             const Unit un = decode_unit(c, S->vprefix, u);
             const int ncp = (un.nc + 15) & ~15;
-            const int b = it & 1;
-            const uint32_t use = (uint32_t)(it >> 1);
+            const bool fused = ncp <= 128;
+            const int tcols = fused ? 2 * ncp : ncp;
+            const int b = it % kBufs;
+            const uint32_t use = (uint32_t)(it / kBufs);
             if (!ptx::mbar_wait(&S->tfull[b], use & 1u, kTimeoutNs)) {
                 fail(c, abort_flag, 8);
                 break;
             }
             ptx::tc_fence_after();
             const size_t row0 = (size_t)c.off[un.f] + un.j0;
+            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * kAccCols);
             for (int ct = 0; ct < un.cg; ++ct) {
-                const int ch = (un.ct0 + ct) * kTileC + q * 32 + lane;
-                for (int j0 = 0; j0 < ncp; j0 += 16) {
-                    uint32_t r[16];
-                    ptx::tmem_ld_32x32b_x16(tmem + ((uint32_t)(q * 32) << 16) +
-                                                (uint32_t)(b * kAccCols + ct * ncp + j0), r);
-                    ptx::tmem_ld_wait();
-                    if (ch < c.D) {
+                const int ch0 = (un.ct0 + ct) * kTileC + q * 32;          // this warp's 32 channels
+                for (int j0 = 0; j0 < ncp; j0 += 32) {
+                    // lane = channel ch0 + lane, registers = tokens j0 .. j0+31
+                    uint32_t v[32];
+                    {
+                        uint32_t h0[16], h1[16];
+                        const uint32_t col = (uint32_t)(ct * tcols + j0);
+                        ptx::tmem_ld_32x32b_x16(tbase + col, h0);
+                        if (j0 + 16 < ncp) ptx::tmem_ld_32x32b_x16(tbase + col + 16, h1);
+                        if (fused) {
+                            uint32_t l0[16], l1[16];
+                            ptx::tmem_ld_32x32b_x16(tbase + col + (uint32_t)ncp, l0);
+                            if (j0 + 16 < ncp) ptx::tmem_ld_32x32b_x16(tbase + col + (uint32_t)ncp + 16, l1);
+                            ptx::tmem_ld_wait();
 #pragma unroll
-                        for (int j = 0; j < 16; ++j)
-                            if (j0 + j < un.nc)
-                                out[(row0 + j0 + j) * (size_t)c.D + ch] = __float2bfloat16_rn(__uint_as_float(r[j]));
+                            for (int j = 0; j < 16; ++j) {
+                                v[j] = __float_as_uint(__uint_as_float(h0[j]) + __uint_as_float(l0[j]));
+                                v[16 + j] = (j0 + 16 < ncp) ? __float_as_uint(__uint_as_float(h1[j]) + __uint_as_float(l1[j])) : 0u;
+                            }
+                        } else {
+                            ptx::tmem_ld_wait();
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) {
+                                v[j] = h0[j];
+                                v[16 + j] = (j0 + 16 < ncp) ? h1[j] : 0u;
+                            }
+                        }
+                    }
+                    // transpose: row t of the tile = 32 channels of token j0 + t
+                    __syncwarp();
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const __nv_bfloat16 bv = __float2bfloat16_rn(__uint_as_float(v[j]));
+                        asm volatile("st.shared.b16 [%0], %1;" ::"r"(tr32 + (uint32_t)(j * 64 + lane * 2)),
+                                     "h"(*reinterpret_cast<const unsigned short *>(&bv)));
+                    }
+                    __syncwarp();
+                    // 16-byte pieces: 4 per token row, 8 tokens per warp instruction
+#pragma unroll
+                    for (int r = 0; r < 4; ++r) {
+                        const int t = r * 8 + (lane >> 2);
+                        const int cc = (lane & 3) * 8;
+                        if (j0 + t < un.nc && ch0 + cc < c.D) {
+                            const uint4 val = ptx::lds128(tr32 + (uint32_t)(t * 64 + cc * 2));
+                            *reinterpret_cast<uint4 *>(out + (row0 + j0 + t) * rowb + (size_t)(ch0 + cc) * 2) = val;
+                        }
                     }
                 }
             }
@@ -276,7 +332,7 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
     __syncthreads();
     if (warp == 1) {
         ptx::tc_fence_after();
-        ptx::tmem_dealloc(tmem, kTmemCols);
+        ptx::tmem_dealloc(tmem, kAccCols * kBufs);
     }
 }
 

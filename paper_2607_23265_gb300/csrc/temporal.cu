@@ -286,7 +286,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         wo += (nloc[k] + 15) & ~15;
     }
     // tensor-core units: per frame, column blocks of <= 256 tokens; per
-    // block, groups of CG 128-channel tiles with CG * round16(nc) <= 256.
+    // block, groups of unit_tiles(round16(nc)) 128-channel tiles.
     if (c.path == WZ_PATH_TENSOR) {
         int ucnt[kPerThread];
         int us = 0;
@@ -296,7 +296,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
                 const int nc = min(kColBlock, nloc[k] - j0);
                 const int ncp = (nc + 15) / 16 * 16;
-                const int cg = max(1, min(4, kColBlock / ncp));
+                const int cg = unit_tiles(ncp);
                 ucnt[k] += (c.n_ct + cg - 1) / cg;
             }
             us += ucnt[k];
@@ -310,7 +310,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
                 const int nc = min(kColBlock, nloc[k] - j0);
                 const int ncp = (nc + 15) / 16 * 16;
-                const int cg = max(1, min(4, kColBlock / ncp));
+                const int cg = unit_tiles(ncp);
                 for (int ct = 0; ct < c.n_ct; ct += cg) {
                     const int g = min(cg, c.n_ct - ct);
                     if (u < c.max_units_v) units[u] = make_int4((int)(base + t), j0, ct, nc | (g << 16));

@@ -13,6 +13,7 @@ constexpr int kMaxTaps = 20;          // Daubechies order <= 10
 constexpr int kG1Max = 2048;          // relevance-pass CTAs (upper bound)
 constexpr int kColBlock = 256;        // output tokens per tensor-core unit
 constexpr int kTileC = 128;           // channels per tensor-core M tile
+constexpr int kTmemCols = 512;        // tensor-memory columns of one condensation CTA
 
 // Per-video parameters written to the workspace by the query-pool kernel.
 struct VideoPar {
@@ -220,6 +221,16 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
 __host__ __device__ __forceinline__ size_t tile_index(int64_t r, int k, int64_t w_rows) {
     return ((((size_t)(k >> 5) * (size_t)(w_rows >> 3) + (size_t)(r >> 3)) * 4 + ((k >> 3) & 3)) * 64) +
            (size_t)(r & 7) * 8 + (size_t)(k & 7);
+}
+
+// Channel tiles per tensor-core work unit for a column block of ncp (padded)
+// output tokens.  Up to 128 tokens, hi and lo are one MMA of N = 2*ncp and
+// take 2*ncp accumulator columns per tile; above, they accumulate into the
+// same ncp columns.  Either way a unit fits one 256-column buffer.
+__host__ __device__ __forceinline__ int unit_tiles(int ncp) {
+    const int cols = ncp <= 128 ? 2 * ncp : ncp;
+    const int cg = 256 / cols;
+    return cg < 1 ? 1 : (cg > 4 ? 4 : cg);
 }
 
 // ---- launchers (one per kernel family) -------------------------------------
