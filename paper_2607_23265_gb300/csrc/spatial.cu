@@ -13,12 +13,14 @@
 //   W_m[(p,q),(i,j)] = sum_v sum_b Q_v[q,b] A'_v[b,j] Y_v[b,i],
 //   Y_v[b,i]         = sum_u sum_a P_u[p,a] A_u[a,i] g_uv[a,b].
 //
-// One CTA per (frame, grid row p) builds the w_m rows of W_m for that grid
-// row in fp32 from tables in shared memory (each thread owns one output
-// token q and input column j and sums only over the few b where A'_v[b, j]
-// is nonzero), writes them as bf16 hi/lo pairs
-// (tensor-core path) or fp32 (CUDA-core path), writes the index map rows,
-// and trailing CTAs fill rows that cannot be produced with -1 / zeros.
+// S CTAs per frame: each builds the frame's tables once (saliency map,
+// gate, analysis matrices, width rows Q_v) and then the rows of W_m for the
+// grid rows p = s, s + S, ... in fp32 (each thread owns one output token q
+// and input column j and sums only over the b where both Q_v[q, b] and
+// A'_v[b, j] are nonzero, and only over the rows i that Y_v reaches), stages
+// them in shared memory and writes them as bf16 hi/lo pairs (tensor-core
+// path) or fp32 (CUDA-core path) in 16-byte groups, with the index map rows.
+// Trailing CTAs fill rows that cannot be produced with -1 / zeros.
 #include <cmath>
 
 #include "wz_internal.cuh"
@@ -27,14 +29,17 @@ namespace wz {
 
 constexpr int kSpatialThreads = 256;
 constexpr int kTailBlocks = 64;
+constexpr int kStageFloats = 8 * 1024;   // staged operator rows (32 KB)
 
 struct SpatialSmem {
-    int N, hp, wp, H, W, HP4;
+    int N, hp, wp, H, W, HP4, K_pad, QB;
     // float offsets
-    int M, G, AHl, AHh, AWl, AWh, PAl, PAh, Yl, Yh, Ql, Qh, red, blo, bhi, total;
-    // Every table starts on a 16-byte boundary (float4 reads of Y).
+    int M, G, AHl, AHh, AWl, AWh, PAl, PAh, Yl, Yh, Ql, Qh, red, blo, bhi, qlo, qhi, stage, total;
+    // Every table starts on a 16-byte boundary (float4 reads of Y, staged rows).
     __host__ __device__ void init(int H_, int W_, int hp_, int wp_) {
         H = H_; W = W_; hp = hp_; wp = wp_; N = H * W;
+        K_pad = (N + 31) & ~31;
+        QB = kStageFloats / K_pad;                 // rows staged at a time (>= 2 for N <= 4096)
         HP4 = (H + 3) & ~3;
         int o = 0;
         auto take = [&](int n) {
@@ -57,6 +62,9 @@ struct SpatialSmem {
         red = take(64);
         blo = take(W);
         bhi = take(W);
+        qlo = take(W);
+        qhi = take(W);
+        stage = take(QB * K_pad);
         total = o;
     }
 };
@@ -66,22 +74,37 @@ __device__ __forceinline__ float synth(const float *rec, int F, int y, int a) {
     return (k >= 0 && k < F) ? rec[k] : 0.f;
 }
 
-// Half-pixel bilinear source (align_corners = false): rows y0, y1, weight of y1.
+// Half-pixel bilinear source (align_corners = false): rows y0, y1, weight of
+// y1.  The source coordinate s = (i + 1/2) in / out - 1/2, clamped at 0, is
+// the rational ((2i + 1) in - out) / (2 out): its floor and remainder are
+// exact in integers, and the weight is the remainder divided in fp32.
 __device__ __forceinline__ void bilinear_src(int i, int in, int out, int &y0, int &y1, float &l) {
-    double s = (i + 0.5) * ((double)in / (double)out) - 0.5;
-    if (s < 0.0) s = 0.0;
-    int f = (int)floor(s);
-    if (f > in - 1) f = in - 1;
+    const int num = (2 * i + 1) * in - out, den = 2 * out;
+    int f = 0, rem = 0;
+    if (num > 0) {
+        f = num / den;
+        rem = num - f * den;
+    }
+    if (f > in - 1) {
+        f = in - 1;
+        rem = 0;
+    }
     y0 = f;
     y1 = f + 1 < in ? f + 1 : in - 1;
-    l = (float)(s - f);
+    l = (float)rem / (float)den;
+}
+
+// Coefficients a with synth(y, a) != 0 for y in {y0, y1}: y + F - 2 - 2a in [0, F).
+__device__ __forceinline__ void synth_support(int y0, int y1, int F, int na, int &lo, int &hi) {
+    lo = y0 >> 1;
+    hi = min(na - 1, (y1 + F - 2) >> 1);
 }
 
 template <int HMAX>
-__global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
+__global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) {
     extern __shared__ float sm[];
     const int tid = threadIdx.x;
-    const int64_t nblk_frames = (int64_t)c.V * c.T * c.H;
+    const int64_t nblk_frames = (int64_t)c.V * c.T * S;
     if ((int64_t)blockIdx.x >= nblk_frames) {
         // rows past the produced count: index -1, zero tokens
         const int tb = (int)(blockIdx.x - nblk_frames);
@@ -98,12 +121,12 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
         }
         return;
     }
-    const int64_t f = blockIdx.x / c.H;
-    const int pi = (int)(blockIdx.x % c.H);
+    const int64_t f = blockIdx.x / S;
+    const int s0 = (int)(blockIdx.x % S);
     const int n = c.n[f];
     if (n <= 0) return;
     const int h = c.hw[2 * f], w = c.hw[2 * f + 1];
-    if (pi >= h) return;
+    if (s0 >= h || s0 * w >= n) return;
     const int H = c.H, W = c.W, N = c.N, hp = c.hp, wp = c.wp, F = c.F;
     SpatialSmem L;
     L.init(H, W, hp, wp);
@@ -112,8 +135,12 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
     float *PAl = sm + L.PAl, *PAh = sm + L.PAh, *Yl = sm + L.Yl, *Yh = sm + L.Yh;
     float *Ql = sm + L.Ql, *Qh = sm + L.Qh, *red = sm + L.red;
     int *blo = reinterpret_cast<int *>(sm + L.blo), *bhi = reinterpret_cast<int *>(sm + L.bhi);
+    int *qlo = reinterpret_cast<int *>(sm + L.qlo), *qhi = reinterpret_cast<int *>(sm + L.qhi);
+    int *irange = reinterpret_cast<int *>(red + 48);
+    float *stg = sm + L.stage;
     const int HP4 = L.HP4;
 
+    // ---- per-frame tables ------------------------------------------------
     // saliency map M (Eq. 6): per-frame min-max of a_{t,n}
     const float *a = c.a + f * N;
     float lo = INFINITY, hi = -INFINITY;
@@ -129,7 +156,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
     }
     if ((tid & 31) == 0) {
         red[tid >> 5] = lo;
-        red[32 + (tid >> 5)] = hi;
+        red[16 + (tid >> 5)] = hi;
     }
     // analysis matrices (zero first)
     for (int k = tid; k < hp * H; k += blockDim.x) AHl[k] = AHh[k] = 0.f;
@@ -139,7 +166,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
     hi = -INFINITY;
     for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
         lo = fminf(lo, red[k]);
-        hi = fmaxf(hi, red[32 + k]);
+        hi = fmaxf(hi, red[16 + k]);
     }
     const float rng = hi - lo;
     for (int k = tid; k < N; k += blockDim.x) M[k] = rng > 0.f ? (M[k] - lo) / rng : 0.f;
@@ -162,6 +189,21 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
             }
         }
     }
+    // bilinear columns through the synthesis: Q_v[q][b] and its support
+    for (int k = tid; k < w * wp; k += blockDim.x) {
+        const int q = k / wp, b = k % wp;
+        int x0, x1;
+        float lx;
+        bilinear_src(q, W, w, x0, x1, lx);
+        Ql[k] = (1.f - lx) * synth(c.rec_lo, F, x0, b) + lx * synth(c.rec_lo, F, x1, b);
+        Qh[k] = (1.f - lx) * synth(c.rec_hi, F, x0, b) + lx * synth(c.rec_hi, F, x1, b);
+        if (b == 0) {
+            int l_, h_;
+            synth_support(x0, x1, F, wp, l_, h_);
+            qlo[q] = l_;
+            qhi[q] = h_;
+        }
+    }
     __syncthreads();
     // gate G = lambda * adaptive-average-pool(M) to hp x wp (Eq. 12)
     for (int k = tid; k < hp * wp; k += blockDim.x) {
@@ -172,25 +214,6 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
         for (int y = r0; y < r1; ++y)
             for (int x = c0; x < c1; ++x) s += M[y * W + x];
         G[k] = c.lambda * (s / (float)((r1 - r0) * (c1 - c0)));
-    }
-    // bilinear rows through the synthesis: P_u[a] for this grid row, Q_v[q][b]
-    int y0, y1;
-    float ly;
-    bilinear_src(pi, H, h, y0, y1, ly);
-    for (int k = tid; k < hp * H; k += blockDim.x) {
-        const int ai = k / H;
-        const float pl = (1.f - ly) * synth(c.rec_lo, F, y0, ai) + ly * synth(c.rec_lo, F, y1, ai);
-        const float ph = (1.f - ly) * synth(c.rec_hi, F, y0, ai) + ly * synth(c.rec_hi, F, y1, ai);
-        PAl[k] = pl * AHl[k];
-        PAh[k] = ph * AHh[k];
-    }
-    for (int k = tid; k < w * wp; k += blockDim.x) {
-        const int q = k / wp, b = k % wp;
-        int x0, x1;
-        float lx;
-        bilinear_src(q, W, w, x0, x1, lx);
-        Ql[k] = (1.f - lx) * synth(c.rec_lo, F, x0, b) + lx * synth(c.rec_lo, F, x1, b);
-        Qh[k] = (1.f - lx) * synth(c.rec_hi, F, x0, b) + lx * synth(c.rec_hi, F, x1, b);
     }
     // support of the width analysis: rows b of A' that reach column j
     for (int j = tid; j < W; j += blockDim.x) {
@@ -203,87 +226,145 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c) {
         blo[j] = lo_b;
         bhi[j] = hi_b;
     }
-    __syncthreads();
-    // Y_v[b][i], rows padded to a multiple of 4 with zeros
-    for (int k = tid; k < wp * HP4; k += blockDim.x) {
-        const int b = k / HP4, i = k % HP4;
-        float yl = 0.f, yh = 0.f;
-        if (i < H) {
-            for (int ai = 0; ai < hp; ++ai) {
-                const float g = G[ai * wp + b];
-                const float pl = PAl[ai * H + i], ph = PAh[ai * H + i];
-                yl += pl + ph * g;
-                yh += (pl + ph) * g;
-            }
-        }
-        Yl[k] = yl;
-        Yh[k] = yh;
-    }
-    __syncthreads();
-    // operator rows of this grid row: p = pi*w + q, q < w, p < n
-    const int nq = min(w, n - pi * w);
-    const int64_t row0 = (int64_t)c.off[f] + (int64_t)pi * w;      // output row
+
     const bool bf = c.path == WZ_PATH_TENSOR;
-    const int64_t wrow0 = bf ? (int64_t)c.woff[f] + (int64_t)pi * w : row0;   // operator row
     __nv_bfloat16 *Whi = static_cast<__nv_bfloat16 *>(c.Wop);
     __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * c.K_pad;
     float *W32 = static_cast<float *>(c.Wop);
-    // one thread per (output q, input column j): all H rows i in registers,
-    // summed over the support of column j only
-    for (int item = tid; item < nq * W; item += blockDim.x) {
-        const int q = item / W, j = item % W;
-        float acc[HMAX];
-#pragma unroll
-        for (int i = 0; i < HMAX; ++i) acc[i] = 0.f;
-        for (int b = blo[j]; b <= bhi[j]; ++b) {
-            const float ql = Ql[q * wp + b] * AWl[b * W + j];
-            const float qh = Qh[q * wp + b] * AWh[b * W + j];
-            const float4 *yl = reinterpret_cast<const float4 *>(Yl + b * HP4);
-            const float4 *yh = reinterpret_cast<const float4 *>(Yh + b * HP4);
-#pragma unroll
-            for (int i4 = 0; i4 < HMAX / 4; ++i4) {
-                if (4 * i4 < H) {
-                    const float4 a = yl[i4], d = yh[i4];
-                    acc[4 * i4 + 0] = fmaf(a.x, ql, fmaf(d.x, qh, acc[4 * i4 + 0]));
-                    acc[4 * i4 + 1] = fmaf(a.y, ql, fmaf(d.y, qh, acc[4 * i4 + 1]));
-                    acc[4 * i4 + 2] = fmaf(a.z, ql, fmaf(d.z, qh, acc[4 * i4 + 2]));
-                    acc[4 * i4 + 3] = fmaf(a.w, ql, fmaf(d.w, qh, acc[4 * i4 + 3]));
-                }
-            }
-        }
-        const size_t rbase = (size_t)(row0 + q) * c.K_pad;
-#pragma unroll
-        for (int i = 0; i < HMAX; ++i) {
-            if (i < H) {
-                const float s = acc[i];
-                if (bf) {
-                    const size_t k = tile_index(wrow0 + q, i * W + j, c.w_rows);
-                    const __nv_bfloat16 hb = __float2bfloat16_rn(s);
-                    Whi[k] = hb;
-                    Wlo[k] = __float2bfloat16_rn(s - __bfloat162float(hb));
-                } else {
-                    W32[rbase + (size_t)i * W + j] = s;
-                }
-            }
-        }
-    }
-    // zero the K padding of these rows, and the index map rows
-    const int padw = c.K_pad - N;
-    for (int k = tid; k < nq * padw; k += blockDim.x) {
-        if (bf) {
-            const size_t idx = tile_index(wrow0 + k / padw, N + (k % padw), c.w_rows);
-            Whi[idx] = __float2bfloat16_rn(0.f);
-            Wlo[idx] = __float2bfloat16_rn(0.f);
-        } else {
-            W32[(size_t)(row0 + k / padw) * c.K_pad + N + (k % padw)] = 0.f;
-        }
-    }
+    const int K_pad = c.K_pad, G8 = K_pad / 8;
     const int t = (int)(f % c.T);
-    for (int q = tid; q < nq; q += blockDim.x) {
-        int *o = c.out_index + (size_t)(row0 + q) * 3;
-        o[0] = t;
-        o[1] = pi;
-        o[2] = q;
+
+    // ---- grid rows p = s0, s0 + S, ... ------------------------------------
+    for (int pi = s0; pi < h && pi * w < n; pi += S) {
+        const int nq = min(w, n - pi * w);
+        // bilinear row through the synthesis: P_u[a] is nonzero for a in [alo, ahi]
+        int y0, y1;
+        float ly;
+        bilinear_src(pi, H, h, y0, y1, ly);
+        int alo, ahi;
+        synth_support(y0, y1, F, hp, alo, ahi);
+        const int na = ahi - alo + 1;
+        __syncthreads();   // previous row's Y / stage reads, the frame tables
+        if (tid == 0) {
+            irange[0] = HMAX;
+            irange[1] = -1;
+        }
+        for (int k = tid; k < na * H; k += blockDim.x) {
+            const int ai = alo + k / H, i = k % H;
+            const float pl = (1.f - ly) * synth(c.rec_lo, F, y0, ai) + ly * synth(c.rec_lo, F, y1, ai);
+            const float ph = (1.f - ly) * synth(c.rec_hi, F, y0, ai) + ly * synth(c.rec_hi, F, y1, ai);
+            PAl[k] = pl * AHl[ai * H + i];
+            PAh[k] = ph * AHh[ai * H + i];
+        }
+        __syncthreads();
+        // Y_v[b][i], rows padded to a multiple of 4 with zeros; [ilo, ihi] = rows it reaches
+        int my_lo = HMAX, my_hi = -1;
+        for (int k = tid; k < wp * HP4; k += blockDim.x) {
+            const int b = k / HP4, i = k % HP4;
+            float yl = 0.f, yh = 0.f;
+            if (i < H) {
+                for (int u = 0; u < na; ++u) {
+                    const float g = G[(alo + u) * wp + b];
+                    const float pl = PAl[u * H + i], ph = PAh[u * H + i];
+                    yl += pl + ph * g;
+                    yh += (pl + ph) * g;
+                }
+                if (yl != 0.f || yh != 0.f) {
+                    my_lo = min(my_lo, i);
+                    my_hi = max(my_hi, i);
+                }
+            }
+            Yl[k] = yl;
+            Yh[k] = yh;
+        }
+        for (int o = 16; o > 0; o >>= 1) {
+            my_lo = min(my_lo, __shfl_xor_sync(0xffffffffu, my_lo, o));
+            my_hi = max(my_hi, __shfl_xor_sync(0xffffffffu, my_hi, o));
+        }
+        if ((tid & 31) == 0 && my_hi >= 0) {
+            atomicMin(&irange[0], my_lo);
+            atomicMax(&irange[1], my_hi);
+        }
+        __syncthreads();
+        const int i4lo = irange[0] >> 2, i4hi = irange[1] >> 2;   // empty when ihi < 0
+        const int64_t row0 = (int64_t)c.off[f] + (int64_t)pi * w;                 // output row
+        const int64_t wrow0 = bf ? (int64_t)c.woff[f] + (int64_t)pi * w : row0;   // operator row
+        // Rows are produced QB at a time: one thread per (output q, input
+        // column j) computes all H rows i in registers into a shared staging
+        // row; then the staged rows go out in 8-column groups (16-byte stores
+        // of the hi and lo halves, or of fp32).
+        for (int q0 = 0; q0 < nq; q0 += L.QB) {
+            const int qn = min(L.QB, nq - q0);
+            for (int item = tid; item < qn * W; item += blockDim.x) {
+                const int ql_ = item / W, j = item % W;
+                const int q = q0 + ql_;
+                float acc[HMAX];
+#pragma unroll
+                for (int i = 0; i < HMAX; ++i) acc[i] = 0.f;
+                const int b1 = min(bhi[j], qhi[q]);
+                for (int b = max(blo[j], qlo[q]); b <= b1; ++b) {
+                    const float ql = Ql[q * wp + b] * AWl[b * W + j];
+                    const float qh = Qh[q * wp + b] * AWh[b * W + j];
+                    const float4 *yl = reinterpret_cast<const float4 *>(Yl + b * HP4);
+                    const float4 *yh = reinterpret_cast<const float4 *>(Yh + b * HP4);
+#pragma unroll
+                    for (int i4 = 0; i4 < HMAX / 4; ++i4) {
+                        if (i4 >= i4lo && i4 <= i4hi) {
+                            const float4 a4 = yl[i4], d4 = yh[i4];
+                            acc[4 * i4 + 0] = fmaf(a4.x, ql, fmaf(d4.x, qh, acc[4 * i4 + 0]));
+                            acc[4 * i4 + 1] = fmaf(a4.y, ql, fmaf(d4.y, qh, acc[4 * i4 + 1]));
+                            acc[4 * i4 + 2] = fmaf(a4.z, ql, fmaf(d4.z, qh, acc[4 * i4 + 2]));
+                            acc[4 * i4 + 3] = fmaf(a4.w, ql, fmaf(d4.w, qh, acc[4 * i4 + 3]));
+                        }
+                    }
+                }
+                float *srow = stg + ql_ * K_pad;
+#pragma unroll
+                for (int i = 0; i < HMAX; ++i)
+                    if (i < H) srow[i * W + j] = acc[i];
+            }
+            for (int k = tid; k < qn * (K_pad - N); k += blockDim.x)
+                stg[(k / (K_pad - N)) * K_pad + N + k % (K_pad - N)] = 0.f;
+            __syncthreads();
+            int ql_ = tid / G8, g = tid % G8;
+            const int gstep = (int)blockDim.x % G8, qstep = (int)blockDim.x / G8;
+            for (; ql_ < qn;) {
+                const float4 v0 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g);
+                const float4 v1 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g + 4);
+                if (bf) {
+                    const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+                    uint32_t hw[4], lw[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+                        const __nv_bfloat162 ll =
+                            __floats2bfloat162_rn(v[2 * e] - __low2float(hh), v[2 * e + 1] - __high2float(hh));
+                        hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
+                        lw[e] = *reinterpret_cast<const uint32_t *>(&ll);
+                    }
+                    const size_t ti = tile_index(wrow0 + q0 + ql_, 8 * g, c.w_rows);
+                    *reinterpret_cast<uint4 *>(Whi + ti) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+                    *reinterpret_cast<uint4 *>(Wlo + ti) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+                } else {
+                    float *dst = W32 + (size_t)(row0 + q0 + ql_) * K_pad + 8 * g;
+                    *reinterpret_cast<float4 *>(dst) = v0;
+                    *reinterpret_cast<float4 *>(dst + 4) = v1;
+                }
+                g += gstep;
+                ql_ += qstep;
+                if (g >= G8) {
+                    g -= G8;
+                    ++ql_;
+                }
+            }
+            if (q0 + L.QB < nq) __syncthreads();
+        }
+        for (int q = tid; q < nq; q += blockDim.x) {
+            int *o = c.out_index + (size_t)(row0 + q) * 3;
+            o[0] = t;
+            o[1] = pi;
+            o[2] = q;
+        }
     }
 }
 
@@ -293,12 +374,21 @@ size_t spatial_smem_bytes(const Ctx &c) {
     return (size_t)L.total * sizeof(float);
 }
 
+// CTAs per frame: enough for about two waves over the SMs, at most 8.
+int spatial_split(const Ctx &c, int resident) {
+    const int64_t frames = (int64_t)c.V * c.T;
+    int64_t S = (2 * (int64_t)resident + frames - 1) / frames;
+    if (S < 1) S = 1;
+    if (S > 8) S = 8;
+    if (S > c.H) S = c.H;
+    return (int)S;
+}
+
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     SpatialSmem L;
     L.init(c.H, c.W, c.hp, c.wp);
-    if ((L.Yl & 3) != 0 || (L.Yh & 3) != 0) return cudaErrorMisalignedAddress;
+    if ((L.Yl & 3) != 0 || (L.Yh & 3) != 0 || (L.stage & 3) != 0 || L.QB < 1) return cudaErrorMisalignedAddress;
     const size_t smem = spatial_smem_bytes(c);
-    const unsigned blocks = (unsigned)((int64_t)c.V * c.T * c.H + kTailBlocks);
     const void *fn;
     if (c.H <= 16) fn = (const void *)spatial_kernel<16>;
     else if (c.H <= 32) fn = (const void *)spatial_kernel<32>;
@@ -306,7 +396,14 @@ cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     else return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    void *args[] = {const_cast<Ctx *>(&c)};
+    int dev = 0, sms = 0, per_sm = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kSpatialThreads, smem)) != cudaSuccess)
+        return e;
+    int S = spatial_split(c, sms * (per_sm > 0 ? per_sm : 1));
+    const unsigned blocks = (unsigned)((int64_t)c.V * c.T * S + kTailBlocks);
+    void *args[] = {const_cast<Ctx *>(&c), &S};
     return cudaLaunchKernel(fn, dim3(blocks), dim3(kSpatialThreads), args, smem, s);
 }
 
