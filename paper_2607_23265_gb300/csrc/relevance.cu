@@ -88,10 +88,10 @@ __device__ __forceinline__ float transpose_reduce(float (&v)[NV]) {
     return r;
 }
 
-// Tokens per TMA chunk: never crosses a frame boundary.
-__device__ __forceinline__ int64_t chunk_len(int64_t tok, int64_t end, int N, int CH) {
-    const int64_t f_end = (tok / N + 1) * (int64_t)N;
-    return min((int64_t)CH, min(end, f_end) - tok);
+// Tokens per TMA chunk starting at token `tok`, index `pos` within its
+// frame: never crosses a frame boundary or the end of the range.
+__device__ __forceinline__ int chunk_len(int pos, int64_t tok, int64_t end, int N, int CH) {
+    return (int)min((int64_t)min(CH, N - pos), end - tok);
 }
 
 constexpr int kRelStages = 3;
@@ -146,8 +146,9 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
             int s = 0;
             uint32_t ph = 0;
             int issued[kRelStages] = {-1, -1, -1};
+            int pos = (int)(start % c.N);   // token index within its frame
             for (int64_t tok = start; tok < end && !abort_flag;) {
-                const int64_t n = chunk_len(tok, end, c.N, CH);
+                const int n = chunk_len(pos, tok, end, c.N, CH);
                 if (!ptx::mbar_wait(&empty[s], ph ^ 1u, kRelTimeoutNs)) {
                     atomicOr(c.status, 16);
                     abort_flag = 1;
@@ -157,6 +158,8 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
                 ptx::bulk_load(rsm + s * stage_bytes, X + (size_t)tok * rowb, (uint32_t)(n * rowb), &full[s], pol);
                 issued[s] = (int)ph;
                 tok += n;
+                pos += n;
+                if (pos == c.N) pos = 0;
                 if (++s == kRelStages) {
                     s = 0;
                     ph ^= 1u;
@@ -178,16 +181,19 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
     f2_t cs[VPT][NP];
     int s = 0;
     uint32_t ph = 0;
-    int64_t cur_f = -1;
     bool dead = false;
     int buf = 0, wcount = 0;
     int64_t wbase = start;
+    // frame f, its position t in the video v, and the token index within the
+    // frame are carried along: no 64-bit divisions inside the loop
+    int64_t f = start / c.N;
+    int pos = (int)(start - f * c.N);
+    int tf = (int)(f % c.T), v = (int)(f / c.T);
+    bool frame_new = true;
     for (int64_t tok = start; tok < end;) {
-        const int64_t f = tok / c.N;
-        const int64_t n = chunk_len(tok, end, c.N, CH);
-        if (f != cur_f) {
-            cur_f = f;
-            const int v = (int)(f / c.T);
+        const int n = chunk_len(pos, tok, end, c.N, CH);
+        if (frame_new) {
+            frame_new = false;
             if (v != cur_v) {
                 cur_v = v;
                 float qq = 0.f;
@@ -274,8 +280,9 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
             ph ^= 1u;
         }
         tok += n;
+        pos += n;
         wcount += nt;
-        const bool frame_done = (tok % c.N == 0) || tok >= end;
+        const bool frame_done = pos == c.N || tok >= end;
         if (frame_done && !dead) {
             // column partial of frame f from this CTA: slot blockIdx.x + f
             float *dst = c.part + ((size_t)blockIdx.x + (size_t)f) * c.D;
@@ -291,9 +298,18 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
                 }
             }
         }
+        if (pos == c.N) {
+            pos = 0;
+            ++f;
+            frame_new = true;
+            if (++tf == c.T) {
+                tf = 0;
+                ++v;
+            }
+        }
         // reduce the window across warps: when it is full, at the end of the
         // range, and before a new video changes u_q
-        const bool new_video = tok < end && (tok / c.N) / c.T != cur_v;
+        const bool new_video = tok < end && v != cur_v;
         if (tok >= end || wcount + CH > WIN || new_video) {
             consumer_sync();
             if (abort_flag) break;
