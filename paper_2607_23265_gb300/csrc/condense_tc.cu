@@ -100,6 +100,51 @@ __device__ __forceinline__ void fail(const Ctx &c, volatile int *abort_flag, int
     atomicOr(c.status, code);
 }
 
+// The MMAs of one unit: KC stages of kKC tokens, each two K = 16 steps over
+// CG channel tiles (hi|lo fused into one MMA, or hi and lo as two).  The
+// pattern is fixed at compile time and the stage descriptors are advanced by
+// a constant, so the issuing thread spends a few instructions per MMA.
+template <int CG, bool FUSED>
+__device__ __forceinline__ bool mma_unit(TcShared *S, uint8_t *ring, const Ctx &c, volatile int *abort_flag, int KC,
+                                         int &stage, uint32_t &phase, uint32_t dbase, int tcols, uint32_t idesc,
+                                         int ncp) {
+    const uint32_t ring32 = ptx::smem_u32(ring);
+    // stage 0 descriptors; the 14-bit start-address field of stage s is
+    // (ring + s * kStageBytes) >> 4, reached by adding to the descriptor
+    const uint64_t a_base = ptx::smem_desc(ring32, 4096, 1024, 2);              // X: MN-major, 128-B swizzle
+    const uint64_t b_base = ptx::smem_desc(ring32 + CG * 8192u, 128, 512, 0);  // W: K-major, no swizzle
+    const uint64_t lo_off = (uint64_t)((ncp * 64) >> 4);
+    constexpr uint64_t kStageDesc = (uint64_t)(kStageBytes >> 4);
+    uint32_t d[CG];
+#pragma unroll
+    for (int ct = 0; ct < CG; ++ct) d[ct] = dbase + (uint32_t)(ct * tcols);
+    for (int kc = 0; kc < KC; ++kc) {
+        if (!ptx::mbar_wait(&S->full[stage], phase, kTimeoutNs)) {
+            fail(c, abort_flag, 4);
+            return false;
+        }
+        ptx::tc_fence_after();
+        const uint64_t so = (uint64_t)stage * kStageDesc;
+        const uint64_t a0 = a_base + so, b0 = b_base + so;
+        const uint32_t acc = kc ? 1u : 0u;
+#pragma unroll
+        for (int s = 0; s < 2; ++s) {
+#pragma unroll
+            for (int ct = 0; ct < CG; ++ct) {
+                const uint64_t a = a0 + (uint64_t)((ct * 8192 + s * 2048) >> 4);
+                ptx::mma_bf16(d[ct], a, b0 + (uint64_t)(s * 16), idesc, acc | (uint32_t)s);
+                if (!FUSED) ptx::mma_bf16(d[ct], a, b0 + lo_off + (uint64_t)(s * 16), idesc, 1u);
+            }
+        }
+        ptx::mma_commit(&S->empty[stage]);
+        if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1u;
+        }
+    }
+    return true;
+}
+
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -213,38 +258,19 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
             ptx::tc_fence_after();
             const uint32_t idesc = ptx::idesc_bf16(128, fused ? 2 * ncp : ncp, true, false);
             const uint32_t dbase = tmem + (uint32_t)(b * kAccCols);
-            bool ok = true;
-            for (int kc = 0; kc < KC; ++kc) {
-                if (!ptx::mbar_wait(&S->full[stage], phase, kTimeoutNs)) {
-                    fail(c, abort_flag, 4);
-                    ok = false;
-                    break;
+            bool ok = false;
+            if (fused) {
+                switch (un.cg) {
+                    case 1: ok = mma_unit<1, true>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp); break;
+                    case 2: ok = mma_unit<2, true>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp); break;
+                    case 3: ok = mma_unit<3, true>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp); break;
+                    case 4: ok = mma_unit<4, true>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp); break;
+                    default: fail(c, abort_flag, 4); break;
                 }
-                ptx::tc_fence_after();
-                // descriptors are built once per stage; the start-address field
-                // is the low 14 bits, so per-MMA operands are constant offsets
-                const uint32_t st = ptx::smem_u32(ring + (size_t)stage * kStageBytes);
-                const uint32_t wh = st + (uint32_t)un.cg * 8192u;
-                const uint64_t a0 = ptx::smem_desc(st, 4096, 1024, 2);
-                const uint64_t bh0 = ptx::smem_desc(wh, 128, 512, 0);       // no swizzle
-                const uint64_t bl0 = bh0 + (uint64_t)((ncp * 64) >> 4);
-#pragma unroll
-                for (int s = 0; s < 2; ++s) {
-                    const uint64_t bh = bh0 + (uint64_t)(s * (256 >> 4));
-                    const uint64_t bl = bl0 + (uint64_t)(s * (256 >> 4));
-                    const uint32_t acc = (kc | s) ? 1u : 0u;
-                    for (int ct = 0; ct < un.cg; ++ct) {
-                        const uint64_t a = a0 + (uint64_t)((ct * 8192 + s * 2048) >> 4);
-                        const uint32_t d = dbase + (uint32_t)(ct * tcols);
-                        ptx::mma_bf16(d, a, bh, idesc, acc);
-                        if (!fused) ptx::mma_bf16(d, a, bl, idesc, 1u);
-                    }
-                }
-                ptx::mma_commit(&S->empty[stage]);
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1u;
-                }
+            } else if (un.cg == 1) {
+                ok = mma_unit<1, false>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp);
+            } else {
+                fail(c, abort_flag, 4);
             }
             if (!ok) break;
             ptx::mma_commit(&S->tfull[b]);
