@@ -27,8 +27,8 @@ bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
 // Sub-buffer offsets of one call's workspace.
 struct Layout {
-    size_t qbar32, qbar64, vpar, a, part, fr, tmp, list, n, off, woff, hw, prod,
-        units, ucount, status, Wop, total;
+    size_t qbar32, qbar64, vpar, a, part, fr, list, n, off, woff, hw, prod,
+        units, ucount, ustart, status, Wop, total;
 };
 
 struct Shape {
@@ -51,7 +51,6 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.a = with_a ? take(VT * s.N * 4) : 0;
     L.part = take(((size_t)kG1Max + VT) * s.D * 4);
     L.fr = take(VT * 4 * 8);
-    L.tmp = take(VT * 4 * 8);
     L.list = take(VT * 2 * 4);
     L.n = take(VT * 4);
     L.off = take(VT * 4);
@@ -60,6 +59,7 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.prod = take((size_t)s.V * 4);
     L.units = take((size_t)s.V * s.max_units_v * 16);
     L.ucount = take((size_t)s.V * 4);
+    L.ustart = take(VT * 4);
     L.status = take(16);
     L.Wop = with_operator ? take((size_t)std::max<int64_t>(s.rows_total, s.w_rows) * s.K_pad * 4) : 0;
     L.total = o;
@@ -150,7 +150,6 @@ void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     if (L.a) c.a = reinterpret_cast<float *>(ws + L.a);
     c.part = reinterpret_cast<float *>(ws + L.part);
     c.fr = reinterpret_cast<double *>(ws + L.fr);
-    c.tmp = reinterpret_cast<double *>(ws + L.tmp);
     c.list = reinterpret_cast<int *>(ws + L.list);
     c.n = reinterpret_cast<int *>(ws + L.n);
     c.off = reinterpret_cast<int *>(ws + L.off);
@@ -159,6 +158,7 @@ void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.prod = reinterpret_cast<int *>(ws + L.prod);
     c.units = reinterpret_cast<int4 *>(ws + L.units);
     c.ucount = reinterpret_cast<int *>(ws + L.ucount);
+    c.ustart = reinterpret_cast<int *>(ws + L.ustart);
     c.status = reinterpret_cast<int *>(ws + L.status);
     if (L.Wop) c.Wop = ws + L.Wop;
 }
@@ -247,6 +247,7 @@ int run_condense(const CondenseRequest &r) {
     c.tau = r.m.tau;
     c.mode = r.m.mode;
     c.path = resolve_path(r.m.path, r.dtype);
+    c.pdl = r.events ? 0 : 1;      // an event between two kernels would break the overlap
     set_filters(c, r.m.wsm_wavelet);
     const Shape s = make_shape(r.V, r.T, r.H, r.W, r.D, r.dtype, c.F, B.data());
     const Layout L = make_layout(s, true, true);

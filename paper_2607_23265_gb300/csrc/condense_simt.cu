@@ -9,6 +9,8 @@ namespace wz {
 
 template <typename Tin>
 __global__ void __launch_bounds__(256) condense_simt_kernel(Ctx c) {
+    pdl_wait();
+    pdl_trigger();
     __shared__ float Ws[16][68];
     __shared__ float Xs[16][68];
     const int64_t f = blockIdx.x;
@@ -63,11 +65,10 @@ __global__ void __launch_bounds__(256) condense_simt_kernel(Ctx c) {
 
 cudaError_t launch_condense_simt(const Ctx &c, cudaStream_t s) {
     const dim3 grid((unsigned)((int64_t)c.V * c.T), (unsigned)((c.N + 63) / 64), (unsigned)((c.D + 63) / 64));
-    if (c.dtype == WZ_DTYPE_BF16)
-        condense_simt_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c);
-    else
-        condense_simt_kernel<float><<<grid, 256, 0, s>>>(c);
-    return cudaGetLastError();
+    void *args[] = {const_cast<Ctx *>(&c)};
+    const void *fn = c.dtype == WZ_DTYPE_BF16 ? (const void *)condense_simt_kernel<__nv_bfloat16>
+                                              : (const void *)condense_simt_kernel<float>;
+    return launch_kernel(fn, grid, dim3(256), 0, s, args, c.pdl != 0);
 }
 
 }  // namespace wz

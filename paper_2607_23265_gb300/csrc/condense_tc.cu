@@ -166,12 +166,6 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
         }
         ptx::mbar_init(&S->drain, 1);
         S->abort = 0;
-        int acc = 0;
-        for (int v = 0; v < c.V; ++v) {
-            S->vprefix[v] = acc;
-            acc += c.ucount[v];
-        }
-        S->vprefix[c.V] = acc;
         ptx::fence_barrier_init();
         ptx::fence_proxy_async_smem();
     }
@@ -184,6 +178,17 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
             for (int g = 0; g < 4; ++g) ptx::prefetch_tmap(&maps.x4[g]);
         else
             ptx::prefetch_tmap(&maps.x3);
+    }
+    // global memory from here on: the previous grid has completed
+    pdl_wait();
+    pdl_trigger();
+    if (threadIdx.x == 0) {
+        int acc = 0;
+        for (int v = 0; v < c.V; ++v) {
+            S->vprefix[v] = acc;
+            acc += c.ucount[v];
+        }
+        S->vprefix[c.V] = acc;
     }
     __syncthreads();
     ptx::tc_fence_after();
@@ -420,8 +425,9 @@ cudaError_t launch_condense_tc(const Ctx &c, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(condense_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess) return e;
-    condense_tc_kernel<<<sms, kThreads, kSmemBytes, s>>>(maps, c);
-    return cudaGetLastError();
+    void *args[] = {&maps, const_cast<Ctx *>(&c)};
+    return launch_kernel((const void *)condense_tc_kernel, dim3(sms), dim3(kThreads), kSmemBytes, s, args,
+                         c.pdl != 0);
 }
 
 }  // namespace wz

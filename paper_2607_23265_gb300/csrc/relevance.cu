@@ -31,6 +31,8 @@ struct VideoParBlock {
 template <typename T>
 __global__ void __launch_bounds__(256) query_pool_kernel(Ctx c, VideoParBlock par) {
     __shared__ float ps[8][32], pe[8][32];
+    pdl_wait();
+    pdl_trigger();
     const int v = blockIdx.y;
     const VideoPar vp = par.v[v];
     if (blockIdx.x == 0 && threadIdx.x == 0) c.vpar[v] = vp;
@@ -107,6 +109,8 @@ constexpr uint64_t kRelTimeoutNs = 2000000000ull;
 // together once per <= 64 tokens, so block barriers are rare.
 template <typename T, int VPT>
 __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kernel(Ctx c, int CH) {
+    pdl_wait();
+    pdl_trigger();
     constexpr int VEC = VecOf<T>::kElems;
     constexpr int GROUP = 8;                 // tokens per warp transpose-reduction
     constexpr int NV = 2 * GROUP;            // GROUP dots + GROUP squared norms
@@ -333,6 +337,8 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
 // threads, then r_t = cos(v_bar_t, u_q) and delta_t = 1 - cos(v_bar_t,
 // v_bar_{t-1}) clamped to [0, 2] (Eq. 7) in fp64.
 __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
+    pdl_wait();
+    pdl_trigger();
     __shared__ double scratch[40];
     const int64_t f = blockIdx.x;
     const int t = (int)(f % c.T);
@@ -380,11 +386,10 @@ cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s
     memset(&blk, 0, sizeof(blk));
     for (int v = 0; v < c.V; ++v) blk.v[v] = hpar[v];
     const dim3 grid((unsigned)((c.D + 31) / 32), (unsigned)c.V);
-    if (c.dtype == WZ_DTYPE_BF16)
-        query_pool_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c, blk);
-    else
-        query_pool_kernel<float><<<grid, 256, 0, s>>>(c, blk);
-    return cudaGetLastError();
+    void *args[] = {const_cast<Ctx *>(&c), &blk};
+    const void *fn = c.dtype == WZ_DTYPE_BF16 ? (const void *)query_pool_kernel<__nv_bfloat16>
+                                              : (const void *)query_pool_kernel<float>;
+    return launch_kernel(fn, grid, dim3(256), 0, s, args, c.pdl != 0);
 }
 
 namespace {
@@ -453,12 +458,12 @@ cudaError_t launch_relevance_pass(const Ctx &c, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     int CH = r.CH;
     void *args[] = {const_cast<Ctx *>(&c), &CH};
-    return cudaLaunchKernel(r.fn, dim3(c.G1), dim3(r.threads), args, r.smem, s);
+    return launch_kernel(r.fn, dim3(c.G1), dim3(r.threads), r.smem, s, args, c.pdl != 0);
 }
 
 cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s) {
-    frame_stats_kernel<<<c.V * c.T, 512, 0, s>>>(c);
-    return cudaGetLastError();
+    void *args[] = {const_cast<Ctx *>(&c)};
+    return launch_kernel((const void *)frame_stats_kernel, dim3(c.V * c.T), dim3(512), 0, s, args, c.pdl != 0);
 }
 
 }  // namespace wz

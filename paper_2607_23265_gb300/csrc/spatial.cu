@@ -102,6 +102,8 @@ __device__ __forceinline__ void synth_support(int y0, int y1, int F, int na, int
 
 template <int HMAX>
 __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) {
+    pdl_wait();
+    pdl_trigger();
     extern __shared__ float sm[];
     const int tid = threadIdx.x;
     const int64_t nblk_frames = (int64_t)c.V * c.T * S;
@@ -127,6 +129,25 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     if (n <= 0) return;
     const int h = c.hw[2 * f], w = c.hw[2 * f + 1];
     if (s0 >= h || s0 * w >= n) return;
+    if (s0 == 0 && c.path == WZ_PATH_TENSOR) {
+        // this frame's tensor-core units (the temporal kernel placed them):
+        // column blocks of <= 256 tokens, each in groups of
+        // unit_tiles(round16(nc)) 128-channel tiles
+        const int v = (int)(f / c.T);
+        int4 *units = c.units + (size_t)v * c.max_units_v;
+        int u0 = c.ustart[f];
+        for (int j0 = 0; j0 < n; j0 += kColBlock) {
+            const int nc = min(kColBlock, n - j0);
+            const int cg = unit_tiles((nc + 15) / 16 * 16);
+            const int cnt = (c.n_ct + cg - 1) / cg;
+            for (int li = tid; li < cnt; li += blockDim.x) {
+                const int ct = li * cg;
+                if (u0 + li < c.max_units_v)
+                    units[u0 + li] = make_int4((int)f, j0, ct, nc | (min(cg, c.n_ct - ct) << 16));
+            }
+            u0 += cnt;
+        }
+    }
     const int H = c.H, W = c.W, N = c.N, hp = c.hp, wp = c.wp, F = c.F;
     SpatialSmem L;
     L.init(H, W, hp, wp);
@@ -404,7 +425,7 @@ cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     int S = spatial_split(c, sms * (per_sm > 0 ? per_sm : 1));
     const unsigned blocks = (unsigned)((int64_t)c.V * c.T * S + kTailBlocks);
     void *args[] = {const_cast<Ctx *>(&c), &S};
-    return cudaLaunchKernel(fn, dim3(blocks), dim3(kSpatialThreads), args, smem, s);
+    return launch_kernel(fn, dim3(blocks), dim3(kSpatialThreads), smem, s, args, c.pdl != 0);
 }
 
 }  // namespace wz

@@ -1,4 +1,5 @@
-// Temporal tail of the condensation pass, one CTA per video, in fp64:
+// Temporal tail of the condensation pass, one CTA per video, in fp64, with
+// the per-video arrays in shared memory:
 //
 //   gamma_t   min-max of delta over the video         Section 3.2.2
 //             (r_t and delta_t, Eq. 7, come from frame_stats)
@@ -18,7 +19,7 @@
 
 namespace wz {
 
-constexpr int kTemporalThreads = 256;
+constexpr int kTemporalThreads = 512;
 
 // Exclusive scan of one int per thread over the block; returns the prefix and
 // writes the block total to *total.
@@ -53,50 +54,63 @@ __device__ int block_excl_scan(int x, int *ws, int *total) {
 // Frames per thread for the scans (T <= 4096 with 256 threads).
 constexpr int kPerThread = WZ_MAX_T / kTemporalThreads;
 
+// h = min(H, ceil(sqrt(n H / W))): a float estimate corrected to the exact
+// smallest h >= 1 with h^2 W >= n H in integers.
 __device__ __forceinline__ int grid_h(int n, int H, int W) {
     if (n <= 0) return 0;
-    long long h = (long long)ceil(sqrt((double)n * H / W));
+    long long h = (long long)ceilf(sqrtf((float)n * (float)H / (float)W));
     if (h < 1) h = 1;
     while (h * h * W < (long long)n * H) ++h;
     while (h > 1 && (h - 1) * (h - 1) * W >= (long long)n * H) --h;
     return (int)(h < H ? h : H);
 }
 
+// Shared-memory arrays of one video, indexed by retained frame m (wgt,
+// keys, lst, nb) or by frame t (nf).
+__host__ __device__ inline size_t temporal_smem_bytes(int T) { return (size_t)T * (8 + 8 + 4 + 4 + 4); }
+
+// Threads of the CTA: one frame per thread up to 512 frames, at most
+// kPerThread frames per thread beyond (fp64 work scales with the warps).
+inline int temporal_threads(int T) { return T <= 512 ? (T < 32 ? 32 : (T + 31) / 32 * 32) : 512; }
+
 __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
+    pdl_wait();
+    pdl_trigger();
+    extern __shared__ __align__(16) unsigned char tsm[];
     __shared__ double dscr[64];
     __shared__ long long lscr[40];
     __shared__ int iscr[72];
-    __shared__ unsigned long long keys[WZ_MAX_T];
     const int v = blockIdx.x;
     const int T = c.T;
     const int64_t base = (int64_t)v * T;
     const VideoPar vp = c.vpar[v];
     double *fr = c.fr + base * 4;          // r, delta, gamma, r~
-    double *ff = c.tmp + base * 4;         // |v|^2, <v, v_prev>, weight, frac
-    int *lst = c.list + 2 * base;          // retained frames, then their budgets
+    double *wgt = reinterpret_cast<double *>(tsm);                        // weight of retained frame m
+    unsigned long long *keys = reinterpret_cast<unsigned long long *>(wgt + T);   // quota / remainder key
+    int *lst = reinterpret_cast<int *>(keys + T);                         // retained frames
+    int *nb = lst + T;                     // budget of retained frame m; -1 while active
+    int *nf = nb + T;                      // budget of frame t
 
-    // r_t and delta_t come from frame_stats; the range of delta (Eq. 7)
-    double lo = INFINITY, hi = -INFINITY;
-    for (int t = threadIdx.x; t < T; t += blockDim.x) {
-        const double d = fr[4 * t + 1];
-        lo = fmin(lo, d);
-        hi = fmax(hi, d);
-    }
-    for (int o = 16; o > 0; o >>= 1) {
-        lo = fmin(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-        hi = fmax(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-    }
-    if ((threadIdx.x & 31) == 0) {
-        dscr[threadIdx.x >> 5] = lo;
-        dscr[32 + (threadIdx.x >> 5)] = hi;
+    // r_t and delta_t come from frame_stats; the range of delta (Eq. 7),
+    // reduced by one warp (fp64 throughput is low: keep it to few warps)
+    if (threadIdx.x < 32) {
+        double lo = INFINITY, hi = -INFINITY;
+        for (int t = threadIdx.x; t < T; t += 32) {
+            const double d = fr[4 * t + 1];
+            lo = fmin(lo, d);
+            hi = fmax(hi, d);
+        }
+        for (int o = 16; o > 0; o >>= 1) {
+            lo = fmin(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+            hi = fmax(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+        }
+        if (threadIdx.x == 0) {
+            dscr[0] = lo;
+            dscr[1] = hi;
+        }
     }
     __syncthreads();
-    lo = INFINITY;
-    hi = -INFINITY;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
-        lo = fmin(lo, dscr[w]);
-        hi = fmax(hi, dscr[32 + w]);
-    }
+    const double lo = dscr[0], hi = dscr[1];
     __syncthreads();
     // gamma_t and the retained set (frame 1 always kept)
     const double tau = (double)c.tau;
@@ -115,6 +129,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             fr[4 * t + 3] = NAN;
             keep[k] = (t == 0 || d >= tau) ? 1 : 0;
             cnt += keep[k];
+            nf[t] = 0;
         }
     }
     int L = 0;
@@ -126,8 +141,10 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
 
     // WTA: Haar DWT of r over the retained sequence, detail gated by the
     // pair mean of gamma, inverse DWT (Eq. 8-10).  Odd L: the last sample
-    // pairs with its mirror image, so its detail is 0.
+    // pairs with its mirror image, so its detail is 0.  Budget weights are
+    // max(r~, 0) (Eq. 5).
     const double s2 = 0.70710678118654752440;
+    int anypos = 0;
     for (int k = threadIdx.x; 2 * k < L; k += blockDim.x) {
         const int i0 = 2 * k, i1 = min(2 * k + 1, L - 1);
         const int a0 = lst[i0], a1 = lst[i1];
@@ -136,27 +153,30 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         const double Dd = s2 * r0 - s2 * r1;
         const double g = 0.5 * (fr[4 * a0 + 2] + fr[4 * a1 + 2]);
         const double Dt = g * Dd;
-        fr[4 * a0 + 3] = s2 * A + s2 * Dt;
-        if (i1 != i0) fr[4 * a1 + 3] = s2 * A - s2 * Dt;
+        const double rt0 = s2 * A + s2 * Dt;
+        fr[4 * a0 + 3] = rt0;
+        wgt[i0] = fmax(rt0, 0.0);
+        anypos |= (rt0 > 0.0);
+        if (i1 != i0) {
+            const double rt1 = s2 * A - s2 * Dt;
+            fr[4 * a1 + 3] = rt1;
+            wgt[i1] = fmax(rt1, 0.0);
+            anypos |= (rt1 > 0.0);
+        }
+    }
+    // uniform weights if none is positive
+    anypos = __syncthreads_or(anypos);
+    for (int m = threadIdx.x; m < L; m += blockDim.x) {
+        nb[m] = -1;
+        if (!anypos) wgt[m] = 1.0;
     }
     __syncthreads();
 
-    // Budgets (Eq. 5, Eq. 15): weights max(r~, 0); uniform if none positive.
+    // Budgets (Eq. 5, Eq. 15): largest-remainder apportionment of B over the
+    // weights, frames whose quota exceeds N capped at N and the rest
+    // re-apportioned.
     const int N = c.N;
     const int B = vp.B;
-    int anypos = 0;
-    for (int m = threadIdx.x; m < L; m += blockDim.x) {
-        const double w = fmax(fr[4 * lst[m] + 3], 0.0);
-        ff[4 * lst[m] + 2] = w;
-        anypos |= (w > 0.0);
-    }
-    anypos = __syncthreads_or(anypos);
-    int *nb = lst + T;                     // budget of retained frame m; -1 while active
-    for (int m = threadIdx.x; m < L; m += blockDim.x) {
-        nb[m] = -1;                        // -1: still active
-        if (!anypos) ff[4 * lst[m] + 2] = 1.0;
-    }
-    __syncthreads();
     if ((long long)L * N <= (long long)B) {
         for (int m = threadIdx.x; m < L; m += blockDim.x) nb[m] = N;
     } else {
@@ -166,8 +186,8 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             double sp = 0.0;
             int npos = 0;
             for (int m = threadIdx.x; m < L; m += blockDim.x)
-                if (nb[m] < 0 && ff[4 * lst[m] + 2] > 0.0) {
-                    sp += ff[4 * lst[m] + 2];
+                if (nb[m] < 0 && wgt[m] > 0.0) {
+                    sp += wgt[m];
                     npos = 1;
                 }
             npos = __syncthreads_or(npos);
@@ -180,22 +200,22 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             } else {
                 S = block_sum(sp, dscr);
             }
+            // quota q_m = remaining * w_m / S of every candidate
             int ncap = 0;
             for (int m = threadIdx.x; m < L; m += blockDim.x) {
-                if (nb[m] >= 0) continue;
-                const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
-                if (!uniform && !(w > 0.0)) continue;
-                const double q = (double)remaining * w / S;
-                if (q > (double)N) ncap += 1;
+                const double w = uniform ? 1.0 : wgt[m];
+                const bool cand = nb[m] < 0 && (uniform || w > 0.0);
+                double q = -1.0;
+                if (cand) {
+                    q = (double)remaining * w / S;
+                    ncap += (q > (double)N);
+                }
+                keys[m] = (unsigned long long)__double_as_longlong(q);
             }
             ncap = (int)block_sum_ll(ncap, lscr);
             if (ncap > 0) {
-                for (int m = threadIdx.x; m < L; m += blockDim.x) {
-                    if (nb[m] >= 0) continue;
-                    const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
-                    if (!uniform && !(w > 0.0)) continue;
-                    if ((double)remaining * w / S > (double)N) nb[m] = N;
-                }
+                for (int m = threadIdx.x; m < L; m += blockDim.x)
+                    if (__longlong_as_double((long long)keys[m]) > (double)N) nb[m] = N;
                 remaining -= (long long)N * ncap;
                 __syncthreads();
                 continue;
@@ -204,14 +224,13 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             // parts (non-negative doubles order like their bit patterns)
             long long fsum = 0;
             for (int m = threadIdx.x; m < L; m += blockDim.x) {
-                const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
-                const bool cand = nb[m] < 0 && (uniform || w > 0.0);
+                const double q = __longlong_as_double((long long)keys[m]);
                 unsigned long long key = ~0ull;
-                if (cand) {
-                    const double q = (double)remaining * w / S;
+                if (q >= 0.0) {
                     const double fl = floor(q);
                     key = (unsigned long long)__double_as_longlong(q - fl);
                     fsum += (long long)fl;
+                    nb[m] = (int)fl;       // floor; the remainder unit is added below
                 }
                 keys[m] = key;
             }
@@ -224,9 +243,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
                     const unsigned long long kk = keys[k];
                     rank += (kk != ~0ull && (kk > km || (kk == km && k < m))) ? 1 : 0;
                 }
-                const double w = uniform ? 1.0 : ff[4 * lst[m] + 2];
-                const long long fl = (long long)floor((double)remaining * w / S);
-                nb[m] = (int)(fl + (rank < R ? 1 : 0));
+                if (rank < R) nb[m] += 1;
             }
             __syncthreads();
             break;
@@ -236,16 +253,14 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     }
     __syncthreads();
     // scatter to frames, offsets, grids
-    for (int t = threadIdx.x; t < T; t += blockDim.x) c.n[base + t] = 0;
-    __syncthreads();
-    for (int m = threadIdx.x; m < L; m += blockDim.x) c.n[base + lst[m]] = nb[m];
+    for (int m = threadIdx.x; m < L; m += blockDim.x) nf[lst[m]] = nb[m];
     __syncthreads();
     int nloc[kPerThread];
     int sum = 0;
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
-        nloc[k] = (k < per && t < T) ? c.n[base + t] : 0;
+        nloc[k] = (k < per && t < T) ? nf[t] : 0;
         sum += nloc[k];
     }
     int produced = 0;
@@ -254,6 +269,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
         if (k < per && t < T) {
+            c.n[base + t] = nloc[k];
             c.off[base + t] = vp.row0 + o;
             const int h = grid_h(nloc[k], c.H, c.W);
             c.hw[2 * (base + t)] = h;
@@ -286,7 +302,9 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         wo += (nloc[k] + 15) & ~15;
     }
     // tensor-core units: per frame, column blocks of <= 256 tokens; per
-    // block, groups of unit_tiles(round16(nc)) 128-channel tiles.
+    // block, groups of unit_tiles(round16(nc)) 128-channel tiles.  Here the
+    // count and the first unit of each frame; the spatial kernel writes the
+    // records.
     if (c.path == WZ_PATH_TENSOR) {
         int ucnt[kPerThread];
         int us = 0;
@@ -303,20 +321,11 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         }
         int total = 0;
         int u = block_excl_scan(us, iscr, &total);
-        int4 *units = c.units + (size_t)v * c.max_units_v;
 #pragma unroll
         for (int k = 0; k < kPerThread; ++k) {
             const int t = t0 + k;
-            for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
-                const int nc = min(kColBlock, nloc[k] - j0);
-                const int ncp = (nc + 15) / 16 * 16;
-                const int cg = unit_tiles(ncp);
-                for (int ct = 0; ct < c.n_ct; ct += cg) {
-                    const int g = min(cg, c.n_ct - ct);
-                    if (u < c.max_units_v) units[u] = make_int4((int)(base + t), j0, ct, nc | (g << 16));
-                    ++u;
-                }
-            }
+            if (k < per && t < T) c.ustart[base + t] = u;
+            u += ucnt[k];
         }
         if (threadIdx.x == 0) {
             c.ucount[v] = min(total, c.max_units_v);
@@ -326,8 +335,12 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
 }
 
 cudaError_t launch_temporal(const Ctx &c, cudaStream_t s) {
-    temporal_kernel<<<c.V, kTemporalThreads, 0, s>>>(c);
-    return cudaGetLastError();
+    const size_t smem = temporal_smem_bytes(c.T);
+    cudaError_t e = cudaFuncSetAttribute(temporal_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    void *args[] = {const_cast<Ctx *>(&c)};
+    return launch_kernel((const void *)temporal_kernel, dim3(c.V), dim3(temporal_threads(c.T)), smem, s, args,
+                         c.pdl != 0);
 }
 
 }  // namespace wz

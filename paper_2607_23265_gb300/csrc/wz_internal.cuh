@@ -48,7 +48,6 @@ struct Ctx {
     float *a;             // [V*T][N] token saliency
     float *part;          // [G1 + V*T][D] column-sum partials
     double *fr;           // [V*T][4] (r, delta, gamma, r~); r, delta from frame_stats
-    double *tmp;          // [V*T][4] temporal-kernel scratch
     int *list;            // [V][2T] retained frames and their budgets
     int *n;               // [V*T] budgets
     int *off;             // [V*T] global output row of the frame's first token
@@ -57,6 +56,7 @@ struct Ctx {
     int *prod;            // [V] produced rows
     int4 *units;          // [V][max_units_v] tensor-core work units
     int *ucount;          // [V]
+    int *ustart;          // [V*T] first unit of each frame in its video's list
     void *Wop;            // operator: tensor path bf16 hi then lo in the tiled
                           // layout of tile_index(), CUDA-core path f32 [rows][K_pad]
     int *status;          // device status word (bounded waits)
@@ -72,10 +72,34 @@ struct Ctx {
     float lambda, tau;
     int mode;             // WZ_MODE_*
     int path;             // resolved WZ_PATH_TENSOR or WZ_PATH_SIMT
+    int pdl;              // host: launch with programmatic stream serialization
     float dec_lo[kMaxTaps], dec_hi[kMaxTaps], rec_lo[kMaxTaps], rec_hi[kMaxTaps];
 };
 
 // ---- device helpers -------------------------------------------------------
+
+// ---- programmatic dependent launch ---------------------------------------
+// Each kernel of the pass waits for the grid before it in the stream before it
+// touches global memory and then lets the next grid be scheduled, so launch
+// latency and prologues overlap the previous kernel's tail.  Launched without
+// the attribute, both instructions return at once.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+inline cudaError_t launch_kernel(const void *fn, dim3 grid, dim3 block, size_t smem, cudaStream_t s, void **args,
+                                 bool pdl) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelExC(&cfg, fn, args);
+}
 
 __device__ __forceinline__ int ext_index(int i, int n, int mode) {
     if (i >= 0 && i < n) return i;
