@@ -50,8 +50,8 @@ def build(verbose: bool = False, force: bool = False) -> str:
     """Compile every .cu under csrc/ and link libwavezip.so; returns its path."""
     os.makedirs(BUILD, exist_ok=True)
     srcs = sources()
-    newest = max(os.path.getmtime(p) for p in srcs + [os.path.join(CSRC, "wz_internal.cuh"),
-                                                        os.path.join(HERE, "..", "include", "wavezip.h")])
+    headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cuh")]
+    newest = max(os.path.getmtime(p) for p in srcs + headers + [os.path.join(HERE, "..", "include", "wavezip.h")])
     if not force and os.path.exists(LIB) and os.path.getmtime(LIB) > newest:
         return LIB
     with cf.ThreadPoolExecutor(max_workers=min(len(srcs), os.cpu_count() or 4)) as pool:

@@ -10,7 +10,7 @@
 #include <cstring>
 #include <vector>
 
-#include "wz_internal.cuh"
+#include "wz_spatial.cuh"
 
 namespace wz {
 
@@ -28,7 +28,7 @@ bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 // Sub-buffer offsets of one call's workspace.
 struct Layout {
     size_t qbar32, qbar64, vpar, a, part, fr, list, n, off, woff, hw, prod,
-        units, ucount, ustart, status, Wop, total;
+        units, ucount, ustart, stab, status, Wop, total;
 };
 
 struct Shape {
@@ -60,6 +60,7 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.units = take((size_t)s.V * s.max_units_v * 16);
     L.ucount = take((size_t)s.V * 4);
     L.ustart = take(VT * 4);
+    L.stab = take(spatial_table_bytes(s.H, s.W, kMaxTaps));   // any wavelet
     L.status = take(16);
     L.Wop = with_operator ? take((size_t)std::max<int64_t>(s.rows_total, s.w_rows) * s.K_pad * 4) : 0;
     L.total = o;
@@ -159,6 +160,7 @@ void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.units = reinterpret_cast<int4 *>(ws + L.units);
     c.ucount = reinterpret_cast<int *>(ws + L.ucount);
     c.ustart = reinterpret_cast<int *>(ws + L.ustart);
+    c.stab = reinterpret_cast<float *>(ws + L.stab);
     c.status = reinterpret_cast<int *>(ws + L.status);
     if (L.Wop) c.Wop = ws + L.Wop;
 }

@@ -23,52 +23,12 @@
 // Trailing CTAs fill rows that cannot be produced with -1 / zeros.
 #include <cmath>
 
-#include "wz_internal.cuh"
+#include "wz_spatial.cuh"
 
 namespace wz {
 
 constexpr int kSpatialThreads = 256;
 constexpr int kTailBlocks = 64;
-constexpr int kStageFloats = 8 * 1024;   // staged operator rows (32 KB)
-
-struct SpatialSmem {
-    int N, hp, wp, H, W, HP4, K_pad, QB;
-    // float offsets
-    int M, G, AHl, AHh, AWl, AWh, PAl, PAh, Yl, Yh, Ql, Qh, red, blo, bhi, qlo, qhi, stage, total;
-    // Every table starts on a 16-byte boundary (float4 reads of Y, staged rows).
-    __host__ __device__ void init(int H_, int W_, int hp_, int wp_) {
-        H = H_; W = W_; hp = hp_; wp = wp_; N = H * W;
-        K_pad = (N + 31) & ~31;
-        QB = kStageFloats / K_pad;                 // rows staged at a time (>= 2 for N <= 4096)
-        HP4 = (H + 3) & ~3;
-        int o = 0;
-        auto take = [&](int n) {
-            const int at = o;
-            o = (o + n + 3) & ~3;
-            return at;
-        };
-        M = take(N);
-        G = take(hp * wp);
-        AHl = take(hp * H);
-        AHh = take(hp * H);
-        AWl = take(wp * W);
-        AWh = take(wp * W);
-        PAl = take(hp * H);
-        PAh = take(hp * H);
-        Yl = take(wp * HP4);
-        Yh = take(wp * HP4);
-        Ql = take(W * wp);
-        Qh = take(W * wp);
-        red = take(64);
-        blo = take(W);
-        bhi = take(W);
-        qlo = take(W);
-        qhi = take(W);
-        stage = take(QB * K_pad);
-        total = o;
-    }
-};
-
 __device__ __forceinline__ float synth(const float *rec, int F, int y, int a) {
     const int k = y + F - 2 - 2 * a;
     return (k >= 0 && k < F) ? rec[k] : 0.f;
@@ -162,6 +122,9 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     const int HP4 = L.HP4;
 
     // ---- per-frame tables ------------------------------------------------
+    // the frame-independent tables (analysis matrices, supports, pooling
+    // windows), built once per pass
+    for (int k = tid; k < L.tables; k += blockDim.x) reinterpret_cast<int *>(sm)[k] = reinterpret_cast<const int *>(c.stab)[k];
     // saliency map M (Eq. 6): per-frame min-max of a_{t,n}
     const float *a = c.a + f * N;
     float lo = INFINITY, hi = -INFINITY;
@@ -179,37 +142,6 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
         red[tid >> 5] = lo;
         red[16 + (tid >> 5)] = hi;
     }
-    // analysis matrices (zero first)
-    for (int k = tid; k < hp * H; k += blockDim.x) AHl[k] = AHh[k] = 0.f;
-    for (int k = tid; k < wp * W; k += blockDim.x) AWl[k] = AWh[k] = 0.f;
-    __syncthreads();
-    lo = INFINITY;
-    hi = -INFINITY;
-    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
-        lo = fminf(lo, red[k]);
-        hi = fmaxf(hi, red[16 + k]);
-    }
-    const float rng = hi - lo;
-    for (int k = tid; k < N; k += blockDim.x) M[k] = rng > 0.f ? (M[k] - lo) / rng : 0.f;
-    // A[a][i] = sum_j dec[j] [ext(2a+1-j) == i]; one thread per row a
-    if (tid < hp) {
-        for (int j = 0; j < F; ++j) {
-            const int i = ext_index(2 * tid + 1 - j, H, c.mode);
-            if (i >= 0) {
-                AHl[tid * H + i] += c.dec_lo[j];
-                AHh[tid * H + i] += c.dec_hi[j];
-            }
-        }
-    } else if (tid >= 128 && tid < 128 + wp) {
-        const int b = tid - 128;
-        for (int j = 0; j < F; ++j) {
-            const int i = ext_index(2 * b + 1 - j, W, c.mode);
-            if (i >= 0) {
-                AWl[b * W + i] += c.dec_lo[j];
-                AWh[b * W + i] += c.dec_hi[j];
-            }
-        }
-    }
     // bilinear columns through the synthesis: Q_v[q][b] and its support
     for (int k = tid; k < w * wp; k += blockDim.x) {
         const int q = k / wp, b = k % wp;
@@ -226,26 +158,25 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
         }
     }
     __syncthreads();
+    lo = INFINITY;
+    hi = -INFINITY;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
+        lo = fminf(lo, red[k]);
+        hi = fmaxf(hi, red[16 + k]);
+    }
+    const float rng = hi - lo;
+    for (int k = tid; k < N; k += blockDim.x) M[k] = rng > 0.f ? (M[k] - lo) / rng : 0.f;
+    __syncthreads();
     // gate G = lambda * adaptive-average-pool(M) to hp x wp (Eq. 12)
+    const int *pr0 = reinterpret_cast<const int *>(sm + L.pr0), *pr1 = reinterpret_cast<const int *>(sm + L.pr1);
+    const int *pc0 = reinterpret_cast<const int *>(sm + L.pc0), *pc1 = reinterpret_cast<const int *>(sm + L.pc1);
     for (int k = tid; k < hp * wp; k += blockDim.x) {
         const int ai = k / wp, bj = k % wp;
-        const int r0 = (ai * H) / hp, r1 = ((ai + 1) * H + hp - 1) / hp;
-        const int c0 = (bj * W) / wp, c1 = ((bj + 1) * W + wp - 1) / wp;
+        const int r0 = pr0[ai], r1 = pr1[ai], c0 = pc0[bj], c1 = pc1[bj];
         float s = 0.f;
         for (int y = r0; y < r1; ++y)
             for (int x = c0; x < c1; ++x) s += M[y * W + x];
         G[k] = c.lambda * (s / (float)((r1 - r0) * (c1 - c0)));
-    }
-    // support of the width analysis: rows b of A' that reach column j
-    for (int j = tid; j < W; j += blockDim.x) {
-        int lo_b = wp, hi_b = -1;
-        for (int b = 0; b < wp; ++b)
-            if (AWl[b * W + j] != 0.f || AWh[b * W + j] != 0.f) {
-                lo_b = min(lo_b, b);
-                hi_b = max(hi_b, b);
-            }
-        blo[j] = lo_b;
-        bhi[j] = hi_b;
     }
 
     const bool bf = c.path == WZ_PATH_TENSOR;
@@ -395,12 +326,11 @@ size_t spatial_smem_bytes(const Ctx &c) {
     return (size_t)L.total * sizeof(float);
 }
 
-// CTAs per frame: enough for about two waves over the SMs, at most 8.
+// CTAs per frame: about four waves over the SMs, at most one per grid row.
 int spatial_split(const Ctx &c, int resident) {
     const int64_t frames = (int64_t)c.V * c.T;
-    int64_t S = (2 * (int64_t)resident + frames - 1) / frames;
+    int64_t S = (4 * (int64_t)resident + frames - 1) / frames;
     if (S < 1) S = 1;
-    if (S > 8) S = 8;
     if (S > c.H) S = c.H;
     return (int)S;
 }

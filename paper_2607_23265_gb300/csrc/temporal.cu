@@ -15,7 +15,7 @@
 // do not depend on scheduling.
 #include <cmath>
 
-#include "wz_internal.cuh"
+#include "wz_spatial.cuh"
 
 namespace wz {
 
@@ -76,6 +76,11 @@ inline int temporal_threads(int T) { return T <= 512 ? (T < 32 ? 32 : (T + 31) /
 __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     pdl_wait();
     pdl_trigger();
+    if ((int)blockIdx.x == c.V) {
+        // the extra CTA: frame-independent tables of the spatial operator
+        build_spatial_tables(c);
+        return;
+    }
     extern __shared__ __align__(16) unsigned char tsm[];
     __shared__ double dscr[64];
     __shared__ long long lscr[40];
@@ -339,7 +344,7 @@ cudaError_t launch_temporal(const Ctx &c, cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(temporal_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     void *args[] = {const_cast<Ctx *>(&c)};
-    return launch_kernel((const void *)temporal_kernel, dim3(c.V), dim3(temporal_threads(c.T)), smem, s, args,
+    return launch_kernel((const void *)temporal_kernel, dim3(c.V + 1), dim3(temporal_threads(c.T)), smem, s, args,
                          c.pdl != 0);
 }
 

@@ -57,6 +57,7 @@ struct Ctx {
     int4 *units;          // [V][max_units_v] tensor-core work units
     int *ucount;          // [V]
     int *ustart;          // [V*T] first unit of each frame in its video's list
+    float *stab;          // frame-independent tables of the spatial operator
     void *Wop;            // operator: tensor path bf16 hi then lo in the tiled
                           // layout of tile_index(), CUDA-core path f32 [rows][K_pad]
     int *status;          // device status word (bounded waits)
