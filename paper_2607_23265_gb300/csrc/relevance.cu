@@ -333,13 +333,14 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
 }
 
 // One block per frame: the frame sums (fixed list of CTA partials) for all
-// channels, fp32 products summed over each thread's channels, fp64 across
-// threads, then r_t = cos(v_bar_t, u_q) and delta_t = 1 - cos(v_bar_t,
-// v_bar_{t-1}) clamped to [0, 2] (Eq. 7) in fp64.
+// channels, read as 16-byte vectors; fp32 products summed over each thread's
+// channels and across each warp, the warp totals in fp64; then
+// r_t = cos(v_bar_t, u_q) and delta_t = 1 - cos(v_bar_t, v_bar_{t-1})
+// clamped to [0, 2] (Eq. 7) in fp64.
 __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     pdl_wait();
     pdl_trigger();
-    __shared__ double scratch[40];
+    __shared__ float wsum[16][5];
     const int64_t f = blockIdx.x;
     const int t = (int)(f % c.T);
     const int v = (int)(f / c.T);
@@ -348,25 +349,59 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     const int64_t g = f - 1;
     const int64_t lo2 = t > 0 ? g * c.N / c.L1 : 0;
     const int64_t hi2 = t > 0 ? min((int64_t)c.G1 - 1, ((g + 1) * c.N - 1) / c.L1) : -1;
+    const int nv = c.D / 4;
+    const float4 *P = reinterpret_cast<const float4 *>(c.part);
+    const float4 *Qv = reinterpret_cast<const float4 *>(c.qbar32 + (size_t)v * c.D);
     float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f, p4 = 0.f;
-    for (int d = threadIdx.x; d < c.D; d += blockDim.x) {
-        float sf = 0.f, sp = 0.f;
-        for (int64_t cc = lo; cc <= hi; ++cc) sf += c.part[(size_t)(cc + f) * c.D + d];
-        for (int64_t cc = lo2; cc <= hi2; ++cc) sp += c.part[(size_t)(cc + g) * c.D + d];
-        const float q = c.qbar32[(size_t)v * c.D + d];
-        if (c.frame_mean) c.frame_mean[(size_t)f * c.D + d] = sf / (float)c.N;
-        p0 = fmaf(sf, q, p0);
-        p1 = fmaf(sf, sf, p1);
-        p2 = fmaf(sf, sp, p2);
-        p3 = fmaf(q, q, p3);
-        p4 = fmaf(sp, sp, p4);
+    for (int i = threadIdx.x; i < nv; i += blockDim.x) {
+        float4 sf = make_float4(0.f, 0.f, 0.f, 0.f), sp = sf;
+        for (int64_t cc = lo; cc <= hi; ++cc) {
+            const float4 x = P[(size_t)(cc + f) * nv + i];
+            sf.x += x.x; sf.y += x.y; sf.z += x.z; sf.w += x.w;
+        }
+        for (int64_t cc = lo2; cc <= hi2; ++cc) {
+            const float4 x = P[(size_t)(cc + g) * nv + i];
+            sp.x += x.x; sp.y += x.y; sp.z += x.z; sp.w += x.w;
+        }
+        const float4 q = Qv[i];
+        if (c.frame_mean) {   // caller's buffer: 4-byte alignment only
+            float *fm = c.frame_mean + (size_t)f * c.D + 4 * i;
+            fm[0] = sf.x / (float)c.N;
+            fm[1] = sf.y / (float)c.N;
+            fm[2] = sf.z / (float)c.N;
+            fm[3] = sf.w / (float)c.N;
+        }
+        p0 = fmaf(sf.x, q.x, fmaf(sf.y, q.y, fmaf(sf.z, q.z, fmaf(sf.w, q.w, p0))));
+        p1 = fmaf(sf.x, sf.x, fmaf(sf.y, sf.y, fmaf(sf.z, sf.z, fmaf(sf.w, sf.w, p1))));
+        p2 = fmaf(sf.x, sp.x, fmaf(sf.y, sp.y, fmaf(sf.z, sp.z, fmaf(sf.w, sp.w, p2))));
+        p3 = fmaf(q.x, q.x, fmaf(q.y, q.y, fmaf(q.z, q.z, fmaf(q.w, q.w, p3))));
+        p4 = fmaf(sp.x, sp.x, fmaf(sp.y, sp.y, fmaf(sp.z, sp.z, fmaf(sp.w, sp.w, p4))));
     }
-    const double vq = block_sum((double)p0, scratch);
-    const double vv = block_sum((double)p1, scratch);
-    const double vp = block_sum((double)p2, scratch);
-    const double qq = block_sum((double)p3, scratch);
-    const double pp = block_sum((double)p4, scratch);
+    for (int o = 16; o > 0; o >>= 1) {
+        p0 += __shfl_xor_sync(0xffffffffu, p0, o);
+        p1 += __shfl_xor_sync(0xffffffffu, p1, o);
+        p2 += __shfl_xor_sync(0xffffffffu, p2, o);
+        p3 += __shfl_xor_sync(0xffffffffu, p3, o);
+        p4 += __shfl_xor_sync(0xffffffffu, p4, o);
+    }
+    const int warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    if ((threadIdx.x & 31) == 0) {
+        wsum[warp][0] = p0;
+        wsum[warp][1] = p1;
+        wsum[warp][2] = p2;
+        wsum[warp][3] = p3;
+        wsum[warp][4] = p4;
+    }
+    __syncthreads();
     if (threadIdx.x == 0) {
+        double vq = 0.0, vv = 0.0, vp = 0.0, qq = 0.0, pp = 0.0;
+        for (int w = 0; w < nw; ++w) {
+            vq += (double)wsum[w][0];
+            vv += (double)wsum[w][1];
+            vp += (double)wsum[w][2];
+            qq += (double)wsum[w][3];
+            pp += (double)wsum[w][4];
+        }
         const double qn = sqrt(qq);
         const double r = (vv > 0.0 && qn > 0.0) ? vq / (sqrt(vv) * qn) : 0.0;
         double d = 0.0;
