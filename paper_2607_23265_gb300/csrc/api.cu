@@ -28,7 +28,7 @@ bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 // Sub-buffer offsets of one call's workspace.
 struct Layout {
     size_t qbar32, qbar64, vpar, a, part, fr, list, n, off, woff, hw, prod,
-        units, ucount, ustart, stab, status, Wop, total;
+        units, ucount, ustart, stab, drange, gate, status, Wop, total;
 };
 
 struct Shape {
@@ -61,6 +61,8 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.ucount = take((size_t)s.V * 4);
     L.ustart = take(VT * 4);
     L.stab = take(spatial_table_bytes(s.H, s.W, kMaxTaps));   // any wavelet
+    L.drange = take((size_t)s.V * 16);
+    L.gate = with_operator ? take(VT * (size_t)((s.H + kMaxTaps - 1) / 2) * ((s.W + kMaxTaps - 1) / 2) * 4) : 0;
     L.status = take(16);
     L.Wop = with_operator ? take((size_t)std::max<int64_t>(s.rows_total, s.w_rows) * s.K_pad * 4) : 0;
     L.total = o;
@@ -161,6 +163,8 @@ void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.ucount = reinterpret_cast<int *>(ws + L.ucount);
     c.ustart = reinterpret_cast<int *>(ws + L.ustart);
     c.stab = reinterpret_cast<float *>(ws + L.stab);
+    c.drange = reinterpret_cast<unsigned long long *>(ws + L.drange);
+    c.gate = L.gate ? reinterpret_cast<float *>(ws + L.gate) : nullptr;
     c.status = reinterpret_cast<int *>(ws + L.status);
     if (L.Wop) c.Wop = ws + L.Wop;
 }

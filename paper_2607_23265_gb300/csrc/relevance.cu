@@ -35,7 +35,13 @@ __global__ void __launch_bounds__(256) query_pool_kernel(Ctx c, VideoParBlock pa
     pdl_trigger();
     const int v = blockIdx.y;
     const VideoPar vp = par.v[v];
-    if (blockIdx.x == 0 && threadIdx.x == 0) c.vpar[v] = vp;
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        c.vpar[v] = vp;
+        if (c.drange) {   // empty range of delta_t, filled by frame_stats
+            c.drange[2 * v] = 0x7ff0000000000000ull;   // +inf
+            c.drange[2 * v + 1] = 0ull;                // +0
+        }
+    }
     const int cl = threadIdx.x & 31, slice = threadIdx.x >> 5;
     const int d = blockIdx.x * 32 + cl;
     float s = 0.f, e = 0.f;
@@ -332,6 +338,52 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
     }
 }
 
+// Gate of the WSM for frame f (Eq. 6, Eq. 12): the saliency map M = min-max
+// normalised a_{t,n} over the frame, average-pooled to the hp x wp grid of
+// the first DWT level and scaled by lambda.  `red` is >= 32 floats of
+// shared scratch.
+__device__ void frame_gate(const Ctx &c, int64_t f, float *red) {
+    __shared__ float M[WZ_MAX_HW * WZ_MAX_HW];
+    const int N = c.N, H = c.H, W = c.W, hp = c.hp, wp = c.wp;
+    const float *a = c.a + f * N;
+    float lo = INFINITY, hi = -INFINITY;
+    for (int k = threadIdx.x; k < N; k += blockDim.x) {
+        const float x = a[k];
+        M[k] = x;
+        lo = fminf(lo, x);
+        hi = fmaxf(hi, x);
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    __syncthreads();   // red is free (the caller's reads are done)
+    if ((threadIdx.x & 31) == 0) {
+        red[threadIdx.x >> 5] = lo;
+        red[16 + (threadIdx.x >> 5)] = hi;
+    }
+    __syncthreads();
+    lo = INFINITY;
+    hi = -INFINITY;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
+        lo = fminf(lo, red[k]);
+        hi = fmaxf(hi, red[16 + k]);
+    }
+    const float rng = hi - lo;
+    for (int k = threadIdx.x; k < N; k += blockDim.x) M[k] = rng > 0.f ? (M[k] - lo) / rng : 0.f;
+    __syncthreads();
+    float *G = c.gate + f * (int64_t)(hp * wp);
+    for (int k = threadIdx.x; k < hp * wp; k += blockDim.x) {
+        const int ai = k / wp, bj = k % wp;
+        const int r0 = (ai * H) / hp, r1 = ((ai + 1) * H + hp - 1) / hp;
+        const int c0 = (bj * W) / wp, c1 = ((bj + 1) * W + wp - 1) / wp;
+        float s = 0.f;
+        for (int y = r0; y < r1; ++y)
+            for (int x = c0; x < c1; ++x) s += M[y * W + x];
+        G[k] = c.lambda * (s / (float)((r1 - r0) * (c1 - c0)));
+    }
+}
+
 // One block per frame: the frame sums (fixed list of CTA partials) for all
 // channels, read as 16-byte vectors; fp32 products summed over each thread's
 // channels and across each warp, the warp totals in fp64; then
@@ -408,12 +460,18 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
         if (t > 0) {
             const double den = sqrt(vv * pp);
             const double cs = den > 0.0 ? vp / den : 0.0;
-            d = fmin(2.0, fmax(0.0, 1.0 - cs));
+            d = fmin(2.0, fmax(0.0, 1.0 - cs)) + 0.0;   // + 0.0: never -0
         }
         c.fr[4 * f + 0] = r;
         c.fr[4 * f + 1] = d;
+        if (c.drange) {   // non-negative doubles order like their bit patterns
+            const unsigned long long bits = (unsigned long long)__double_as_longlong(d);
+            atomicMin(&c.drange[2 * v], bits);
+            atomicMax(&c.drange[2 * v + 1], bits);
+        }
         if (c.frame_scores) c.frame_scores[f] = (float)r;
     }
+    if (c.gate) frame_gate(c, f, wsum[0]);
 }
 
 cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s) {

@@ -111,7 +111,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     const int H = c.H, W = c.W, N = c.N, hp = c.hp, wp = c.wp, F = c.F;
     SpatialSmem L;
     L.init(H, W, hp, wp);
-    float *M = sm + L.M, *G = sm + L.G;
+    float *G = sm + L.G;
     float *AHl = sm + L.AHl, *AHh = sm + L.AHh, *AWl = sm + L.AWl, *AWh = sm + L.AWh;
     float *PAl = sm + L.PAl, *PAh = sm + L.PAh, *Yl = sm + L.Yl, *Yh = sm + L.Yh;
     float *Ql = sm + L.Ql, *Qh = sm + L.Qh, *red = sm + L.red;
@@ -122,26 +122,12 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     const int HP4 = L.HP4;
 
     // ---- per-frame tables ------------------------------------------------
-    // the frame-independent tables (analysis matrices, supports, pooling
-    // windows), built once per pass
+    // the frame-independent tables (analysis matrices, supports), built once
+    // per pass
     for (int k = tid; k < L.tables; k += blockDim.x) reinterpret_cast<int *>(sm)[k] = reinterpret_cast<const int *>(c.stab)[k];
-    // saliency map M (Eq. 6): per-frame min-max of a_{t,n}
-    const float *a = c.a + f * N;
-    float lo = INFINITY, hi = -INFINITY;
-    for (int k = tid; k < N; k += blockDim.x) {
-        const float x = a[k];
-        M[k] = x;
-        lo = fminf(lo, x);
-        hi = fmaxf(hi, x);
-    }
-    for (int o = 16; o > 0; o >>= 1) {
-        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-    }
-    if ((tid & 31) == 0) {
-        red[tid >> 5] = lo;
-        red[16 + (tid >> 5)] = hi;
-    }
+    // gate G of this frame (Eq. 6, Eq. 12), pooled by frame_stats
+    const float *Gf = c.gate + f * (int64_t)(hp * wp);
+    for (int k = tid; k < hp * wp; k += blockDim.x) G[k] = Gf[k];
     // bilinear columns through the synthesis: Q_v[q][b] and its support
     for (int k = tid; k < w * wp; k += blockDim.x) {
         const int q = k / wp, b = k % wp;
@@ -156,27 +142,6 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
             qlo[q] = l_;
             qhi[q] = h_;
         }
-    }
-    __syncthreads();
-    lo = INFINITY;
-    hi = -INFINITY;
-    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
-        lo = fminf(lo, red[k]);
-        hi = fmaxf(hi, red[16 + k]);
-    }
-    const float rng = hi - lo;
-    for (int k = tid; k < N; k += blockDim.x) M[k] = rng > 0.f ? (M[k] - lo) / rng : 0.f;
-    __syncthreads();
-    // gate G = lambda * adaptive-average-pool(M) to hp x wp (Eq. 12)
-    const int *pr0 = reinterpret_cast<const int *>(sm + L.pr0), *pr1 = reinterpret_cast<const int *>(sm + L.pr1);
-    const int *pc0 = reinterpret_cast<const int *>(sm + L.pc0), *pc1 = reinterpret_cast<const int *>(sm + L.pc1);
-    for (int k = tid; k < hp * wp; k += blockDim.x) {
-        const int ai = k / wp, bj = k % wp;
-        const int r0 = pr0[ai], r1 = pr1[ai], c0 = pc0[bj], c1 = pc1[bj];
-        float s = 0.f;
-        for (int y = r0; y < r1; ++y)
-            for (int x = c0; x < c1; ++x) s += M[y * W + x];
-        G[k] = c.lambda * (s / (float)((r1 - r0) * (c1 - c0)));
     }
 
     const bool bf = c.path == WZ_PATH_TENSOR;

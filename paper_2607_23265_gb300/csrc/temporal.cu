@@ -96,27 +96,10 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     int *nb = lst + T;                     // budget of retained frame m; -1 while active
     int *nf = nb + T;                      // budget of frame t
 
-    // r_t and delta_t come from frame_stats; the range of delta (Eq. 7),
-    // reduced by one warp (fp64 throughput is low: keep it to few warps)
-    if (threadIdx.x < 32) {
-        double lo = INFINITY, hi = -INFINITY;
-        for (int t = threadIdx.x; t < T; t += 32) {
-            const double d = fr[4 * t + 1];
-            lo = fmin(lo, d);
-            hi = fmax(hi, d);
-        }
-        for (int o = 16; o > 0; o >>= 1) {
-            lo = fmin(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-            hi = fmax(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-        }
-        if (threadIdx.x == 0) {
-            dscr[0] = lo;
-            dscr[1] = hi;
-        }
-    }
-    __syncthreads();
-    const double lo = dscr[0], hi = dscr[1];
-    __syncthreads();
+    // r_t and delta_t come from frame_stats, which also kept the range of
+    // delta over the video (Eq. 7)
+    const double lo = __longlong_as_double((long long)c.drange[2 * v]);
+    const double hi = __longlong_as_double((long long)c.drange[2 * v + 1]);
     // gamma_t and the retained set (frame 1 always kept)
     const double tau = (double)c.tau;
     // each thread owns `per` consecutive frames (per <= kPerThread)
@@ -226,14 +209,16 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
                 continue;
             }
             // largest remainder among the candidates: rank the fractional
-            // parts (non-negative doubles order like their bit patterns)
+            // parts (non-negative doubles order like their bit patterns; a
+            // candidate's key is its pattern + 1, others 0, so non-candidates
+            // rank below every candidate)
             long long fsum = 0;
             for (int m = threadIdx.x; m < L; m += blockDim.x) {
                 const double q = __longlong_as_double((long long)keys[m]);
-                unsigned long long key = ~0ull;
+                unsigned long long key = 0ull;
                 if (q >= 0.0) {
                     const double fl = floor(q);
-                    key = (unsigned long long)__double_as_longlong(q - fl);
+                    key = (unsigned long long)__double_as_longlong(q - fl) + 1ull;
                     fsum += (long long)fl;
                     nb[m] = (int)fl;       // floor; the remainder unit is added below
                 }
@@ -242,13 +227,25 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             const long long R = remaining - block_sum_ll(fsum, lscr);
             for (int m = threadIdx.x; m < L; m += blockDim.x) {
                 const unsigned long long km = keys[m];
-                if (km == ~0ull) continue;
-                int rank = 0;
-                for (int k = 0; k < L; ++k) {
-                    const unsigned long long kk = keys[k];
-                    rank += (kk != ~0ull && (kk > km || (kk == km && k < m))) ? 1 : 0;
+                if (km == 0ull) continue;
+                // rank = #{k : key_k > key_m, or key_k == key_m and k < m}
+                int r0 = 0, r1 = 0, r2 = 0, r3 = 0;
+                int k = 0;
+                for (; k + 4 <= m; k += 4) {   // k < m: ties count
+                    r0 += keys[k] >= km;
+                    r1 += keys[k + 1] >= km;
+                    r2 += keys[k + 2] >= km;
+                    r3 += keys[k + 3] >= km;
                 }
-                if (rank < R) nb[m] += 1;
+                for (; k < m; ++k) r0 += keys[k] >= km;
+                for (k = m + 1; k + 4 <= L; k += 4) {   // k > m: ties do not count
+                    r0 += keys[k] > km;
+                    r1 += keys[k + 1] > km;
+                    r2 += keys[k + 2] > km;
+                    r3 += keys[k + 3] > km;
+                }
+                for (; k < L; ++k) r0 += keys[k] > km;
+                if (r0 + r1 + r2 + r3 < R) nb[m] += 1;
             }
             __syncthreads();
             break;

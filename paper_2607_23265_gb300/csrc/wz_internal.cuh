@@ -58,6 +58,8 @@ struct Ctx {
     int *ucount;          // [V]
     int *ustart;          // [V*T] first unit of each frame in its video's list
     float *stab;          // frame-independent tables of the spatial operator
+    unsigned long long *drange;   // [V][2] min / max of delta_t as bit patterns (delta >= +0)
+    float *gate;          // [V*T][hp*wp] gate G of each frame (Eq. 12)
     void *Wop;            // operator: tensor path bf16 hi then lo in the tiled
                           // layout of tile_index(), CUDA-core path f32 [rows][K_pad]
     int *status;          // device status word (bounded waits)

@@ -1,8 +1,7 @@
 // Shared-memory layout of the spatial-operator CTA and the frame-independent
 // tables it starts from (Eq. 11-14): the db analysis matrices along height
-// and width with the boundary extension folded in, the rows of the width
-// analysis that reach each column, and the adaptive-pooling windows of the
-// gate.  The tables depend only on (H, W, filter, extension); one CTA builds
+// and width with the boundary extension folded in, and the rows of the width
+// analysis that reach each column.  The tables depend only on (H, W, filter, extension); one CTA builds
 // them per pass into global memory with the same layout as the head of the
 // shared-memory block, so each spatial CTA copies them in one loop.
 #pragma once
@@ -16,8 +15,8 @@ constexpr int kStageFloats = 8 * 1024;   // staged operator rows (32 KB)
 struct SpatialSmem {
     int N, hp, wp, H, W, HP4, K_pad, QB;
     // float offsets; [0, tables) is the frame-independent part
-    int AHl, AHh, AWl, AWh, blo, bhi, pr0, pr1, pc0, pc1, tables;
-    int M, G, PAl, PAh, Yl, Yh, Ql, Qh, red, qlo, qhi, stage, total;
+    int AHl, AHh, AWl, AWh, blo, bhi, tables;
+    int G, PAl, PAh, Yl, Yh, Ql, Qh, red, qlo, qhi, stage, total;
     // Every table starts on a 16-byte boundary (float4 reads of Y, staged rows).
     __host__ __device__ void init(int H_, int W_, int hp_, int wp_) {
         H = H_; W = W_; hp = hp_; wp = wp_; N = H * W;
@@ -36,12 +35,7 @@ struct SpatialSmem {
         AWh = take(wp * W);
         blo = take(W);
         bhi = take(W);
-        pr0 = take(hp);
-        pr1 = take(hp);
-        pc0 = take(wp);
-        pc1 = take(wp);
         tables = o;
-        M = take(N);
         G = take(hp * wp);
         PAl = take(hp * H);
         PAh = take(hp * H);
@@ -68,7 +62,6 @@ inline size_t spatial_table_bytes(int H, int W, int F) {
 //   A[a][i] = sum_j dec[j] [ext(2a + 1 - j) == i]   (analysis along a side)
 //   blo/bhi[j] = first / last row b of A' with A'[b][j] != 0 (shared-memory
 //                atomics while A' is formed)
-//   pooling window of gate cell (a, b): rows [pr0, pr1), columns [pc0, pc1)
 __device__ inline void build_spatial_tables(const Ctx &c) {
     SpatialSmem L;
     L.init(c.H, c.W, c.hp, c.wp);
@@ -106,14 +99,6 @@ __device__ inline void build_spatial_tables(const Ctx &c) {
             atomicMin(&s_blo[i], b);
             atomicMax(&s_bhi[i], b);
         }
-    }
-    for (int k = threadIdx.x; k < hp; k += blockDim.x) {
-        ti[L.pr0 + k] = (k * H) / hp;
-        ti[L.pr1 + k] = ((k + 1) * H + hp - 1) / hp;
-    }
-    for (int k = threadIdx.x; k < wp; k += blockDim.x) {
-        ti[L.pc0 + k] = (k * W) / wp;
-        ti[L.pc1 + k] = ((k + 1) * W + wp - 1) / wp;
     }
     __syncthreads();
     for (int j = threadIdx.x; j < W; j += blockDim.x) {
