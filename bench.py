@@ -98,8 +98,15 @@ def measured_peak():
 
 
 def source_hash(fname):
-    with open(os.path.join(ROOT, "paper_2607_23265_gb300", "csrc", fname), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    """Hash of a kernel's source file and every shared header it can include."""
+    csrc = os.path.join(ROOT, "paper_2607_23265_gb300", "csrc")
+    paths = [os.path.join(csrc, fname)] + sorted(os.path.join(csrc, h) for h in os.listdir(csrc) if h.endswith(".cuh"))
+    paths.append(os.path.join(ROOT, "include", "wavezip.h"))
+    h = hashlib.sha256()
+    for p in paths:
+        with open(p, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def recorded_traffic(kernel):

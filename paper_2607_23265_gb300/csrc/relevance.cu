@@ -188,7 +188,10 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
     int cur_v = -1;
     f2_t q[VPT][NP];
     float qn = 0.f;
-    f2_t cs[VPT][NP];
+    // column sums, split by token parity when registers allow (two shorter
+    // dependent chains per group)
+    constexpr int CSP = VPT == 1 ? 2 : 1;
+    f2_t cs[CSP][VPT][NP];
     int s = 0;
     uint32_t ph = 0;
     bool dead = false;
@@ -229,7 +232,7 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
 #pragma unroll
             for (int vi = 0; vi < VPT; ++vi)
 #pragma unroll
-                for (int e = 0; e < NP; ++e) cs[vi][e] = 0ull;
+                for (int e = 0; e < NP; ++e) cs[0][vi][e] = cs[CSP - 1][vi][e] = 0ull;
         }
         // this warp waits for the chunk itself (bounded)
         int ok = 1;
@@ -264,7 +267,7 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
                                 unpack_pairs(raw, x, (T *)nullptr);
 #pragma unroll
                                 for (int e = 0; e < NP; ++e) {
-                                    cs[vi][e] = add2(cs[vi][e], x[e]);
+                                    cs[k & (CSP - 1)][vi][e] = add2(cs[k & (CSP - 1)][vi][e], x[e]);
                                     dd = fma2(x[e], q[vi][e], dd);
                                     nn = fma2(x[e], x[e], nn);
                                 }
@@ -302,7 +305,12 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
                 if (vidx < n_vec) {
 #pragma unroll
                     for (int e = 0; e < NP; e += 2) {
-                        const float2 a = unpack2(cs[vi][e]), b = unpack2(cs[vi][e + 1]);
+                        f2_t s0 = cs[0][vi][e], s1 = cs[0][vi][e + 1];
+                        if (CSP == 2) {
+                            s0 = add2(s0, cs[CSP - 1][vi][e]);
+                            s1 = add2(s1, cs[CSP - 1][vi][e + 1]);
+                        }
+                        const float2 a = unpack2(s0), b = unpack2(s1);
                         *reinterpret_cast<float4 *>(dst + vidx * VEC + 2 * e) = make_float4(a.x, a.y, b.x, b.y);
                     }
                 }
