@@ -47,11 +47,23 @@ __global__ void __launch_bounds__(256) query_pool_kernel(Ctx c, VideoParBlock pa
     float s = 0.f, e = 0.f;
     if (d < c.D) {
         const T *Q = static_cast<const T *>(c.Q) + (size_t)vp.q_row0 * c.D + d;
-        for (int j = slice; j < vp.Lq; j += 8) {
-            float t, err;
-            two_sum(s, load_scalar<T>(Q + (size_t)j * c.D), t, err);
-            s = t;
-            e += err;
+        // rows slice, slice + 8, ...: loaded 8 at a time, then summed in order
+        for (int j0 = slice; j0 < vp.Lq; j0 += 64) {
+            float x[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int j = j0 + 8 * k;
+                x[k] = j < vp.Lq ? load_scalar<T>(Q + (size_t)j * c.D) : 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                if (j0 + 8 * k < vp.Lq) {
+                    float t, err;
+                    two_sum(s, x[k], t, err);
+                    s = t;
+                    e += err;
+                }
+            }
         }
     }
     ps[slice][cl] = s;

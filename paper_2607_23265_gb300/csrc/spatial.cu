@@ -149,6 +149,8 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * c.K_pad;
     float *W32 = static_cast<float *>(c.Wop);
     const int K_pad = c.K_pad, G8 = K_pad / 8;
+    const int wsh = W <= 32 ? 5 : 6;
+    const size_t kstride = (size_t)(c.w_rows >> 3) * 256;   // tile_index step of 32 columns
     const int t = (int)(f % c.T);
 
     // ---- grid rows p = s0, s0 + S, ... ------------------------------------
@@ -212,8 +214,10 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
         // of the hi and lo halves, or of fp32).
         for (int q0 = 0; q0 < nq; q0 += L.QB) {
             const int qn = min(L.QB, nq - q0);
-            for (int item = tid; item < qn * W; item += blockDim.x) {
-                const int ql_ = item / W, j = item % W;
+            // items (q, j): j is the lane within a stride of 32 or 64 columns
+            for (int item = tid; item < (qn << wsh); item += blockDim.x) {
+                const int ql_ = item >> wsh, j = item & ((1 << wsh) - 1);
+                if (j >= W) continue;
                 const int q = q0 + ql_;
                 float acc[HMAX];
 #pragma unroll
@@ -259,7 +263,10 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
                         hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
                         lw[e] = *reinterpret_cast<const uint32_t *>(&ll);
                     }
-                    const size_t ti = tile_index(wrow0 + q0 + ql_, 8 * g, c.w_rows);
+                    // tile_index(r, 8 g, w_rows), row part and column part apart
+                    const int64_t r = wrow0 + q0 + ql_;
+                    const size_t ti = (size_t)(g >> 2) * kstride + (size_t)(r >> 3) * 256 + (size_t)(r & 7) * 8 +
+                                      (size_t)(g & 3) * 64;
                     *reinterpret_cast<uint4 *>(Whi + ti) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
                     *reinterpret_cast<uint4 *>(Wlo + ti) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
                 } else {
