@@ -228,7 +228,9 @@ def algorithmic_bytes(spec, budgets, B, K_pad):
     return {
         "relevance": T * N * D * esz + T * N * 4,
         "condense": active * N * D * esz + B * D * esz + B * K_pad * 4,
-        "spatial": B * K_pad * 4 + active * N * 4,
+        # operator rows written (bf16 hi + lo) and the pooled gate of each
+        # active frame read (db4: (H + 7) / 2 x (W + 7) / 2)
+        "spatial": B * K_pad * 4 + active * ((spec.H + 7) // 2) * ((spec.W + 7) // 2) * 4,
         "frame_stats": None, "query_pool": None, "temporal": None,
     }
 
