@@ -74,6 +74,8 @@ def _random_case(wz, T, H, W, D, Lq, ratio, seed=0, dtype="bf16", **kw):
     (12, 13, 13, 256, 16, 0.002),  # B = 4 tokens
     (3, 64, 64, 32, 2, 0.05),     # largest map
     (33, 14, 14, 96, 5, 0.25),
+    (600, 3, 4, 16, 2, 0.3),      # more frames than temporal threads: 2 frames per thread
+    (4096, 2, 2, 8, 1, 0.4),      # longest video: 8 frames per thread, 4096-way ranking
 ])
 def test_shapes(wz, T, H, W, D, Lq, ratio):
     _random_case(wz, T, H, W, D, Lq, ratio, seed=T * 7 + H)
