@@ -58,6 +58,15 @@ fact; the same list is kept in the design notes):
       order are kept; the index map records (t, i, j).
   R17 the output dtype is the input dtype; rows that cannot be produced
       (B > sum of budgets) carry index -1 and zero tokens.
+  R18 the ablation modes of Section 4 ("Ablation Study") and Appendix B:
+      temporal "raw" (Raw Top-k) apportions B with the same rule over
+      max(r_t, 0) of the retained frames instead of max(r~, 0); temporal
+      "uniform" apportions B over the retained frames with equal weights (the
+      quotas are then exactly equal and the tie rule alone decides, so their
+      rounding is not a decision margin); spatial "saliency" (Saliency-Only)
+      replaces the WSM by the plain saliency weighting X~_m = lambda * M_m * X_m
+      in the token domain; spatial "none" (the module ablation's Uniform / WTA
+      rows) condenses X_m itself.  The default modes are the full method.
 """
 
 from __future__ import annotations
@@ -437,15 +446,22 @@ def psi(Xt_tilde: np.ndarray, n: int):
 # Whole pass C_WaveZip(X, Q) (Section 3.2, Eq. 18)
 # ----------------------------------------------------------------------------
 
+TEMPORAL_MODES = ("wta", "raw", "uniform")
+SPATIAL_MODES = ("wsm", "saliency", "none")
+
+
 def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
              wta_wavelet: int = 1, wsm_wavelet: int = 4, mode: str = "symmetric",
-             token_frames=None) -> dict:
+             token_frames=None, temporal_mode: str = "wta", spatial_mode: str = "wsm") -> dict:
     """Condense features X (T, H, W, D) for query Q (Lq, D) to B tokens.
 
     token_frames: optional iterable of frame indices; when given, the WSM and
     Psi steps run only for those frames (budgets, offsets and the index map are
     always complete), and out_tokens rows of other frames are left as NaN.
+    temporal_mode / spatial_mode: the ablation modes of reading R18.
     """
+    if temporal_mode not in TEMPORAL_MODES or spatial_mode not in SPATIAL_MODES:
+        raise ValueError("unknown mode")
     X = np.asarray(X, dtype=np.float64)
     T, H, W, D = X.shape
     N = H * W
@@ -461,7 +477,13 @@ def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
     keep = frame_filter(delta, as_float32(tau))
     r_tilde_M = wta(r[keep], gamma[keep], wta_wavelet)
     B = global_budget(ratio, T, N)
-    n_M, margins = allocate_budget(r_tilde_M, B, N)
+    if temporal_mode == "wta":
+        n_M, margins = allocate_budget(r_tilde_M, B, N)
+    elif temporal_mode == "raw":
+        n_M, margins = allocate_budget(r[keep], B, N)
+    else:
+        n_M, margins = allocate_budget(np.ones(len(keep)), B, N)
+        margins["alloc_gap"] = math.inf        # equal quotas: the tie rule decides (R18)
     budgets = np.zeros(T, dtype=np.int64)
     r_tilde = np.full(T, np.nan)
     for k, t in enumerate(keep):
@@ -481,7 +503,12 @@ def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
         for p in range(n):
             out_index[offsets[t] + p] = (t, p // w, p % w)
         if t in frames:
-            Xt = wsm(X[t], saliency_map(a[t], H, W), lam, wsm_wavelet, mode)
+            if spatial_mode == "wsm":
+                Xt = wsm(X[t], saliency_map(a[t], H, W), lam, wsm_wavelet, mode)
+            elif spatial_mode == "saliency":
+                Xt = lam * saliency_map(a[t], H, W)[:, :, None] * X[t]
+            else:
+                Xt = X[t]
             tok, _ = psi(Xt, n)
             out_tokens[offsets[t]:offsets[t] + n] = tok
         else:

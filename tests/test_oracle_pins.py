@@ -507,6 +507,103 @@ def test_condense_tail_rows_when_filter_drops_frames():
 
 
 # ----------------------------------------------------------------------------
+# Ablation modes (Section 4 "Ablation Study", Appendix B; reading R18)
+# ----------------------------------------------------------------------------
+
+def _aligned_video(T=10, H=4, W=5, D=6, seed=3):
+    """Frames whose pooled vector leans on the query by a frame-dependent
+    amount, so that r_t spreads over both signs."""
+    g = np.random.default_rng(seed)
+    Q = g.standard_normal((2, D))
+    u = Q.mean(axis=0) / np.linalg.norm(Q.mean(axis=0))
+    X = 0.3 * g.standard_normal((T, H, W, D))
+    X += np.linspace(-1.0, 1.5, T)[:, None, None, None] * u
+    return X, Q
+
+
+def check_uniform_mode(o):
+    X = RNG.standard_normal((9, 4, 5, 6))
+    Q = RNG.standard_normal((2, 6))
+    res = o.condense(X, Q, 0.37, temporal_mode="uniform")
+    B, keep = res["B"], res["keep"]
+    base, extra = divmod(B, len(keep))
+    expect = np.zeros(9, dtype=np.int64)
+    for k, t in enumerate(keep):                          # ties go to the earlier frame
+        expect[t] = base + (1 if k < extra else 0)
+    assert np.array_equal(res["budgets"], expect)
+
+
+def check_raw_mode(o):
+    X, Q = _aligned_video()
+    res = o.condense(X, Q, 0.2, temporal_mode="raw")
+    keep, B = res["keep"], res["B"]
+    w = np.maximum(res["r"][keep], 0.0)
+    q = B * w / w.sum()                                   # Eq. 15 quotas on the raw relevance
+    n = res["budgets"][keep]
+    assert n.sum() == B and np.all(q < 20)                # no cap binds at this ratio
+    assert np.all((n == np.floor(q)) | (n == np.floor(q) + 1))
+    frac = q - np.floor(q)
+    got = n - np.floor(q)
+    # the units beyond the floors went to the largest fractional parts
+    assert frac[got == 1].min(initial=np.inf) >= frac[got == 0].max(initial=-np.inf)
+
+
+def _torch_psi(Xt, n):
+    H, W = Xt.shape[:2]
+    h, w = OM.grid_shape(n, H, W)
+    g = torch.nn.functional.interpolate(torch.from_numpy(Xt).permute(2, 0, 1)[None], size=(h, w),
+                                        mode="bilinear", align_corners=False, antialias=False)
+    return g[0].permute(1, 2, 0).reshape(h * w, -1)[:n].numpy()
+
+
+def check_spatial_none(o):
+    X, Q = _aligned_video()
+    res = o.condense(X, Q, 0.4, spatial_mode="none")
+    for t in range(X.shape[0]):
+        lo, hi = res["offsets"][t], res["offsets"][t + 1]
+        if hi > lo:
+            assert np.allclose(res["out_tokens"][lo:hi], _torch_psi(X[t], hi - lo), atol=1e-12)
+
+
+def check_spatial_saliency(o):
+    X, Q = _aligned_video()
+    lam = 1.3
+    res = o.condense(X, Q, 0.4, lam=lam, spatial_mode="saliency")
+    for t in range(X.shape[0]):
+        lo, hi = res["offsets"][t], res["offsets"][t + 1]
+        if hi > lo:
+            A = torch.from_numpy(res["a"][t].reshape(X.shape[1], X.shape[2]))
+            M = (A - A.min()) / (A.max() - A.min())
+            Xw = lam * M.numpy()[:, :, None] * X[t]
+            assert np.allclose(res["out_tokens"][lo:hi], _torch_psi(Xw, hi - lo), atol=1e-12)
+
+
+def test_uniform_mode_budgets_closed_form():
+    check_uniform_mode(O)
+
+
+def test_raw_mode_apportions_raw_relevance():
+    check_raw_mode(O)
+
+
+def test_spatial_none_is_bilinear_of_features():
+    check_spatial_none(O)
+
+
+def test_spatial_saliency_is_bilinear_of_weighted_features():
+    check_spatial_saliency(O)
+
+
+def test_full_mode_differs_from_ablations():
+    X, Q = _aligned_video()
+    full = O.condense(X, Q, 0.4)
+    for sm in ("saliency", "none"):
+        abl = O.condense(X, Q, 0.4, spatial_mode=sm)
+        assert np.array_equal(abl["budgets"], full["budgets"])
+        assert not np.allclose(abl["out_tokens"], full["out_tokens"])
+
+
+# ----------------------------------------------------------------------------
 # Mutation tests: a planted mistake in the oracle makes a pin fail
 # ----------------------------------------------------------------------------
 
@@ -616,3 +713,17 @@ def test_mutation_tie_rule_breaks_pin():
         n, info = src(np.asarray(r)[::-1], B, N)
         return n[::-1].copy(), info
     assert _fails(check_budget_ties_to_earlier, _mutant(allocate_budget=alloc_bad))
+
+
+def test_mutation_saliency_map_without_normalisation_breaks_saliency_pin():
+    m = _mutant(saliency_map=lambda a_t, H, W: np.asarray(a_t, dtype=np.float64).reshape(H, W))
+    assert _fails(check_spatial_saliency, m)
+
+
+def test_mutation_budget_without_remainders_breaks_uniform_pin():
+    def floors_only(r_tilde, B, N):
+        w = np.maximum(np.asarray(r_tilde, dtype=np.float64), 0.0)
+        n = np.floor(B * w / w.sum()).astype(np.int64)
+        return n, {"alloc_gap": math.inf, "cap_gap": math.inf, "max_r": 1.0}
+    m = _mutant(allocate_budget=floors_only)
+    assert _fails(check_uniform_mode, m)
