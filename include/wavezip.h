@@ -88,6 +88,15 @@ typedef struct CUstream_st *wz_stream_t;
 #define WZ_KERNEL_CONDENSE       5 /* Z_m = W_m X_m, packed                     */
 #define WZ_NUM_KERNELS           6
 
+/* Ablation modes (Section 4 "Ablation Study", Appendix B).  The defaults
+ * (0, 0) are the method itself. */
+#define WZ_TEMPORAL_WTA      0 /* budgets from the WTA-rectified relevance r~      */
+#define WZ_TEMPORAL_RAW      1 /* "Raw Top-k": budgets from the raw relevance r_t   */
+#define WZ_TEMPORAL_UNIFORM  2 /* equal budgets over the retained frames          */
+#define WZ_SPATIAL_WSM       0 /* wavelet spatial modulator (Eq. 11-14)            */
+#define WZ_SPATIAL_SALIENCY  1 /* "Saliency-Only": lambda * M_t * X_t, no wavelets */
+#define WZ_SPATIAL_NONE      2 /* no modulation: Psi of the features itself       */
+
 /* Wavelets are Daubechies filters named by their vanishing moments p
  * (2p taps): 1 = Haar, 4 = db4.  1 <= p <= 10. */
 #define WZ_WAVELET_HAAR 1
@@ -138,6 +147,8 @@ typedef struct {
     int wsm_wavelet;         /* Daubechies order 1..10, default 4            */
     int mode;                /* WZ_MODE_* extension for the WSM DWT          */
     int path;                /* WZ_PATH_*                                    */
+    int temporal_mode;       /* WZ_TEMPORAL_*, default WTA                   */
+    int spatial_mode;        /* WZ_SPATIAL_*, default WSM                    */
     void *out_tokens;        /* [B][D], dtype                                */
     int32_t *out_index;      /* [B][3]                                       */
     int32_t *out_budgets;    /* [T] n_t (0 for filtered frames); nullable    */
@@ -186,6 +197,7 @@ typedef struct {
     const float *ratio;      /* host */
     float lambda, tau;
     int wta_wavelet, wsm_wavelet, mode, path;
+    int temporal_mode, spatial_mode;   /* WZ_TEMPORAL_*, WZ_SPATIAL_* */
     void *out_tokens;
     int32_t *out_index;
     int64_t *row_offsets;    /* host, [V+1], nullable */

@@ -112,7 +112,7 @@ Shape make_shape(int V, int T, int H, int W, int D, int dtype, int F, const int6
 
 struct Common {
     float lambda, tau;
-    int wta_wavelet, wsm_wavelet, mode, path;
+    int wta_wavelet, wsm_wavelet, mode, path, temporal_mode, spatial_mode;
 };
 
 int check_common(const Common &m, int dtype) {
@@ -123,6 +123,8 @@ int check_common(const Common &m, int dtype) {
     if (m.mode < WZ_MODE_SYMMETRIC || m.mode > WZ_MODE_PERIODIC) return WZ_ERR_INVALID_ARG;
     if (m.path < WZ_PATH_AUTO || m.path > WZ_PATH_SIMT) return WZ_ERR_INVALID_ARG;
     if (m.path == WZ_PATH_TENSOR && dtype != WZ_DTYPE_BF16) return WZ_ERR_UNSUPPORTED;
+    if (m.temporal_mode < WZ_TEMPORAL_WTA || m.temporal_mode > WZ_TEMPORAL_UNIFORM) return WZ_ERR_INVALID_ARG;
+    if (m.spatial_mode < WZ_SPATIAL_WSM || m.spatial_mode > WZ_SPATIAL_NONE) return WZ_ERR_INVALID_ARG;
     return WZ_OK;
 }
 
@@ -253,6 +255,8 @@ int run_condense(const CondenseRequest &r) {
     c.tau = r.m.tau;
     c.mode = r.m.mode;
     c.path = resolve_path(r.m.path, r.dtype);
+    c.temporal_mode = r.m.temporal_mode;
+    c.spatial_mode = r.m.spatial_mode;
     c.pdl = r.events ? 0 : 1;      // an event between two kernels would break the overlap
     set_filters(c, r.m.wsm_wavelet);
     const Shape s = make_shape(r.V, r.T, r.H, r.W, r.D, r.dtype, c.F, B.data());
@@ -376,7 +380,8 @@ int wz_condense_ex(const wz_condense_args *a) {
     r.queries = a->query;
     r.Lq.assign(1, a->Lq);
     r.ratio.assign(1, a->ratio);
-    r.m = Common{a->lambda, a->tau, a->wta_wavelet, a->wsm_wavelet, a->mode, a->path};
+    r.m = Common{a->lambda, a->tau, a->wta_wavelet, a->wsm_wavelet, a->mode, a->path, a->temporal_mode,
+                 a->spatial_mode};
     r.out_tokens = a->out_tokens;
     r.out_index = a->out_index;
     r.out_budgets = a->out_budgets;
@@ -430,7 +435,8 @@ int wz_condense_batch(const wz_batch_args *a) {
     r.queries = a->queries;
     r.Lq.assign(a->Lq, a->Lq + a->V);
     r.ratio.assign(a->ratio, a->ratio + a->V);
-    r.m = Common{a->lambda, a->tau, a->wta_wavelet, a->wsm_wavelet, a->mode, a->path};
+    r.m = Common{a->lambda, a->tau, a->wta_wavelet, a->wsm_wavelet, a->mode, a->path, a->temporal_mode,
+                 a->spatial_mode};
     r.out_tokens = a->out_tokens;
     r.out_index = a->out_index;
     r.out_budgets = a->out_budgets;

@@ -491,7 +491,7 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
         }
         if (c.frame_scores) c.frame_scores[f] = (float)r;
     }
-    if (c.gate) frame_gate(c, f, wsum[0]);
+    if (c.gate && c.spatial_mode == WZ_SPATIAL_WSM) frame_gate(c, f, wsum[0]);
 }
 
 cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s) {

@@ -60,7 +60,129 @@ __device__ __forceinline__ void synth_support(int y0, int y1, int F, int na, int
     hi = min(na - 1, (y1 + F - 2) >> 1);
 }
 
-template <int HMAX>
+// Staged rows [0, qn) of a grid row go out in 8-column groups: bf16 hi and
+// lo halves at tile_index(r, 8 g, w_rows) (tensor path; r = r_first + row,
+// split into a row part and a column part) or fp32 rows (CUDA-core path).
+__device__ __forceinline__ void write_rows(const float *stg, int qn, int K_pad, int64_t r_first, bool bf,
+                                           __nv_bfloat16 *Whi, __nv_bfloat16 *Wlo, float *W32, size_t kstride) {
+    const int G8 = K_pad / 8;
+    int ql_ = (int)threadIdx.x / G8, g = (int)threadIdx.x % G8;
+    const int gstep = (int)blockDim.x % G8, qstep = (int)blockDim.x / G8;
+    for (; ql_ < qn;) {
+        const float4 v0 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g);
+        const float4 v1 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g + 4);
+        const int64_t r = r_first + ql_;
+        if (bf) {
+            const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+            uint32_t hw[4], lw[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+                const __nv_bfloat162 ll =
+                    __floats2bfloat162_rn(v[2 * e] - __low2float(hh), v[2 * e + 1] - __high2float(hh));
+                hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
+                lw[e] = *reinterpret_cast<const uint32_t *>(&ll);
+            }
+            const size_t ti = (size_t)(g >> 2) * kstride + (size_t)(r >> 3) * 256 + (size_t)(r & 7) * 8 +
+                              (size_t)(g & 3) * 64;
+            *reinterpret_cast<uint4 *>(Whi + ti) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+            *reinterpret_cast<uint4 *>(Wlo + ti) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        } else {
+            float *dst = W32 + (size_t)r * K_pad + 8 * g;
+            *reinterpret_cast<float4 *>(dst) = v0;
+            *reinterpret_cast<float4 *>(dst + 4) = v1;
+        }
+        g += gstep;
+        ql_ += qstep;
+        if (g >= G8) {
+            g -= G8;
+            ++ql_;
+        }
+    }
+}
+
+// Operator rows of the ablation modes without the WSM (spatial "saliency" and
+// "none"): W[(p,q),(y,x)] = Ry[p][y] Rx[q][x] s(y, x), the bilinear weights of
+// Eq. 16 times s = lambda * M_t (Eq. 6 map) or 1.  Same staging, layout and
+// index rows as the WSM operator.
+__device__ void plain_operator_rows(const Ctx &c, const SpatialSmem &L, float *sm, int64_t f, int s0, int S, int n,
+                                    int h, int w) {
+    const int tid = threadIdx.x, H = c.H, W = c.W, N = c.N, K_pad = c.K_pad;
+    float *stg = sm + L.stage, *M = sm + L.M, *red = sm + L.red;
+    const bool sal = c.spatial_mode == WZ_SPATIAL_SALIENCY;
+    if (sal) {
+        const float *a = c.a + f * N;
+        float lo = INFINITY, hi = -INFINITY;
+        for (int k = tid; k < N; k += blockDim.x) {
+            const float x = a[k];
+            M[k] = x;
+            lo = fminf(lo, x);
+            hi = fmaxf(hi, x);
+        }
+        for (int o = 16; o > 0; o >>= 1) {
+            lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+            hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+        }
+        if ((tid & 31) == 0) {
+            red[tid >> 5] = lo;
+            red[16 + (tid >> 5)] = hi;
+        }
+        __syncthreads();
+        lo = INFINITY;
+        hi = -INFINITY;
+        for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
+            lo = fminf(lo, red[k]);
+            hi = fmaxf(hi, red[16 + k]);
+        }
+        const float rng = hi - lo;
+        for (int k = tid; k < N; k += blockDim.x) M[k] = c.lambda * (rng > 0.f ? (M[k] - lo) / rng : 0.f);
+    }
+    const bool bf = c.path == WZ_PATH_TENSOR;
+    __nv_bfloat16 *Whi = static_cast<__nv_bfloat16 *>(c.Wop);
+    __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * K_pad;
+    float *W32 = static_cast<float *>(c.Wop);
+    const size_t kstride = (size_t)(c.w_rows >> 3) * 256;
+    const int t = (int)(f % c.T);
+    for (int pi = s0; pi < h && pi * w < n; pi += S) {
+        const int nq = min(w, n - pi * w);
+        int y0, y1;
+        float ly;
+        bilinear_src(pi, H, h, y0, y1, ly);
+        const int64_t row0 = (int64_t)c.off[f] + (int64_t)pi * w;
+        const int64_t wrow0 = bf ? (int64_t)c.woff[f] + (int64_t)pi * w : row0;
+        for (int q0 = 0; q0 < nq; q0 += L.QB) {
+            const int qn = min(L.QB, nq - q0);
+            __syncthreads();   // M, and the previous batch's reads of the stage
+            for (int k = tid; k < qn * K_pad; k += blockDim.x) stg[k] = 0.f;
+            __syncthreads();
+            for (int ql_ = tid; ql_ < qn; ql_ += blockDim.x) {
+                int x0, x1;
+                float lx;
+                bilinear_src(q0 + ql_, W, w, x0, x1, lx);
+                float *row = stg + ql_ * K_pad;
+                const int ys[2] = {y0, y1}, xs[2] = {x0, x1};
+                const float wy[2] = {1.f - ly, ly}, wx[2] = {1.f - lx, lx};
+#pragma unroll
+                for (int u = 0; u < 2; ++u)
+#pragma unroll
+                    for (int v = 0; v < 2; ++v) {
+                        const int k = ys[u] * W + xs[v];
+                        row[k] += wy[u] * wx[v] * (sal ? M[k] : 1.f);
+                    }
+            }
+            __syncthreads();
+            write_rows(stg, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
+        }
+        for (int q = tid; q < nq; q += blockDim.x) {
+            int *o = c.out_index + (size_t)(row0 + q) * 3;
+            o[0] = t;
+            o[1] = pi;
+            o[2] = q;
+        }
+    }
+}
+
+template <int HMAX, bool PLAIN>
 __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) {
     pdl_wait();
     pdl_trigger();
@@ -111,6 +233,10 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     const int H = c.H, W = c.W, N = c.N, hp = c.hp, wp = c.wp, F = c.F;
     SpatialSmem L;
     L.init(H, W, hp, wp);
+    if constexpr (PLAIN) {   // ablation modes without the WSM
+        plain_operator_rows(c, L, sm, f, s0, S, n, h, w);
+        return;
+    }
     float *G = sm + L.G;
     float *AHl = sm + L.AHl, *AHh = sm + L.AHh, *AWl = sm + L.AWl, *AWh = sm + L.AWh;
     float *PAl = sm + L.PAl, *PAh = sm + L.PAh, *Yl = sm + L.Yl, *Yh = sm + L.Yh;
@@ -148,7 +274,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     __nv_bfloat16 *Whi = static_cast<__nv_bfloat16 *>(c.Wop);
     __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * c.K_pad;
     float *W32 = static_cast<float *>(c.Wop);
-    const int K_pad = c.K_pad, G8 = K_pad / 8;
+    const int K_pad = c.K_pad;
     const int wsh = W <= 32 ? 5 : 6;
     const size_t kstride = (size_t)(c.w_rows >> 3) * 256;   // tile_index step of 32 columns
     const int t = (int)(f % c.T);
@@ -247,40 +373,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
             for (int k = tid; k < qn * (K_pad - N); k += blockDim.x)
                 stg[(k / (K_pad - N)) * K_pad + N + k % (K_pad - N)] = 0.f;
             __syncthreads();
-            int ql_ = tid / G8, g = tid % G8;
-            const int gstep = (int)blockDim.x % G8, qstep = (int)blockDim.x / G8;
-            for (; ql_ < qn;) {
-                const float4 v0 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g);
-                const float4 v1 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g + 4);
-                if (bf) {
-                    const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-                    uint32_t hw[4], lw[4];
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
-                        const __nv_bfloat162 ll =
-                            __floats2bfloat162_rn(v[2 * e] - __low2float(hh), v[2 * e + 1] - __high2float(hh));
-                        hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
-                        lw[e] = *reinterpret_cast<const uint32_t *>(&ll);
-                    }
-                    // tile_index(r, 8 g, w_rows), row part and column part apart
-                    const int64_t r = wrow0 + q0 + ql_;
-                    const size_t ti = (size_t)(g >> 2) * kstride + (size_t)(r >> 3) * 256 + (size_t)(r & 7) * 8 +
-                                      (size_t)(g & 3) * 64;
-                    *reinterpret_cast<uint4 *>(Whi + ti) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-                    *reinterpret_cast<uint4 *>(Wlo + ti) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-                } else {
-                    float *dst = W32 + (size_t)(row0 + q0 + ql_) * K_pad + 8 * g;
-                    *reinterpret_cast<float4 *>(dst) = v0;
-                    *reinterpret_cast<float4 *>(dst + 4) = v1;
-                }
-                g += gstep;
-                ql_ += qstep;
-                if (g >= G8) {
-                    g -= G8;
-                    ++ql_;
-                }
-            }
+            write_rows(stg, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
             if (q0 + L.QB < nq) __syncthreads();
         }
         for (int q = tid; q < nq; q += blockDim.x) {
@@ -313,9 +406,11 @@ cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     if ((L.Yl & 3) != 0 || (L.Yh & 3) != 0 || (L.stage & 3) != 0 || L.QB < 1) return cudaErrorMisalignedAddress;
     const size_t smem = spatial_smem_bytes(c);
     const void *fn;
-    if (c.H <= 16) fn = (const void *)spatial_kernel<16>;
-    else if (c.H <= 32) fn = (const void *)spatial_kernel<32>;
-    else if (c.H <= 64) fn = (const void *)spatial_kernel<64>;
+    const bool plain = c.spatial_mode != WZ_SPATIAL_WSM;
+    if (plain) fn = (const void *)spatial_kernel<4, true>;   // HMAX unused without the WSM
+    else if (c.H <= 16) fn = (const void *)spatial_kernel<16, false>;
+    else if (c.H <= 32) fn = (const void *)spatial_kernel<32, false>;
+    else if (c.H <= 64) fn = (const void *)spatial_kernel<64, false>;
     else return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

@@ -130,7 +130,8 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     // WTA: Haar DWT of r over the retained sequence, detail gated by the
     // pair mean of gamma, inverse DWT (Eq. 8-10).  Odd L: the last sample
     // pairs with its mirror image, so its detail is 0.  Budget weights are
-    // max(r~, 0) (Eq. 5).
+    // max(r~, 0) (Eq. 5); the ablation modes use max(r, 0) ("raw") or 1
+    // ("uniform") instead.
     const double s2 = 0.70710678118654752440;
     int anypos = 0;
     for (int k = threadIdx.x; 2 * k < L; k += blockDim.x) {
@@ -143,13 +144,16 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         const double Dt = g * Dd;
         const double rt0 = s2 * A + s2 * Dt;
         fr[4 * a0 + 3] = rt0;
-        wgt[i0] = fmax(rt0, 0.0);
-        anypos |= (rt0 > 0.0);
+        const double w0 = c.temporal_mode == WZ_TEMPORAL_WTA ? rt0 : c.temporal_mode == WZ_TEMPORAL_RAW ? r0 : 1.0;
+        wgt[i0] = fmax(w0, 0.0);
+        anypos |= (w0 > 0.0);
         if (i1 != i0) {
             const double rt1 = s2 * A - s2 * Dt;
             fr[4 * a1 + 3] = rt1;
-            wgt[i1] = fmax(rt1, 0.0);
-            anypos |= (rt1 > 0.0);
+            const double w1 =
+                c.temporal_mode == WZ_TEMPORAL_WTA ? rt1 : c.temporal_mode == WZ_TEMPORAL_RAW ? r1 : 1.0;
+            wgt[i1] = fmax(w1, 0.0);
+            anypos |= (w1 > 0.0);
         }
     }
     // uniform weights if none is positive

@@ -75,6 +75,8 @@ struct Ctx {
     float lambda, tau;
     int mode;             // WZ_MODE_*
     int path;             // resolved WZ_PATH_TENSOR or WZ_PATH_SIMT
+    int temporal_mode;    // WZ_TEMPORAL_*
+    int spatial_mode;     // WZ_SPATIAL_*
     int pdl;              // host: launch with programmatic stream serialization
     float dec_lo[kMaxTaps], dec_hi[kMaxTaps], rec_lo[kMaxTaps], rec_hi[kMaxTaps];
 };

@@ -16,7 +16,7 @@ struct SpatialSmem {
     int N, hp, wp, H, W, HP4, K_pad, QB;
     // float offsets; [0, tables) is the frame-independent part
     int AHl, AHh, AWl, AWh, blo, bhi, tables;
-    int G, PAl, PAh, Yl, Yh, Ql, Qh, red, qlo, qhi, stage, total;
+    int G, PAl, PAh, Yl, Yh, Ql, Qh, red, qlo, qhi, M, stage, total;
     // Every table starts on a 16-byte boundary (float4 reads of Y, staged rows).
     __host__ __device__ void init(int H_, int W_, int hp_, int wp_) {
         H = H_; W = W_; hp = hp_; wp = wp_; N = H * W;
@@ -46,6 +46,7 @@ struct SpatialSmem {
         red = take(64);
         qlo = take(W);
         qhi = take(W);
+        M = take(N);                               // saliency map (ablation mode "saliency")
         stage = take(QB * K_pad);
         total = o;
     }

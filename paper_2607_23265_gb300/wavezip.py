@@ -23,6 +23,14 @@ MODE_SYMMETRIC, MODE_ZERO, MODE_PERIODIC = 0, 1, 2
 PATH_AUTO, PATH_TENSOR, PATH_SIMT = 0, 1, 2
 MODES = {"symmetric": MODE_SYMMETRIC, "zero": MODE_ZERO, "periodic": MODE_PERIODIC}
 PATHS = {"auto": PATH_AUTO, "tensor": PATH_TENSOR, "simt": PATH_SIMT}
+TEMPORAL_WTA, TEMPORAL_RAW, TEMPORAL_UNIFORM = 0, 1, 2
+SPATIAL_WSM, SPATIAL_SALIENCY, SPATIAL_NONE = 0, 1, 2
+TEMPORAL_MODES = {"wta": TEMPORAL_WTA, "raw": TEMPORAL_RAW, "uniform": TEMPORAL_UNIFORM}
+SPATIAL_MODES = {"wsm": SPATIAL_WSM, "saliency": SPATIAL_SALIENCY, "none": SPATIAL_NONE}
+
+
+def _enum(table, v):
+    return table[v] if isinstance(v, str) else int(v)
 
 
 class WaveZipError(RuntimeError):
@@ -36,7 +44,8 @@ class CondenseArgs(C.Structure):
         ("features", C.c_void_p), ("T", C.c_int), ("H", C.c_int), ("W", C.c_int), ("D", C.c_int),
         ("dtype", C.c_int), ("query", C.c_void_p), ("Lq", C.c_int), ("ratio", C.c_float),
         ("lam", C.c_float), ("tau", C.c_float), ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int),
-        ("mode", C.c_int), ("path", C.c_int), ("out_tokens", C.c_void_p), ("out_index", C.c_void_p),
+        ("mode", C.c_int), ("path", C.c_int), ("temporal_mode", C.c_int), ("spatial_mode", C.c_int),
+        ("out_tokens", C.c_void_p), ("out_index", C.c_void_p),
         ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
         ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
         ("kernel_events", C.POINTER(C.c_void_p)), ("stream", C.c_void_p),
@@ -49,6 +58,7 @@ class BatchArgs(C.Structure):
         ("D", C.c_int), ("dtype", C.c_int), ("queries", C.c_void_p), ("Lq", C.POINTER(C.c_int32)),
         ("ratio", C.POINTER(C.c_float)), ("lam", C.c_float), ("tau", C.c_float),
         ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int), ("mode", C.c_int), ("path", C.c_int),
+        ("temporal_mode", C.c_int), ("spatial_mode", C.c_int),
         ("out_tokens", C.c_void_p), ("out_index", C.c_void_p), ("row_offsets", C.POINTER(C.c_int64)),
         ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
         ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
@@ -160,6 +170,7 @@ def wz_condense(features: torch.Tensor, query: torch.Tensor, ratio: float, strea
 
 def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *, lam: float = 1.5,
                    tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
+                   temporal_mode="wta", spatial_mode="wsm",
                    workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
                    device_status: torch.Tensor | None = None, kernel_events=None, stream=None):
     """wz_condense_ex.  Returns a dict with tokens, index, budgets, count and relevance.
@@ -186,6 +197,8 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
     a.lam, a.tau, a.wsm_wavelet = lam, tau, wsm_wavelet
     a.mode = MODES[mode] if isinstance(mode, str) else int(mode)
     a.path = PATHS[path] if isinstance(path, str) else int(path)
+    a.temporal_mode = _enum(TEMPORAL_MODES, temporal_mode)
+    a.spatial_mode = _enum(SPATIAL_MODES, spatial_mode)
     a.out_tokens, a.out_index = tokens.data_ptr(), index.data_ptr()
     a.out_budgets, a.out_count, a.out_relevance = budgets.data_ptr(), count.data_ptr(), rel.data_ptr()
     if workspace is not None:
@@ -210,6 +223,7 @@ def wz_batch_rows(V, T, H, W, ratios):
 
 def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios, *, lam: float = 1.5,
                       tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
+                      temporal_mode="wta", spatial_mode="wsm",
                       workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
                       stream=None):
     """wz_condense_batch: features [V,T,H,W,D], queries [sum Lq, D]."""
@@ -234,6 +248,8 @@ def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios,
     a.lam, a.tau, a.wsm_wavelet = lam, tau, wsm_wavelet
     a.mode = MODES[mode] if isinstance(mode, str) else int(mode)
     a.path = PATHS[path] if isinstance(path, str) else int(path)
+    a.temporal_mode = _enum(TEMPORAL_MODES, temporal_mode)
+    a.spatial_mode = _enum(SPATIAL_MODES, spatial_mode)
     a.out_tokens, a.out_index, a.row_offsets = tokens.data_ptr(), index.data_ptr(), ro
     a.out_budgets, a.out_count, a.out_relevance = budgets.data_ptr(), count.data_ptr(), rel.data_ptr()
     if workspace is not None:

@@ -19,14 +19,15 @@ def oracle_run(X, Q, ratio, **kw):
     return O.condense(to_np64(X), to_np64(Q), ratio, **kw)
 
 
-def accepted_video(spec: wl.VideoSpec, tries: int = 8):
+def accepted_video(spec: wl.VideoSpec, tries: int = 8, **kw):
     """Generate the spec's video, advancing the seed by 10000 until every
-    integer decision of the oracle is at least MIN_MARGIN from its boundary."""
+    integer decision of the oracle (with options kw) is at least MIN_MARGIN
+    from its boundary."""
     seed = spec.seed
     for _ in range(tries):
         s = wl.VideoSpec(**{**spec.__dict__, "seed": seed})
         X, Q, meta = wl.make_video(s)
-        ref = oracle_run(X, Q, s.ratio, token_frames=[])
+        ref = oracle_run(X, Q, s.ratio, token_frames=[], **kw)
         if O.decision_margins(ref) >= MIN_MARGIN:
             return s, X, Q, ref
         seed += 10000

@@ -47,6 +47,7 @@ def test_struct_layout_matches_defaults(wz):
     a = wz.CondenseArgs()
     wz._lib.wz_condense_args_init(C.byref(a))
     assert (a.lam, a.tau, a.wta_wavelet, a.wsm_wavelet, a.mode, a.path, a.dtype) == (1.5, 0.0, 1, 4, 0, 0, 0)
+    assert (a.temporal_mode, a.spatial_mode) == (wz.TEMPORAL_WTA, wz.SPATIAL_WSM)
     b = wz.BatchArgs()
     wz._lib.wz_batch_args_init(C.byref(b))
     assert (b.lam, b.wta_wavelet, b.wsm_wavelet) == (1.5, 1, 4)
@@ -111,6 +112,7 @@ def _args(wz, **over):
     (dict(ratio=1.01), -1), (dict(ratio=float("nan")), -1), (dict(lam=-1.0), -1),
     (dict(lam=float("inf")), -1), (dict(wta_wavelet=4), -2), (dict(wta_wavelet=0), -1),
     (dict(wsm_wavelet=11), -1), (dict(mode=3), -1), (dict(path=7), -1), (dict(dtype=5), -1),
+    (dict(temporal_mode=3), -1), (dict(temporal_mode=-1), -1), (dict(spatial_mode=3), -1),
     (dict(dtype=1, path=1), -2), (dict(features=P + 4), -1), (dict(out_tokens=3 * P + 8), -1),
     (dict(workspace=5 * P, workspace_bytes=16), -5), (dict(workspace=5 * P + 64, workspace_bytes=1 << 30), -1),
 ])

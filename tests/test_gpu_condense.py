@@ -56,7 +56,7 @@ def test_config_256_frames_sampled(wz):
 
 
 def _random_case(wz, T, H, W, D, Lq, ratio, seed=0, dtype="bf16", **kw):
-    okw = {k: v for k, v in kw.items() if k in ("lam", "tau", "wsm_wavelet", "mode")}
+    okw = {k: v for k, v in kw.items() if k in ("lam", "tau", "wsm_wavelet", "mode", "temporal_mode", "spatial_mode")}
     X, Q = accepted_random(T, H, W, D, Lq, ratio, seed=seed, dtype=dtype, **okw)
     ref = oracle_run(X, Q, ratio, **okw)
     out = run(wz, X, Q, ratio, **kw)
@@ -85,6 +85,28 @@ def test_shapes(wz, T, H, W, D, Lq, ratio):
                                 dict(mode="zero"), dict(mode="periodic"), dict(path="simt")])
 def test_options(wz, kw):
     _random_case(wz, 10, 13, 13, 128, 6, 0.2, seed=5, **kw)
+
+
+@pytest.mark.parametrize("kw", [dict(temporal_mode="raw"), dict(temporal_mode="uniform"),
+                                dict(spatial_mode="saliency"), dict(spatial_mode="none"),
+                                dict(spatial_mode="saliency", lam=0.7, temporal_mode="raw"),
+                                dict(temporal_mode="uniform", spatial_mode="none", path="simt")])
+def test_ablation_modes(wz, kw):
+    _random_case(wz, 10, 13, 13, 128, 6, 0.2, seed=5, **kw)
+
+
+@pytest.mark.parametrize("tm,sm", [("raw", "wsm"), ("uniform", "saliency"), ("raw", "none")])
+def test_ablation_modes_structured_video(wz, tm, sm):
+    kw = dict(temporal_mode=tm, spatial_mode=sm)
+    spec = wl.VideoSpec(T=24, H=13, W=13, D=256, Lq=8, ratio=0.15, cuts=2, patches=2, seed=77)
+    s, X, Q, _ = accepted_video(spec, **kw)
+    ref = oracle_run(X, Q, s.ratio, **kw)
+    out = run(wz, X, Q, s.ratio, **kw)
+    compare_condense(out, ref, X.dtype)
+
+
+def test_ablation_saliency_fp32(wz):
+    _random_case(wz, 6, 9, 11, 64, 4, 0.3, seed=11, dtype="f32", spatial_mode="saliency")
 
 
 def test_fp32_features(wz):
