@@ -143,7 +143,8 @@ typedef struct {
     float ratio;             /* rho in (0, 1]                                */
     float lambda;            /* WSM gate strength (Eq. 12), default 1.5      */
     float tau;               /* frame-filter threshold on delta, default 0   */
-    int wta_wavelet;         /* must be WZ_WAVELET_HAAR                      */
+    int wta_wavelet;         /* Daubechies order 1..10 of the WTA DWT,       */
+                             /* default 1 (Haar, Eq. 8-10)                   */
     int wsm_wavelet;         /* Daubechies order 1..10, default 4            */
     int mode;                /* WZ_MODE_* extension for the WSM DWT          */
     int path;                /* WZ_PATH_*                                    */

@@ -117,8 +117,7 @@ struct Common {
 
 int check_common(const Common &m, int dtype) {
     if (!std::isfinite(m.lambda) || m.lambda < 0.f || !std::isfinite(m.tau)) return WZ_ERR_INVALID_ARG;
-    if (m.wta_wavelet != WZ_WAVELET_HAAR) return m.wta_wavelet >= 1 && m.wta_wavelet <= 10
-                                                      ? WZ_ERR_UNSUPPORTED : WZ_ERR_INVALID_ARG;
+    if (m.wta_wavelet < 1 || m.wta_wavelet > 10) return WZ_ERR_INVALID_ARG;
     if (m.wsm_wavelet < 1 || m.wsm_wavelet > 10) return WZ_ERR_INVALID_ARG;
     if (m.mode < WZ_MODE_SYMMETRIC || m.mode > WZ_MODE_PERIODIC) return WZ_ERR_INVALID_ARG;
     if (m.path < WZ_PATH_AUTO || m.path > WZ_PATH_SIMT) return WZ_ERR_INVALID_ARG;
@@ -142,6 +141,18 @@ void set_filters(Ctx &c, int p) {
         c.dec_hi[k] = k < c.F ? (float)dh[k] : 0.f;
         c.rec_lo[k] = k < c.F ? (float)rl[k] : 0.f;
         c.rec_hi[k] = k < c.F ? (float)rh[k] : 0.f;
+    }
+}
+
+void set_wta_filters(Ctx &c, int p) {
+    double dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
+    daubechies(p, dl, dh, rl, rh);
+    c.wta_F = 2 * p;
+    for (int k = 0; k < kMaxTaps; ++k) {
+        c.wta_dec_lo[k] = k < c.wta_F ? dl[k] : 0.0;
+        c.wta_dec_hi[k] = k < c.wta_F ? dh[k] : 0.0;
+        c.wta_rec_lo[k] = k < c.wta_F ? rl[k] : 0.0;
+        c.wta_rec_hi[k] = k < c.wta_F ? rh[k] : 0.0;
     }
 }
 
@@ -259,6 +270,7 @@ int run_condense(const CondenseRequest &r) {
     c.spatial_mode = r.m.spatial_mode;
     c.pdl = r.events ? 0 : 1;      // an event between two kernels would break the overlap
     set_filters(c, r.m.wsm_wavelet);
+    set_wta_filters(c, r.m.wta_wavelet);
     const Shape s = make_shape(r.V, r.T, r.H, r.W, r.D, r.dtype, c.F, B.data());
     const Layout L = make_layout(s, true, true);
     Scratch ws;

@@ -67,7 +67,10 @@ __device__ __forceinline__ int grid_h(int n, int H, int W) {
 
 // Shared-memory arrays of one video, indexed by retained frame m (wgt,
 // keys, lst, nb) or by frame t (nf).
-__host__ __device__ inline size_t temporal_smem_bytes(int T) { return (size_t)T * (8 + 8 + 4 + 4 + 4); }
+__host__ __device__ inline size_t temporal_smem_offset_coef(int T) { return ((size_t)T * (8 + 8 + 4 + 4 + 4) + 7) & ~(size_t)7; }
+__host__ __device__ inline size_t temporal_smem_bytes(int T) {
+    return temporal_smem_offset_coef(T) + 2 * sizeof(double) * (size_t)((T + kMaxTaps - 1) / 2);
+}
 
 // Threads of the CTA: one frame per thread up to 512 frames, at most
 // kPerThread frames per thread beyond (fp64 work scales with the warps).
@@ -95,6 +98,8 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     int *lst = reinterpret_cast<int *>(keys + T);                         // retained frames
     int *nb = lst + T;                     // budget of retained frame m; -1 while active
     int *nf = nb + T;                      // budget of frame t
+    double *cA = reinterpret_cast<double *>(tsm + temporal_smem_offset_coef(T));   // WTA approximation
+    double *cD = cA + (T + kMaxTaps - 1) / 2;                                       // gated WTA detail
 
     // r_t and delta_t come from frame_stats, which also kept the range of
     // delta over the video (Eq. 7)
@@ -127,34 +132,42 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         if (k < per && keep[k]) lst[pos++] = t0 + k;
     __syncthreads();
 
-    // WTA: Haar DWT of r over the retained sequence, detail gated by the
-    // pair mean of gamma, inverse DWT (Eq. 8-10).  Odd L: the last sample
-    // pairs with its mirror image, so its detail is 0.  Budget weights are
-    // max(r~, 0) (Eq. 5); the ablation modes use max(r, 0) ("raw") or 1
-    // ("uniform") instead.
-    const double s2 = 0.70710678118654752440;
-    int anypos = 0;
-    for (int k = threadIdx.x; 2 * k < L; k += blockDim.x) {
-        const int i0 = 2 * k, i1 = min(2 * k + 1, L - 1);
-        const int a0 = lst[i0], a1 = lst[i1];
-        const double r0 = fr[4 * a0], r1 = fr[4 * a1];
-        const double A = s2 * r0 + s2 * r1;
-        const double Dd = s2 * r0 - s2 * r1;
-        const double g = 0.5 * (fr[4 * a0 + 2] + fr[4 * a1 + 2]);
-        const double Dt = g * Dd;
-        const double rt0 = s2 * A + s2 * Dt;
-        fr[4 * a0 + 3] = rt0;
-        const double w0 = c.temporal_mode == WZ_TEMPORAL_WTA ? rt0 : c.temporal_mode == WZ_TEMPORAL_RAW ? r0 : 1.0;
-        wgt[i0] = fmax(w0, 0.0);
-        anypos |= (w0 > 0.0);
-        if (i1 != i0) {
-            const double rt1 = s2 * A - s2 * Dt;
-            fr[4 * a1 + 3] = rt1;
-            const double w1 =
-                c.temporal_mode == WZ_TEMPORAL_WTA ? rt1 : c.temporal_mode == WZ_TEMPORAL_RAW ? r1 : 1.0;
-            wgt[i1] = fmax(w1, 0.0);
-            anypos |= (w1 > 0.0);
+    // WTA (Eq. 8-10): DWT of r over the retained sequence with the WTA
+    // wavelet (Daubechies p, 2p taps; half-sample symmetric extension, as the
+    // WSM's), each detail coefficient k gated by the mean of the extended gate
+    // samples 2k and 2k+1, inverse DWT.  For Haar an odd last sample pairs
+    // with its mirror image, so its detail is 0 and it passes through.
+    // Budget weights are max(r~, 0) (Eq. 5); the ablation modes use max(r, 0)
+    // ("raw") or 1 ("uniform") instead.
+    const int FT = c.wta_F;
+    const int K = (L + FT - 1) / 2;
+    for (int k = threadIdx.x; k < K; k += blockDim.x) {
+        double ca = 0.0, cd = 0.0;
+        for (int j = 0; j < FT; ++j) {
+            const double x = fr[4 * lst[ext_index(2 * k + 1 - j, L, WZ_MODE_SYMMETRIC)]];
+            ca += c.wta_dec_lo[j] * x;
+            cd += c.wta_dec_hi[j] * x;
         }
+        const int m0 = ext_index(2 * k, L, WZ_MODE_SYMMETRIC), m1 = ext_index(2 * k + 1, L, WZ_MODE_SYMMETRIC);
+        const double g = 0.5 * (fr[4 * lst[m0] + 2] + fr[4 * lst[m1] + 2]);
+        cA[k] = ca;
+        cD[k] = g * cd;
+    }
+    __syncthreads();
+    int anypos = 0;
+    for (int m = threadIdx.x; m < L; m += blockDim.x) {
+        double rt = 0.0;
+        const int alo = m >> 1, ahi = min(K - 1, (m + FT - 2) >> 1);
+        for (int ai = alo; ai <= ahi; ++ai) {
+            const int kk = m + FT - 2 - 2 * ai;       // synthesis tap, 0 <= kk < FT
+            rt += c.wta_rec_lo[kk] * cA[ai] + c.wta_rec_hi[kk] * cD[ai];
+        }
+        const int t = lst[m];
+        fr[4 * t + 3] = rt;
+        const double wv = c.temporal_mode == WZ_TEMPORAL_WTA ? rt
+                          : c.temporal_mode == WZ_TEMPORAL_RAW ? fr[4 * t] : 1.0;
+        wgt[m] = fmax(wv, 0.0);
+        anypos |= (wv > 0.0);
     }
     // uniform weights if none is positive
     anypos = __syncthreads_or(anypos);

@@ -79,6 +79,8 @@ struct Ctx {
     int spatial_mode;     // WZ_SPATIAL_*
     int pdl;              // host: launch with programmatic stream serialization
     float dec_lo[kMaxTaps], dec_hi[kMaxTaps], rec_lo[kMaxTaps], rec_hi[kMaxTaps];
+    int wta_F;            // WTA filter taps (temporal DWT, fp64)
+    double wta_dec_lo[kMaxTaps], wta_dec_hi[kMaxTaps], wta_rec_lo[kMaxTaps], wta_rec_hi[kMaxTaps];
 };
 
 // ---- device helpers -------------------------------------------------------

@@ -170,7 +170,7 @@ def wz_condense(features: torch.Tensor, query: torch.Tensor, ratio: float, strea
 
 def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *, lam: float = 1.5,
                    tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
-                   temporal_mode="wta", spatial_mode="wsm",
+                   temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1,
                    workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
                    device_status: torch.Tensor | None = None, kernel_events=None, stream=None):
     """wz_condense_ex.  Returns a dict with tokens, index, budgets, count and relevance.
@@ -194,7 +194,7 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
     a.features, a.T, a.H, a.W, a.D = features.data_ptr(), T, H, W, D
     a.dtype = _dtype_code(features)
     a.query, a.Lq, a.ratio = query.data_ptr(), query.shape[0], ratio
-    a.lam, a.tau, a.wsm_wavelet = lam, tau, wsm_wavelet
+    a.lam, a.tau, a.wsm_wavelet, a.wta_wavelet = lam, tau, wsm_wavelet, wta_wavelet
     a.mode = MODES[mode] if isinstance(mode, str) else int(mode)
     a.path = PATHS[path] if isinstance(path, str) else int(path)
     a.temporal_mode = _enum(TEMPORAL_MODES, temporal_mode)
@@ -223,7 +223,7 @@ def wz_batch_rows(V, T, H, W, ratios):
 
 def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios, *, lam: float = 1.5,
                       tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
-                      temporal_mode="wta", spatial_mode="wsm",
+                      temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1,
                       workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
                       stream=None):
     """wz_condense_batch: features [V,T,H,W,D], queries [sum Lq, D]."""
@@ -245,7 +245,7 @@ def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios,
     a.V, a.features, a.T, a.H, a.W, a.D = V, features.data_ptr(), T, H, W, D
     a.dtype = _dtype_code(features)
     a.queries, a.Lq, a.ratio = queries.data_ptr(), lq, rt
-    a.lam, a.tau, a.wsm_wavelet = lam, tau, wsm_wavelet
+    a.lam, a.tau, a.wsm_wavelet, a.wta_wavelet = lam, tau, wsm_wavelet, wta_wavelet
     a.mode = MODES[mode] if isinstance(mode, str) else int(mode)
     a.path = PATHS[path] if isinstance(path, str) else int(path)
     a.temporal_mode = _enum(TEMPORAL_MODES, temporal_mode)

@@ -110,7 +110,7 @@ def _args(wz, **over):
     (dict(out_index=None), -1), (dict(T=0), -1), (dict(H=0), -1), (dict(D=12), -2),
     (dict(H=65), -2), (dict(T=5000), -2), (dict(Lq=0), -1), (dict(ratio=0.0), -1),
     (dict(ratio=1.01), -1), (dict(ratio=float("nan")), -1), (dict(lam=-1.0), -1),
-    (dict(lam=float("inf")), -1), (dict(wta_wavelet=4), -2), (dict(wta_wavelet=0), -1),
+    (dict(lam=float("inf")), -1), (dict(wta_wavelet=11), -1), (dict(wta_wavelet=0), -1),
     (dict(wsm_wavelet=11), -1), (dict(mode=3), -1), (dict(path=7), -1), (dict(dtype=5), -1),
     (dict(temporal_mode=3), -1), (dict(temporal_mode=-1), -1), (dict(spatial_mode=3), -1),
     (dict(dtype=1, path=1), -2), (dict(features=P + 4), -1), (dict(out_tokens=3 * P + 8), -1),

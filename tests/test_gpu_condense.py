@@ -56,7 +56,8 @@ def test_config_256_frames_sampled(wz):
 
 
 def _random_case(wz, T, H, W, D, Lq, ratio, seed=0, dtype="bf16", **kw):
-    okw = {k: v for k, v in kw.items() if k in ("lam", "tau", "wsm_wavelet", "mode", "temporal_mode", "spatial_mode")}
+    okw = {k: v for k, v in kw.items()
+           if k in ("lam", "tau", "wta_wavelet", "wsm_wavelet", "mode", "temporal_mode", "spatial_mode")}
     X, Q = accepted_random(T, H, W, D, Lq, ratio, seed=seed, dtype=dtype, **okw)
     ref = oracle_run(X, Q, ratio, **okw)
     out = run(wz, X, Q, ratio, **kw)
@@ -82,7 +83,9 @@ def test_shapes(wz, T, H, W, D, Lq, ratio):
 
 
 @pytest.mark.parametrize("kw", [dict(lam=0.0), dict(lam=2.0), dict(wsm_wavelet=1), dict(wsm_wavelet=2),
-                                dict(mode="zero"), dict(mode="periodic"), dict(path="simt")])
+                                dict(mode="zero"), dict(mode="periodic"), dict(path="simt"),
+                                dict(wta_wavelet=4), dict(wta_wavelet=2, wsm_wavelet=1),
+                                dict(wta_wavelet=10, temporal_mode="wta")])
 def test_options(wz, kw):
     _random_case(wz, 10, 13, 13, 128, 6, 0.2, seed=5, **kw)
 

@@ -346,6 +346,22 @@ def test_wta_closed_form():
     check_wta_closed_form(O)
 
 
+@pytest.mark.parametrize("p", [2, 4, 10])
+def test_wta_daubechies_unit_gate_is_identity(p):
+    r = RNG.standard_normal(23)
+    assert np.allclose(O.wta(r, np.ones(23), p), r, atol=1e-12)      # perfect reconstruction
+
+
+@pytest.mark.parametrize("p", [2, 4])
+def test_wta_daubechies_zero_gate_keeps_smooth_signals(p):
+    # a polynomial of degree < p has no detail away from the borders, so the
+    # gate cannot change the interior of the rectified sequence
+    x = np.arange(40, dtype=np.float64)
+    r = 0.3 + 0.01 * x - (0.0002 * x * x if p > 2 else 0.0)
+    out = O.wta(r, np.zeros(40), p)
+    assert np.allclose(out[2 * p:-2 * p], r[2 * p:-2 * p], atol=1e-9)
+
+
 def test_wta_two_element():
     out = O.wta(np.array([1.0, 0.0]), np.array([0.0, 0.5]))
     assert np.allclose(out, [0.5 + 0.25 * 0.5, 0.5 - 0.25 * 0.5])
