@@ -67,6 +67,10 @@ fact; the same list is kept in the design notes):
       replaces the WSM by the plain saliency weighting X~_m = lambda * M_m * X_m
       in the token domain; spatial "none" (the module ablation's Uniform / WTA
       rows) condenses X_m itself.  The default modes are the full method.
+  R19 an external scorer (Section 3.2.1 names BLIP-style matchers as
+      alternatives to the similarity branch) may supply the token saliency
+      a_{t,n} and / or the frame relevance r_t; the pooled features still come
+      from X, since delta_t (Eq. 7) compares frames, not scores.
 """
 
 from __future__ import annotations
@@ -452,13 +456,16 @@ SPATIAL_MODES = ("wsm", "saliency", "none")
 
 def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
              wta_wavelet: int = 1, wsm_wavelet: int = 4, mode: str = "symmetric",
-             token_frames=None, temporal_mode: str = "wta", spatial_mode: str = "wsm") -> dict:
+             token_frames=None, temporal_mode: str = "wta", spatial_mode: str = "wsm",
+             token_scores=None, frame_scores=None) -> dict:
     """Condense features X (T, H, W, D) for query Q (Lq, D) to B tokens.
 
     token_frames: optional iterable of frame indices; when given, the WSM and
     Psi steps run only for those frames (budgets, offsets and the index map are
     always complete), and out_tokens rows of other frames are left as NaN.
     temporal_mode / spatial_mode: the ablation modes of reading R18.
+    token_scores (T, N) / frame_scores (T,): an external scorer's a_{t,n} and
+    r_t (reading R19), replacing the similarity branch's values.
     """
     if temporal_mode not in TEMPORAL_MODES or spatial_mode not in SPATIAL_MODES:
         raise ValueError("unknown mode")
@@ -473,6 +480,10 @@ def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
         U = X[t].reshape(N, D)
         a[t] = token_saliency(U, u_q)
         r[t], vbar[t] = frame_relevance(U, u_q)
+    if token_scores is not None:
+        a = np.asarray(token_scores, dtype=np.float64).reshape(T, N).copy()
+    if frame_scores is not None:
+        r = np.asarray(frame_scores, dtype=np.float64).reshape(T).copy()
     delta, gamma = visual_change(vbar)
     keep = frame_filter(delta, as_float32(tau))
     r_tilde_M = wta(r[keep], gamma[keep], wta_wavelet)

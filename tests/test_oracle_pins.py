@@ -619,6 +619,27 @@ def test_full_mode_differs_from_ablations():
         assert not np.allclose(abl["out_tokens"], full["out_tokens"])
 
 
+def test_external_constant_frame_scores_give_uniform_budgets():
+    # constant r: the Haar details vanish, r~ = r, every quota is equal
+    X = RNG.standard_normal((8, 4, 5, 6))
+    Q = RNG.standard_normal((2, 6))
+    ext = O.condense(X, Q, 0.3, frame_scores=np.full(8, 0.4))
+    uni = O.condense(X, Q, 0.3, temporal_mode="uniform")
+    assert np.array_equal(ext["budgets"], uni["budgets"])
+    assert np.allclose(ext["r"], 0.4) and np.allclose(ext["r_tilde"], 0.4)
+
+
+def test_external_flat_token_scores_remove_the_details():
+    # a flat saliency map is M = 0 (R11), so G = 0 and the WSM keeps LL only:
+    # the same tokens as lambda = 0
+    X = RNG.standard_normal((3, 4, 5, 6))
+    Q = RNG.standard_normal((2, 6))
+    flat = O.condense(X, Q, 0.5, token_scores=np.full((3, 20), 0.7))
+    low = O.condense(X, Q, 0.5, lam=0.0)
+    assert np.array_equal(flat["budgets"], low["budgets"])
+    assert np.allclose(flat["out_tokens"], low["out_tokens"], atol=1e-12)
+
+
 # ----------------------------------------------------------------------------
 # Mutation tests: a planted mistake in the oracle makes a pin fail
 # ----------------------------------------------------------------------------
