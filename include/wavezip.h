@@ -150,6 +150,10 @@ typedef struct {
     int path;                /* WZ_PATH_*                                    */
     int temporal_mode;       /* WZ_TEMPORAL_*, default WTA                   */
     int spatial_mode;        /* WZ_SPATIAL_*, default WSM                    */
+    const float *token_scores; /* [T][N] f32 device, an external scorer's    */
+                             /* a_{t,n} (Section 3.2.1) replacing the        */
+                             /* similarity branch's; nullable                */
+    const float *frame_scores; /* [T] f32 device, external r_t; nullable     */
     void *out_tokens;        /* [B][D], dtype                                */
     int32_t *out_index;      /* [B][3]                                       */
     int32_t *out_budgets;    /* [T] n_t (0 for filtered frames); nullable    */
@@ -199,6 +203,8 @@ typedef struct {
     float lambda, tau;
     int wta_wavelet, wsm_wavelet, mode, path;
     int temporal_mode, spatial_mode;   /* WZ_TEMPORAL_*, WZ_SPATIAL_* */
+    const float *token_scores;         /* [V][T][N] device, nullable   */
+    const float *frame_scores;         /* [V][T] device, nullable      */
     void *out_tokens;
     int32_t *out_index;
     int64_t *row_offsets;    /* host, [V+1], nullable */

@@ -223,6 +223,7 @@ struct CondenseRequest {
     std::vector<int> Lq;
     std::vector<float> ratio;
     Common m;
+    const float *token_scores = nullptr, *frame_scores = nullptr;
     void *out_tokens;
     int32_t *out_index, *out_budgets, *out_count, *device_status;
     float *out_relevance;
@@ -239,6 +240,7 @@ int validate(const CondenseRequest &r, std::vector<int64_t> &B, int64_t &rows) {
     if (st != WZ_OK) return st;
     if (!r.features || !r.queries) return WZ_ERR_INVALID_ARG;
     if (!aligned(r.features, 16) || !aligned(r.queries, 16)) return WZ_ERR_INVALID_ARG;
+    if (!aligned(r.token_scores, 4) || !aligned(r.frame_scores, 4)) return WZ_ERR_INVALID_ARG;
     B.assign(r.V, 0);
     rows = 0;
     int64_t qrows = 0;
@@ -268,6 +270,8 @@ int run_condense(const CondenseRequest &r) {
     c.path = resolve_path(r.m.path, r.dtype);
     c.temporal_mode = r.m.temporal_mode;
     c.spatial_mode = r.m.spatial_mode;
+    c.ext_a = r.token_scores;
+    c.ext_r = r.frame_scores;
     c.pdl = r.events ? 0 : 1;      // an event between two kernels would break the overlap
     set_filters(c, r.m.wsm_wavelet);
     set_wta_filters(c, r.m.wta_wavelet);
@@ -394,6 +398,8 @@ int wz_condense_ex(const wz_condense_args *a) {
     r.ratio.assign(1, a->ratio);
     r.m = Common{a->lambda, a->tau, a->wta_wavelet, a->wsm_wavelet, a->mode, a->path, a->temporal_mode,
                  a->spatial_mode};
+    r.token_scores = a->token_scores;
+    r.frame_scores = a->frame_scores;
     r.out_tokens = a->out_tokens;
     r.out_index = a->out_index;
     r.out_budgets = a->out_budgets;
@@ -449,6 +455,8 @@ int wz_condense_batch(const wz_batch_args *a) {
     r.ratio.assign(a->ratio, a->ratio + a->V);
     r.m = Common{a->lambda, a->tau, a->wta_wavelet, a->wsm_wavelet, a->mode, a->path, a->temporal_mode,
                  a->spatial_mode};
+    r.token_scores = a->token_scores;
+    r.frame_scores = a->frame_scores;
     r.out_tokens = a->out_tokens;
     r.out_index = a->out_index;
     r.out_budgets = a->out_budgets;

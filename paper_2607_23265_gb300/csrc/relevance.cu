@@ -365,7 +365,7 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
 __device__ void frame_gate(const Ctx &c, int64_t f, float *red) {
     __shared__ float M[WZ_MAX_HW * WZ_MAX_HW];
     const int N = c.N, H = c.H, W = c.W, hp = c.hp, wp = c.wp;
-    const float *a = c.a + f * N;
+    const float *a = (c.ext_a ? c.ext_a : c.a) + f * N;   // an external scorer's a_{t,n} if given
     float lo = INFINITY, hi = -INFINITY;
     for (int k = threadIdx.x; k < N; k += blockDim.x) {
         const float x = a[k];
@@ -475,7 +475,8 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
             pp += (double)wsum[w][4];
         }
         const double qn = sqrt(qq);
-        const double r = (vv > 0.0 && qn > 0.0) ? vq / (sqrt(vv) * qn) : 0.0;
+        const double r = c.ext_r ? (double)c.ext_r[f]                      // an external scorer's r_t
+                                 : (vv > 0.0 && qn > 0.0) ? vq / (sqrt(vv) * qn) : 0.0;
         double d = 0.0;
         if (t > 0) {
             const double den = sqrt(vv * pp);

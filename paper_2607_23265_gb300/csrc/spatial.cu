@@ -111,7 +111,7 @@ __device__ void plain_operator_rows(const Ctx &c, const SpatialSmem &L, float *s
     float *stg = sm + L.stage, *M = sm + L.M, *red = sm + L.red;
     const bool sal = c.spatial_mode == WZ_SPATIAL_SALIENCY;
     if (sal) {
-        const float *a = c.a + f * N;
+        const float *a = (c.ext_a ? c.ext_a : c.a) + f * N;
         float lo = INFINITY, hi = -INFINITY;
         for (int k = tid; k < N; k += blockDim.x) {
             const float x = a[k];

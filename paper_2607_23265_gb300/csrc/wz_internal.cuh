@@ -77,6 +77,8 @@ struct Ctx {
     int path;             // resolved WZ_PATH_TENSOR or WZ_PATH_SIMT
     int temporal_mode;    // WZ_TEMPORAL_*
     int spatial_mode;     // WZ_SPATIAL_*
+    const float *ext_a;   // [V*T][N] external token scores, or null
+    const float *ext_r;   // [V*T] external frame scores, or null
     int pdl;              // host: launch with programmatic stream serialization
     float dec_lo[kMaxTaps], dec_hi[kMaxTaps], rec_lo[kMaxTaps], rec_hi[kMaxTaps];
     int wta_F;            // WTA filter taps (temporal DWT, fp64)

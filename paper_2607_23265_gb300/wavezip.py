@@ -33,6 +33,12 @@ def _enum(table, v):
     return table[v] if isinstance(v, str) else int(v)
 
 
+def _f32_scores(x: torch.Tensor, shape, name: str) -> torch.Tensor:
+    if x.dtype != torch.float32 or not x.is_cuda or tuple(x.shape) != tuple(shape):
+        raise ValueError(f"{name} must be a float32 CUDA tensor of shape {tuple(shape)}")
+    return x.contiguous()
+
+
 class WaveZipError(RuntimeError):
     def __init__(self, status: int, where: str):
         self.status = status
@@ -45,6 +51,7 @@ class CondenseArgs(C.Structure):
         ("dtype", C.c_int), ("query", C.c_void_p), ("Lq", C.c_int), ("ratio", C.c_float),
         ("lam", C.c_float), ("tau", C.c_float), ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int),
         ("mode", C.c_int), ("path", C.c_int), ("temporal_mode", C.c_int), ("spatial_mode", C.c_int),
+        ("token_scores", C.c_void_p), ("frame_scores", C.c_void_p),
         ("out_tokens", C.c_void_p), ("out_index", C.c_void_p),
         ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
         ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
@@ -59,6 +66,7 @@ class BatchArgs(C.Structure):
         ("ratio", C.POINTER(C.c_float)), ("lam", C.c_float), ("tau", C.c_float),
         ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int), ("mode", C.c_int), ("path", C.c_int),
         ("temporal_mode", C.c_int), ("spatial_mode", C.c_int),
+        ("token_scores", C.c_void_p), ("frame_scores", C.c_void_p),
         ("out_tokens", C.c_void_p), ("out_index", C.c_void_p), ("row_offsets", C.POINTER(C.c_int64)),
         ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
         ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
@@ -171,12 +179,15 @@ def wz_condense(features: torch.Tensor, query: torch.Tensor, ratio: float, strea
 def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *, lam: float = 1.5,
                    tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
                    temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1,
+                   token_scores: torch.Tensor | None = None, frame_scores: torch.Tensor | None = None,
                    workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
                    device_status: torch.Tensor | None = None, kernel_events=None, stream=None):
     """wz_condense_ex.  Returns a dict with tokens, index, budgets, count and relevance.
 
     kernel_events: optional list of 2*NUM_KERNELS recorded torch.cuda.Event
-    objects; event 2k / 2k+1 is recorded right before / after kernel k."""
+    objects; event 2k / 2k+1 is recorded right before / after kernel k.
+    token_scores [T, H*W] / frame_scores [T]: float32 device tensors of an
+    external scorer (None: the similarity branch's own scores)."""
     features = _cuda_contig(features, "features")
     query = _cuda_contig(query, "query")
     T, H, W, D = features.shape
@@ -199,6 +210,12 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
     a.path = PATHS[path] if isinstance(path, str) else int(path)
     a.temporal_mode = _enum(TEMPORAL_MODES, temporal_mode)
     a.spatial_mode = _enum(SPATIAL_MODES, spatial_mode)
+    if token_scores is not None:
+        token_scores = _f32_scores(token_scores, (T, H * W), "token_scores")
+        a.token_scores = token_scores.data_ptr()
+    if frame_scores is not None:
+        frame_scores = _f32_scores(frame_scores, (T,), "frame_scores")
+        a.frame_scores = frame_scores.data_ptr()
     a.out_tokens, a.out_index = tokens.data_ptr(), index.data_ptr()
     a.out_budgets, a.out_count, a.out_relevance = budgets.data_ptr(), count.data_ptr(), rel.data_ptr()
     if workspace is not None:

@@ -112,6 +112,29 @@ def test_ablation_saliency_fp32(wz):
     _random_case(wz, 6, 9, 11, 64, 4, 0.3, seed=11, dtype="f32", spatial_mode="saliency")
 
 
+@pytest.mark.parametrize("which", ["both", "tokens", "frames"])
+def test_external_scores(wz, which):
+    from helpers import MIN_MARGIN
+    g = np.random.default_rng(21)
+    T, H, W, D, Lq, ratio = 10, 13, 13, 128, 6, 0.2
+    for attempt in range(20):
+        a_ext = g.random((T, H * W)).astype(np.float32)
+        r_ext = g.normal(0.1, 0.2, T).astype(np.float32)
+        kw = {}
+        if which in ("both", "tokens"):
+            kw["token_scores"] = a_ext
+        if which in ("both", "frames"):
+            kw["frame_scores"] = r_ext
+        X, Q = wl.random_video(T, H, W, D, Lq, seed=40 + attempt)
+        ref = oracle_run(X, Q, ratio, **kw)
+        if O.decision_margins(ref) >= MIN_MARGIN:
+            break
+    out = run(wz, X, Q, ratio, **{k: torch.from_numpy(v).cuda() for k, v in kw.items()})
+    compare_condense(out, ref, X.dtype)
+    if "frame_scores" in kw:
+        assert np.allclose(out["relevance"][:, 0].cpu().numpy(), r_ext, atol=0)
+
+
 def test_fp32_features(wz):
     _random_case(wz, 6, 14, 14, 96, 4, 0.25, seed=3, dtype="f32")
 
