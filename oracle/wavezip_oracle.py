@@ -67,6 +67,10 @@ fact; the same list is kept in the design notes):
       replaces the WSM by the plain saliency weighting X~_m = lambda * M_m * X_m
       in the token domain; spatial "none" (the module ablation's Uniform / WTA
       rows) condenses X_m itself.  The default modes are the full method.
+  R20 "bior4.4" is the biorthogonal CDF 9/7 pair (the PyWavelets name, as
+      for db4), with 10-tap arrays laid out as in that library: analysis
+      lowpass in dec_lo[1..9], synthesis lowpass in rec_lo[1..7]; the paper
+      evaluates it for both WTA and WSM ("Wavelet Basis" ablation).
   R19 an external scorer (Section 3.2.1 names BLIP-style matchers as
       alternatives to the similarity branch) may supply the token saliency
       a_{t,n} and / or the frame relevance r_t; the pooled features still come
@@ -110,12 +114,57 @@ def daubechies_lowpass(p: int) -> np.ndarray:
     return h * (math.sqrt(2.0) / h.sum())
 
 
-def wavelet_filters(p: int) -> dict:
-    """Analysis / synthesis filter bank of the orthogonal wavelet db<p>.
+BIOR44 = 44     # identifier of the biorthogonal wavelet bior4.4 (CDF 9/7)
 
-    rec_lo is the minimum-phase filter, dec_lo its reverse, and the high-pass
-    pair is the alternating flip: rec_hi[k] = (-1)^k rec_lo[F-1-k].
+
+def cdf97_lowpass():
+    """(h, h~): the 7-tap synthesis and 9-tap analysis lowpass filters of bior4.4.
+
+    Same product polynomial as db4 (p = 4): cos^8(w/2) P(sin^2(w/2)), split
+    into two symmetric (zero-phase) factors cos^4 q(sin^2) and cos^4 q~(sin^2)
+    with q q~ = P: the real root of P goes to q (7 taps), the complex pair to
+    q~ (9 taps) (Cohen, Daubechies, Feauveau 1992).  sin^2(w/2) is
+    (-z + 2 - 1/z) / 4 and cos^2(w/2) is (z + 2 + 1/z) / 4; each filter is
+    normalised to sum sqrt(2).
     """
+    P = [comb(3 + k, k) for k in range(4)]               # 1 + 4y + 10y^2 + 20y^3
+    roots = np.roots(P[::-1])
+    y_r = float(np.real(roots[np.argmin(np.abs(np.imag(roots)))]))
+    y_c = roots[np.argmax(np.imag(roots))]
+    cos4 = np.array([1.0, 4.0, 6.0, 4.0, 1.0]) / 16.0
+    s_taps = np.array([-1.0, 2.0, -1.0]) / 4.0            # sin^2(w/2)
+    q = np.array([0.0, 1.0, 0.0]) - s_taps / y_r
+    alpha = float(np.real(1.0 / y_c + 1.0 / np.conj(y_c)))
+    beta = float(np.real(1.0 / (y_c * np.conj(y_c))))
+    qt = (np.array([0.0, 0.0, 1.0, 0.0, 0.0]) - alpha * np.pad(s_taps, 1)
+          + beta * np.convolve(s_taps, s_taps))
+    h = np.convolve(cos4, q)
+    ht = np.convolve(cos4, qt)
+    return h * (math.sqrt(2.0) / h.sum()), ht * (math.sqrt(2.0) / ht.sum())
+
+
+def wavelet_filters(p: int) -> dict:
+    """Analysis / synthesis filter bank of the orthogonal wavelet db<p>, or of
+    bior4.4 for p = BIOR44.
+
+    db<p>: rec_lo is the minimum-phase filter, dec_lo its reverse, and the
+    high-pass pair is the alternating flip: rec_hi[k] = (-1)^k rec_lo[F-1-k].
+    bior4.4 (reading R20): F = 10 taps; the 9-tap analysis lowpass occupies
+    dec_lo[1..9] and the 7-tap synthesis lowpass rec_lo[1..7]; each high-pass
+    filter is the alternating flip of the OTHER side's lowpass
+    (rec_hi[k] = (-1)^k dec_lo[F-1-k] reversed, dec_hi from rec_lo).
+    """
+    if p == BIOR44:
+        h, ht = cdf97_lowpass()
+        F = 10
+        rec_lo = np.zeros(F)
+        rec_lo[1:8] = h
+        ht_pad = np.zeros(F)
+        ht_pad[0:9] = ht
+        dec_lo = ht_pad[::-1].copy()
+        rec_hi = np.array([(-1.0) ** k * ht_pad[F - 1 - k] for k in range(F)])
+        g = np.array([(-1.0) ** k * rec_lo[F - 1 - k] for k in range(F)])
+        return {"dec_lo": dec_lo, "dec_hi": g[::-1].copy(), "rec_lo": rec_lo, "rec_hi": rec_hi, "F": F}
     rec_lo = daubechies_lowpass(p)
     F = rec_lo.size
     rec_hi = np.array([(-1.0) ** k * rec_lo[F - 1 - k] for k in range(F)])

@@ -89,6 +89,42 @@ def test_db4_published_taps(golden_dir):
     check_db4_table(O, golden_dir)
 
 
+def check_bior44_published(o, golden_dir):
+    rows = _golden(os.path.join(golden_dir, "cdf97_taps.txt"))
+    f = o.wavelet_filters(o.BIOR44)
+    assert f["F"] == 10
+    ana = f["dec_lo"][1:10] / math.sqrt(2.0)             # DC gain 1, 9 taps
+    syn = f["rec_lo"][1:8] * math.sqrt(2.0)              # DC gain 2, 7 taps
+    for taps, row in ((ana, rows[0]), (syn, rows[1])):
+        c = taps.size // 2
+        for k, v in enumerate(row):
+            assert abs(taps[c + k] - v) < 1e-12 and abs(taps[c - k] - v) < 1e-12
+
+
+def test_bior44_published_taps(golden_dir):
+    check_bior44_published(O, golden_dir)
+
+
+def test_bior44_biorthogonality_and_moments():
+    f = O.wavelet_filters(O.BIOR44)
+    F = f["F"]
+    # analysis and synthesis lowpass are dual: sum_k h~[k] h[k + 2m] = delta_m
+    # (as z-transforms aligned by the layout); checked through perfect
+    # reconstruction of every length and of shifted impulses
+    for n in (1, 2, 3, 4, 7, 16, 27, 33):
+        for mode in ("symmetric", "periodic", "zero"):
+            if mode == "periodic" and n < 2:
+                continue
+            x = RNG.standard_normal(n)
+            A, D = O.dwt1d(x, f, mode)
+            assert np.allclose(O.idwt1d(A, D, n, f), x, atol=1e-12) or mode == "zero"
+    # four vanishing moments on both sides
+    k = np.arange(F, dtype=np.float64)
+    for hp in (f["dec_hi"], f["rec_hi"]):
+        for m in range(4):
+            assert abs(np.sum(hp * k ** m)) < 1e-9 * (F ** m)
+
+
 @pytest.mark.parametrize("p", [1, 2, 3, 4, 5, 6, 8])
 def test_filter_identities(p):
     check_filter_identities(O, p)
@@ -764,3 +800,11 @@ def test_mutation_budget_without_remainders_breaks_uniform_pin():
         return n, {"alloc_gap": math.inf, "cap_gap": math.inf, "max_r": 1.0}
     m = _mutant(allocate_budget=floors_only)
     assert _fails(check_uniform_mode, m)
+
+
+def test_mutation_bior44_normalisation_breaks_published_pin(golden_dir):
+    def unit_sum():
+        h, ht = OM.cdf97_lowpass()
+        return h / h.sum(), ht / ht.sum()                # a plausible slip: DC gain 1, not sqrt(2)
+    m = _mutant(cdf97_lowpass=unit_sum)
+    assert _fails(check_bior44_published, m, golden_dir)
