@@ -97,10 +97,13 @@ typedef struct CUstream_st *wz_stream_t;
 #define WZ_SPATIAL_SALIENCY  1 /* "Saliency-Only": lambda * M_t * X_t, no wavelets */
 #define WZ_SPATIAL_NONE      2 /* no modulation: Psi of the features itself       */
 
-/* Wavelets are Daubechies filters named by their vanishing moments p
- * (2p taps): 1 = Haar, 4 = db4.  1 <= p <= 10. */
-#define WZ_WAVELET_HAAR 1
-#define WZ_WAVELET_DB4  4
+/* Wavelets: Daubechies filters named by their vanishing moments p (2p
+ * taps), 1 = Haar, 4 = db4, 1 <= p <= 10; and the biorthogonal bior4.4
+ * (CDF 9/7, 10-tap arrays), the third basis of the paper's "Wavelet Basis"
+ * ablation (Section 4). */
+#define WZ_WAVELET_HAAR   1
+#define WZ_WAVELET_DB4    4
+#define WZ_WAVELET_BIOR44 44
 
 /* Limits of this build (WZ_ERR_UNSUPPORTED beyond them). */
 #define WZ_MAX_HW      64    /* H, W <= 64                                  */
@@ -143,9 +146,10 @@ typedef struct {
     float ratio;             /* rho in (0, 1]                                */
     float lambda;            /* WSM gate strength (Eq. 12), default 1.5      */
     float tau;               /* frame-filter threshold on delta, default 0   */
-    int wta_wavelet;         /* Daubechies order 1..10 of the WTA DWT,       */
+    int wta_wavelet;         /* WTA wavelet: 1..10 or WZ_WAVELET_BIOR44,     */
                              /* default 1 (Haar, Eq. 8-10)                   */
-    int wsm_wavelet;         /* Daubechies order 1..10, default 4            */
+    int wsm_wavelet;         /* WSM wavelet: 1..10 or WZ_WAVELET_BIOR44,     */
+                             /* default 4 (db4)                              */
     int mode;                /* WZ_MODE_* extension for the WSM DWT          */
     int path;                /* WZ_PATH_*                                    */
     int temporal_mode;       /* WZ_TEMPORAL_*, default WTA                   */
@@ -277,15 +281,18 @@ WZ_API int wz_relevance_static(const void *features, int T, int H, int W, int D,
 /* Single-level DWT (Eq. 8, 10, 11, 14)                                      */
 /* ------------------------------------------------------------------------ */
 
-/* Coefficients per band for a length-n signal: floor((n + 2p - 1) / 2).
- * Returns -1 for n < 1 or an unsupported wavelet. */
+/* Coefficients per band for a length-n signal: floor((n + F - 1) / 2), F the
+ * wavelet's taps (2p, or 10 for bior4.4).  Returns -1 for n < 1 or an
+ * unsupported wavelet. */
 WZ_API int wz_dwt_len(int n, int wavelet);
 
 /*
- * Filter bank of db<wavelet> as derived by this library (HOST arrays of 2p
- * doubles each; any may be NULL).  rec_lo is minimum phase with sum sqrt(2);
- * dec_lo is its reverse; rec_hi[k] = (-1)^k rec_lo[2p-1-k]; dec_hi reverses
- * rec_hi.
+ * Filter bank of the wavelet as derived by this library (HOST arrays of F
+ * doubles each; any may be NULL).  db<p>: rec_lo is minimum phase with sum
+ * sqrt(2); dec_lo is its reverse; rec_hi[k] = (-1)^k rec_lo[2p-1-k]; dec_hi
+ * reverses rec_hi.  bior4.4: the 9-tap analysis lowpass in dec_lo[1..9], the
+ * 7-tap synthesis lowpass in rec_lo[1..7], both with sum sqrt(2); each
+ * high-pass filter is the alternating flip of the other side's lowpass.
  */
 WZ_API int wz_wavelet_filters(int wavelet, double *dec_lo, double *dec_hi,
                        double *rec_lo, double *rec_hi);

@@ -117,8 +117,7 @@ struct Common {
 
 int check_common(const Common &m, int dtype) {
     if (!std::isfinite(m.lambda) || m.lambda < 0.f || !std::isfinite(m.tau)) return WZ_ERR_INVALID_ARG;
-    if (m.wta_wavelet < 1 || m.wta_wavelet > 10) return WZ_ERR_INVALID_ARG;
-    if (m.wsm_wavelet < 1 || m.wsm_wavelet > 10) return WZ_ERR_INVALID_ARG;
+    if (wavelet_taps(m.wta_wavelet) == 0 || wavelet_taps(m.wsm_wavelet) == 0) return WZ_ERR_INVALID_ARG;
     if (m.mode < WZ_MODE_SYMMETRIC || m.mode > WZ_MODE_PERIODIC) return WZ_ERR_INVALID_ARG;
     if (m.path < WZ_PATH_AUTO || m.path > WZ_PATH_SIMT) return WZ_ERR_INVALID_ARG;
     if (m.path == WZ_PATH_TENSOR && dtype != WZ_DTYPE_BF16) return WZ_ERR_UNSUPPORTED;
@@ -134,8 +133,8 @@ int resolve_path(int path, int dtype) {
 
 void set_filters(Ctx &c, int p) {
     double dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
-    daubechies(p, dl, dh, rl, rh);
-    c.F = 2 * p;
+    wavelet_bank(p, dl, dh, rl, rh);
+    c.F = wavelet_taps(p);
     for (int k = 0; k < kMaxTaps; ++k) {
         c.dec_lo[k] = k < c.F ? (float)dl[k] : 0.f;
         c.dec_hi[k] = k < c.F ? (float)dh[k] : 0.f;
@@ -146,8 +145,8 @@ void set_filters(Ctx &c, int p) {
 
 void set_wta_filters(Ctx &c, int p) {
     double dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
-    daubechies(p, dl, dh, rl, rh);
-    c.wta_F = 2 * p;
+    wavelet_bank(p, dl, dh, rl, rh);
+    c.wta_F = wavelet_taps(p);
     for (int k = 0; k < kMaxTaps; ++k) {
         c.wta_dec_lo[k] = k < c.wta_F ? dl[k] : 0.0;
         c.wta_dec_hi[k] = k < c.wta_F ? dh[k] : 0.0;
@@ -515,19 +514,20 @@ int wz_relevance(const void *features, int T, int H, int W, int D, int dtype, co
 }
 
 int wz_dwt_len(int n, int wavelet) {
-    if (n < 1 || wavelet < 1 || wavelet > 10) return -1;
-    return (n + 2 * wavelet - 1) / 2;
+    const int F = wavelet_taps(wavelet);
+    if (n < 1 || F == 0) return -1;
+    return (n + F - 1) / 2;
 }
 
 int wz_wavelet_filters(int wavelet, double *dec_lo, double *dec_hi, double *rec_lo, double *rec_hi) {
-    if (wavelet < 1 || wavelet > 10) return WZ_ERR_INVALID_ARG;
-    return daubechies(wavelet, dec_lo, dec_hi, rec_lo, rec_hi) ? WZ_OK : WZ_ERR_INVALID_ARG;
+    if (wavelet_taps(wavelet) == 0) return WZ_ERR_INVALID_ARG;
+    return wavelet_bank(wavelet, dec_lo, dec_hi, rec_lo, rec_hi) ? WZ_OK : WZ_ERR_INVALID_ARG;
 }
 
 static void float_taps(int p, float *dl, float *dh, float *rl, float *rh) {
     double a[kMaxTaps], b[kMaxTaps], c[kMaxTaps], d[kMaxTaps];
-    daubechies(p, a, b, c, d);
-    for (int k = 0; k < 2 * p; ++k) {
+    wavelet_bank(p, a, b, c, d);
+    for (int k = 0; k < wavelet_taps(p); ++k) {
         dl[k] = (float)a[k];
         dh[k] = (float)b[k];
         rl[k] = (float)c[k];
@@ -537,46 +537,46 @@ static void float_taps(int p, float *dl, float *dh, float *rl, float *rh) {
 
 int wz_dwt1d(const float *x, int rows, int L, int wavelet, int mode, float *cA, float *cD,
              wz_stream_t stream) {
-    if (rows < 0 || L < 1 || wavelet < 1 || wavelet > 10 || mode < 0 || mode > 2) return WZ_ERR_INVALID_ARG;
+    if (rows < 0 || L < 1 || wavelet_taps(wavelet) == 0 || mode < 0 || mode > 2) return WZ_ERR_INVALID_ARG;
     if (rows > 0 && (!x || !cA || !cD)) return WZ_ERR_INVALID_ARG;
     float dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
     float_taps(wavelet, dl, dh, rl, rh);
-    WZ_CUDA(launch_dwt1d(x, rows, L, 2 * wavelet, mode, dl, dh, cA, cD, (cudaStream_t)stream));
+    WZ_CUDA(launch_dwt1d(x, rows, L, wavelet_taps(wavelet), mode, dl, dh, cA, cD, (cudaStream_t)stream));
     return WZ_OK;
 }
 
 int wz_idwt1d(const float *cA, const float *cD, int rows, int L, int wavelet, float *x,
               wz_stream_t stream) {
-    if (rows < 0 || L < 1 || wavelet < 1 || wavelet > 10) return WZ_ERR_INVALID_ARG;
+    if (rows < 0 || L < 1 || wavelet_taps(wavelet) == 0) return WZ_ERR_INVALID_ARG;
     if (rows > 0 && (!x || !cA || !cD)) return WZ_ERR_INVALID_ARG;
     float dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
     float_taps(wavelet, dl, dh, rl, rh);
-    WZ_CUDA(launch_idwt1d(cA, cD, rows, L, 2 * wavelet, rl, rh, x, (cudaStream_t)stream));
+    WZ_CUDA(launch_idwt1d(cA, cD, rows, L, wavelet_taps(wavelet), rl, rh, x, (cudaStream_t)stream));
     return WZ_OK;
 }
 
 int wz_dwt2d(const void *features, int T, int H, int W, int D, int dtype, int wavelet, int mode,
              float *LL, float *LH, float *HL, float *HH, wz_stream_t stream) {
-    if (T < 1 || H < 1 || W < 1 || D < 1 || wavelet < 1 || wavelet > 10 || mode < 0 || mode > 2)
+    if (T < 1 || H < 1 || W < 1 || D < 1 || wavelet_taps(wavelet) == 0 || mode < 0 || mode > 2)
         return WZ_ERR_INVALID_ARG;
     if (dtype != WZ_DTYPE_BF16 && dtype != WZ_DTYPE_F32) return WZ_ERR_INVALID_ARG;
     if (H > WZ_MAX_HW || W > WZ_MAX_HW || T > 65535) return WZ_ERR_UNSUPPORTED;
     if (!features || !LL || !LH || !HL || !HH) return WZ_ERR_INVALID_ARG;
     float dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
     float_taps(wavelet, dl, dh, rl, rh);
-    WZ_CUDA(launch_dwt2d(features, dtype, T, H, W, D, 2 * wavelet, mode, dl, dh, LL, LH, HL, HH,
+    WZ_CUDA(launch_dwt2d(features, dtype, T, H, W, D, wavelet_taps(wavelet), mode, dl, dh, LL, LH, HL, HH,
                          (cudaStream_t)stream));
     return WZ_OK;
 }
 
 int wz_idwt2d(const float *LL, const float *LH, const float *HL, const float *HH, int T, int H, int W,
               int D, int wavelet, float *out, wz_stream_t stream) {
-    if (T < 1 || H < 1 || W < 1 || D < 1 || wavelet < 1 || wavelet > 10) return WZ_ERR_INVALID_ARG;
+    if (T < 1 || H < 1 || W < 1 || D < 1 || wavelet_taps(wavelet) == 0) return WZ_ERR_INVALID_ARG;
     if (H > WZ_MAX_HW || W > WZ_MAX_HW || T > 65535) return WZ_ERR_UNSUPPORTED;
     if (!out || !LL || !LH || !HL || !HH) return WZ_ERR_INVALID_ARG;
     float dl[kMaxTaps], dh[kMaxTaps], rl[kMaxTaps], rh[kMaxTaps];
     float_taps(wavelet, dl, dh, rl, rh);
-    WZ_CUDA(launch_idwt2d(LL, LH, HL, HH, T, H, W, D, 2 * wavelet, rl, rh, out, (cudaStream_t)stream));
+    WZ_CUDA(launch_idwt2d(LL, LH, HL, HH, T, H, W, D, wavelet_taps(wavelet), rl, rh, out, (cudaStream_t)stream));
     return WZ_OK;
 }
 

@@ -1,4 +1,5 @@
-// Daubechies filter banks by spectral factorisation (host code).
+// Wavelet filter banks by spectral factorisation (host code): Daubechies
+// db1-db10 and the biorthogonal bior4.4.
 //
 // The WSM uses db4 and the WTA Haar (Section 4.1; Fig. "wavelet ablation"
 // names the bases).  The filter of order p is the minimum-phase square root
@@ -109,6 +110,69 @@ bool daubechies(int p, double *dec_lo, double *dec_hi, double *rec_lo, double *r
         if (dec_hi) dec_hi[F - 1 - k] = (double)g;
     }
     return true;
+}
+
+// bior4.4 (CDF 9/7): the product filter of db4, cos^8(w/2) P(sin^2(w/2)) with
+// P(y) = 1 + 4y + 10y^2 + 20y^3, split into two zero-phase factors
+// cos^4 q(sin^2) (7 taps, q from the real root of P) and cos^4 q~(sin^2)
+// (9 taps, q~ from the complex pair), each normalised to sum sqrt(2); in z,
+// cos^2(w/2) = (z + 2 + 1/z) / 4 and sin^2(w/2) = (-z + 2 - 1/z) / 4.
+// 10-tap layout: analysis lowpass in dec_lo[1..9], synthesis lowpass in
+// rec_lo[1..7]; each high-pass is the alternating flip of the other side's
+// lowpass.
+bool bior44(double *dec_lo, double *dec_hi, double *rec_lo, double *rec_hi) {
+    const std::vector<long double> P = {1.0L, 4.0L, 10.0L, 20.0L};
+    const std::vector<cld> roots = poly_roots(P);
+    cld yr = roots[0], yc = roots[0];
+    for (const cld &y : roots) {
+        if (std::fabs(y.imag()) < std::fabs(yr.imag())) yr = y;
+        if (y.imag() > yc.imag()) yc = y;
+    }
+    auto conv = [](const std::vector<long double> &a, const std::vector<long double> &b) {
+        std::vector<long double> r(a.size() + b.size() - 1, 0.0L);
+        for (size_t i = 0; i < a.size(); ++i)
+            for (size_t j = 0; j < b.size(); ++j) r[i + j] += a[i] * b[j];
+        return r;
+    };
+    const std::vector<long double> cos4 = {1.0L / 16, 4.0L / 16, 6.0L / 16, 4.0L / 16, 1.0L / 16};
+    const std::vector<long double> s2 = {-0.25L, 0.5L, -0.25L};           // sin^2(w/2)
+    const long double inv_r = 1.0L / yr.real();
+    const std::vector<long double> q = {-s2[0] * inv_r, 1.0L - s2[1] * inv_r, -s2[2] * inv_r};
+    const cld inv_c = 1.0L / yc;
+    const long double alpha = 2.0L * inv_c.real();                      // 1/y + 1/conj(y)
+    const long double beta = std::norm(inv_c);                            // 1/|y|^2
+    const std::vector<long double> ss = conv(s2, s2);
+    std::vector<long double> qt(5, 0.0L);
+    qt[2] = 1.0L;
+    for (int k = 0; k < 3; ++k) qt[k + 1] -= alpha * s2[k];
+    for (int k = 0; k < 5; ++k) qt[k] += beta * ss[k];
+    std::vector<long double> h = conv(cos4, q), ht = conv(cos4, qt);   // 7 and 9 taps
+    long double sh = 0.0L, sht = 0.0L;
+    for (long double v : h) sh += v;
+    for (long double v : ht) sht += v;
+    const int F = 10;
+    long double rl[F] = {}, htp[F] = {};
+    for (int k = 0; k < 7; ++k) rl[1 + k] = h[k] * std::sqrt(2.0L) / sh;
+    for (int k = 0; k < 9; ++k) htp[k] = ht[k] * std::sqrt(2.0L) / sht;
+    for (int k = 0; k < F; ++k) {
+        const long double sg = (k & 1) ? -1.0L : 1.0L;
+        if (rec_lo) rec_lo[k] = (double)rl[k];
+        if (dec_lo) dec_lo[k] = (double)htp[F - 1 - k];
+        if (rec_hi) rec_hi[k] = (double)(sg * htp[F - 1 - k]);
+        if (dec_hi) dec_hi[F - 1 - k] = (double)(sg * rl[F - 1 - k]);
+    }
+    return true;
+}
+
+int wavelet_taps(int wavelet) {
+    if (wavelet >= 1 && 2 * wavelet <= kMaxTaps) return 2 * wavelet;
+    if (wavelet == WZ_WAVELET_BIOR44) return 10;
+    return 0;
+}
+
+bool wavelet_bank(int wavelet, double *dec_lo, double *dec_hi, double *rec_lo, double *rec_hi) {
+    if (wavelet == WZ_WAVELET_BIOR44) return bior44(dec_lo, dec_hi, rec_lo, rec_hi);
+    return daubechies(wavelet, dec_lo, dec_hi, rec_lo, rec_hi);
 }
 
 }  // namespace wz

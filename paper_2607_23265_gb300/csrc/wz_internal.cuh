@@ -290,5 +290,8 @@ cudaError_t launch_idwt2d(const float *LL, const float *LH, const float *HL, con
 
 // Host: Daubechies filter bank of order p (2p taps); false if p is out of range.
 bool daubechies(int p, double *dec_lo, double *dec_hi, double *rec_lo, double *rec_hi);
+bool bior44(double *dec_lo, double *dec_hi, double *rec_lo, double *rec_hi);
+int wavelet_taps(int wavelet);   // 2p for db<p>, 10 for bior4.4, 0 if unsupported
+bool wavelet_bank(int wavelet, double *dec_lo, double *dec_hi, double *rec_lo, double *rec_hi);
 
 }  // namespace wz

@@ -23,6 +23,7 @@ MODE_SYMMETRIC, MODE_ZERO, MODE_PERIODIC = 0, 1, 2
 PATH_AUTO, PATH_TENSOR, PATH_SIMT = 0, 1, 2
 MODES = {"symmetric": MODE_SYMMETRIC, "zero": MODE_ZERO, "periodic": MODE_PERIODIC}
 PATHS = {"auto": PATH_AUTO, "tensor": PATH_TENSOR, "simt": PATH_SIMT}
+WAVELET_HAAR, WAVELET_DB4, WAVELET_BIOR44 = 1, 4, 44
 TEMPORAL_WTA, TEMPORAL_RAW, TEMPORAL_UNIFORM = 0, 1, 2
 SPATIAL_WSM, SPATIAL_SALIENCY, SPATIAL_NONE = 0, 1, 2
 TEMPORAL_MODES = {"wta": TEMPORAL_WTA, "raw": TEMPORAL_RAW, "uniform": TEMPORAL_UNIFORM}
@@ -328,8 +329,12 @@ def wz_dwt_len(n: int, wavelet: int = 4) -> int:
     return int(_lib.wz_dwt_len(n, wavelet))
 
 
+def wavelet_taps(wavelet: int) -> int:
+    return 10 if wavelet == WAVELET_BIOR44 else 2 * wavelet
+
+
 def wz_wavelet_filters(wavelet: int = 4):
-    F = 2 * wavelet
+    F = wavelet_taps(wavelet)
     bufs = [(C.c_double * F)() for _ in range(4)]
     _check(_lib.wz_wavelet_filters(wavelet, *bufs), "wz_wavelet_filters")
     return {k: [float(x) for x in b] for k, b in zip(("dec_lo", "dec_hi", "rec_lo", "rec_hi"), bufs)}

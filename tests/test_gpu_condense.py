@@ -85,7 +85,8 @@ def test_shapes(wz, T, H, W, D, Lq, ratio):
 @pytest.mark.parametrize("kw", [dict(lam=0.0), dict(lam=2.0), dict(wsm_wavelet=1), dict(wsm_wavelet=2),
                                 dict(mode="zero"), dict(mode="periodic"), dict(path="simt"),
                                 dict(wta_wavelet=4), dict(wta_wavelet=2, wsm_wavelet=1),
-                                dict(wta_wavelet=10, temporal_mode="wta")])
+                                dict(wta_wavelet=10, temporal_mode="wta"), dict(wsm_wavelet=44),
+                                dict(wta_wavelet=44, wsm_wavelet=44), dict(wsm_wavelet=44, path="simt")])
 def test_options(wz, kw):
     _random_case(wz, 10, 13, 13, 128, 6, 0.2, seed=5, **kw)
 
@@ -248,7 +249,8 @@ def test_relevance_entry_point(wz):
     assert np.allclose(fm.cpu().double().numpy(), ref["vbar"], atol=1e-5)
 
 
-@pytest.mark.parametrize("p,mode", [(1, "symmetric"), (4, "symmetric"), (4, "zero"), (4, "periodic"), (2, "symmetric")])
+@pytest.mark.parametrize("p,mode", [(1, "symmetric"), (4, "symmetric"), (4, "zero"), (4, "periodic"), (2, "symmetric"),
+                                    (44, "symmetric"), (44, "periodic")])
 def test_dwt_entry_points(wz, p, mode):
     g = torch.Generator().manual_seed(p)
     x = torch.randn((5, 27), generator=g)
