@@ -71,6 +71,10 @@ fact; the same list is kept in the design notes):
       for db4), with 10-tap arrays laid out as in that library: analysis
       lowpass in dec_lo[1..9], synthesis lowpass in rec_lo[1..7]; the paper
       evaluates it for both WTA and WSM ("Wavelet Basis" ablation).
+  R21 the projector P of Eq. 17 (applied after Psi, Eq. 16-18) is the two-
+      layer MLP of LLaVA-style models, P(z) = W2 GELU(W1 z + b1) + b2 with the
+      exact (erf) GELU; its weights are the caller's.  The hidden layer is
+      rounded to the tokens' dtype (bf16), as a bf16 model stores it.
   R19 an external scorer (Section 3.2.1 names BLIP-style matchers as
       alternatives to the similarity branch) may supply the token saliency
       a_{t,n} and / or the frame relevance r_t; the pooled features still come
@@ -593,3 +597,38 @@ def decision_margins(result: dict) -> float:
     vals = [m.get("alloc_gap", math.inf), m.get("cap_gap", math.inf),
             abs(m.get("max_r", math.inf)), m.get("tau_gap", math.inf)]
     return float(min(vals))
+
+
+# ----------------------------------------------------------------------------
+# Projector P (Eq. 17), applied to the condensed tokens (reading R21)
+# ----------------------------------------------------------------------------
+
+def gelu(x: np.ndarray) -> np.ndarray:
+    """GELU(x) = x Phi(x) = x (1 + erf(x / sqrt 2)) / 2, elementwise."""
+    x = np.asarray(x, dtype=np.float64)
+    return np.array([0.5 * v * (1.0 + math.erf(v / math.sqrt(2.0))) for v in x.ravel()]).reshape(x.shape)
+
+
+def round_bf16(x: np.ndarray) -> np.ndarray:
+    """Round to bfloat16 (nearest, ties to even) and back to float64."""
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float64)).to(torch.bfloat16).double().numpy()
+
+
+def project(Z: np.ndarray, W1: np.ndarray, b1, W2: np.ndarray, b2, hidden_bf16: bool = True) -> np.ndarray:
+    """P(Z) = GELU(Z W1^T + b1) W2^T + b2 for tokens Z (B, D), W1 (C, D), W2 (E, C).
+
+    A bias of None is zero.  With hidden_bf16 the hidden layer is rounded to
+    bfloat16 between the two layers (reading R21).
+    """
+    Z = np.asarray(Z, dtype=np.float64)
+    Hd = Z @ np.asarray(W1, dtype=np.float64).T
+    if b1 is not None:
+        Hd = Hd + np.asarray(b1, dtype=np.float64)[None, :]
+    Hd = gelu(Hd)
+    if hidden_bf16:
+        Hd = round_bf16(Hd)
+    out = Hd @ np.asarray(W2, dtype=np.float64).T
+    if b2 is not None:
+        out = out + np.asarray(b2, dtype=np.float64)[None, :]
+    return out

@@ -677,6 +677,44 @@ def test_external_flat_token_scores_remove_the_details():
 
 
 # ----------------------------------------------------------------------------
+# Projector P (Eq. 17, reading R21) against torch's CPU routines
+# ----------------------------------------------------------------------------
+
+def check_gelu(o):
+    x = np.linspace(-6.0, 6.0, 241)
+    ref = torch.nn.functional.gelu(torch.from_numpy(x), approximate="none").numpy()
+    assert np.allclose(o.gelu(x), ref, atol=1e-15, rtol=1e-14)
+
+
+def check_project(o):
+    g = np.random.default_rng(5)
+    Z = g.standard_normal((7, 24))
+    W1, b1 = g.standard_normal((40, 24)) / 5, g.standard_normal(40)
+    W2, b2 = g.standard_normal((16, 40)) / 6, g.standard_normal(16)
+    t = lambda a: torch.from_numpy(a)
+    hid = torch.nn.functional.gelu(torch.nn.functional.linear(t(Z), t(W1), t(b1)))
+    ref = torch.nn.functional.linear(hid.to(torch.bfloat16).double(), t(W2), t(b2)).numpy()
+    assert np.allclose(o.project(Z, W1, b1, W2, b2), ref, atol=1e-12)
+    ref32 = torch.nn.functional.linear(hid, t(W2), t(b2)).numpy()
+    assert np.allclose(o.project(Z, W1, b1, W2, b2, hidden_bf16=False), ref32, atol=1e-12)
+
+
+def test_gelu_matches_torch():
+    check_gelu(O)
+
+
+def test_project_matches_torch_linear():
+    check_project(O)
+
+
+def test_project_identity_weights():
+    Z = RNG.standard_normal((5, 8))
+    eye = np.eye(8)
+    out = O.project(Z, eye, None, eye, None)
+    assert np.allclose(out, O.round_bf16(O.gelu(Z)), atol=0)
+
+
+# ----------------------------------------------------------------------------
 # Mutation tests: a planted mistake in the oracle makes a pin fail
 # ----------------------------------------------------------------------------
 
@@ -808,3 +846,15 @@ def test_mutation_bior44_normalisation_breaks_published_pin(golden_dir):
         return h / h.sum(), ht / ht.sum()                # a plausible slip: DC gain 1, not sqrt(2)
     m = _mutant(cdf97_lowpass=unit_sum)
     assert _fails(check_bior44_published, m, golden_dir)
+
+
+def test_mutation_tanh_gelu_breaks_gelu_pin():
+    tanh_gelu = lambda x: 0.5 * np.asarray(x) * (1 + np.tanh(math.sqrt(2 / math.pi) * (np.asarray(x) + 0.044715 * np.asarray(x) ** 3)))
+    m = _mutant(gelu=tanh_gelu)
+    assert _fails(check_gelu, m)
+
+
+def test_mutation_dropped_bias_breaks_project_pin():
+    original = OM.project
+    m = _mutant(project=lambda Z, W1, b1, W2, b2, hidden_bf16=True: original(Z, W1, None, W2, b2, hidden_bf16))
+    assert _fails(check_project, m)
