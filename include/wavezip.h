@@ -278,6 +278,43 @@ WZ_API int wz_relevance_static(const void *features, int T, int H, int W, int D,
                                float *frame_mean, wz_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
+/* Projector P (Eq. 17): the condensed tokens through the model's MLP         */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * out = GELU(tokens W1^T + b1) W2^T + b2, the two-layer projector of
+ * LLaVA-style models that Eq. 17 applies after the condensation Psi, with
+ * the exact (erf) GELU.  bf16 operands, fp32 accumulation on the tensor
+ * cores (tcgen05), bf16 results; the hidden layer [B][C] is stored in bf16
+ * in the workspace (as a bf16 model stores it).
+ *   tokens [B][D], w1 [C][D], w2 [E][C] bf16 (torch.nn.Linear weights,
+ *   out x in); b1 [C], b2 [E] f32, nullable; out [B][E] bf16.
+ *   D, C, E: multiples of 64, at most 65536; every pointer 16-byte aligned.
+ * Errors: WZ_ERR_INVALID_ARG (null, misaligned, bad size), WZ_ERR_WORKSPACE,
+ * WZ_ERR_NO_MEMORY, WZ_ERR_CUDA; nothing is launched on an argument error.
+ */
+typedef struct {
+    const void *tokens;      /* [B][D] bf16                                  */
+    int64_t B;
+    int D;
+    const void *w1;          /* [C][D] bf16                                  */
+    const float *b1;         /* [C] or NULL                                  */
+    int C;
+    const void *w2;          /* [E][C] bf16                                  */
+    const float *b2;         /* [E] or NULL                                  */
+    int E;
+    void *out;               /* [B][E] bf16                                  */
+    void *workspace;         /* >= wz_project_workspace_size(B, C), 256-B    */
+    size_t workspace_bytes;  /* aligned; NULL = cudaMallocAsync on stream    */
+    int32_t *device_status;  /* [1] set nonzero on a bounded-wait timeout;   */
+                             /* nullable                                     */
+    wz_stream_t stream;
+} wz_project_args;
+
+WZ_API size_t wz_project_workspace_size(int64_t B, int C);
+WZ_API int wz_project(const wz_project_args *a);
+
+/* ------------------------------------------------------------------------ */
 /* Single-level DWT (Eq. 8, 10, 11, 14)                                      */
 /* ------------------------------------------------------------------------ */
 

@@ -513,6 +513,37 @@ int wz_relevance(const void *features, int T, int H, int W, int D, int dtype, co
     return WZ_OK;
 }
 
+size_t wz_project_workspace_size(int64_t B, int C) {
+    if (B < 0 || C < 1) return 0;
+    return align_up((size_t)B * (size_t)C * 2) + kAlign;   // hidden layer, then the status word
+}
+
+int wz_project(const wz_project_args *a) {
+    if (!a) return WZ_ERR_INVALID_ARG;
+    const auto dim_ok = [](int x) { return x >= 64 && x <= 65536 && x % 64 == 0; };
+    if (a->B < 0 || a->B > (int64_t)INT32_MAX || !dim_ok(a->D) || !dim_ok(a->C) || !dim_ok(a->E))
+        return WZ_ERR_INVALID_ARG;
+    if (a->B == 0) return WZ_OK;
+    if (!a->tokens || !a->w1 || !a->w2 || !a->out) return WZ_ERR_INVALID_ARG;
+    if (!aligned(a->tokens, 16) || !aligned(a->w1, 16) || !aligned(a->w2, 16) || !aligned(a->out, 16) ||
+        !aligned(a->b1, 16) || !aligned(a->b2, 16) || !aligned(a->device_status, 4))
+        return WZ_ERR_INVALID_ARG;
+    const cudaStream_t s = (cudaStream_t)a->stream;
+    const size_t need = wz_project_workspace_size(a->B, a->C);
+    Scratch ws;
+    int st = ws.acquire(a->workspace, a->workspace_bytes, need, s);
+    if (st != WZ_OK) return st;
+    int *status = a->device_status;
+    if (!status) {
+        status = reinterpret_cast<int *>(ws.ptr + align_up((size_t)a->B * (size_t)a->C * 2));
+        WZ_CUDA(cudaMemsetAsync(status, 0, sizeof(int), s));
+    }
+    const int M = (int)a->B;
+    WZ_CUDA(launch_project_gemm(a->tokens, M, a->D, a->w1, a->C, a->b1, ws.ptr, true, status, false, s));
+    WZ_CUDA(launch_project_gemm(ws.ptr, M, a->C, a->w2, a->E, a->b2, a->out, false, status, true, s));
+    return WZ_OK;
+}
+
 int wz_dwt_len(int n, int wavelet) {
     const int F = wavelet_taps(wavelet);
     if (n < 1 || F == 0) return -1;

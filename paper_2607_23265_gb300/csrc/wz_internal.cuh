@@ -273,6 +273,8 @@ cudaError_t launch_relevance_pass(const Ctx &c, cudaStream_t s);
 cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s);
 cudaError_t launch_temporal(const Ctx &c, cudaStream_t s);
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s);
+cudaError_t launch_project_gemm(const void *A, int M, int K, const void *B, int N, const float *bias, void *out,
+                                bool gelu, int *status, bool pdl, cudaStream_t s);
 cudaError_t launch_condense_simt(const Ctx &c, cudaStream_t s);
 cudaError_t launch_condense_tc(const Ctx &c, cudaStream_t s);
 int relevance_grid(const Ctx &c);   // CTAs for the relevance pass on this device

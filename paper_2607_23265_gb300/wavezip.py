@@ -74,6 +74,15 @@ class BatchArgs(C.Structure):
         ("kernel_events", C.POINTER(C.c_void_p)), ("stream", C.c_void_p),
     ]
 
+class ProjectArgs(C.Structure):
+    _fields_ = [
+        ("tokens", C.c_void_p), ("B", C.c_int64), ("D", C.c_int), ("w1", C.c_void_p), ("b1", C.c_void_p),
+        ("C", C.c_int), ("w2", C.c_void_p), ("b2", C.c_void_p), ("E", C.c_int), ("out", C.c_void_p),
+        ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
+        ("stream", C.c_void_p),
+    ]
+
+
 NUM_KERNELS = 6
 KERNEL_NAMES = ("query_pool", "relevance", "frame_stats", "temporal", "spatial", "condense")
 
@@ -97,6 +106,8 @@ def _load():
         "wz_relevance": (i, [vp, i, i, i, i, i, vp, i, vp, vp, vp, vp, sz, vp]),
         "wz_relevance_workspace_size": (sz, [i, i, i, i]),
         "wz_relevance_static": (i, [vp, i, i, i, i, i, vp, i, vp, vp, vp, vp]),
+        "wz_project_workspace_size": (sz, [i64, i]),
+        "wz_project": (i, [C.POINTER(ProjectArgs)]),
         "wz_dwt_len": (i, [i, i]),
         "wz_wavelet_filters": (i, [i] + [C.POINTER(C.c_double)] * 4),
         "wz_dwt1d": (i, [vp, i, i, i, i, vp, vp, vp]),
@@ -386,3 +397,40 @@ def wz_idwt2d(LL, LH, HL, HH, H: int, W: int, wavelet: int = 4, stream=None):
 
 def wz_version() -> int:
     return int(_lib.wz_version())
+
+
+def wz_project_workspace_size(B: int, C_: int) -> int:
+    return int(_lib.wz_project_workspace_size(int(B), int(C_)))
+
+
+def wz_project(tokens: torch.Tensor, w1: torch.Tensor, b1, w2: torch.Tensor, b2, *, out=None,
+               workspace: torch.Tensor | None = None, device_status: torch.Tensor | None = None, stream=None):
+    """wz_project: GELU(tokens w1^T + b1) w2^T + b2, bf16 in and out (b1, b2 float32 or None)."""
+    tokens = _cuda_contig(tokens, "tokens")
+    w1 = _cuda_contig(w1, "w1")
+    w2 = _cuda_contig(w2, "w2")
+    for t, name in ((tokens, "tokens"), (w1, "w1"), (w2, "w2")):
+        if t.dtype != torch.bfloat16:
+            raise TypeError(f"{name} must be bfloat16")
+    B, D = tokens.shape
+    C_, E = w1.shape[0], w2.shape[0]
+    if w1.shape[1] != D or w2.shape[1] != C_:
+        raise ValueError("shapes: tokens [B, D], w1 [C, D], w2 [E, C]")
+    biases = []
+    for b, n, name in ((b1, C_, "b1"), (b2, E, "b2")):
+        if b is not None:
+            b = _cuda_contig(b, name)
+            if b.dtype != torch.float32 or b.shape != (n,):
+                raise ValueError(f"{name} must be float32 of shape ({n},)")
+        biases.append(b)
+    res = out if out is not None else torch.empty((B, E), dtype=torch.bfloat16, device=tokens.device)
+    a = ProjectArgs()
+    a.tokens, a.B, a.D, a.w1, a.C, a.w2, a.E = tokens.data_ptr(), B, D, w1.data_ptr(), C_, w2.data_ptr(), E
+    a.b1, a.b2 = _ptr(biases[0]), _ptr(biases[1])
+    a.out = res.data_ptr()
+    if workspace is not None:
+        a.workspace, a.workspace_bytes = workspace.data_ptr(), workspace.numel() * workspace.element_size()
+    a.device_status = _ptr(device_status)
+    a.stream = _stream(stream, tokens.device)
+    _check(_lib.wz_project(C.byref(a)), "wz_project")
+    return res
