@@ -49,6 +49,8 @@ def parse():
     p.add_argument("--path", default="auto", choices=["auto", "tensor", "simt"])
     p.add_argument("--e2e-steps", type=int, default=5)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--projector-steps", type=int, default=10,
+                   help="also time the projector P (Eq. 17) on the condensed tokens; 0 skips it")
     return p.parse_args()
 
 
@@ -95,6 +97,48 @@ def measured_peak():
             return float(json.load(f)["hbm_gbs"]), "measured"
     except (OSError, KeyError, ValueError):
         return 6800.0, "fallback"
+
+
+def measured_tensor_peak():
+    """Measured dense bf16 TFLOP/s (burst, sustained) of the GB300s."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 1900.0, 1700.0, "fallback"
+
+
+def time_projector(wz, tokens, steps, dev):
+    """P (Eq. 17) on this step's condensed tokens [B][D] with random weights of
+    an LLM-sized MLP (C = E = D), timed with CUDA events after warm-up."""
+    import torch
+    B, D = tokens.shape
+    g = torch.Generator(device=dev).manual_seed(17)
+    w1 = (torch.randn((D, D), device=dev, generator=g) / D ** 0.5).to(torch.bfloat16)
+    w2 = (torch.randn((D, D), device=dev, generator=g) / D ** 0.5).to(torch.bfloat16)
+    b1 = torch.zeros(D, device=dev)
+    b2 = torch.zeros(D, device=dev)
+    ws = torch.empty((wz.wz_project_workspace_size(B, D),), dtype=torch.uint8, device=dev)
+    out = torch.empty((B, D), dtype=torch.bfloat16, device=dev)
+    for _ in range(3):
+        wz.wz_project(tokens, w1, b1, w2, b2, out=out, workspace=ws)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        wz.wz_project(tokens, w1, b1, w2, b2, out=out, workspace=ws)
+    e1.record()
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1) / steps
+    flop = 2 * 2.0 * B * D * D
+    burst, sustained, kind = measured_tensor_peak()
+    achieved = flop / (ms * 1e-3) / 1e12
+    return {"config": {"B": B, "D": D, "C": D, "E": D, "hidden": "bf16", "activation": "gelu (erf)"},
+            "ms": round(ms, 5), "bound": "tensor", "achieved": round(achieved, 1), "unit": "TFLOP/s",
+            "peak": sustained, "frac": round(achieved / sustained, 4), "frac_of_burst": round(achieved / burst, 4),
+            "peak_source": kind + " (sustained: a kernel timed in a back-to-back loop)", "launches": 2 * steps}
 
 
 def source_hash(fname):
@@ -337,6 +381,8 @@ def run_ours(args, spec, world, rank, local):
     barrier()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.e2e_steps, world, dev)
 
+    projector = time_projector(wz, tokens, args.projector_steps, dev) if args.projector_steps > 0 else None
+
     if rank == 0:
         peak, peak_kind = measured_peak()
         ab = algorithmic_bytes(spec, budgets, B, K_pad)
@@ -368,6 +414,7 @@ def run_ours(args, spec, world, rank, local):
                     "d2h_bytes_per_step": tokens.numel() * tokens.element_size() + index.numel() * 4},
             "clocks": clocks,
             "gpu_launches": len(KERNELS) * args.steps,
+            "projector": projector,
         }
         if world == 1 and not args.no_cpu_baseline:
             out["cpu_baseline"] = cpu_baseline(spec, CPU_SAMPLE_FRAMES)
