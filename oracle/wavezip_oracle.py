@@ -75,6 +75,10 @@ fact; the same list is kept in the design notes):
       layer MLP of LLaVA-style models, P(z) = W2 GELU(W1 z + b1) + b2 with the
       exact (erf) GELU; its weights are the caller's.  The hidden layer is
       rounded to the tokens' dtype (bf16), as a bf16 model stores it.
+  R22 a max-over-query scorer ("maxsim") for queries of several rows: the
+      query is not pooled; a_{t,n} = max_j cos(u_{t,n}, q_j) and
+      r_t = max_j cos(v_bar_t, q_j) over the Lq rows q_j (with one row it is
+      the similarity branch itself).
   R19 an external scorer (Section 3.2.1 names BLIP-style matchers as
       alternatives to the similarity branch) may supply the token saliency
       a_{t,n} and / or the frame relevance r_t; the pooled features still come
@@ -510,7 +514,7 @@ SPATIAL_MODES = ("wsm", "saliency", "none")
 def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
              wta_wavelet: int = 1, wsm_wavelet: int = 4, mode: str = "symmetric",
              token_frames=None, temporal_mode: str = "wta", spatial_mode: str = "wsm",
-             token_scores=None, frame_scores=None) -> dict:
+             token_scores=None, frame_scores=None, relevance: str = "mean") -> dict:
     """Condense features X (T, H, W, D) for query Q (Lq, D) to B tokens.
 
     token_frames: optional iterable of frame indices; when given, the WSM and
@@ -519,8 +523,9 @@ def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
     temporal_mode / spatial_mode: the ablation modes of reading R18.
     token_scores (T, N) / frame_scores (T,): an external scorer's a_{t,n} and
     r_t (reading R19), replacing the similarity branch's values.
+    relevance: "mean" (u_q = mean query row, R1) or "maxsim" (reading R22).
     """
-    if temporal_mode not in TEMPORAL_MODES or spatial_mode not in SPATIAL_MODES:
+    if temporal_mode not in TEMPORAL_MODES or spatial_mode not in SPATIAL_MODES or relevance not in ("mean", "maxsim"):
         raise ValueError("unknown mode")
     X = np.asarray(X, dtype=np.float64)
     T, H, W, D = X.shape
@@ -533,6 +538,10 @@ def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
         U = X[t].reshape(N, D)
         a[t] = token_saliency(U, u_q)
         r[t], vbar[t] = frame_relevance(U, u_q)
+        if relevance == "maxsim":
+            Qr = np.asarray(Q, dtype=np.float64)
+            a[t] = np.max([token_saliency(U, q) for q in Qr], axis=0)
+            r[t] = max(cosine(vbar[t], q) for q in Qr)
     if token_scores is not None:
         a = np.asarray(token_scores, dtype=np.float64).reshape(T, N).copy()
     if frame_scores is not None:

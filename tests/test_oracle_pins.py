@@ -676,6 +676,37 @@ def test_external_flat_token_scores_remove_the_details():
     assert np.allclose(flat["out_tokens"], low["out_tokens"], atol=1e-12)
 
 
+def check_maxsim_hand_case(o):
+    # two orthonormal query rows; one token equal to q_1, one to q_2, one along q_1 + q_2
+    D = 4
+    Q = np.array([[1.0, 0, 0, 0], [0, 1.0, 0, 0]])
+    X = np.zeros((1, 1, 3, D))
+    X[0, 0, 0] = [2.0, 0, 0, 0]
+    X[0, 0, 1] = [0, 3.0, 0, 0]
+    X[0, 0, 2] = [1.0, 1.0, 0, 0]
+    res = o.condense(X, Q, 1.0, relevance="maxsim")
+    assert np.allclose(res["a"][0], [1.0, 1.0, 1 / math.sqrt(2)], atol=1e-15)
+    mean = o.condense(X, Q, 1.0)
+    assert np.allclose(mean["a"][0], [1 / math.sqrt(2), 1 / math.sqrt(2), 1.0], atol=1e-15)
+    # v_bar = (1, 4/3, 0, 0)/1: r = max of its cosines with q_1 and q_2
+    v = np.array([3.0, 4.0, 0, 0]) / 3
+    assert abs(res["r"][0] - 4.0 / 5.0) < 1e-15 and abs(mean["r"][0] - 7.0 / (5 * math.sqrt(2))) < 1e-15
+    assert np.allclose(res["vbar"][0], v)
+
+
+def test_maxsim_hand_case():
+    check_maxsim_hand_case(O)
+
+
+def test_maxsim_with_one_query_row_is_the_similarity_branch():
+    X = RNG.standard_normal((6, 4, 5, 8))
+    Q = RNG.standard_normal((1, 8))
+    a, b = O.condense(X, Q, 0.3, relevance="maxsim"), O.condense(X, Q, 0.3)
+    assert np.array_equal(a["budgets"], b["budgets"])
+    assert np.allclose(a["a"], b["a"], atol=1e-15) and np.allclose(a["r"], b["r"], atol=1e-15)
+    assert np.allclose(a["out_tokens"], b["out_tokens"], atol=1e-13)
+
+
 # ----------------------------------------------------------------------------
 # Projector P (Eq. 17, reading R21) against torch's CPU routines
 # ----------------------------------------------------------------------------
@@ -858,3 +889,18 @@ def test_mutation_dropped_bias_breaks_project_pin():
     original = OM.project
     m = _mutant(project=lambda Z, W1, b1, W2, b2, hidden_bf16=True: original(Z, W1, None, W2, b2, hidden_bf16))
     assert _fails(check_project, m)
+
+
+def test_mutation_maxsim_min_breaks_hand_case():
+    original = OM.condense
+
+    def min_condense(X, Q, ratio, **kw):
+        res = original(X, Q, ratio, **kw)
+        if kw.get("relevance") == "maxsim":              # planted: min over the rows instead of max
+            Xr = np.asarray(X, dtype=np.float64)
+            T, H, W, D = Xr.shape
+            res["a"] = np.array([np.min([OM.token_saliency(Xr[t].reshape(H * W, D), q) for q in Q], axis=0)
+                                 for t in range(T)])
+        return res
+    m = _mutant(condense=min_condense)
+    assert _fails(check_maxsim_hand_case, m)
