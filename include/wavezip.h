@@ -97,6 +97,14 @@ typedef struct CUstream_st *wz_stream_t;
 #define WZ_SPATIAL_SALIENCY  1 /* "Saliency-Only": lambda * M_t * X_t, no wavelets */
 #define WZ_SPATIAL_NONE      2 /* no modulation: Psi of the features itself       */
 
+/* Relevance scorer.  MEAN: the similarity branch with the mean query row
+ * u_q (Section 3.2.1); MAXSIM: no pooling of the query, the maximum cosine
+ * over its rows for both a_{t,n} and r_t (bf16 features, D % 64 == 0,
+ * Lq <= WZ_MAX_LQ_MAXSIM; the token x row cosines run on the tensor cores). */
+#define WZ_RELEVANCE_MEAN    0
+#define WZ_RELEVANCE_MAXSIM  1
+#define WZ_MAX_LQ_MAXSIM     128
+
 /* Wavelets: Daubechies filters named by their vanishing moments p (2p
  * taps), 1 = Haar, 4 = db4, 1 <= p <= 10; and the biorthogonal bior4.4
  * (CDF 9/7, 10-tap arrays), the third basis of the paper's "Wavelet Basis"
@@ -158,6 +166,7 @@ typedef struct {
                              /* a_{t,n} (Section 3.2.1) replacing the        */
                              /* similarity branch's; nullable                */
     const float *frame_scores; /* [T] f32 device, external r_t; nullable     */
+    int relevance_mode;      /* WZ_RELEVANCE_*, default MEAN                 */
     void *out_tokens;        /* [B][D], dtype                                */
     int32_t *out_index;      /* [B][3]                                       */
     int32_t *out_budgets;    /* [T] n_t (0 for filtered frames); nullable    */
@@ -209,6 +218,7 @@ typedef struct {
     int temporal_mode, spatial_mode;   /* WZ_TEMPORAL_*, WZ_SPATIAL_* */
     const float *token_scores;         /* [V][T][N] device, nullable   */
     const float *frame_scores;         /* [V][T] device, nullable      */
+    int relevance_mode;                /* WZ_RELEVANCE_*               */
     void *out_tokens;
     int32_t *out_index;
     int64_t *row_offsets;    /* host, [V+1], nullable */

@@ -28,7 +28,7 @@ bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 // Sub-buffer offsets of one call's workspace.
 struct Layout {
     size_t qbar32, qbar64, vpar, a, part, fr, list, n, off, woff, hw, prod,
-        units, ucount, ustart, stab, drange, gate, status, Wop, total;
+        units, ucount, ustart, stab, drange, gate, qnorm, qhl, status, Wop, total;
 };
 
 struct Shape {
@@ -62,6 +62,8 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.ustart = take(VT * 4);
     L.stab = take(spatial_table_bytes(s.H, s.W, kMaxTaps));   // any wavelet
     L.drange = take((size_t)s.V * 16);
+    L.qnorm = take((size_t)s.V * WZ_MAX_LQ_MAXSIM * 4);
+    L.qhl = take((size_t)2 * WZ_MAX_LQ_MAXSIM * s.D * 2);
     L.gate = with_operator ? take(VT * (size_t)((s.H + kMaxTaps - 1) / 2) * ((s.W + kMaxTaps - 1) / 2) * 4) : 0;
     L.status = take(16);
     L.Wop = with_operator ? take((size_t)std::max<int64_t>(s.rows_total, s.w_rows) * s.K_pad * 4) : 0;
@@ -113,6 +115,7 @@ Shape make_shape(int V, int T, int H, int W, int D, int dtype, int F, const int6
 struct Common {
     float lambda, tau;
     int wta_wavelet, wsm_wavelet, mode, path, temporal_mode, spatial_mode;
+    int relevance_mode = WZ_RELEVANCE_MEAN;
 };
 
 int check_common(const Common &m, int dtype) {
@@ -176,6 +179,8 @@ void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.ustart = reinterpret_cast<int *>(ws + L.ustart);
     c.stab = reinterpret_cast<float *>(ws + L.stab);
     c.drange = reinterpret_cast<unsigned long long *>(ws + L.drange);
+    c.qnorm = reinterpret_cast<float *>(ws + L.qnorm);
+    c.qhl = reinterpret_cast<__nv_bfloat16 *>(ws + L.qhl);
     c.gate = L.gate ? reinterpret_cast<float *>(ws + L.gate) : nullptr;
     c.status = reinterpret_cast<int *>(ws + L.status);
     if (L.Wop) c.Wop = ws + L.Wop;
@@ -240,6 +245,12 @@ int validate(const CondenseRequest &r, std::vector<int64_t> &B, int64_t &rows) {
     if (!r.features || !r.queries) return WZ_ERR_INVALID_ARG;
     if (!aligned(r.features, 16) || !aligned(r.queries, 16)) return WZ_ERR_INVALID_ARG;
     if (!aligned(r.token_scores, 4) || !aligned(r.frame_scores, 4)) return WZ_ERR_INVALID_ARG;
+    if (r.m.relevance_mode != WZ_RELEVANCE_MEAN && r.m.relevance_mode != WZ_RELEVANCE_MAXSIM) return WZ_ERR_INVALID_ARG;
+    if (r.m.relevance_mode == WZ_RELEVANCE_MAXSIM) {
+        if (r.dtype != WZ_DTYPE_BF16 || r.D % 64 != 0) return WZ_ERR_UNSUPPORTED;
+        for (int v = 0; v < r.V; ++v)
+            if (r.Lq[v] > WZ_MAX_LQ_MAXSIM) return WZ_ERR_UNSUPPORTED;
+    }
     B.assign(r.V, 0);
     rows = 0;
     int64_t qrows = 0;
@@ -271,6 +282,7 @@ int run_condense(const CondenseRequest &r) {
     c.spatial_mode = r.m.spatial_mode;
     c.ext_a = r.token_scores;
     c.ext_r = r.frame_scores;
+    c.relevance_mode = r.m.relevance_mode;
     c.pdl = r.events ? 0 : 1;      // an event between two kernels would break the overlap
     set_filters(c, r.m.wsm_wavelet);
     set_wta_filters(c, r.m.wta_wavelet);
@@ -318,6 +330,17 @@ int run_condense(const CondenseRequest &r) {
     WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE));
     WZ_CUDA(launch_relevance_pass(c, r.stream));
     WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE + 1));
+    if (c.relevance_mode == WZ_RELEVANCE_MAXSIM) {
+        // the token x query-row cosines on the tensor cores, video by video
+        // (the relevance pass left ||u|| in c.a)
+        for (int v = 0; v < r.V; ++v) {
+            const int Lq = r.Lq[v], Lqp = (Lq + 15) / 16 * 16;
+            const int64_t tok = (int64_t)s.T * s.N;
+            WZ_CUDA(launch_query_rows(c, v, par[v].q_row0, Lq, Lqp, r.stream));
+            WZ_CUDA(launch_maxsim_gemm(static_cast<const char *>(r.features) + (size_t)v * tok * s.D * 2, (int)tok,
+                                       s.D, c.qhl, Lq, Lqp, c.a + v * tok, c.status, c.pdl != 0, r.stream));
+        }
+    }
     WZ_CUDA(mark(2 * WZ_KERNEL_FRAME_STATS));
     WZ_CUDA(launch_frame_stats(c, r.stream));
     WZ_CUDA(mark(2 * WZ_KERNEL_FRAME_STATS + 1));
@@ -399,6 +422,7 @@ int wz_condense_ex(const wz_condense_args *a) {
                  a->spatial_mode};
     r.token_scores = a->token_scores;
     r.frame_scores = a->frame_scores;
+    r.m.relevance_mode = a->relevance_mode;
     r.out_tokens = a->out_tokens;
     r.out_index = a->out_index;
     r.out_budgets = a->out_budgets;
@@ -456,6 +480,7 @@ int wz_condense_batch(const wz_batch_args *a) {
                  a->spatial_mode};
     r.token_scores = a->token_scores;
     r.frame_scores = a->frame_scores;
+    r.m.relevance_mode = a->relevance_mode;
     r.out_tokens = a->out_tokens;
     r.out_index = a->out_index;
     r.out_budgets = a->out_budgets;

@@ -15,6 +15,9 @@
 //   warp 1     TMEM allocation and the MMA issuer (one thread)
 //   warps 2-5  epilogue: tcgen05.ld (TMEM lane = row m, columns = n) -> + bias
 //              -> activation -> bf16 -> 16-byte stores of contiguous row pieces
+// The same kernel with a row-max epilogue computes the max-over-query
+// relevance: the token x query-row cosines (B = the normalised query rows as
+// bf16 hi and lo halves, N = 2 Lqp), maximum over the rows per token.
 // Every mbarrier wait is bounded; on a timeout the kernel records a status
 // bit, drains what it issued, frees tensor memory and exits.
 #include <cuda.h>
@@ -57,9 +60,16 @@ struct PMaps {
 
 struct PArgs {
     int M, N, K;
+    int tileN;           // MMA N of a tile (<= 256, multiple of 32); the B box height
+    // epilogue 0 (projector): out = act(acc + bias)
     const float *bias;   // [N] or null
     __nv_bfloat16 *out;  // [M][N]
     int gelu;            // 1: exact GELU after the bias
+    // epilogue 1 (max-over-query relevance): columns [0, Lqp) and [Lqp, 2 Lqp)
+    // hold the hi and lo parts of the dots with the normalised query rows;
+    // a[m] = max_{j < Lq} (hi_j + lo_j) / a[m] (a[m] holds ||u_m|| on entry)
+    float *a;
+    int Lq, Lqp;
     int *status;
 };
 
@@ -70,6 +80,7 @@ __device__ __forceinline__ void pfail(const PArgs &p, volatile int *abort_flag, 
 
 }  // namespace
 
+template <int EPI>
 __global__ void __launch_bounds__(kPThreads, 1)
 project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
     extern __shared__ uint8_t smem_raw[];
@@ -105,7 +116,7 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = S->tmem_base;
-    const int mt = (p.M + kPM - 1) / kPM, nt = (p.N + kPN - 1) / kPN;
+    const int mt = (p.M + kPM - 1) / kPM, nt = (p.N + p.tileN - 1) / p.tileN;
     const int tiles = mt * nt;
     const int KS = p.K / kPK;
 
@@ -118,7 +129,8 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
         int issued_parity[kPStages];
         for (int s = 0; s < kPStages; ++s) issued_parity[s] = -1;
         for (int t = blockIdx.x; t < tiles && !*abort_flag; t += gridDim.x) {
-            const int m0 = (t / nt) * kPM, n0 = (t % nt) * kPN;
+            const int m0 = (t / nt) * kPM, n0 = (t % nt) * p.tileN;
+            const uint32_t stage_bytes = (uint32_t)(kPM + p.tileN) * kPK * 2;
             bool ok = true;
             for (int ks = 0; ks < KS; ++ks) {
                 if (!ptx::mbar_wait(&S->empty[stage], phase ^ 1u, kPTimeoutNs)) {
@@ -127,7 +139,7 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
                     break;
                 }
                 uint8_t *st = ring + (size_t)stage * kPStageBytes;
-                ptx::mbar_arrive_expect_tx(&S->full[stage], (uint32_t)kPStageBytes);
+                ptx::mbar_arrive_expect_tx(&S->full[stage], stage_bytes);
                 ptx::tma_load_2d(st, &maps.a, &S->full[stage], ks * kPK, m0, pol_a);
                 ptx::tma_load_2d(st + kPABytes, &maps.b, &S->full[stage], ks * kPK, n0, pol_b);
                 issued_parity[stage] = (int)phase;
@@ -142,7 +154,7 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
             if (issued_parity[s] >= 0) ptx::mbar_wait(&S->full[s], (uint32_t)issued_parity[s], kPTimeoutNs);
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer ----------------
-        constexpr uint32_t idesc = ptx::idesc_bf16(kPM, kPN, false, false);   // both K-major
+        const uint32_t idesc = ptx::idesc_bf16(kPM, p.tileN, false, false);   // both K-major
         const uint32_t ring32 = ptx::smem_u32(ring);
         const uint64_t a_base = ptx::smem_desc(ring32, 16, 1024, 2);              // 128-B swizzle
         const uint64_t b_base = ptx::smem_desc(ring32 + kPABytes, 16, 1024, 2);
@@ -195,9 +207,25 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
                 break;
             }
             ptx::tc_fence_after();
-            const int m0 = (t / nt) * kPM, n0 = (t % nt) * kPN;
+            const int m0 = (t / nt) * kPM, n0 = (t % nt) * p.tileN;
             const int row = m0 + q * 32 + lane;
             const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * kPAccCols);
+            if constexpr (EPI == 1) {
+                float best = -INFINITY;
+                for (int c0 = 0; c0 < p.Lqp; c0 += 16) {
+                    uint32_t hi[16], lo[16];
+                    ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)c0, hi);
+                    ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)(p.Lqp + c0), lo);
+                    ptx::tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                        if (c0 + j < p.Lq) best = fmaxf(best, __uint_as_float(hi[j]) + __uint_as_float(lo[j]));
+                }
+                if (row < p.M) {
+                    const float nrm = p.a[row];
+                    p.a[row] = nrm > 0.f ? best / nrm : 0.f;
+                }
+            } else
             for (int c0 = 0; c0 < kPN && n0 + c0 < p.N; c0 += 32) {
                 uint32_t v0[16], v1[16];
                 ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)c0, v0);
@@ -287,18 +315,50 @@ cudaError_t launch_project_gemm(const void *A, int M, int K, const void *B, int 
     memset(&maps, 0, sizeof(maps));
     if (!encode_2d(enc, &maps.a, A, M, K, kPM) || !encode_2d(enc, &maps.b, B, N, K, kPN))
         return cudaErrorInvalidValue;
-    PArgs p{M, N, K, bias, static_cast<__nv_bfloat16 *>(out), gelu ? 1 : 0, status};
+    PArgs p{};
+    p.M = M; p.N = N; p.K = K; p.tileN = kPN;
+    p.bias = bias; p.out = static_cast<__nv_bfloat16 *>(out); p.gelu = gelu ? 1 : 0; p.status = status;
     int dev = 0, sms = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(project_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPSmemBytes);
+    e = cudaFuncSetAttribute(project_gemm_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPSmemBytes);
     if (e != cudaSuccess) return e;
     const int tiles = ((M + kPM - 1) / kPM) * ((N + kPN - 1) / kPN);
     const int grid = tiles < sms ? tiles : sms;
     void *args[] = {&maps, &p};
-    return launch_kernel((const void *)project_gemm_kernel, dim3(grid), dim3(kPThreads), kPSmemBytes, s, args, pdl);
+    return launch_kernel((const void *)project_gemm_kernel<0>, dim3(grid), dim3(kPThreads), kPSmemBytes, s, args,
+                         pdl);
+}
+
+// Max-over-query relevance of M tokens X [M][K] against the hi/lo rows
+// QHL [2 Lqp][K] of the normalised queries: a[m] = max_j <x_m, q^_j> / a[m].
+cudaError_t launch_maxsim_gemm(const void *X, int M, int K, const void *QHL, int Lq, int Lqp, float *a, int *status,
+                               bool pdl, cudaStream_t s) {
+    if (M < 1) return cudaSuccess;
+    if (Lq < 1 || Lqp % 16 != 0 || Lq > Lqp || 2 * Lqp > kPN || K % kPK != 0) return cudaErrorInvalidValue;
+    auto enc = project_encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    PMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    if (!encode_2d(enc, &maps.a, X, M, K, kPM) || !encode_2d(enc, &maps.b, QHL, 2 * Lqp, K, 2 * Lqp))
+        return cudaErrorInvalidValue;
+    PArgs p{};
+    p.M = M; p.N = 2 * Lqp; p.K = K; p.tileN = 2 * Lqp;
+    p.a = a; p.Lq = Lq; p.Lqp = Lqp; p.status = status;
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(project_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPSmemBytes);
+    if (e != cudaSuccess) return e;
+    const int tiles = (M + kPM - 1) / kPM;
+    const int grid = tiles < sms ? tiles : sms;
+    void *args[] = {&maps, &p};
+    return launch_kernel((const void *)project_gemm_kernel<1>, dim3(grid), dim3(kPThreads), kPSmemBytes, s, args,
+                         pdl);
 }
 
 }  // namespace wz

@@ -9,6 +9,14 @@
 //                   in a fixed order and forms r_t and delta_t (Eq. 7) from
 //                   <v_t,u_q>, <v_t,v_t>, <v_t,v_{t-1}>, <v_{t-1},v_{t-1}>
 //                   and <u_q,u_q>, reduced in fp64.
+//   query_rows      (max-over-query scorer) the norms of the query rows and
+//                   the rows scaled to unit length, split into bf16 hi + lo
+//                   halves: the B operand of the token x row cosine GEMM.
+//
+// With the max-over-query scorer the relevance pass stores ||u|| in place of
+// a_{t,n}; the tensor-core GEMM that follows divides max_j <u, q_j/||q_j||>
+// by it, and frame_stats takes r_t = max_j cos(v_bar_t, q_j) from the raw
+// rows and their norms.
 //
 // The relevance pass is HBM bound: it reads T*H*W*D elements once, streamed
 // by TMA bulk copies through a shared-memory ring; each CTA owns one
@@ -83,6 +91,43 @@ __global__ void __launch_bounds__(256) query_pool_kernel(Ctx c, VideoParBlock pa
     }
 }
 
+// Query rows of video v for the max-over-query scorer: block j < Lq writes
+// ||q_j|| (fp64 sum of fp32 squares) to qnorm and q_j / ||q_j|| as bf16 hi
+// (row j of qhl) and lo = bf16(x - hi) (row Lqp + j); blocks Lq <= j < Lqp
+// write zero rows, so the GEMM's padding columns are zero.  bf16 rows.
+__global__ void __launch_bounds__(256) query_rows_kernel(Ctx c, int v, int q_row0, int Lq, int Lqp) {
+    __shared__ double red[33];
+    pdl_wait();
+    pdl_trigger();
+    const int j = blockIdx.x;
+    const int D = c.D;
+    __nv_bfloat16 *hi = c.qhl + (size_t)j * D;
+    __nv_bfloat16 *lo = c.qhl + (size_t)(Lqp + j) * D;
+    const __nv_bfloat16 zero = __float2bfloat16_rn(0.f);
+    if (j >= Lq) {
+        for (int d = threadIdx.x; d < D; d += blockDim.x) {
+            hi[d] = zero;
+            lo[d] = zero;
+        }
+        return;
+    }
+    const __nv_bfloat16 *q = static_cast<const __nv_bfloat16 *>(c.Q) + (size_t)(q_row0 + j) * D;
+    float ss = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) {
+        const float x = __bfloat162float(q[d]);
+        ss = fmaf(x, x, ss);
+    }
+    const double qn = sqrt(block_sum((double)ss, red));
+    if (threadIdx.x == 0) c.qnorm[(size_t)v * WZ_MAX_LQ_MAXSIM + j] = (float)qn;
+    const float inv = qn > 0.0 ? (float)(1.0 / qn) : 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) {
+        const float x = __bfloat162float(q[d]) * inv;
+        const __nv_bfloat16 h = __float2bfloat16_rn(x);
+        hi[d] = h;
+        lo[d] = __float2bfloat16_rn(x - __bfloat162float(h));
+    }
+}
+
 // Reduce the NV values held by every lane across the warp (NV a power of
 // two <= 32).  Each of the first log2(NV) steps halves the values a lane
 // keeps; the remaining steps are plain butterflies.  On return lane l holds
@@ -143,6 +188,7 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
     const int nw = NC >> 5;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int n_vec = c.D / VEC;
+    const bool maxsim = c.relevance_mode == WZ_RELEVANCE_MAXSIM;
     const size_t rowb = (size_t)c.D * sizeof(T);
     const size_t stage_bytes = (size_t)CH * rowb;
     const int64_t total = (int64_t)c.V * c.T * c.N;
@@ -349,7 +395,8 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
                     dot += wpart[buf][w][0][t];
                     nrm += wpart[buf][w][1][t];
                 }
-                c.a[wbase + t] = (nrm > 0.f && qn > 0.f) ? dot / (sqrtf(nrm) * qn) : 0.f;
+                c.a[wbase + t] = maxsim ? sqrtf(nrm)   // ||u||, divided out by the row-max GEMM
+                                        : (nrm > 0.f && qn > 0.f) ? dot / (sqrtf(nrm) * qn) : 0.f;
             }
             buf ^= 1;
             wbase = tok;
@@ -409,10 +456,18 @@ __device__ void frame_gate(const Ctx &c, int64_t f, float *red) {
 // channels and across each warp, the warp totals in fp64; then
 // r_t = cos(v_bar_t, u_q) and delta_t = 1 - cos(v_bar_t, v_bar_{t-1})
 // clamped to [0, 2] (Eq. 7) in fp64.
+//
+// With the max-over-query scorer the frame sums are kept in shared memory
+// (D floats of dynamic shared memory) and every warp takes query rows j:
+// <v_t, q_j> with fp32 products per 8 channels summed in fp64, divided by
+// ||q_j||; r_t = max_j of that / ||v_t||.
 __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     pdl_wait();
     pdl_trigger();
     __shared__ float wsum[16][5];
+    __shared__ double wmax[16];
+    extern __shared__ float4 sfs[];   // [D/4] frame sums (max-over-query scorer only)
+    const bool maxsim = c.relevance_mode == WZ_RELEVANCE_MAXSIM;
     const int64_t f = blockIdx.x;
     const int t = (int)(f % c.T);
     const int v = (int)(f / c.T);
@@ -436,6 +491,7 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
             sp.x += x.x; sp.y += x.y; sp.z += x.z; sp.w += x.w;
         }
         const float4 q = Qv[i];
+        if (maxsim) sfs[i] = sf;
         if (c.frame_mean) {   // caller's buffer: 4-byte alignment only
             float *fm = c.frame_mean + (size_t)f * c.D + 4 * i;
             fm[0] = sf.x / (float)c.N;
@@ -457,6 +513,30 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
         p4 += __shfl_xor_sync(0xffffffffu, p4, o);
     }
     const int warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    if (maxsim) {
+        __syncthreads();   // sfs complete
+        const int lane = threadIdx.x & 31;
+        const VideoPar vp = c.vpar[v];
+        const int n8 = c.D / 8;
+        double best = -INFINITY;
+        for (int j = warp; j < vp.Lq; j += nw) {
+            const uint4 *qr = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(c.Q) +
+                                                              (size_t)(vp.q_row0 + j) * c.D);
+            double acc = 0.0;
+            for (int i = lane; i < n8; i += 32) {
+                float qf[8];
+                unpack(__ldg(qr + i), qf, (__nv_bfloat16 *)nullptr);
+                const float4 s0 = sfs[2 * i], s1 = sfs[2 * i + 1];
+                const float pp = fmaf(s0.x, qf[0], fmaf(s0.y, qf[1], fmaf(s0.z, qf[2], fmaf(s0.w, qf[3],
+                                 fmaf(s1.x, qf[4], fmaf(s1.y, qf[5], fmaf(s1.z, qf[6], s1.w * qf[7])))))));
+                acc += (double)pp;
+            }
+            for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+            const double qn = (double)c.qnorm[(size_t)v * WZ_MAX_LQ_MAXSIM + j];
+            best = fmax(best, qn > 0.0 ? acc / qn : 0.0);
+        }
+        if (lane == 0) wmax[warp] = best;
+    }
     if ((threadIdx.x & 31) == 0) {
         wsum[warp][0] = p0;
         wsum[warp][1] = p1;
@@ -475,8 +555,13 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
             pp += (double)wsum[w][4];
         }
         const double qn = sqrt(qq);
-        const double r = c.ext_r ? (double)c.ext_r[f]                      // an external scorer's r_t
-                                 : (vv > 0.0 && qn > 0.0) ? vq / (sqrt(vv) * qn) : 0.0;
+        double r = (vv > 0.0 && qn > 0.0) ? vq / (sqrt(vv) * qn) : 0.0;
+        if (maxsim) {
+            double best = -INFINITY;
+            for (int w = 0; w < nw; ++w) best = fmax(best, wmax[w]);
+            r = vv > 0.0 ? best / sqrt(vv) : 0.0;
+        }
+        if (c.ext_r) r = (double)c.ext_r[f];   // an external scorer's r_t
         double d = 0.0;
         if (t > 0) {
             const double den = sqrt(vv * pp);
@@ -577,7 +662,18 @@ cudaError_t launch_relevance_pass(const Ctx &c, cudaStream_t s) {
 
 cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s) {
     void *args[] = {const_cast<Ctx *>(&c)};
-    return launch_kernel((const void *)frame_stats_kernel, dim3(c.V * c.T), dim3(512), 0, s, args, c.pdl != 0);
+    const size_t smem = c.relevance_mode == WZ_RELEVANCE_MAXSIM ? (size_t)c.D * 4 : 0;
+    if (smem > 0) {
+        const cudaError_t e =
+            cudaFuncSetAttribute((const void *)frame_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    return launch_kernel((const void *)frame_stats_kernel, dim3(c.V * c.T), dim3(512), smem, s, args, c.pdl != 0);
+}
+
+cudaError_t launch_query_rows(const Ctx &c, int v, int q_row0, int Lq, int Lqp, cudaStream_t s) {
+    void *args[] = {const_cast<Ctx *>(&c), &v, &q_row0, &Lq, &Lqp};
+    return launch_kernel((const void *)query_rows_kernel, dim3((unsigned)Lqp), dim3(256), 0, s, args, c.pdl != 0);
 }
 
 }  // namespace wz

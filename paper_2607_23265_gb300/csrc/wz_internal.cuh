@@ -79,6 +79,9 @@ struct Ctx {
     int spatial_mode;     // WZ_SPATIAL_*
     const float *ext_a;   // [V*T][N] external token scores, or null
     const float *ext_r;   // [V*T] external frame scores, or null
+    int relevance_mode;   // WZ_RELEVANCE_*
+    float *qnorm;         // [V][WZ_MAX_LQ_MAXSIM] query row norms (max-over-query scorer)
+    __nv_bfloat16 *qhl;   // [2 WZ_MAX_LQ_MAXSIM][D] normalised rows, bf16 hi then lo (one video at a time)
     int pdl;              // host: launch with programmatic stream serialization
     float dec_lo[kMaxTaps], dec_hi[kMaxTaps], rec_lo[kMaxTaps], rec_hi[kMaxTaps];
     int wta_F;            // WTA filter taps (temporal DWT, fp64)
@@ -275,6 +278,9 @@ cudaError_t launch_temporal(const Ctx &c, cudaStream_t s);
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s);
 cudaError_t launch_project_gemm(const void *A, int M, int K, const void *B, int N, const float *bias, void *out,
                                 bool gelu, int *status, bool pdl, cudaStream_t s);
+cudaError_t launch_maxsim_gemm(const void *X, int M, int K, const void *QHL, int Lq, int Lqp, float *a, int *status,
+                               bool pdl, cudaStream_t s);
+cudaError_t launch_query_rows(const Ctx &c, int v, int q_row0, int Lq, int Lqp, cudaStream_t s);
 cudaError_t launch_condense_simt(const Ctx &c, cudaStream_t s);
 cudaError_t launch_condense_tc(const Ctx &c, cudaStream_t s);
 int relevance_grid(const Ctx &c);   // CTAs for the relevance pass on this device

@@ -28,6 +28,9 @@ TEMPORAL_WTA, TEMPORAL_RAW, TEMPORAL_UNIFORM = 0, 1, 2
 SPATIAL_WSM, SPATIAL_SALIENCY, SPATIAL_NONE = 0, 1, 2
 TEMPORAL_MODES = {"wta": TEMPORAL_WTA, "raw": TEMPORAL_RAW, "uniform": TEMPORAL_UNIFORM}
 SPATIAL_MODES = {"wsm": SPATIAL_WSM, "saliency": SPATIAL_SALIENCY, "none": SPATIAL_NONE}
+RELEVANCE_MEAN, RELEVANCE_MAXSIM = 0, 1
+RELEVANCE_MODES = {"mean": RELEVANCE_MEAN, "maxsim": RELEVANCE_MAXSIM}
+MAX_LQ_MAXSIM = 128
 
 
 def _enum(table, v):
@@ -52,7 +55,7 @@ class CondenseArgs(C.Structure):
         ("dtype", C.c_int), ("query", C.c_void_p), ("Lq", C.c_int), ("ratio", C.c_float),
         ("lam", C.c_float), ("tau", C.c_float), ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int),
         ("mode", C.c_int), ("path", C.c_int), ("temporal_mode", C.c_int), ("spatial_mode", C.c_int),
-        ("token_scores", C.c_void_p), ("frame_scores", C.c_void_p),
+        ("token_scores", C.c_void_p), ("frame_scores", C.c_void_p), ("relevance_mode", C.c_int),
         ("out_tokens", C.c_void_p), ("out_index", C.c_void_p),
         ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
         ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
@@ -67,7 +70,7 @@ class BatchArgs(C.Structure):
         ("ratio", C.POINTER(C.c_float)), ("lam", C.c_float), ("tau", C.c_float),
         ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int), ("mode", C.c_int), ("path", C.c_int),
         ("temporal_mode", C.c_int), ("spatial_mode", C.c_int),
-        ("token_scores", C.c_void_p), ("frame_scores", C.c_void_p),
+        ("token_scores", C.c_void_p), ("frame_scores", C.c_void_p), ("relevance_mode", C.c_int),
         ("out_tokens", C.c_void_p), ("out_index", C.c_void_p), ("row_offsets", C.POINTER(C.c_int64)),
         ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
         ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
@@ -192,14 +195,16 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
                    tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
                    temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1,
                    token_scores: torch.Tensor | None = None, frame_scores: torch.Tensor | None = None,
-                   workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
+                   relevance="mean", workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
                    device_status: torch.Tensor | None = None, kernel_events=None, stream=None):
     """wz_condense_ex.  Returns a dict with tokens, index, budgets, count and relevance.
 
     kernel_events: optional list of 2*NUM_KERNELS recorded torch.cuda.Event
     objects; event 2k / 2k+1 is recorded right before / after kernel k.
     token_scores [T, H*W] / frame_scores [T]: float32 device tensors of an
-    external scorer (None: the similarity branch's own scores)."""
+    external scorer (None: the similarity branch's own scores).
+    relevance: "mean" (the mean query row) or "maxsim" (maximum cosine over
+    the query rows; bf16 features, D % 64 == 0, at most 128 query rows)."""
     features = _cuda_contig(features, "features")
     query = _cuda_contig(query, "query")
     T, H, W, D = features.shape
@@ -222,6 +227,7 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
     a.path = PATHS[path] if isinstance(path, str) else int(path)
     a.temporal_mode = _enum(TEMPORAL_MODES, temporal_mode)
     a.spatial_mode = _enum(SPATIAL_MODES, spatial_mode)
+    a.relevance_mode = _enum(RELEVANCE_MODES, relevance)
     if token_scores is not None:
         token_scores = _f32_scores(token_scores, (T, H * W), "token_scores")
         a.token_scores = token_scores.data_ptr()
@@ -252,7 +258,7 @@ def wz_batch_rows(V, T, H, W, ratios):
 
 def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios, *, lam: float = 1.5,
                       tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
-                      temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1,
+                      temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1, relevance="mean",
                       workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
                       stream=None):
     """wz_condense_batch: features [V,T,H,W,D], queries [sum Lq, D]."""
@@ -279,6 +285,7 @@ def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios,
     a.path = PATHS[path] if isinstance(path, str) else int(path)
     a.temporal_mode = _enum(TEMPORAL_MODES, temporal_mode)
     a.spatial_mode = _enum(SPATIAL_MODES, spatial_mode)
+    a.relevance_mode = _enum(RELEVANCE_MODES, relevance)
     a.out_tokens, a.out_index, a.row_offsets = tokens.data_ptr(), index.data_ptr(), ro
     a.out_budgets, a.out_count, a.out_relevance = budgets.data_ptr(), count.data_ptr(), rel.data_ptr()
     if workspace is not None:

@@ -48,6 +48,7 @@ def test_struct_layout_matches_defaults(wz):
     wz._lib.wz_condense_args_init(C.byref(a))
     assert (a.lam, a.tau, a.wta_wavelet, a.wsm_wavelet, a.mode, a.path, a.dtype) == (1.5, 0.0, 1, 4, 0, 0, 0)
     assert (a.temporal_mode, a.spatial_mode) == (wz.TEMPORAL_WTA, wz.SPATIAL_WSM)
+    assert a.relevance_mode == wz.RELEVANCE_MEAN
     b = wz.BatchArgs()
     wz._lib.wz_batch_args_init(C.byref(b))
     assert (b.lam, b.wta_wavelet, b.wsm_wavelet) == (1.5, 1, 4)
@@ -113,6 +114,8 @@ def _args(wz, **over):
     (dict(lam=float("inf")), -1), (dict(wta_wavelet=11), -1), (dict(wta_wavelet=0), -1),
     (dict(wsm_wavelet=11), -1), (dict(mode=3), -1), (dict(path=7), -1), (dict(dtype=5), -1),
     (dict(temporal_mode=3), -1), (dict(temporal_mode=-1), -1), (dict(spatial_mode=3), -1),
+    (dict(relevance_mode=2), -1), (dict(relevance_mode=1), -2),                 # max-over-query: D % 64
+    (dict(relevance_mode=1, D=64, dtype=1), -2), (dict(relevance_mode=1, D=64, Lq=129), -2),
     (dict(dtype=1, path=1), -2), (dict(features=P + 4), -1), (dict(out_tokens=3 * P + 8), -1),
     (dict(workspace=5 * P, workspace_bytes=16), -5), (dict(workspace=5 * P + 64, workspace_bytes=1 << 30), -1),
 ])
@@ -146,6 +149,11 @@ def test_batch_argument_errors(wz):
     b.V = 2000
     assert wz._lib.wz_condense_batch(C.byref(b)) == -2          # too many videos
     b.V = 2
+    b.relevance_mode = wz.RELEVANCE_MAXSIM
+    assert wz._lib.wz_condense_batch(C.byref(b)) == -2          # max-over-query wants D % 64 == 0
+    b.D, lq[1] = 64, 200
+    assert wz._lib.wz_condense_batch(C.byref(b)) == -2          # and at most 128 query rows
+    b.D, lq[1], b.relevance_mode = 16, 4, wz.RELEVANCE_MEAN
     b.workspace, b.workspace_bytes = 5 * P, 8
     assert wz._lib.wz_condense_batch(C.byref(b)) == -5
 
