@@ -51,6 +51,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--projector-steps", type=int, default=10,
                    help="also time the projector P (Eq. 17) on the condensed tokens; 0 skips it")
+    p.add_argument("--maxsim-steps", type=int, default=10,
+                   help="also time the step with the max-over-query scorer; 0 skips it")
     return p.parse_args()
 
 
@@ -139,6 +141,59 @@ def time_projector(wz, tokens, steps, dev):
             "ms": round(ms, 5), "bound": "tensor", "achieved": round(achieved, 1), "unit": "TFLOP/s",
             "peak": sustained, "frac": round(achieved / sustained, 4), "frac_of_burst": round(achieved / burst, 4),
             "peak_source": kind + " (sustained: a kernel timed in a back-to-back loop)", "launches": 2 * steps}
+
+
+def time_maxsim(wz, X, Q, ratio, ws, status, steps, dev):
+    """The whole step with the max-over-query scorer (same workload), plain
+    and with kernel events; the token x query-row GEMM (and the small
+    query-row kernel before it) is the span between the relevance pass's
+    end event and frame_stats' start event."""
+    import torch
+    stream = torch.cuda.current_stream(dev)
+    T, H, W, D = X.shape
+    Lq = Q.shape[0]
+    Lqp = (Lq + 15) // 16 * 16
+
+    def step(events=None):
+        return wz.wz_condense_ex(X, Q, ratio, workspace=ws, device_status=status, relevance="maxsim",
+                                 kernel_events=events)
+
+    for _ in range(3):
+        res = step()
+    torch.cuda.synchronize(dev)
+    active = int((res["budgets"] > 0).sum())
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(steps):
+        step()
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = t0.elapsed_time(t1) / steps
+    rel, fs = KERNELS.index("relevance"), KERNELS.index("frame_stats")
+    spans, kern = [], {k: [] for k in KERNELS}
+    for _ in range(steps):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * len(KERNELS))]
+        for e in ev:
+            e.record(stream)   # creates the CUDA event behind the handle
+        step(ev)
+        torch.cuda.synchronize(dev)
+        spans.append(ev[2 * rel + 1].elapsed_time(ev[2 * fs]))
+        for j, k in enumerate(KERNELS):
+            kern[k].append(ev[2 * j].elapsed_time(ev[2 * j + 1]))
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())}: a bounded wait timed out")
+    gemm_ms = statistics.mean(spans)
+    tok = T * H * W
+    nbytes = tok * D * X.element_size() + 2 * 4 * tok   # features once, ||u|| in and a_{t,n} out
+    flop = 2.0 * tok * D * (2 * Lqp)                     # hi and lo halves of the Lqp padded rows
+    peak, peak_kind = measured_peak()
+    gb_s = nbytes / (gemm_ms * 1e-3) / 1e9
+    return {"Lq": Lq, "active_frames": active, "ms_per_step": round(ms, 5), "frames_per_s": round(T / (ms * 1e-3), 1),
+            "gemm": {"ms": round(gemm_ms, 5), "bound": "hbm", "achieved": round(gb_s, 1), "unit": "GB/s",
+                     "peak": peak, "frac": round(gb_s / peak, 4), "peak_source": peak_kind,
+                     "tflop_s": round(flop / (gemm_ms * 1e-3) / 1e12, 1)},
+            "kernels_ms": {k: round(statistics.mean(v), 5) for k, v in kern.items()},
+            "launches_per_step": len(KERNELS) + 2}
 
 
 def source_hash(fname):
@@ -382,6 +437,8 @@ def run_ours(args, spec, world, rank, local):
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.e2e_steps, world, dev)
 
     projector = time_projector(wz, tokens, args.projector_steps, dev) if args.projector_steps > 0 else None
+    maxsim = time_maxsim(wz, X, Q, spec.ratio, ws, status, args.maxsim_steps, dev) \
+        if args.maxsim_steps > 0 and X.dtype == torch.bfloat16 and D % 64 == 0 else None
 
     if rank == 0:
         peak, peak_kind = measured_peak()
@@ -415,6 +472,7 @@ def run_ours(args, spec, world, rank, local):
             "clocks": clocks,
             "gpu_launches": len(KERNELS) * args.steps,
             "projector": projector,
+            "maxsim": maxsim,
         }
         if world == 1 and not args.no_cpu_baseline:
             out["cpu_baseline"] = cpu_baseline(spec, CPU_SAMPLE_FRAMES)

@@ -33,7 +33,8 @@ namespace wz {
 namespace {
 
 constexpr int kPM = 128, kPN = 256, kPK = 64;
-constexpr int kPStages = 4;
+constexpr int kPStages = 4;                          // projector ring (48 KB stages)
+constexpr int kPMaxStages = 8;                       // smaller stages of the row-max GEMM
 constexpr int kPABytes = kPM * kPK * 2;             // 16 KB
 constexpr int kPBBytes = kPN * kPK * 2;             // 32 KB
 constexpr int kPStageBytes = kPABytes + kPBBytes;
@@ -42,8 +43,8 @@ constexpr int kPAccCols = 256;
 constexpr uint64_t kPTimeoutNs = 2000000000ull;
 
 struct PShared {
-    uint64_t full[kPStages];
-    uint64_t empty[kPStages];
+    uint64_t full[kPMaxStages];
+    uint64_t empty[kPMaxStages];
     uint64_t tfull[2];
     uint64_t tempty[2];
     uint64_t drain;
@@ -61,6 +62,8 @@ struct PMaps {
 struct PArgs {
     int M, N, K;
     int tileN;           // MMA N of a tile (<= 256, multiple of 32); the B box height
+    int stages;          // ring stages (<= kPMaxStages, stages * stage_stride <= the ring)
+    int stage_stride;    // bytes per stage: (kPM + tileN) * kPK * 2 rounded to 1 KB
     // epilogue 0 (projector): out = act(acc + bias)
     const float *bias;   // [N] or null
     __nv_bfloat16 *out;  // [M][N]
@@ -90,7 +93,7 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kPStages; ++s) {
+        for (int s = 0; s < p.stages; ++s) {
             ptx::mbar_init(&S->full[s], 1);
             ptx::mbar_init(&S->empty[s], 1);
         }
@@ -126,8 +129,8 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
         const uint64_t pol_b = ptx::policy_evict_last();
         int stage = 0;
         uint32_t phase = 0;
-        int issued_parity[kPStages];
-        for (int s = 0; s < kPStages; ++s) issued_parity[s] = -1;
+        int issued_parity[kPMaxStages];
+        for (int s = 0; s < kPMaxStages; ++s) issued_parity[s] = -1;
         for (int t = blockIdx.x; t < tiles && !*abort_flag; t += gridDim.x) {
             const int m0 = (t / nt) * kPM, n0 = (t % nt) * p.tileN;
             const uint32_t stage_bytes = (uint32_t)(kPM + p.tileN) * kPK * 2;
@@ -138,19 +141,19 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
                     ok = false;
                     break;
                 }
-                uint8_t *st = ring + (size_t)stage * kPStageBytes;
+                uint8_t *st = ring + (size_t)stage * p.stage_stride;
                 ptx::mbar_arrive_expect_tx(&S->full[stage], stage_bytes);
                 ptx::tma_load_2d(st, &maps.a, &S->full[stage], ks * kPK, m0, pol_a);
                 ptx::tma_load_2d(st + kPABytes, &maps.b, &S->full[stage], ks * kPK, n0, pol_b);
                 issued_parity[stage] = (int)phase;
-                if (++stage == kPStages) {
+                if (++stage == p.stages) {
                     stage = 0;
                     phase ^= 1u;
                 }
             }
             if (!ok) break;
         }
-        for (int s = 0; s < kPStages; ++s)
+        for (int s = 0; s < p.stages; ++s)
             if (issued_parity[s] >= 0) ptx::mbar_wait(&S->full[s], (uint32_t)issued_parity[s], kPTimeoutNs);
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer ----------------
@@ -158,7 +161,7 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
         const uint32_t ring32 = ptx::smem_u32(ring);
         const uint64_t a_base = ptx::smem_desc(ring32, 16, 1024, 2);              // 128-B swizzle
         const uint64_t b_base = ptx::smem_desc(ring32 + kPABytes, 16, 1024, 2);
-        constexpr uint64_t kStageDesc = (uint64_t)(kPStageBytes >> 4);
+        const uint64_t stage_desc = (uint64_t)(p.stage_stride >> 4);
         int stage = 0;
         uint32_t phase = 0;
         int it = 0;
@@ -179,13 +182,13 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
                     break;
                 }
                 ptx::tc_fence_after();
-                const uint64_t so = (uint64_t)stage * kStageDesc;
+                const uint64_t so = (uint64_t)stage * stage_desc;
 #pragma unroll
                 for (int k = 0; k < kPK / 16; ++k)   // K = 16 per MMA: 32 bytes along the swizzled row
                     ptx::mma_bf16(d, a_base + so + (uint64_t)(2 * k), b_base + so + (uint64_t)(2 * k), idesc,
                                   (ks | k) ? 1u : 0u);
                 ptx::mma_commit(&S->empty[stage]);
-                if (++stage == kPStages) {
+                if (++stage == p.stages) {
                     stage = 0;
                     phase ^= 1u;
                 }
@@ -317,6 +320,8 @@ cudaError_t launch_project_gemm(const void *A, int M, int K, const void *B, int 
         return cudaErrorInvalidValue;
     PArgs p{};
     p.M = M; p.N = N; p.K = K; p.tileN = kPN;
+    p.stages = kPStages;
+    p.stage_stride = kPStageBytes;
     p.bias = bias; p.out = static_cast<__nv_bfloat16 *>(out); p.gelu = gelu ? 1 : 0; p.status = status;
     int dev = 0, sms = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -346,6 +351,11 @@ cudaError_t launch_maxsim_gemm(const void *X, int M, int K, const void *QHL, int
         return cudaErrorInvalidValue;
     PArgs p{};
     p.M = M; p.N = 2 * Lqp; p.K = K; p.tileN = 2 * Lqp;
+    // a narrower B tile: more, smaller stages in the same ring keep more of the
+    // feature stream in flight (the GEMM is HBM bound at N <= 256)
+    p.stage_stride = (kPM + p.tileN) * kPK * 2;   // multiple of 4 KB (tileN % 32 == 0)
+    p.stages = (kPStages * kPStageBytes) / p.stage_stride;
+    if (p.stages > kPMaxStages) p.stages = kPMaxStages;
     p.a = a; p.Lq = Lq; p.Lqp = Lqp; p.status = status;
     int dev = 0, sms = 0;
     cudaError_t e = cudaGetDevice(&dev);

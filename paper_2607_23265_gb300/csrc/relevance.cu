@@ -459,8 +459,8 @@ __device__ void frame_gate(const Ctx &c, int64_t f, float *red) {
 //
 // With the max-over-query scorer the frame sums are kept in shared memory
 // (D floats of dynamic shared memory) and every warp takes query rows j:
-// <v_t, q_j> with fp32 products per 8 channels summed in fp64, divided by
-// ||q_j||; r_t = max_j of that / ||v_t||.
+// <v_t, q_j> in fp32 (as the per-warp partials of the mean scorer), divided
+// by ||q_j|| in fp64; r_t = max_j of that / ||v_t||.
 __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     pdl_wait();
     pdl_trigger();
@@ -519,21 +519,34 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
         const VideoPar vp = c.vpar[v];
         const int n8 = c.D / 8;
         double best = -INFINITY;
-        for (int j = warp; j < vp.Lq; j += nw) {
+        const int rot = (int)(f % vp.Lq);   // frames start on different rows: no hot L2 lines
+        for (int jr = warp; jr < vp.Lq; jr += nw) {
+            const int j = jr + rot < vp.Lq ? jr + rot : jr + rot - vp.Lq;
             const uint4 *qr = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(c.Q) +
                                                               (size_t)(vp.q_row0 + j) * c.D);
-            double acc = 0.0;
-            for (int i = lane; i < n8; i += 32) {
-                float qf[8];
-                unpack(__ldg(qr + i), qf, (__nv_bfloat16 *)nullptr);
-                const float4 s0 = sfs[2 * i], s1 = sfs[2 * i + 1];
-                const float pp = fmaf(s0.x, qf[0], fmaf(s0.y, qf[1], fmaf(s0.z, qf[2], fmaf(s0.w, qf[3],
-                                 fmaf(s1.x, qf[4], fmaf(s1.y, qf[5], fmaf(s1.z, qf[6], s1.w * qf[7])))))));
-                acc += (double)pp;
+            float acc = 0.f;
+            for (int i0 = lane; i0 < n8; i0 += 32 * 8) {   // 8 loads in flight per lane (L2 latency)
+                uint4 qv[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int i = i0 + 32 * u;
+                    qv[u] = i < n8 ? __ldg(qr + i) : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int i = i0 + 32 * u;
+                    if (i < n8) {
+                        float qf[8];
+                        unpack(qv[u], qf, (__nv_bfloat16 *)nullptr);
+                        const float4 s0 = sfs[2 * i], s1 = sfs[2 * i + 1];
+                        acc = fmaf(s0.x, qf[0], fmaf(s0.y, qf[1], fmaf(s0.z, qf[2], fmaf(s0.w, qf[3],
+                              fmaf(s1.x, qf[4], fmaf(s1.y, qf[5], fmaf(s1.z, qf[6], fmaf(s1.w, qf[7], acc))))))));
+                    }
+                }
             }
             for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
             const double qn = (double)c.qnorm[(size_t)v * WZ_MAX_LQ_MAXSIM + j];
-            best = fmax(best, qn > 0.0 ? acc / qn : 0.0);
+            best = fmax(best, qn > 0.0 ? (double)acc / qn : 0.0);
         }
         if (lane == 0) wmax[warp] = best;
     }
