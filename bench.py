@@ -290,6 +290,35 @@ def cpu_baseline(spec, frames):
             "seconds": r["seconds"]}
 
 
+def cpu_baseline_parallel(spec, frames):
+    """The oracle's per-frame steps spread over every host core (spawned
+    processes, frames sharing one block of shared memory), the coupling steps
+    in the parent: the second CPU baseline.  Same video as cpu_baseline."""
+    code = (
+        "import json,os,sys,time; sys.path.insert(0, %r)\n"
+        "import numpy as np, torch, workload as wl\n"
+        "from oracle.parallel import condense_parallel\n"
+        "s = wl.VideoSpec(T=%d, H=%d, W=%d, D=%d, dtype=%r, Lq=%d, ratio=%r, ar=%r, cuts=%d, seed=%d)\n"
+        "X, Q, _ = wl.make_video(s)\n"
+        "bits, q = X.view(torch.int16).numpy().view(np.uint16), Q.double().numpy()\n"
+        "n = os.cpu_count()\n"
+        "t = time.perf_counter(); condense_parallel(bits, q, s.ratio, n); dt = time.perf_counter() - t\n"
+        "print(json.dumps({'seconds': dt, 'frames': s.T, 'cores': n}))\n"
+    ) % (ROOT, frames, spec.H, spec.W, spec.D, spec.dtype, spec.Lq, spec.ratio, spec.ar,
+         max(1, spec.cuts * frames // spec.T), spec.seed)
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    if spec.dtype != "bf16":
+        return None
+    res = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=900)
+    if res.returncode != 0:
+        return {"value": None, "unit": UNIT, "kind": "oracle, frames over a process pool", "error": res.stderr[-400:]}
+    r = json.loads(res.stdout.strip().splitlines()[-1])
+    return {"value": r["frames"] / r["seconds"], "unit": UNIT, "cores": r["cores"],
+            "kind": "oracle, per-frame steps over a process pool (one process per core)",
+            "sample": f"the same {frames}-frame video as cpu_baseline", "seconds": r["seconds"]}
+
+
 def run_reference(args, spec, world, rank):
     """The oracle, timed on the host cores, on a bounded sample per step."""
     if rank != 0:
@@ -476,6 +505,7 @@ def run_ours(args, spec, world, rank, local):
         }
         if world == 1 and not args.no_cpu_baseline:
             out["cpu_baseline"] = cpu_baseline(spec, CPU_SAMPLE_FRAMES)
+            out["cpu_baseline_parallel"] = cpu_baseline_parallel(spec, CPU_SAMPLE_FRAMES)
         print(json.dumps(out))
     if world > 1:
         dist.destroy_process_group()
