@@ -79,6 +79,14 @@ fact; the same list is kept in the design notes):
       query is not pooled; a_{t,n} = max_j cos(u_{t,n}, q_j) and
       r_t = max_j cos(v_bar_t, q_j) over the Lq rows q_j (with one row it is
       the similarity branch itself).
+  R23 a multi-level option for both wavelet modules (the paper keeps one
+      level, Section 4 "Wavelet Basis"; one level stays the default).  With
+      J levels the DWT cascades on the approximation band.  WTA: the gate of
+      level j's details is the pairwise mean (R8) of level j-1's gate, the
+      gate of level 0 being gamma; the inverse cascades back.  WSM: the
+      detail bands of level j are gated by G_j = lambda * P_down(M_m) with
+      P_down the adaptive average pool (R14) of the saliency map to level
+      j's subband grid; the approximation of level J is not gated.
   R19 an external scorer (Section 3.2.1 names BLIP-style matchers as
       alternatives to the similarity branch) may supply the token saliency
       a_{t,n} and / or the frame relevance r_t; the pooled features still come
@@ -336,20 +344,30 @@ def frame_filter(delta: np.ndarray, tau: float) -> list:
 # Wavelet Temporal Allocator (Eq. 8-10)
 # ----------------------------------------------------------------------------
 
-def wta(r_M: np.ndarray, gamma_M: np.ndarray, p: int = 1) -> np.ndarray:
+def wta(r_M: np.ndarray, gamma_M: np.ndarray, p: int = 1, levels: int = 1) -> np.ndarray:
     """Rectified relevance r~ = IDWT(A, Gamma_bar * D) with (A, D) = DWT(r).
 
     Gamma_bar_k is the mean of the extended gate samples 2k and 2k+1 (R8); the
-    extension is the DWT's half-sample symmetric one (R7).
+    extension is the DWT's half-sample symmetric one (R7).  With levels > 1
+    (R23) the DWT cascades on A, level j's gate is the same pairwise mean of
+    level j-1's gate, and the inverse cascades back.
     """
-    r_M = np.asarray(r_M, dtype=np.float64)
-    L = r_M.size
+    A = np.asarray(r_M, dtype=np.float64)
+    g = np.asarray(gamma_M, dtype=np.float64)
     filt = wavelet_filters(p)
-    A, D = dwt1d(r_M, filt, "symmetric")
-    gbar = np.array([0.5 * (gamma_M[extend_index(2 * k, L, "symmetric")]
-                            + gamma_M[extend_index(2 * k + 1, L, "symmetric")])
-                     for k in range(D.size)])
-    return idwt1d(A, gbar * D, L, filt)
+    details, lengths = [], []
+    for _ in range(levels):
+        n = A.size
+        A_next, D = dwt1d(A, filt, "symmetric")
+        gbar = np.array([0.5 * (g[extend_index(2 * k, n, "symmetric")]
+                                + g[extend_index(2 * k + 1, n, "symmetric")])
+                         for k in range(D.size)])
+        details.append(gbar * D)
+        lengths.append(n)
+        A, g = A_next, gbar
+    for j in reversed(range(levels)):
+        A = idwt1d(A, details[j], lengths[j], filt)
+    return A
 
 
 # ----------------------------------------------------------------------------
@@ -441,14 +459,25 @@ def adaptive_avg_pool2d(M: np.ndarray, oh: int, ow: int) -> np.ndarray:
 
 
 def wsm(X_m: np.ndarray, M_m: np.ndarray, lam: float = 1.5, p: int = 4,
-        mode: str = "symmetric") -> np.ndarray:
-    """X~_m = IDWT2(LL, G*LH, G*HL, G*HH) with G = lambda * P_down(M_m)."""
-    H, W = X_m.shape[:2]
+        mode: str = "symmetric", levels: int = 1) -> np.ndarray:
+    """X~_m = IDWT2(LL, G*LH, G*HL, G*HH) with G = lambda * P_down(M_m).
+
+    levels > 1 (R23): the DWT2 cascades on LL; level j's detail bands are
+    gated by lambda * P_down(M_m) pooled to level j's subband grid.
+    """
     filt = wavelet_filters(p)
-    LL, LH, HL, HH = dwt2d(X_m, filt, mode)
-    G = as_float32(lam) * adaptive_avg_pool2d(M_m, LL.shape[0], LL.shape[1])
-    G = G.reshape(G.shape + (1,) * (X_m.ndim - 2))
-    return idwt2d(LL, G * LH, G * HL, G * HH, H, W, filt)
+    LL = X_m
+    bands, sizes = [], []
+    for _ in range(levels):
+        sizes.append(LL.shape[:2])
+        LL, LH, HL, HH = dwt2d(LL, filt, mode)
+        G = as_float32(lam) * adaptive_avg_pool2d(M_m, LL.shape[0], LL.shape[1])
+        G = G.reshape(G.shape + (1,) * (X_m.ndim - 2))
+        bands.append((G * LH, G * HL, G * HH))
+    for j in reversed(range(levels)):
+        H, W = sizes[j]
+        LL = idwt2d(LL, *bands[j], H, W, filt)
+    return LL
 
 
 # ----------------------------------------------------------------------------
@@ -514,7 +543,8 @@ SPATIAL_MODES = ("wsm", "saliency", "none")
 def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
              wta_wavelet: int = 1, wsm_wavelet: int = 4, mode: str = "symmetric",
              token_frames=None, temporal_mode: str = "wta", spatial_mode: str = "wsm",
-             token_scores=None, frame_scores=None, relevance: str = "mean") -> dict:
+             token_scores=None, frame_scores=None, relevance: str = "mean",
+             wta_levels: int = 1, wsm_levels: int = 1) -> dict:
     """Condense features X (T, H, W, D) for query Q (Lq, D) to B tokens.
 
     token_frames: optional iterable of frame indices; when given, the WSM and
@@ -524,6 +554,7 @@ def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
     token_scores (T, N) / frame_scores (T,): an external scorer's a_{t,n} and
     r_t (reading R19), replacing the similarity branch's values.
     relevance: "mean" (u_q = mean query row, R1) or "maxsim" (reading R22).
+    wta_levels / wsm_levels: decomposition levels of the two modules (R23).
     """
     if temporal_mode not in TEMPORAL_MODES or spatial_mode not in SPATIAL_MODES or relevance not in ("mean", "maxsim"):
         raise ValueError("unknown mode")
@@ -548,7 +579,7 @@ def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
         r = np.asarray(frame_scores, dtype=np.float64).reshape(T).copy()
     delta, gamma = visual_change(vbar)
     keep = frame_filter(delta, as_float32(tau))
-    r_tilde_M = wta(r[keep], gamma[keep], wta_wavelet)
+    r_tilde_M = wta(r[keep], gamma[keep], wta_wavelet, wta_levels)
     B = global_budget(ratio, T, N)
     if temporal_mode == "wta":
         n_M, margins = allocate_budget(r_tilde_M, B, N)
@@ -577,7 +608,7 @@ def condense(X, Q, ratio: float, lam: float = 1.5, tau: float = 0.0,
             out_index[offsets[t] + p] = (t, p // w, p % w)
         if t in frames:
             if spatial_mode == "wsm":
-                Xt = wsm(X[t], saliency_map(a[t], H, W), lam, wsm_wavelet, mode)
+                Xt = wsm(X[t], saliency_map(a[t], H, W), lam, wsm_wavelet, mode, wsm_levels)
             elif spatial_mode == "saliency":
                 Xt = lam * saliency_map(a[t], H, W)[:, :, None] * X[t]
             else:

@@ -746,6 +746,82 @@ def test_project_identity_weights():
 
 
 # ----------------------------------------------------------------------------
+# Multi-level option of the wavelet modules (reading R23)
+# ----------------------------------------------------------------------------
+
+def check_multilevel_wta_hand_case(o):
+    """Haar, two levels, on one block of four samples (worked by hand): the
+    level-1 gates are the pair means of gamma (0.4, 0.5), the level-2 gate
+    their mean (0.45); block mean 3, pair means 2 and 4."""
+    r = np.array([1.0, 3.0, 2.0, 6.0])
+    g = np.array([0.2, 0.6, 1.0, 0.0])
+    # pair means after level 2: 3 -/+ 0.45 * (2 - 4) / 2; then -/+ gate * half-difference
+    assert np.allclose(o.wta(r, g, 1, 2), [2.15, 2.95, 2.45, 4.45], atol=1e-12)
+
+
+def check_multilevel_zero_gate_is_block_mean(o):
+    r = np.array([1.0, 3.0, 2.0, 6.0, 0.0, 4.0, 8.0, 8.0])
+    assert np.allclose(o.wta(r, np.zeros(8), 1, 2), np.repeat([3.0, 5.0], 4), atol=1e-12)
+    assert np.allclose(o.wta(r, np.zeros(8), 1, 3), np.full(8, 4.0), atol=1e-12)
+    X = RNG.standard_normal((8, 8, 2))
+    blocks = X.reshape(2, 4, 2, 4, 2).mean(axis=(1, 3))
+    expect = np.repeat(np.repeat(blocks, 4, axis=0), 4, axis=1)
+    assert np.allclose(o.wsm(X, np.ones((8, 8)), lam=0.0, p=1, levels=2), expect, atol=1e-12)
+
+
+def check_multilevel_wsm_level2_gate(o):
+    """Haar, two levels, a 4x4 map constant on 2x2 blocks (no level-1 detail):
+    the blocks b become mean + G_2 (b - mean) with G_2 = lambda * mean(M),
+    the saliency map pooled to the 1x1 grid of level 2."""
+    b = np.array([[1.0, -2.0], [0.5, 3.5]])
+    X = np.repeat(np.repeat(b, 2, axis=0), 2, axis=1)[:, :, None]
+    M = np.linspace(0.0, 1.0, 16).reshape(4, 4)
+    lam = 1.25
+    g2 = lam * M.mean()
+    mu = b.mean()
+    expect = np.repeat(np.repeat(mu + g2 * (b - mu), 2, axis=0), 2, axis=1)[:, :, None]
+    assert np.allclose(o.wsm(X, M, lam=lam, p=1, levels=2), expect, atol=1e-12)
+
+
+def test_multilevel_wta_hand_case():
+    check_multilevel_wta_hand_case(O)
+
+
+def test_multilevel_zero_gate_is_block_mean():
+    check_multilevel_zero_gate_is_block_mean(O)
+
+
+def test_multilevel_wsm_level2_gate():
+    check_multilevel_wsm_level2_gate(O)
+
+
+@pytest.mark.parametrize("p", [1, 2, 4, 44])
+@pytest.mark.parametrize("levels", [2, 3, 4])
+def test_multilevel_unit_gate_is_identity(p, levels):
+    for L in (1, 2, 5, 23, 64):
+        r = RNG.standard_normal(L)
+        assert np.allclose(O.wta(r, np.ones(L), p, levels), r, atol=1e-11)
+    for H, W in ((4, 4), (9, 11), (27, 27)):
+        X = RNG.standard_normal((H, W, 2))
+        assert np.allclose(O.wsm(X, np.ones((H, W)), lam=1.0, p=p, levels=levels), X, atol=1e-10)
+
+
+def test_multilevel_one_level_is_the_single_level_module():
+    r, g = RNG.standard_normal(19), RNG.random(19)
+    X, M = RNG.standard_normal((13, 13, 3)), RNG.random((13, 13))
+    assert np.array_equal(O.wta(r, g, 4, 1), O.wta(r, g, 4))
+    assert np.array_equal(O.wsm(X, M, 1.5, 4, "symmetric", 1), O.wsm(X, M, 1.5, 4))
+
+
+def test_multilevel_condense_invariants():
+    X = RNG.standard_normal((9, 7, 8, 4))
+    Q = RNG.standard_normal((3, 4))
+    res = O.condense(X, Q, 0.3, wta_levels=3, wsm_levels=2)
+    assert res["budgets"].sum() == O.global_budget(0.3, 9, 56)
+    assert np.all(np.isfinite(res["out_tokens"]))
+
+
+# ----------------------------------------------------------------------------
 # Mutation tests: a planted mistake in the oracle makes a pin fail
 # ----------------------------------------------------------------------------
 
@@ -904,3 +980,38 @@ def test_mutation_maxsim_min_breaks_hand_case():
         return res
     m = _mutant(condense=min_condense)
     assert _fails(check_maxsim_hand_case, m)
+
+
+def test_mutation_level2_gate_from_gamma_breaks_multilevel_pin():
+    def wta_bad(r_M, gamma_M, p=1, levels=1):         # planted: every level gated by gamma's pair means
+        A = np.asarray(r_M, dtype=np.float64)
+        filt = OM.wavelet_filters(p)
+        n0 = A.size
+        g1 = lambda k: 0.5 * (gamma_M[OM.extend_index(2 * k, n0, "symmetric")]
+                              + gamma_M[OM.extend_index(2 * k + 1, n0, "symmetric")])
+        details, lengths = [], []
+        for _ in range(levels):
+            n = A.size
+            A_next, D = OM.dwt1d(A, filt, "symmetric")
+            details.append(np.array([g1(k) for k in range(D.size)]) * D)
+            lengths.append(n)
+            A = A_next
+        for j in reversed(range(levels)):
+            A = OM.idwt1d(A, details[j], lengths[j], filt)
+        return A
+    assert _fails(check_multilevel_wta_hand_case, _mutant(wta=wta_bad))
+
+
+def test_mutation_gated_level1_approximation_breaks_multilevel_pin():
+    original = OM.wsm
+
+    def wsm_bad(X_m, M_m, lam=1.5, p=4, mode="symmetric", levels=1):   # planted: LL of level 1 gated too
+        if levels == 1:
+            return original(X_m, M_m, lam, p, mode)
+        filt = OM.wavelet_filters(p)
+        LL, LH, HL, HH = OM.dwt2d(X_m, filt, mode)
+        G = OM.as_float32(lam) * OM.adaptive_avg_pool2d(M_m, LL.shape[0], LL.shape[1])
+        G = G.reshape(G.shape + (1,) * (X_m.ndim - 2))
+        inner = original(LL, OM.adaptive_avg_pool2d(M_m, LL.shape[0], LL.shape[1]), lam, p, mode, levels - 1)
+        return OM.idwt2d(G * inner, G * LH, G * HL, G * HH, X_m.shape[0], X_m.shape[1], filt)
+    assert _fails(check_multilevel_zero_gate_is_block_mean, _mutant(wsm=wsm_bad))
