@@ -105,6 +105,12 @@ typedef struct CUstream_st *wz_stream_t;
 #define WZ_RELEVANCE_MAXSIM  1
 #define WZ_MAX_LQ_MAXSIM     128
 
+/* Decomposition levels of the WTA and the WSM (the paper's modules use one;
+ * with J > 1 the DWT cascades on the approximation band, level j's details
+ * gated by the pairwise mean of level j-1's gate (WTA) or by the saliency
+ * map pooled to level j's subband grid (WSM)). */
+#define WZ_MAX_LEVELS 4
+
 /* Wavelets: Daubechies filters named by their vanishing moments p (2p
  * taps), 1 = Haar, 4 = db4, 1 <= p <= 10; and the biorthogonal bior4.4
  * (CDF 9/7, 10-tap arrays), the third basis of the paper's "Wavelet Basis"
@@ -167,6 +173,8 @@ typedef struct {
                              /* similarity branch's; nullable                */
     const float *frame_scores; /* [T] f32 device, external r_t; nullable     */
     int relevance_mode;      /* WZ_RELEVANCE_*, default MEAN                 */
+    int wta_levels;          /* 1..WZ_MAX_LEVELS, default 1                  */
+    int wsm_levels;          /* 1..WZ_MAX_LEVELS, default 1                  */
     void *out_tokens;        /* [B][D], dtype                                */
     int32_t *out_index;      /* [B][3]                                       */
     int32_t *out_budgets;    /* [T] n_t (0 for filtered frames); nullable    */
@@ -219,6 +227,7 @@ typedef struct {
     const float *token_scores;         /* [V][T][N] device, nullable   */
     const float *frame_scores;         /* [V][T] device, nullable      */
     int relevance_mode;                /* WZ_RELEVANCE_*               */
+    int wta_levels, wsm_levels;        /* 1..WZ_MAX_LEVELS             */
     void *out_tokens;
     int32_t *out_index;
     int64_t *row_offsets;    /* host, [V+1], nullable */

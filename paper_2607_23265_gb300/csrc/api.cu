@@ -60,11 +60,12 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.units = take((size_t)s.V * s.max_units_v * 16);
     L.ucount = take((size_t)s.V * 4);
     L.ustart = take(VT * 4);
-    L.stab = take(spatial_table_bytes(s.H, s.W, kMaxTaps));   // any wavelet
+    L.stab = take(std::max(spatial_table_bytes(s.H, s.W, kMaxTaps),            // any wavelet,
+                           ml_table_bytes(s.H, s.W, kMaxTaps, kMaxLevels)));   // any level count
     L.drange = take((size_t)s.V * 16);
     L.qnorm = take((size_t)s.V * WZ_MAX_LQ_MAXSIM * 4);
     L.qhl = take((size_t)2 * WZ_MAX_LQ_MAXSIM * s.D * 2);
-    L.gate = with_operator ? take(VT * (size_t)((s.H + kMaxTaps - 1) / 2) * ((s.W + kMaxTaps - 1) / 2) * 4) : 0;
+    L.gate = with_operator ? take(VT * (size_t)gate_floats(s.H, s.W, kMaxTaps, kMaxLevels) * 4) : 0;
     L.status = take(16);
     L.Wop = with_operator ? take((size_t)std::max<int64_t>(s.rows_total, s.w_rows) * s.K_pad * 4) : 0;
     L.total = o;
@@ -116,6 +117,7 @@ struct Common {
     float lambda, tau;
     int wta_wavelet, wsm_wavelet, mode, path, temporal_mode, spatial_mode;
     int relevance_mode = WZ_RELEVANCE_MEAN;
+    int wta_levels = 1, wsm_levels = 1;
 };
 
 int check_common(const Common &m, int dtype) {
@@ -126,6 +128,8 @@ int check_common(const Common &m, int dtype) {
     if (m.path == WZ_PATH_TENSOR && dtype != WZ_DTYPE_BF16) return WZ_ERR_UNSUPPORTED;
     if (m.temporal_mode < WZ_TEMPORAL_WTA || m.temporal_mode > WZ_TEMPORAL_UNIFORM) return WZ_ERR_INVALID_ARG;
     if (m.spatial_mode < WZ_SPATIAL_WSM || m.spatial_mode > WZ_SPATIAL_NONE) return WZ_ERR_INVALID_ARG;
+    if (m.wta_levels < 1 || m.wta_levels > kMaxLevels || m.wsm_levels < 1 || m.wsm_levels > kMaxLevels)
+        return WZ_ERR_INVALID_ARG;
     return WZ_OK;
 }
 
@@ -156,6 +160,22 @@ void set_wta_filters(Ctx &c, int p) {
         c.wta_rec_lo[k] = k < c.wta_F ? rl[k] : 0.0;
         c.wta_rec_hi[k] = k < c.wta_F ? rh[k] : 0.0;
     }
+}
+
+// Level counts and the WSM subband grids of every level (c.F set).
+void set_levels(Ctx &c, int H, int W, int wta_levels, int wsm_levels) {
+    c.wta_levels = wta_levels;
+    c.wsm_levels = wsm_levels;
+    int off = 0;
+    for (int l = 0; l <= kMaxLevels; ++l) {
+        c.lvl_h[l] = level_size(H, c.F, l);
+        c.lvl_w[l] = level_size(W, c.F, l);
+        if (l >= 1) {
+            c.goff[l - 1] = off;
+            if (l <= wsm_levels) off += c.lvl_h[l] * c.lvl_w[l];
+        }
+    }
+    c.gate_stride = off;
 }
 
 void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
@@ -246,6 +266,9 @@ int validate(const CondenseRequest &r, std::vector<int64_t> &B, int64_t &rows) {
     if (!aligned(r.features, 16) || !aligned(r.queries, 16)) return WZ_ERR_INVALID_ARG;
     if (!aligned(r.token_scores, 4) || !aligned(r.frame_scores, 4)) return WZ_ERR_INVALID_ARG;
     if (r.m.relevance_mode != WZ_RELEVANCE_MEAN && r.m.relevance_mode != WZ_RELEVANCE_MAXSIM) return WZ_ERR_INVALID_ARG;
+    if (r.m.wsm_levels > 1 && r.m.spatial_mode == WZ_SPATIAL_WSM &&
+        spatial_ml_smem_bytes(r.H, r.W, wavelet_taps(r.m.wsm_wavelet), r.m.wsm_levels) == 0)
+        return WZ_ERR_UNSUPPORTED;   // the multi-level tables of this map do not fit one CTA
     if (r.m.relevance_mode == WZ_RELEVANCE_MAXSIM) {
         if (r.dtype != WZ_DTYPE_BF16 || r.D % 64 != 0) return WZ_ERR_UNSUPPORTED;
         for (int v = 0; v < r.V; ++v)
@@ -286,6 +309,7 @@ int run_condense(const CondenseRequest &r) {
     c.pdl = r.events ? 0 : 1;      // an event between two kernels would break the overlap
     set_filters(c, r.m.wsm_wavelet);
     set_wta_filters(c, r.m.wta_wavelet);
+    set_levels(c, r.H, r.W, r.m.wta_levels, r.m.spatial_mode == WZ_SPATIAL_WSM ? r.m.wsm_levels : 1);
     const Shape s = make_shape(r.V, r.T, r.H, r.W, r.D, r.dtype, c.F, B.data());
     const Layout L = make_layout(s, true, true);
     Scratch ws;
@@ -392,6 +416,8 @@ void wz_condense_args_init(wz_condense_args *a) {
     a->wsm_wavelet = WZ_WAVELET_DB4;
     a->mode = WZ_MODE_SYMMETRIC;
     a->path = WZ_PATH_AUTO;
+    a->wta_levels = 1;
+    a->wsm_levels = 1;
 }
 
 void wz_batch_args_init(wz_batch_args *a) {
@@ -404,6 +430,8 @@ void wz_batch_args_init(wz_batch_args *a) {
     a->wsm_wavelet = WZ_WAVELET_DB4;
     a->mode = WZ_MODE_SYMMETRIC;
     a->path = WZ_PATH_AUTO;
+    a->wta_levels = 1;
+    a->wsm_levels = 1;
 }
 
 size_t wz_condense_workspace_size(int T, int H, int W, int D, int dtype, float ratio) {
@@ -423,6 +451,8 @@ int wz_condense_ex(const wz_condense_args *a) {
     r.token_scores = a->token_scores;
     r.frame_scores = a->frame_scores;
     r.m.relevance_mode = a->relevance_mode;
+    r.m.wta_levels = a->wta_levels;
+    r.m.wsm_levels = a->wsm_levels;
     r.out_tokens = a->out_tokens;
     r.out_index = a->out_index;
     r.out_budgets = a->out_budgets;
@@ -481,6 +511,8 @@ int wz_condense_batch(const wz_batch_args *a) {
     r.token_scores = a->token_scores;
     r.frame_scores = a->frame_scores;
     r.m.relevance_mode = a->relevance_mode;
+    r.m.wta_levels = a->wta_levels;
+    r.m.wsm_levels = a->wsm_levels;
     r.out_tokens = a->out_tokens;
     r.out_index = a->out_index;
     r.out_budgets = a->out_budgets;

@@ -406,12 +406,12 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
 }
 
 // Gate of the WSM for frame f (Eq. 6, Eq. 12): the saliency map M = min-max
-// normalised a_{t,n} over the frame, average-pooled to the hp x wp grid of
-// the first DWT level and scaled by lambda.  `red` is >= 32 floats of
-// shared scratch.
+// normalised a_{t,n} over the frame, average-pooled to the subband grid of
+// each DWT level (hp x wp for the first) and scaled by lambda.  `red` is >= 32
+// floats of shared scratch.
 __device__ void frame_gate(const Ctx &c, int64_t f, float *red) {
     __shared__ float M[WZ_MAX_HW * WZ_MAX_HW];
-    const int N = c.N, H = c.H, W = c.W, hp = c.hp, wp = c.wp;
+    const int N = c.N, H = c.H, W = c.W;
     const float *a = (c.ext_a ? c.ext_a : c.a) + f * N;   // an external scorer's a_{t,n} if given
     float lo = INFINITY, hi = -INFINITY;
     for (int k = threadIdx.x; k < N; k += blockDim.x) {
@@ -439,15 +439,18 @@ __device__ void frame_gate(const Ctx &c, int64_t f, float *red) {
     const float rng = hi - lo;
     for (int k = threadIdx.x; k < N; k += blockDim.x) M[k] = rng > 0.f ? (M[k] - lo) / rng : 0.f;
     __syncthreads();
-    float *G = c.gate + f * (int64_t)(hp * wp);
-    for (int k = threadIdx.x; k < hp * wp; k += blockDim.x) {
-        const int ai = k / wp, bj = k % wp;
-        const int r0 = (ai * H) / hp, r1 = ((ai + 1) * H + hp - 1) / hp;
-        const int c0 = (bj * W) / wp, c1 = ((bj + 1) * W + wp - 1) / wp;
-        float s = 0.f;
-        for (int y = r0; y < r1; ++y)
-            for (int x = c0; x < c1; ++x) s += M[y * W + x];
-        G[k] = c.lambda * (s / (float)((r1 - r0) * (c1 - c0)));
+    for (int l = 1; l <= c.wsm_levels; ++l) {
+        const int hp = c.lvl_h[l], wp = c.lvl_w[l];
+        float *G = c.gate + f * (int64_t)c.gate_stride + c.goff[l - 1];
+        for (int k = threadIdx.x; k < hp * wp; k += blockDim.x) {
+            const int ai = k / wp, bj = k % wp;
+            const int r0 = (ai * H) / hp, r1 = ((ai + 1) * H + hp - 1) / hp;
+            const int c0 = (bj * W) / wp, c1 = ((bj + 1) * W + wp - 1) / wp;
+            float s = 0.f;
+            for (int y = r0; y < r1; ++y)
+                for (int x = c0; x < c1; ++x) s += M[y * W + x];
+            G[k] = c.lambda * (s / (float)((r1 - r0) * (c1 - c0)));
+        }
     }
 }
 

@@ -27,80 +27,6 @@
 
 namespace wz {
 
-constexpr int kSpatialThreads = 256;
-constexpr int kTailBlocks = 64;
-__device__ __forceinline__ float synth(const float *rec, int F, int y, int a) {
-    const int k = y + F - 2 - 2 * a;
-    return (k >= 0 && k < F) ? rec[k] : 0.f;
-}
-
-// Half-pixel bilinear source (align_corners = false): rows y0, y1, weight of
-// y1.  The source coordinate s = (i + 1/2) in / out - 1/2, clamped at 0, is
-// the rational ((2i + 1) in - out) / (2 out): its floor and remainder are
-// exact in integers, and the weight is the remainder divided in fp32.
-__device__ __forceinline__ void bilinear_src(int i, int in, int out, int &y0, int &y1, float &l) {
-    const int num = (2 * i + 1) * in - out, den = 2 * out;
-    int f = 0, rem = 0;
-    if (num > 0) {
-        f = num / den;
-        rem = num - f * den;
-    }
-    if (f > in - 1) {
-        f = in - 1;
-        rem = 0;
-    }
-    y0 = f;
-    y1 = f + 1 < in ? f + 1 : in - 1;
-    l = (float)rem / (float)den;
-}
-
-// Coefficients a with synth(y, a) != 0 for y in {y0, y1}: y + F - 2 - 2a in [0, F).
-__device__ __forceinline__ void synth_support(int y0, int y1, int F, int na, int &lo, int &hi) {
-    lo = y0 >> 1;
-    hi = min(na - 1, (y1 + F - 2) >> 1);
-}
-
-// Staged rows [0, qn) of a grid row go out in 8-column groups: bf16 hi and
-// lo halves at tile_index(r, 8 g, w_rows) (tensor path; r = r_first + row,
-// split into a row part and a column part) or fp32 rows (CUDA-core path).
-__device__ __forceinline__ void write_rows(const float *stg, int qn, int K_pad, int64_t r_first, bool bf,
-                                           __nv_bfloat16 *Whi, __nv_bfloat16 *Wlo, float *W32, size_t kstride) {
-    const int G8 = K_pad / 8;
-    int ql_ = (int)threadIdx.x / G8, g = (int)threadIdx.x % G8;
-    const int gstep = (int)blockDim.x % G8, qstep = (int)blockDim.x / G8;
-    for (; ql_ < qn;) {
-        const float4 v0 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g);
-        const float4 v1 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g + 4);
-        const int64_t r = r_first + ql_;
-        if (bf) {
-            const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-            uint32_t hw[4], lw[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
-                const __nv_bfloat162 ll =
-                    __floats2bfloat162_rn(v[2 * e] - __low2float(hh), v[2 * e + 1] - __high2float(hh));
-                hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
-                lw[e] = *reinterpret_cast<const uint32_t *>(&ll);
-            }
-            const size_t ti = (size_t)(g >> 2) * kstride + (size_t)(r >> 3) * 256 + (size_t)(r & 7) * 8 +
-                              (size_t)(g & 3) * 64;
-            *reinterpret_cast<uint4 *>(Whi + ti) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-            *reinterpret_cast<uint4 *>(Wlo + ti) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-        } else {
-            float *dst = W32 + (size_t)r * K_pad + 8 * g;
-            *reinterpret_cast<float4 *>(dst) = v0;
-            *reinterpret_cast<float4 *>(dst + 4) = v1;
-        }
-        g += gstep;
-        ql_ += qstep;
-        if (g >= G8) {
-            g -= G8;
-            ++ql_;
-        }
-    }
-}
-
 // Operator rows of the ablation modes without the WSM (spatial "saliency" and
 // "none"): W[(p,q),(y,x)] = Ry[p][y] Rx[q][x] s(y, x), the bilinear weights of
 // Eq. 16 times s = lambda * M_t (Eq. 6 map) or 1.  Same staging, layout and
@@ -190,19 +116,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     const int tid = threadIdx.x;
     const int64_t nblk_frames = (int64_t)c.V * c.T * S;
     if ((int64_t)blockIdx.x >= nblk_frames) {
-        // rows past the produced count: index -1, zero tokens
-        const int tb = (int)(blockIdx.x - nblk_frames);
-        const size_t esz = c.dtype == WZ_DTYPE_BF16 ? 2 : 4;
-        const int nvec = (int)((size_t)c.D * esz / 16);
-        for (int v = 0; v < c.V; ++v) {
-            const int r0 = c.vpar[v].row0 + c.prod[v];
-            const int r1 = c.vpar[v].row0 + c.vpar[v].B;
-            for (int r = r0 + tb; r < r1; r += kTailBlocks) {
-                uint4 *o = reinterpret_cast<uint4 *>(static_cast<char *>(c.out) + (size_t)r * c.D * esz);
-                for (int k = tid; k < nvec; k += blockDim.x) o[k] = make_uint4(0u, 0u, 0u, 0u);
-                if (tid < 3) c.out_index[(size_t)r * 3 + tid] = -1;
-            }
-        }
+        tail_rows(c, (int)(blockIdx.x - nblk_frames));
         return;
     }
     const int64_t f = blockIdx.x / S;
@@ -211,25 +125,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     if (n <= 0) return;
     const int h = c.hw[2 * f], w = c.hw[2 * f + 1];
     if (s0 >= h || s0 * w >= n) return;
-    if (s0 == 0 && c.path == WZ_PATH_TENSOR) {
-        // this frame's tensor-core units (the temporal kernel placed them):
-        // column blocks of <= 256 tokens, each in groups of
-        // unit_tiles(round16(nc)) 128-channel tiles
-        const int v = (int)(f / c.T);
-        int4 *units = c.units + (size_t)v * c.max_units_v;
-        int u0 = c.ustart[f];
-        for (int j0 = 0; j0 < n; j0 += kColBlock) {
-            const int nc = min(kColBlock, n - j0);
-            const int cg = unit_tiles((nc + 15) / 16 * 16);
-            const int cnt = (c.n_ct + cg - 1) / cg;
-            for (int li = tid; li < cnt; li += blockDim.x) {
-                const int ct = li * cg;
-                if (u0 + li < c.max_units_v)
-                    units[u0 + li] = make_int4((int)f, j0, ct, nc | (min(cg, c.n_ct - ct) << 16));
-            }
-            u0 += cnt;
-        }
-    }
+    if (s0 == 0 && c.path == WZ_PATH_TENSOR) unit_records(c, f, n);
     const int H = c.H, W = c.W, N = c.N, hp = c.hp, wp = c.wp, F = c.F;
     SpatialSmem L;
     L.init(H, W, hp, wp);
@@ -252,7 +148,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     // per pass
     for (int k = tid; k < L.tables; k += blockDim.x) reinterpret_cast<int *>(sm)[k] = reinterpret_cast<const int *>(c.stab)[k];
     // gate G of this frame (Eq. 6, Eq. 12), pooled by frame_stats
-    const float *Gf = c.gate + f * (int64_t)(hp * wp);
+    const float *Gf = c.gate + f * (int64_t)c.gate_stride;
     for (int k = tid; k < hp * wp; k += blockDim.x) G[k] = Gf[k];
     // bilinear columns through the synthesis: Q_v[q][b] and its support
     for (int k = tid; k < w * wp; k += blockDim.x) {
@@ -401,6 +297,7 @@ int spatial_split(const Ctx &c, int resident) {
 }
 
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
+    if (c.spatial_mode == WZ_SPATIAL_WSM && c.wsm_levels > 1) return launch_spatial_ml(c, s);
     SpatialSmem L;
     L.init(c.H, c.W, c.hp, c.wp);
     if ((L.Yl & 3) != 0 || (L.Yh & 3) != 0 || (L.stage & 3) != 0 || L.QB < 1) return cudaErrorMisalignedAddress;

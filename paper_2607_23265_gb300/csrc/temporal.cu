@@ -68,8 +68,22 @@ __device__ __forceinline__ int grid_h(int n, int H, int W) {
 // Shared-memory arrays of one video, indexed by retained frame m (wgt,
 // keys, lst, nb) or by frame t (nf).
 __host__ __device__ inline size_t temporal_smem_offset_coef(int T) { return ((size_t)T * (8 + 8 + 4 + 4 + 4) + 7) & ~(size_t)7; }
-__host__ __device__ inline size_t temporal_smem_bytes(int T) {
-    return temporal_smem_offset_coef(T) + 2 * sizeof(double) * (size_t)((T + kMaxTaps - 1) / 2);
+// WTA coefficient arrays: the longest subband of any level (any filter).
+__host__ __device__ inline int temporal_coef_len(int T, int J) {
+    const int k = (T + kMaxTaps - 1) / 2;
+    return J > 1 && k < kMaxTaps ? kMaxTaps : k;
+}
+// Detail coefficients of all J levels, back to back (lengths halve, plus at
+// most F/2 per level).
+__host__ __device__ inline int temporal_detail_len(int T, int J) {
+    const int k = temporal_coef_len(T, J);
+    return J > 1 ? 2 * k + J * kMaxTaps : k;
+}
+// The coefficient part: approximation A0 | details | (J > 1) A1 | G0 | G1.
+__host__ __device__ inline size_t temporal_smem_bytes(int T, int J) {
+    const size_t k = (size_t)temporal_coef_len(T, J);
+    const size_t coef = k + (size_t)temporal_detail_len(T, J) + (J > 1 ? 3 * k : 0);
+    return temporal_smem_offset_coef(T) + sizeof(double) * coef;
 }
 
 // Threads of the CTA: one frame per thread up to 512 frames, at most
@@ -81,7 +95,8 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     pdl_trigger();
     if ((int)blockIdx.x == c.V) {
         // the extra CTA: frame-independent tables of the spatial operator
-        build_spatial_tables(c);
+        if (c.wsm_levels > 1) build_ml_tables(c);
+        else build_spatial_tables(c);
         return;
     }
     extern __shared__ __align__(16) unsigned char tsm[];
@@ -98,8 +113,12 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     int *lst = reinterpret_cast<int *>(keys + T);                         // retained frames
     int *nb = lst + T;                     // budget of retained frame m; -1 while active
     int *nf = nb + T;                      // budget of frame t
-    double *cA = reinterpret_cast<double *>(tsm + temporal_smem_offset_coef(T));   // WTA approximation
-    double *cD = cA + (T + kMaxTaps - 1) / 2;                                       // gated WTA detail
+    const int J = c.wta_levels;
+    const int KH = temporal_coef_len(T, J);
+    double *A0 = reinterpret_cast<double *>(tsm + temporal_smem_offset_coef(T));   // WTA approximation
+    double *dall = A0 + KH;                                                         // gated details, all levels
+    double *A1 = dall + temporal_detail_len(T, J);                                  // (J > 1) ping-pong
+    double *G0 = A1 + KH, *G1 = G0 + KH;                                            // (J > 1) gates of a level
 
     // r_t and delta_t come from frame_stats, which also kept the range of
     // delta over the video (Eq. 7)
@@ -136,31 +155,69 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     // wavelet (Daubechies p, 2p taps; half-sample symmetric extension, as the
     // WSM's), each detail coefficient k gated by the mean of the extended gate
     // samples 2k and 2k+1, inverse DWT.  For Haar an odd last sample pairs
-    // with its mirror image, so its detail is 0 and it passes through.
+    // with its mirror image, so its detail is 0 and it passes through.  With
+    // J > 1 levels the DWT cascades on the approximation and level j's gate is
+    // the same pairwise mean of level j-1's gate; the inverse cascades back.
     // Budget weights are max(r~, 0) (Eq. 5); the ablation modes use max(r, 0)
     // ("raw") or 1 ("uniform") instead.
     const int FT = c.wta_F;
-    const int K = (L + FT - 1) / 2;
-    for (int k = threadIdx.x; k < K; k += blockDim.x) {
-        double ca = 0.0, cd = 0.0;
-        for (int j = 0; j < FT; ++j) {
-            const double x = fr[4 * lst[ext_index(2 * k + 1 - j, L, WZ_MODE_SYMMETRIC)]];
-            ca += c.wta_dec_lo[j] * x;
-            cd += c.wta_dec_hi[j] * x;
-        }
-        const int m0 = ext_index(2 * k, L, WZ_MODE_SYMMETRIC), m1 = ext_index(2 * k + 1, L, WZ_MODE_SYMMETRIC);
-        const double g = 0.5 * (fr[4 * lst[m0] + 2] + fr[4 * lst[m1] + 2]);
-        cA[k] = ca;
-        cD[k] = g * cd;
+    int lens[kMaxLevels + 1], doff[kMaxLevels];
+    lens[0] = L;
+    for (int j = 1, o = 0; j <= J; ++j) {
+        lens[j] = (lens[j - 1] + FT - 1) / 2;
+        doff[j - 1] = o;
+        o += lens[j];
     }
-    __syncthreads();
+    const double *ain = nullptr, *gin = nullptr;   // level 1 reads r and gamma of the retained frames
+    double *aout = A0, *gout = G0;
+    for (int j = 1; j <= J; ++j) {
+        const int n = lens[j - 1], K = lens[j];
+        for (int k = threadIdx.x; k < K; k += blockDim.x) {
+            double ca = 0.0, cd = 0.0;
+            for (int i = 0; i < FT; ++i) {
+                const int m = ext_index(2 * k + 1 - i, n, WZ_MODE_SYMMETRIC);
+                const double x = ain ? ain[m] : fr[4 * lst[m]];
+                ca += c.wta_dec_lo[i] * x;
+                cd += c.wta_dec_hi[i] * x;
+            }
+            const int m0 = ext_index(2 * k, n, WZ_MODE_SYMMETRIC), m1 = ext_index(2 * k + 1, n, WZ_MODE_SYMMETRIC);
+            const double g = gin ? 0.5 * (gin[m0] + gin[m1]) : 0.5 * (fr[4 * lst[m0] + 2] + fr[4 * lst[m1] + 2]);
+            aout[k] = ca;
+            if (j < J) gout[k] = g;
+            dall[doff[j - 1] + k] = g * cd;
+        }
+        __syncthreads();
+        ain = aout;
+        gin = gout;
+        aout = aout == A0 ? A1 : A0;
+        gout = gout == G0 ? G1 : G0;
+    }
+    // inverse of levels J .. 2 into the free approximation buffer
+    for (int j = J; j >= 2; --j) {
+        const int n = lens[j - 1], K = lens[j];
+        const double *dj = dall + doff[j - 1];
+        for (int m = threadIdx.x; m < n; m += blockDim.x) {
+            double x = 0.0;
+            const int alo = m >> 1, ahi = min(K - 1, (m + FT - 2) >> 1);
+            for (int ai = alo; ai <= ahi; ++ai) {
+                const int kk = m + FT - 2 - 2 * ai;
+                x += c.wta_rec_lo[kk] * ain[ai] + c.wta_rec_hi[kk] * dj[ai];
+            }
+            aout[m] = x;
+        }
+        __syncthreads();
+        const double *t_ = ain;
+        ain = aout;
+        aout = const_cast<double *>(t_);
+    }
+    const int K = lens[1];
     int anypos = 0;
     for (int m = threadIdx.x; m < L; m += blockDim.x) {
         double rt = 0.0;
         const int alo = m >> 1, ahi = min(K - 1, (m + FT - 2) >> 1);
         for (int ai = alo; ai <= ahi; ++ai) {
             const int kk = m + FT - 2 - 2 * ai;       // synthesis tap, 0 <= kk < FT
-            rt += c.wta_rec_lo[kk] * cA[ai] + c.wta_rec_hi[kk] * cD[ai];
+            rt += c.wta_rec_lo[kk] * ain[ai] + c.wta_rec_hi[kk] * dall[ai];
         }
         const int t = lst[m];
         fr[4 * t + 3] = rt;
@@ -354,7 +411,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
 }
 
 cudaError_t launch_temporal(const Ctx &c, cudaStream_t s) {
-    const size_t smem = temporal_smem_bytes(c.T);
+    const size_t smem = temporal_smem_bytes(c.T, c.wta_levels);
     cudaError_t e = cudaFuncSetAttribute(temporal_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     void *args[] = {const_cast<Ctx *>(&c)};

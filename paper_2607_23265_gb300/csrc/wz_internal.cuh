@@ -10,6 +10,7 @@
 namespace wz {
 
 constexpr int kMaxTaps = 20;          // Daubechies order <= 10
+constexpr int kMaxLevels = WZ_MAX_LEVELS;   // decomposition levels of the WTA / WSM
 constexpr int kG1Max = 2048;          // relevance-pass CTAs (upper bound)
 constexpr int kColBlock = 256;        // output tokens per tensor-core unit
 constexpr int kTileC = 128;           // channels per tensor-core M tile
@@ -82,6 +83,11 @@ struct Ctx {
     int relevance_mode;   // WZ_RELEVANCE_*
     float *qnorm;         // [V][WZ_MAX_LQ_MAXSIM] query row norms (max-over-query scorer)
     __nv_bfloat16 *qhl;   // [2 WZ_MAX_LQ_MAXSIM][D] normalised rows, bf16 hi then lo (one video at a time)
+    int wta_levels;       // WTA decomposition levels (1 = the paper's single level)
+    int wsm_levels;       // WSM decomposition levels
+    int gate_stride;      // floats of c.gate per frame: sum over levels of lvl_h * lvl_w
+    int lvl_h[kMaxLevels + 1], lvl_w[kMaxLevels + 1];   // WSM subband grid of level l (l = 0: H x W)
+    int goff[kMaxLevels]; // offset of level l+1's gate within a frame's gate
     int pdl;              // host: launch with programmatic stream serialization
     float dec_lo[kMaxTaps], dec_hi[kMaxTaps], rec_lo[kMaxTaps], rec_hi[kMaxTaps];
     int wta_F;            // WTA filter taps (temporal DWT, fp64)
@@ -263,6 +269,19 @@ __host__ __device__ __forceinline__ size_t tile_index(int64_t r, int k, int64_t 
 // output tokens.  Up to 128 tokens, hi and lo are one MMA of N = 2*ncp and
 // take 2*ncp accumulator columns per tile; above, they accumulate into the
 // same ncp columns.  Either way a unit fits one 256-column buffer.
+// Subband length after l cascaded levels of an F-tap DWT: n_l = (n_{l-1} + F - 1) / 2.
+__host__ __device__ __forceinline__ int level_size(int n, int F, int l) {
+    for (int k = 0; k < l; ++k) n = (n + F - 1) / 2;
+    return n;
+}
+
+// Floats of one frame's WSM gates over J levels (level l: h_l x w_l).
+__host__ __device__ __forceinline__ int gate_floats(int H, int W, int F, int J) {
+    int s = 0;
+    for (int l = 1; l <= J; ++l) s += level_size(H, F, l) * level_size(W, F, l);
+    return s;
+}
+
 __host__ __device__ __forceinline__ int unit_tiles(int ncp) {
     const int cols = ncp <= 128 ? 2 * ncp : ncp;
     const int cg = 256 / cols;
@@ -276,6 +295,8 @@ cudaError_t launch_relevance_pass(const Ctx &c, cudaStream_t s);
 cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s);
 cudaError_t launch_temporal(const Ctx &c, cudaStream_t s);
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s);
+cudaError_t launch_spatial_ml(const Ctx &c, cudaStream_t s);
+size_t spatial_ml_smem_bytes(int H, int W, int F, int J);   // 0 if the layout does not fit
 cudaError_t launch_project_gemm(const void *A, int M, int K, const void *B, int N, const float *bias, void *out,
                                 bool gelu, int *status, bool pdl, cudaStream_t s);
 cudaError_t launch_maxsim_gemm(const void *X, int M, int K, const void *QHL, int Lq, int Lqp, float *a, int *status,

@@ -52,6 +52,119 @@ struct SpatialSmem {
     }
 };
 
+// Synthesis weight of coefficient a at sample y (upsample, filter, keep the
+// samples from offset F - 2).
+__device__ __forceinline__ float synth(const float *rec, int F, int y, int a) {
+    const int k = y + F - 2 - 2 * a;
+    return (k >= 0 && k < F) ? rec[k] : 0.f;
+}
+
+// Half-pixel bilinear source (align_corners = false): rows y0, y1, weight of
+// y1.  The source coordinate s = (i + 1/2) in / out - 1/2, clamped at 0, is
+// the rational ((2i + 1) in - out) / (2 out): its floor and remainder are
+// exact in integers, and the weight is the remainder divided in fp32.
+__device__ __forceinline__ void bilinear_src(int i, int in, int out, int &y0, int &y1, float &l) {
+    const int num = (2 * i + 1) * in - out, den = 2 * out;
+    int f = 0, rem = 0;
+    if (num > 0) {
+        f = num / den;
+        rem = num - f * den;
+    }
+    if (f > in - 1) {
+        f = in - 1;
+        rem = 0;
+    }
+    y0 = f;
+    y1 = f + 1 < in ? f + 1 : in - 1;
+    l = (float)rem / (float)den;
+}
+
+// Coefficients a with synth(y, a) != 0 for y in {y0, y1}: y + F - 2 - 2a in [0, F).
+__device__ __forceinline__ void synth_support(int y0, int y1, int F, int na, int &lo, int &hi) {
+    lo = y0 >> 1;
+    hi = min(na - 1, (y1 + F - 2) >> 1);
+}
+
+// Staged rows [0, qn) of a grid row go out in 8-column groups: bf16 hi and
+// lo halves at tile_index(r, 8 g, w_rows) (tensor path; r = r_first + row,
+// split into a row part and a column part) or fp32 rows (CUDA-core path).
+__device__ __forceinline__ void write_rows(const float *stg, int qn, int K_pad, int64_t r_first, bool bf,
+                                           __nv_bfloat16 *Whi, __nv_bfloat16 *Wlo, float *W32, size_t kstride) {
+    const int G8 = K_pad / 8;
+    int ql_ = (int)threadIdx.x / G8, g = (int)threadIdx.x % G8;
+    const int gstep = (int)blockDim.x % G8, qstep = (int)blockDim.x / G8;
+    for (; ql_ < qn;) {
+        const float4 v0 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g);
+        const float4 v1 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g + 4);
+        const int64_t r = r_first + ql_;
+        if (bf) {
+            const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+            uint32_t hw[4], lw[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+                const __nv_bfloat162 ll =
+                    __floats2bfloat162_rn(v[2 * e] - __low2float(hh), v[2 * e + 1] - __high2float(hh));
+                hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
+                lw[e] = *reinterpret_cast<const uint32_t *>(&ll);
+            }
+            const size_t ti = (size_t)(g >> 2) * kstride + (size_t)(r >> 3) * 256 + (size_t)(r & 7) * 8 +
+                              (size_t)(g & 3) * 64;
+            *reinterpret_cast<uint4 *>(Whi + ti) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+            *reinterpret_cast<uint4 *>(Wlo + ti) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        } else {
+            float *dst = W32 + (size_t)r * K_pad + 8 * g;
+            *reinterpret_cast<float4 *>(dst) = v0;
+            *reinterpret_cast<float4 *>(dst + 4) = v1;
+        }
+        g += gstep;
+        ql_ += qstep;
+        if (g >= G8) {
+            g -= G8;
+            ++ql_;
+        }
+    }
+}
+
+constexpr int kSpatialThreads = 256;
+constexpr int kTailBlocks = 64;
+
+// Rows past the produced count (tau > 0): index -1, zero tokens.  Tail CTA
+// tb of kTailBlocks.
+__device__ inline void tail_rows(const Ctx &c, int tb) {
+    const size_t esz = c.dtype == WZ_DTYPE_BF16 ? 2 : 4;
+    const int nvec = (int)((size_t)c.D * esz / 16);
+    for (int v = 0; v < c.V; ++v) {
+        const int r0 = c.vpar[v].row0 + c.prod[v];
+        const int r1 = c.vpar[v].row0 + c.vpar[v].B;
+        for (int r = r0 + tb; r < r1; r += kTailBlocks) {
+            uint4 *o = reinterpret_cast<uint4 *>(static_cast<char *>(c.out) + (size_t)r * c.D * esz);
+            for (int k = threadIdx.x; k < nvec; k += blockDim.x) o[k] = make_uint4(0u, 0u, 0u, 0u);
+            if (threadIdx.x < 3) c.out_index[(size_t)r * 3 + threadIdx.x] = -1;
+        }
+    }
+}
+
+// The tensor-core work units of frame f (the temporal kernel placed them):
+// column blocks of <= 256 tokens, each in groups of unit_tiles(round16(nc))
+// 128-channel tiles.
+__device__ inline void unit_records(const Ctx &c, int64_t f, int n) {
+    const int v = (int)(f / c.T);
+    int4 *units = c.units + (size_t)v * c.max_units_v;
+    int u0 = c.ustart[f];
+    for (int j0 = 0; j0 < n; j0 += kColBlock) {
+        const int nc = min(kColBlock, n - j0);
+        const int cg = unit_tiles((nc + 15) / 16 * 16);
+        const int cnt = (c.n_ct + cg - 1) / cg;
+        for (int li = threadIdx.x; li < cnt; li += blockDim.x) {
+            const int ct = li * cg;
+            if (u0 + li < c.max_units_v)
+                units[u0 + li] = make_int4((int)f, j0, ct, nc | (min(cg, c.n_ct - ct) << 16));
+        }
+        u0 += cnt;
+    }
+}
+
 // Bytes of the frame-independent tables for an image of H x W and F taps.
 inline size_t spatial_table_bytes(int H, int W, int F) {
     SpatialSmem L;
@@ -105,6 +218,200 @@ __device__ inline void build_spatial_tables(const Ctx &c) {
     for (int j = threadIdx.x; j < W; j += blockDim.x) {
         ti[L.blo + j] = s_blo[j];
         ti[L.bhi + j] = s_bhi[j];
+    }
+}
+
+}  // namespace wz
+
+namespace wz {
+
+// ---- multi-level WSM --------------------------------------------------------
+// With J levels the DWT2 cascades on LL (level l of an h_{l-1} x w_{l-1} band
+// gives h_l x w_l subbands).  Folded into matrices along one side, level l's
+// analysis rows are AH_u^l = A_u^l AH_L^{l-1} (h_l x H, AH_L^0 = I, A_u^l the
+// single-level analysis of length h_{l-1}, extension folded in) and its
+// synthesis columns SH_u^l = SH_L^{l-1} S_u^l (H x h_l).  The operator is
+//
+//   W_m[(p,q),(i,j)] = sum_l sum_v sum_b Q_v^l[q,b] AW_v^l[b,j] Y_v^l[b,i],
+//   Y_v^l[b,i]       = sum_u sum_a P_u^l[p,a] AH_u^l[a,i] g_uv^l[a,b],
+//
+// P_u^l = R_y SH_u^l, Q_v^l = R_x SW_v^l, g_LH = g_HL = g_HH = G_l (the gate
+// of level l), g_LL = 1 at level J and 0 above it (that band is decomposed
+// further).  One level gives the single-level operator.
+struct MLTables {
+    int J, H, W;
+    int h[kMaxLevels + 1], w[kMaxLevels + 1];
+    // copied into shared memory: [0, copy)
+    int AHl[kMaxLevels], AHh[kMaxLevels];   // [h_l][H]
+    int AWl[kMaxLevels], AWh[kMaxLevels];   // [w_l][W]
+    int blo[kMaxLevels], bhi[kMaxLevels];   // [W] int: rows b of AW^l nonzero at column j
+    int copy;
+    // read from global memory
+    int SHl[kMaxLevels], SHh[kMaxLevels];   // [H][h_l]
+    int SWl[kMaxLevels], SWh[kMaxLevels];   // [W][w_l]
+    int slo[kMaxLevels], shi[kMaxLevels];   // [H] int: columns a of SH^l nonzero at row y
+    int xlo[kMaxLevels], xhi[kMaxLevels];   // [W] int: columns b of SW^l nonzero at row x
+    int total;
+    __host__ __device__ void init(int H_, int W_, int F, int J_) {
+        J = J_; H = H_; W = W_;
+        for (int l = 0; l <= kMaxLevels; ++l) {
+            h[l] = level_size(H, F, l);
+            w[l] = level_size(W, F, l);
+        }
+        int o = 0;
+        auto take = [&](int n) {
+            const int at = o;
+            o = (o + n + 3) & ~3;
+            return at;
+        };
+        for (int l = 0; l < J; ++l) {
+            AHl[l] = take(h[l + 1] * H);
+            AHh[l] = take(h[l + 1] * H);
+            AWl[l] = take(w[l + 1] * W);
+            AWh[l] = take(w[l + 1] * W);
+            blo[l] = take(W);
+            bhi[l] = take(W);
+        }
+        copy = o;
+        for (int l = 0; l < J; ++l) {
+            SHl[l] = take(H * h[l + 1]);
+            SHh[l] = take(H * h[l + 1]);
+            SWl[l] = take(W * w[l + 1]);
+            SWh[l] = take(W * w[l + 1]);
+            slo[l] = take(H);
+            shi[l] = take(H);
+            xlo[l] = take(W);
+            xhi[l] = take(W);
+        }
+        total = o;
+    }
+};
+
+inline size_t ml_table_bytes(int H, int W, int F, int J) {
+    MLTables T;
+    T.init(H, W, F, J);
+    return (size_t)T.total * 4;
+}
+
+// Shared memory of one multi-level spatial CTA.
+struct MLSmem {
+    int HP4, K_pad, QB;
+    int G;                                  // the frame's gates, levels 1..J (c.goff layout)
+    int Ql[kMaxLevels], Qh[kMaxLevels];     // [w][w_l] (w <= W)
+    int qlo[kMaxLevels], qhi[kMaxLevels];   // [W] int
+    int PAl, PAh;                           // [h_1][H], one level at a time
+    int Yl[kMaxLevels], Yh[kMaxLevels];     // [w_l][HP4]
+    int red, stage, total;
+    __host__ __device__ void init(const MLTables &T) {
+        const int H = T.H, W = T.W, N = H * W;
+        K_pad = (N + 31) & ~31;
+        QB = kStageFloats / K_pad;
+        HP4 = (H + 3) & ~3;
+        int o = T.copy;
+        auto take = [&](int n) {
+            const int at = o;
+            o = (o + n + 3) & ~3;
+            return at;
+        };
+        int gs = 0;
+        for (int l = 1; l <= T.J; ++l) gs += T.h[l] * T.w[l];
+        G = take(gs);
+        for (int l = 0; l < T.J; ++l) {
+            Ql[l] = take(W * T.w[l + 1]);
+            Qh[l] = take(W * T.w[l + 1]);
+            qlo[l] = take(W);
+            qhi[l] = take(W);
+            Yl[l] = take(T.w[l + 1] * HP4);
+            Yh[l] = take(T.w[l + 1] * HP4);
+        }
+        int hmax = 0;
+        for (int l = 1; l <= T.J; ++l) hmax = T.h[l] > hmax ? T.h[l] : hmax;
+        PAl = take(hmax * H);
+        PAh = take(hmax * H);
+        red = take(64);
+        stage = take(QB * K_pad);
+        total = o;
+    }
+};
+
+// Build the multi-level tables into c.stab (one CTA).  Level l's matrices
+// are formed from level l-1's in global memory; a block barrier separates
+// the levels (global writes of the block are visible to it after the barrier).
+__device__ inline void build_ml_tables(const Ctx &c) {
+    MLTables T;
+    T.init(c.H, c.W, c.F, c.wsm_levels);
+    float *tb = c.stab;
+    int *ti = reinterpret_cast<int *>(c.stab);
+    const int F = c.F, H = c.H, W = c.W;
+    for (int l = 0; l < T.J; ++l) {
+        // analysis rows: AX_u^{l+1}[a][i] = sum_j dec_u[j] AX_L^l[ext(2a + 1 - j)][i]
+        for (int side = 0; side < 2; ++side) {
+            const int n = side ? W : H, nin = side ? T.w[l] : T.h[l], nout = side ? T.w[l + 1] : T.h[l + 1];
+            float *lo = tb + (side ? T.AWl[l] : T.AHl[l]), *hi = tb + (side ? T.AWh[l] : T.AHh[l]);
+            const float *prev = l ? tb + (side ? T.AWl[l - 1] : T.AHl[l - 1]) : nullptr;
+            for (int k = threadIdx.x; k < nout * n; k += blockDim.x) {
+                const int a = k / n, i = k % n;
+                float sl = 0.f, sh = 0.f;
+                for (int j = 0; j < F; ++j) {
+                    const int e = ext_index(2 * a + 1 - j, nin, c.mode);
+                    if (e < 0) continue;
+                    const float x = prev ? prev[e * n + i] : (e == i ? 1.f : 0.f);
+                    sl += c.dec_lo[j] * x;
+                    sh += c.dec_hi[j] * x;
+                }
+                lo[k] = sl;
+                hi[k] = sh;
+            }
+            // synthesis columns: SX_u^{l+1}[y][a] = sum_k SX_L^l[y][k] rec_u[k + F - 2 - 2a]
+            float *slo_ = tb + (side ? T.SWl[l] : T.SHl[l]), *shi_ = tb + (side ? T.SWh[l] : T.SHh[l]);
+            const float *sprev = l ? tb + (side ? T.SWl[l - 1] : T.SHl[l - 1]) : nullptr;
+            for (int k = threadIdx.x; k < n * nout; k += blockDim.x) {
+                const int y = k / nout, a = k % nout;
+                float sl = 0.f, sh = 0.f;
+                const int k0 = max(0, 2 * a - F + 2), k1 = min(nin - 1, 2 * a + 1);
+                for (int kk = k0; kk <= k1; ++kk) {
+                    const float x = sprev ? sprev[y * nin + kk] : (y == kk ? 1.f : 0.f);
+                    sl += x * c.rec_lo[kk + F - 2 - 2 * a];
+                    sh += x * c.rec_hi[kk + F - 2 - 2 * a];
+                }
+                slo_[k] = sl;
+                shi_[k] = sh;
+            }
+        }
+        __syncthreads();
+    }
+    // supports
+    for (int l = 0; l < T.J; ++l) {
+        for (int j = threadIdx.x; j < W; j += blockDim.x) {   // rows b of AW^l at column j
+            int lo = T.w[l + 1], hi = -1;
+            for (int b = 0; b < T.w[l + 1]; ++b)
+                if (tb[T.AWl[l] + b * W + j] != 0.f || tb[T.AWh[l] + b * W + j] != 0.f) {
+                    lo = min(lo, b);
+                    hi = max(hi, b);
+                }
+            ti[T.blo[l] + j] = lo;
+            ti[T.bhi[l] + j] = hi;
+        }
+        for (int y = threadIdx.x; y < H; y += blockDim.x) {   // columns a of SH^l at row y
+            int lo = T.h[l + 1], hi = -1;
+            for (int a = 0; a < T.h[l + 1]; ++a)
+                if (tb[T.SHl[l] + y * T.h[l + 1] + a] != 0.f || tb[T.SHh[l] + y * T.h[l + 1] + a] != 0.f) {
+                    lo = min(lo, a);
+                    hi = max(hi, a);
+                }
+            ti[T.slo[l] + y] = lo;
+            ti[T.shi[l] + y] = hi;
+        }
+        for (int x = threadIdx.x; x < W; x += blockDim.x) {   // columns b of SW^l at row x
+            int lo = T.w[l + 1], hi = -1;
+            for (int b = 0; b < T.w[l + 1]; ++b)
+                if (tb[T.SWl[l] + x * T.w[l + 1] + b] != 0.f || tb[T.SWh[l] + x * T.w[l + 1] + b] != 0.f) {
+                    lo = min(lo, b);
+                    hi = max(hi, b);
+                }
+            ti[T.xlo[l] + x] = lo;
+            ti[T.xhi[l] + x] = hi;
+        }
     }
 }
 

@@ -31,6 +31,7 @@ SPATIAL_MODES = {"wsm": SPATIAL_WSM, "saliency": SPATIAL_SALIENCY, "none": SPATI
 RELEVANCE_MEAN, RELEVANCE_MAXSIM = 0, 1
 RELEVANCE_MODES = {"mean": RELEVANCE_MEAN, "maxsim": RELEVANCE_MAXSIM}
 MAX_LQ_MAXSIM = 128
+MAX_LEVELS = 4
 
 
 def _enum(table, v):
@@ -56,6 +57,7 @@ class CondenseArgs(C.Structure):
         ("lam", C.c_float), ("tau", C.c_float), ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int),
         ("mode", C.c_int), ("path", C.c_int), ("temporal_mode", C.c_int), ("spatial_mode", C.c_int),
         ("token_scores", C.c_void_p), ("frame_scores", C.c_void_p), ("relevance_mode", C.c_int),
+        ("wta_levels", C.c_int), ("wsm_levels", C.c_int),
         ("out_tokens", C.c_void_p), ("out_index", C.c_void_p),
         ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
         ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
@@ -71,6 +73,7 @@ class BatchArgs(C.Structure):
         ("wta_wavelet", C.c_int), ("wsm_wavelet", C.c_int), ("mode", C.c_int), ("path", C.c_int),
         ("temporal_mode", C.c_int), ("spatial_mode", C.c_int),
         ("token_scores", C.c_void_p), ("frame_scores", C.c_void_p), ("relevance_mode", C.c_int),
+        ("wta_levels", C.c_int), ("wsm_levels", C.c_int),
         ("out_tokens", C.c_void_p), ("out_index", C.c_void_p), ("row_offsets", C.POINTER(C.c_int64)),
         ("out_budgets", C.c_void_p), ("out_count", C.c_void_p), ("out_relevance", C.c_void_p),
         ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("device_status", C.c_void_p),
@@ -195,7 +198,7 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
                    tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
                    temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1,
                    token_scores: torch.Tensor | None = None, frame_scores: torch.Tensor | None = None,
-                   relevance="mean", workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
+                   relevance="mean", wta_levels: int = 1, wsm_levels: int = 1, workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
                    device_status: torch.Tensor | None = None, kernel_events=None, stream=None):
     """wz_condense_ex.  Returns a dict with tokens, index, budgets, count and relevance.
 
@@ -204,7 +207,9 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
     token_scores [T, H*W] / frame_scores [T]: float32 device tensors of an
     external scorer (None: the similarity branch's own scores).
     relevance: "mean" (the mean query row) or "maxsim" (maximum cosine over
-    the query rows; bf16 features, D % 64 == 0, at most 128 query rows)."""
+    the query rows; bf16 features, D % 64 == 0, at most 128 query rows).
+    wta_levels / wsm_levels: decomposition levels of the two wavelet modules
+    (1..4; the DWT cascades on the approximation band)."""
     features = _cuda_contig(features, "features")
     query = _cuda_contig(query, "query")
     T, H, W, D = features.shape
@@ -228,6 +233,7 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
     a.temporal_mode = _enum(TEMPORAL_MODES, temporal_mode)
     a.spatial_mode = _enum(SPATIAL_MODES, spatial_mode)
     a.relevance_mode = _enum(RELEVANCE_MODES, relevance)
+    a.wta_levels, a.wsm_levels = wta_levels, wsm_levels
     if token_scores is not None:
         token_scores = _f32_scores(token_scores, (T, H * W), "token_scores")
         a.token_scores = token_scores.data_ptr()
@@ -259,7 +265,7 @@ def wz_batch_rows(V, T, H, W, ratios):
 def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios, *, lam: float = 1.5,
                       tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
                       temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1, relevance="mean",
-                      workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
+                      wta_levels: int = 1, wsm_levels: int = 1, workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
                       stream=None):
     """wz_condense_batch: features [V,T,H,W,D], queries [sum Lq, D]."""
     features = _cuda_contig(features, "features")
@@ -286,6 +292,7 @@ def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios,
     a.temporal_mode = _enum(TEMPORAL_MODES, temporal_mode)
     a.spatial_mode = _enum(SPATIAL_MODES, spatial_mode)
     a.relevance_mode = _enum(RELEVANCE_MODES, relevance)
+    a.wta_levels, a.wsm_levels = wta_levels, wsm_levels
     a.out_tokens, a.out_index, a.row_offsets = tokens.data_ptr(), index.data_ptr(), ro
     a.out_budgets, a.out_count, a.out_relevance = budgets.data_ptr(), count.data_ptr(), rel.data_ptr()
     if workspace is not None:

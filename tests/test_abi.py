@@ -49,6 +49,7 @@ def test_struct_layout_matches_defaults(wz):
     assert (a.lam, a.tau, a.wta_wavelet, a.wsm_wavelet, a.mode, a.path, a.dtype) == (1.5, 0.0, 1, 4, 0, 0, 0)
     assert (a.temporal_mode, a.spatial_mode) == (wz.TEMPORAL_WTA, wz.SPATIAL_WSM)
     assert a.relevance_mode == wz.RELEVANCE_MEAN
+    assert (a.wta_levels, a.wsm_levels) == (1, 1)
     b = wz.BatchArgs()
     wz._lib.wz_batch_args_init(C.byref(b))
     assert (b.lam, b.wta_wavelet, b.wsm_wavelet) == (1.5, 1, 4)
@@ -115,6 +116,8 @@ def _args(wz, **over):
     (dict(wsm_wavelet=11), -1), (dict(mode=3), -1), (dict(path=7), -1), (dict(dtype=5), -1),
     (dict(temporal_mode=3), -1), (dict(temporal_mode=-1), -1), (dict(spatial_mode=3), -1),
     (dict(relevance_mode=2), -1), (dict(relevance_mode=1), -2),                 # max-over-query: D % 64
+    (dict(wta_levels=0), -1), (dict(wta_levels=5), -1), (dict(wsm_levels=5), -1),
+    (dict(H=64, W=64, wsm_levels=4, wsm_wavelet=10), -2),                      # level tables exceed a CTA
     (dict(relevance_mode=1, D=64, dtype=1), -2), (dict(relevance_mode=1, D=64, Lq=129), -2),
     (dict(dtype=1, path=1), -2), (dict(features=P + 4), -1), (dict(out_tokens=3 * P + 8), -1),
     (dict(workspace=5 * P, workspace_bytes=16), -5), (dict(workspace=5 * P + 64, workspace_bytes=1 << 30), -1),

@@ -57,7 +57,8 @@ def test_config_256_frames_sampled(wz):
 
 def _random_case(wz, T, H, W, D, Lq, ratio, seed=0, dtype="bf16", **kw):
     okw = {k: v for k, v in kw.items()
-           if k in ("lam", "tau", "wta_wavelet", "wsm_wavelet", "mode", "temporal_mode", "spatial_mode")}
+           if k in ("lam", "tau", "wta_wavelet", "wsm_wavelet", "mode", "temporal_mode", "spatial_mode",
+                    "relevance", "wta_levels", "wsm_levels")}
     X, Q = accepted_random(T, H, W, D, Lq, ratio, seed=seed, dtype=dtype, **okw)
     ref = oracle_run(X, Q, ratio, **okw)
     out = run(wz, X, Q, ratio, **kw)
@@ -89,6 +90,25 @@ def test_shapes(wz, T, H, W, D, Lq, ratio):
                                 dict(wta_wavelet=44, wsm_wavelet=44), dict(wsm_wavelet=44, path="simt")])
 def test_options(wz, kw):
     _random_case(wz, 10, 13, 13, 128, 6, 0.2, seed=5, **kw)
+
+
+@pytest.mark.parametrize("kw", [dict(wta_levels=2), dict(wta_levels=3, wta_wavelet=2), dict(wta_levels=4, wta_wavelet=4),
+                                dict(wsm_levels=2), dict(wsm_levels=3, wsm_wavelet=1), dict(wsm_levels=2, wsm_wavelet=44),
+                                dict(wsm_levels=2, path="simt"), dict(wsm_levels=2, mode="zero"),
+                                dict(wsm_levels=3, mode="periodic", wsm_wavelet=2),
+                                dict(wta_levels=4, wsm_levels=4, wsm_wavelet=1)])
+def test_levels(wz, kw):
+    _random_case(wz, 10, 13, 13, 128, 6, 0.2, seed=5, **kw)
+
+
+@pytest.mark.parametrize("T,H,W,D,kw", [
+    (24, 27, 27, 256, dict(wsm_levels=3)),                    # the 27x27 map, three db4 levels
+    (9, 7, 9, 64, dict(wsm_levels=2, wta_levels=2)),          # non-square, subbands wider than the map
+    (5, 64, 64, 32, dict(wsm_levels=2, wsm_wavelet=1)),       # the largest map
+    (600, 3, 4, 16, dict(wta_levels=3)),                      # two frames per temporal thread
+])
+def test_levels_shapes(wz, T, H, W, D, kw):
+    _random_case(wz, T, H, W, D, 4, 0.25, seed=T + H, **kw)
 
 
 @pytest.mark.parametrize("kw", [dict(temporal_mode="raw"), dict(temporal_mode="uniform"),
