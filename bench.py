@@ -53,6 +53,8 @@ def parse():
                    help="also time the projector P (Eq. 17) on the condensed tokens; 0 skips it")
     p.add_argument("--maxsim-steps", type=int, default=10,
                    help="also time the step with the max-over-query scorer; 0 skips it")
+    p.add_argument("--variant-steps", type=int, default=5,
+                   help="also time the wavelet, level, ablation and external-score variants; 0 skips them")
     return p.parse_args()
 
 
@@ -194,6 +196,65 @@ def time_maxsim(wz, X, Q, ratio, ws, status, steps, dev):
                      "tflop_s": round(flop / (gemm_ms * 1e-3) / 1e12, 1)},
             "kernels_ms": {k: round(statistics.mean(v), 5) for k, v in kern.items()},
             "launches_per_step": len(KERNELS) + 2}
+
+
+VARIANTS = [   # (name, wz_condense_ex options): the paper's variant rows on the same video
+    ("wta_db4", dict(wta_wavelet=4)),
+    ("wsm_haar", dict(wsm_wavelet=1)),
+    ("wsm_bior44", dict(wsm_wavelet=44)),
+    ("wta_levels3", dict(wta_levels=3)),
+    ("wsm_levels2", dict(wsm_levels=2)),
+    ("wsm_levels3", dict(wsm_levels=3)),
+    ("alloc_raw", dict(temporal_mode="raw")),
+    ("alloc_uniform", dict(temporal_mode="uniform")),
+    ("spatial_saliency_only", dict(spatial_mode="saliency")),
+    ("spatial_none", dict(spatial_mode="none")),
+    ("external_scores", None),   # caller-supplied a_{t,n} and r_t
+]
+
+
+def time_variants(wz, X, Q, ratio, ws, status, steps, dev):
+    """Each variant: 3 warm-up steps, `steps` plain timed steps, then the same
+    steps with kernel events for the per-kernel times."""
+    import torch
+    stream = torch.cuda.current_stream(dev)
+    T, H, W, D = X.shape
+    g = torch.Generator(device=dev).manual_seed(23)
+    ext = dict(token_scores=torch.rand((T, H * W), device=dev, generator=g),
+               frame_scores=0.1 + 0.2 * torch.randn((T,), device=dev, generator=g))
+    out = {}
+    for name, kw in VARIANTS:
+        kw = ext if kw is None else kw
+
+        def step(events=None):
+            return wz.wz_condense_ex(X, Q, ratio, workspace=ws, device_status=status, kernel_events=events, **kw)
+
+        for _ in range(3):
+            res = step()
+        torch.cuda.synchronize(dev)
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(steps):
+            step()
+        t1.record(stream)
+        torch.cuda.synchronize(dev)
+        ms = t0.elapsed_time(t1) / steps
+        kern = {k: [] for k in KERNELS}
+        for _ in range(steps):
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * len(KERNELS))]
+            for e in ev:
+                e.record(stream)
+            step(ev)
+            torch.cuda.synchronize(dev)
+            for j, k in enumerate(KERNELS):
+                kern[k].append(ev[2 * j].elapsed_time(ev[2 * j + 1]))
+        out[name] = {"options": {k: v for k, v in kw.items() if not hasattr(v, "shape")} or "external a, r",
+                     "ms_per_step": round(ms, 5), "frames_per_s": round(T / (ms * 1e-3), 1),
+                     "active_frames": int((res["budgets"] > 0).sum()),
+                     "kernels_ms": {k: round(statistics.mean(v), 5) for k, v in kern.items()}}
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())}: a bounded wait timed out")
+    return out
 
 
 def source_hash(fname):
@@ -468,6 +529,8 @@ def run_ours(args, spec, world, rank, local):
     projector = time_projector(wz, tokens, args.projector_steps, dev) if args.projector_steps > 0 else None
     maxsim = time_maxsim(wz, X, Q, spec.ratio, ws, status, args.maxsim_steps, dev) \
         if args.maxsim_steps > 0 and X.dtype == torch.bfloat16 and D % 64 == 0 else None
+    variants = time_variants(wz, X, Q, spec.ratio, ws, status, args.variant_steps, dev) \
+        if args.variant_steps > 0 else None
 
     if rank == 0:
         peak, peak_kind = measured_peak()
@@ -502,6 +565,7 @@ def run_ours(args, spec, world, rank, local):
             "gpu_launches": len(KERNELS) * args.steps,
             "projector": projector,
             "maxsim": maxsim,
+            "variants": variants,
         }
         if world == 1 and not args.no_cpu_baseline:
             out["cpu_baseline"] = cpu_baseline(spec, CPU_SAMPLE_FRAMES)

@@ -90,6 +90,66 @@ __host__ __device__ inline size_t temporal_smem_bytes(int T, int J) {
 // kPerThread frames per thread beyond (fp64 work scales with the warps).
 inline int temporal_threads(int T) { return T <= 512 ? (T < 32 ? 32 : (T + 31) / 32 * 32) : 512; }
 
+// WTA levels 2..J (J > 1): level 1 left its approximation in A0, its gate in
+// G0 and its gated details in dall[0, K1).  Each further level analyses the
+// previous approximation (gate: the pairwise mean of the previous gate) and
+// appends its gated details to dall; the inverse then cascades back to level
+// 1's approximation, whose buffer is returned.  Called by the whole block.
+__device__ __noinline__ const double *wta_deeper_levels(const Ctx &c, double *A0, double *A1, double *G0, double *G1,
+                                                         double *dall, int K1, int J) {
+    const int FT = c.wta_F;
+    int lens[kMaxLevels + 1], doff[kMaxLevels];
+    lens[1] = K1;
+    doff[0] = 0;
+    for (int j = 2, o = K1; j <= J; ++j) {
+        lens[j] = (lens[j - 1] + FT - 1) / 2;
+        doff[j - 1] = o;
+        o += lens[j];
+    }
+    double *ain = A0, *gin = G0, *aout = A1, *gout = G1;
+    for (int j = 2; j <= J; ++j) {
+        const int n = lens[j - 1], K = lens[j];
+        for (int k = threadIdx.x; k < K; k += blockDim.x) {
+            double ca = 0.0, cd = 0.0;
+            for (int i = 0; i < FT; ++i) {
+                const double x = ain[ext_index(2 * k + 1 - i, n, WZ_MODE_SYMMETRIC)];
+                ca += c.wta_dec_lo[i] * x;
+                cd += c.wta_dec_hi[i] * x;
+            }
+            const double g = 0.5 * (gin[ext_index(2 * k, n, WZ_MODE_SYMMETRIC)] +
+                                    gin[ext_index(2 * k + 1, n, WZ_MODE_SYMMETRIC)]);
+            aout[k] = ca;
+            if (j < J) gout[k] = g;
+            dall[doff[j - 1] + k] = g * cd;
+        }
+        __syncthreads();
+        double *t_ = ain;
+        ain = aout;
+        aout = t_;
+        t_ = gin;
+        gin = gout;
+        gout = t_;
+    }
+    for (int j = J; j >= 2; --j) {   // inverse of levels J .. 2
+        const int n = lens[j - 1], K = lens[j];
+        const double *dj = dall + doff[j - 1];
+        for (int m = threadIdx.x; m < n; m += blockDim.x) {
+            double x = 0.0;
+            const int alo = m >> 1, ahi = min(K - 1, (m + FT - 2) >> 1);
+            for (int ai = alo; ai <= ahi; ++ai) {
+                const int kk = m + FT - 2 - 2 * ai;
+                x += c.wta_rec_lo[kk] * ain[ai] + c.wta_rec_hi[kk] * dj[ai];
+            }
+            aout[m] = x;
+        }
+        __syncthreads();
+        double *t_ = ain;
+        ain = aout;
+        aout = t_;
+    }
+    return ain;
+}
+
 __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     pdl_wait();
     pdl_trigger();
@@ -161,56 +221,22 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     // Budget weights are max(r~, 0) (Eq. 5); the ablation modes use max(r, 0)
     // ("raw") or 1 ("uniform") instead.
     const int FT = c.wta_F;
-    int lens[kMaxLevels + 1], doff[kMaxLevels];
-    lens[0] = L;
-    for (int j = 1, o = 0; j <= J; ++j) {
-        lens[j] = (lens[j - 1] + FT - 1) / 2;
-        doff[j - 1] = o;
-        o += lens[j];
-    }
-    const double *ain = nullptr, *gin = nullptr;   // level 1 reads r and gamma of the retained frames
-    double *aout = A0, *gout = G0;
-    for (int j = 1; j <= J; ++j) {
-        const int n = lens[j - 1], K = lens[j];
-        for (int k = threadIdx.x; k < K; k += blockDim.x) {
-            double ca = 0.0, cd = 0.0;
-            for (int i = 0; i < FT; ++i) {
-                const int m = ext_index(2 * k + 1 - i, n, WZ_MODE_SYMMETRIC);
-                const double x = ain ? ain[m] : fr[4 * lst[m]];
-                ca += c.wta_dec_lo[i] * x;
-                cd += c.wta_dec_hi[i] * x;
-            }
-            const int m0 = ext_index(2 * k, n, WZ_MODE_SYMMETRIC), m1 = ext_index(2 * k + 1, n, WZ_MODE_SYMMETRIC);
-            const double g = gin ? 0.5 * (gin[m0] + gin[m1]) : 0.5 * (fr[4 * lst[m0] + 2] + fr[4 * lst[m1] + 2]);
-            aout[k] = ca;
-            if (j < J) gout[k] = g;
-            dall[doff[j - 1] + k] = g * cd;
+    const int K = (L + FT - 1) / 2;
+    for (int k = threadIdx.x; k < K; k += blockDim.x) {
+        double ca = 0.0, cd = 0.0;
+        for (int j = 0; j < FT; ++j) {
+            const double x = fr[4 * lst[ext_index(2 * k + 1 - j, L, WZ_MODE_SYMMETRIC)]];
+            ca += c.wta_dec_lo[j] * x;
+            cd += c.wta_dec_hi[j] * x;
         }
-        __syncthreads();
-        ain = aout;
-        gin = gout;
-        aout = aout == A0 ? A1 : A0;
-        gout = gout == G0 ? G1 : G0;
+        const int m0 = ext_index(2 * k, L, WZ_MODE_SYMMETRIC), m1 = ext_index(2 * k + 1, L, WZ_MODE_SYMMETRIC);
+        const double g = 0.5 * (fr[4 * lst[m0] + 2] + fr[4 * lst[m1] + 2]);
+        A0[k] = ca;
+        dall[k] = g * cd;
+        if (J > 1) G0[k] = g;
     }
-    // inverse of levels J .. 2 into the free approximation buffer
-    for (int j = J; j >= 2; --j) {
-        const int n = lens[j - 1], K = lens[j];
-        const double *dj = dall + doff[j - 1];
-        for (int m = threadIdx.x; m < n; m += blockDim.x) {
-            double x = 0.0;
-            const int alo = m >> 1, ahi = min(K - 1, (m + FT - 2) >> 1);
-            for (int ai = alo; ai <= ahi; ++ai) {
-                const int kk = m + FT - 2 - 2 * ai;
-                x += c.wta_rec_lo[kk] * ain[ai] + c.wta_rec_hi[kk] * dj[ai];
-            }
-            aout[m] = x;
-        }
-        __syncthreads();
-        const double *t_ = ain;
-        ain = aout;
-        aout = const_cast<double *>(t_);
-    }
-    const int K = lens[1];
+    __syncthreads();
+    const double *ain = J > 1 ? wta_deeper_levels(c, A0, A1, G0, G1, dall, K, J) : A0;
     int anypos = 0;
     for (int m = threadIdx.x; m < L; m += blockDim.x) {
         double rt = 0.0;

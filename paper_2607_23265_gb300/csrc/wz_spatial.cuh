@@ -337,7 +337,7 @@ struct MLSmem {
 // Build the multi-level tables into c.stab (one CTA).  Level l's matrices
 // are formed from level l-1's in global memory; a block barrier separates
 // the levels (global writes of the block are visible to it after the barrier).
-__device__ inline void build_ml_tables(const Ctx &c) {
+static __device__ __noinline__ void build_ml_tables(const Ctx &c) {
     MLTables T;
     T.init(c.H, c.W, c.F, c.wsm_levels);
     float *tb = c.stab;
