@@ -47,6 +47,18 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_ml_kernel(Ctx c, int 
     float *G = sm + L.G, *PAl = sm + L.PAl, *PAh = sm + L.PAh, *red = sm + L.red, *stg = sm + L.stage;
     int *irange = reinterpret_cast<int *>(red + 48);
     const int HP4 = L.HP4;
+    // per-level offsets for the inner loop, read as shared-memory broadcasts
+    enum { kWl, kQl, kQh, kAWl, kAWh, kYl, kYh, kBlo, kBhi, kQlo, kQhi, kMeta };
+    __shared__ int meta[kMaxLevels][kMeta];
+    if (tid < J) {
+        int *m = meta[tid];
+        m[kWl] = T.w[tid + 1];
+        m[kQl] = L.Ql[tid]; m[kQh] = L.Qh[tid];
+        m[kAWl] = T.AWl[tid]; m[kAWh] = T.AWh[tid];
+        m[kYl] = L.Yl[tid]; m[kYh] = L.Yh[tid];
+        m[kBlo] = T.blo[tid]; m[kBhi] = T.bhi[tid];
+        m[kQlo] = L.qlo[tid]; m[kQhi] = L.qhi[tid];
+    }
 
     // ---- per-frame tables ------------------------------------------------
     for (int k = tid; k < T.copy; k += blockDim.x) si[k] = gi[k];
@@ -149,13 +161,15 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_ml_kernel(Ctx c, int 
                 float acc[HMAX];
 #pragma unroll
                 for (int i = 0; i < HMAX; ++i) acc[i] = 0.f;
+#pragma unroll 1
                 for (int l = 0; l < J; ++l) {
-                    const int wl = T.w[l + 1];
-                    const float *Ql = sm + L.Ql[l], *Qh = sm + L.Qh[l];
-                    const float *AWl = sm + T.AWl[l], *AWh = sm + T.AWh[l];
-                    const float *Yl = sm + L.Yl[l], *Yh = sm + L.Yh[l];
-                    const int b1 = min(si[T.bhi[l] + j], si[L.qhi[l] + q]);
-                    for (int b = max(si[T.blo[l] + j], si[L.qlo[l] + q]); b <= b1; ++b) {
+                    const int *m = meta[l];
+                    const int wl = m[kWl];
+                    const float *Ql = sm + m[kQl], *Qh = sm + m[kQh];
+                    const float *AWl = sm + m[kAWl], *AWh = sm + m[kAWh];
+                    const float *Yl = sm + m[kYl], *Yh = sm + m[kYh];
+                    const int b1 = min(si[m[kBhi] + j], si[m[kQhi] + q]);
+                    for (int b = max(si[m[kBlo] + j], si[m[kQlo] + q]); b <= b1; ++b) {
                         const float ql = Ql[q * wl + b] * AWl[b * W + j];
                         const float qh = Qh[q * wl + b] * AWh[b * W + j];
                         const float4 *yl = reinterpret_cast<const float4 *>(Yl + b * HP4);

@@ -343,6 +343,14 @@ static __device__ __noinline__ void build_ml_tables(const Ctx &c) {
     float *tb = c.stab;
     int *ti = reinterpret_cast<int *>(c.stab);
     const int F = c.F, H = c.H, W = c.W;
+    // supports, gathered with shared-memory atomics while the tables are formed
+    __shared__ int sup[6][kMaxLevels][WZ_MAX_HW];   // blo, bhi (AW rows), slo, shi (SH), xlo, xhi (SW)
+    for (int k = threadIdx.x; k < kMaxLevels * WZ_MAX_HW; k += blockDim.x) {
+        const int l = k / WZ_MAX_HW, x = k % WZ_MAX_HW;
+        sup[0][l][x] = sup[2][l][x] = sup[4][l][x] = 1 << 30;
+        sup[1][l][x] = sup[3][l][x] = sup[5][l][x] = -1;
+    }
+    __syncthreads();
     for (int l = 0; l < T.J; ++l) {
         // analysis rows: AX_u^{l+1}[a][i] = sum_j dec_u[j] AX_L^l[ext(2a + 1 - j)][i]
         for (int side = 0; side < 2; ++side) {
@@ -352,6 +360,7 @@ static __device__ __noinline__ void build_ml_tables(const Ctx &c) {
             for (int k = threadIdx.x; k < nout * n; k += blockDim.x) {
                 const int a = k / n, i = k % n;
                 float sl = 0.f, sh = 0.f;
+#pragma unroll 4
                 for (int j = 0; j < F; ++j) {
                     const int e = ext_index(2 * a + 1 - j, nin, c.mode);
                     if (e < 0) continue;
@@ -361,6 +370,10 @@ static __device__ __noinline__ void build_ml_tables(const Ctx &c) {
                 }
                 lo[k] = sl;
                 hi[k] = sh;
+                if (side && (sl != 0.f || sh != 0.f)) {
+                    atomicMin(&sup[0][l][i], a);
+                    atomicMax(&sup[1][l][i], a);
+                }
             }
             // synthesis columns: SX_u^{l+1}[y][a] = sum_k SX_L^l[y][k] rec_u[k + F - 2 - 2a]
             float *slo_ = tb + (side ? T.SWl[l] : T.SHl[l]), *shi_ = tb + (side ? T.SWh[l] : T.SHh[l]);
@@ -369,6 +382,7 @@ static __device__ __noinline__ void build_ml_tables(const Ctx &c) {
                 const int y = k / nout, a = k % nout;
                 float sl = 0.f, sh = 0.f;
                 const int k0 = max(0, 2 * a - F + 2), k1 = min(nin - 1, 2 * a + 1);
+#pragma unroll 4
                 for (int kk = k0; kk <= k1; ++kk) {
                     const float x = sprev ? sprev[y * nin + kk] : (y == kk ? 1.f : 0.f);
                     sl += x * c.rec_lo[kk + F - 2 - 2 * a];
@@ -376,41 +390,25 @@ static __device__ __noinline__ void build_ml_tables(const Ctx &c) {
                 }
                 slo_[k] = sl;
                 shi_[k] = sh;
+                if (sl != 0.f || sh != 0.f) {
+                    atomicMin(&sup[side ? 4 : 2][l][y], a);
+                    atomicMax(&sup[side ? 5 : 3][l][y], a);
+                }
             }
         }
         __syncthreads();
     }
-    // supports
+    // supports (empty: lo = the band length, hi = -1)
     for (int l = 0; l < T.J; ++l) {
-        for (int j = threadIdx.x; j < W; j += blockDim.x) {   // rows b of AW^l at column j
-            int lo = T.w[l + 1], hi = -1;
-            for (int b = 0; b < T.w[l + 1]; ++b)
-                if (tb[T.AWl[l] + b * W + j] != 0.f || tb[T.AWh[l] + b * W + j] != 0.f) {
-                    lo = min(lo, b);
-                    hi = max(hi, b);
-                }
-            ti[T.blo[l] + j] = lo;
-            ti[T.bhi[l] + j] = hi;
+        for (int x = threadIdx.x; x < W; x += blockDim.x) {
+            ti[T.blo[l] + x] = min(sup[0][l][x], T.w[l + 1]);
+            ti[T.bhi[l] + x] = sup[1][l][x];
+            ti[T.xlo[l] + x] = min(sup[4][l][x], T.w[l + 1]);
+            ti[T.xhi[l] + x] = sup[5][l][x];
         }
-        for (int y = threadIdx.x; y < H; y += blockDim.x) {   // columns a of SH^l at row y
-            int lo = T.h[l + 1], hi = -1;
-            for (int a = 0; a < T.h[l + 1]; ++a)
-                if (tb[T.SHl[l] + y * T.h[l + 1] + a] != 0.f || tb[T.SHh[l] + y * T.h[l + 1] + a] != 0.f) {
-                    lo = min(lo, a);
-                    hi = max(hi, a);
-                }
-            ti[T.slo[l] + y] = lo;
-            ti[T.shi[l] + y] = hi;
-        }
-        for (int x = threadIdx.x; x < W; x += blockDim.x) {   // columns b of SW^l at row x
-            int lo = T.w[l + 1], hi = -1;
-            for (int b = 0; b < T.w[l + 1]; ++b)
-                if (tb[T.SWl[l] + x * T.w[l + 1] + b] != 0.f || tb[T.SWh[l] + x * T.w[l + 1] + b] != 0.f) {
-                    lo = min(lo, b);
-                    hi = max(hi, b);
-                }
-            ti[T.xlo[l] + x] = lo;
-            ti[T.xhi[l] + x] = hi;
+        for (int y = threadIdx.x; y < H; y += blockDim.x) {
+            ti[T.slo[l] + y] = min(sup[2][l][y], T.h[l + 1]);
+            ti[T.shi[l] + y] = sup[3][l][y];
         }
     }
 }
