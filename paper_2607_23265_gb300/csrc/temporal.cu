@@ -51,6 +51,48 @@ __device__ int block_excl_scan(int x, int *ws, int *total) {
     return r;
 }
 
+// Three exclusive block scans at once (same barriers as one); ws holds
+// >= 3 * 33 ints.  Returns the exclusive prefixes and the totals.
+__device__ void block_excl_scan3(const int (&x)[3], int *ws, int (&excl)[3], int (&total)[3]) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nw = blockDim.x >> 5;
+    int incl[3] = {x[0], x[1], x[2]};
+    for (int o = 1; o < 32; o <<= 1) {
+#pragma unroll
+        for (int k = 0; k < 3; ++k) {
+            const int y = __shfl_up_sync(0xffffffffu, incl[k], o);
+            if (lane >= o) incl[k] += y;
+        }
+    }
+    __syncthreads();
+    if (lane == 31) {
+#pragma unroll
+        for (int k = 0; k < 3; ++k) ws[33 * k + warp] = incl[k];
+    }
+    __syncthreads();
+    if (warp == 0) {
+#pragma unroll
+        for (int k = 0; k < 3; ++k) {
+            const int w = lane < nw ? ws[33 * k + lane] : 0;
+            int wi = w;
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xffffffffu, wi, o);
+                if (lane >= o) wi += y;
+            }
+            __syncwarp();
+            if (lane < nw) ws[33 * k + lane] = wi - w;
+            if (lane == nw - 1) ws[33 * k + 32] = wi;
+        }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+        excl[k] = ws[33 * k + warp] + incl[k] - x[k];
+        total[k] = ws[33 * k + 32];
+    }
+    __syncthreads();
+}
+
 // Frames per thread for the scans (T <= 4096 with 256 threads).
 constexpr int kPerThread = WZ_MAX_T / kTemporalThreads;
 
@@ -161,8 +203,8 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     }
     extern __shared__ __align__(16) unsigned char tsm[];
     __shared__ double dscr[64];
-    __shared__ long long lscr[40];
-    __shared__ int iscr[72];
+    __shared__ long long lscr[66];
+    __shared__ int iscr[3 * 33];
     const int v = blockIdx.x;
     const int T = c.T;
     const int64_t base = (int64_t)v * T;
@@ -288,43 +330,40 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             } else {
                 S = block_sum(sp, dscr);
             }
-            // quota q_m = remaining * w_m / S of every candidate
-            int ncap = 0;
+            // quota q_m = remaining * w_m / S of every candidate; in the same
+            // pass the caps that bind and, for the largest remainder, the
+            // floors and the fractional parts (non-negative doubles order like
+            // their bit patterns; a candidate's key is its pattern + 1, others
+            // 0, so non-candidates rank below every candidate)
+            long long ncap = 0, fsum = 0;
             for (int m = threadIdx.x; m < L; m += blockDim.x) {
                 const double w = uniform ? 1.0 : wgt[m];
-                const bool cand = nb[m] < 0 && (uniform || w > 0.0);
-                double q = -1.0;
-                if (cand) {
-                    q = (double)remaining * w / S;
+                unsigned long long key = 0ull;
+                if (nb[m] < 0 && (uniform || w > 0.0)) {
+                    const double q = (double)remaining * w / S;
+                    const double fl = floor(q);
                     ncap += (q > (double)N);
+                    fsum += (long long)fl;
+                    key = (unsigned long long)__double_as_longlong(q - fl) + 1ull;
                 }
-                keys[m] = (unsigned long long)__double_as_longlong(q);
+                keys[m] = key;
             }
-            ncap = (int)block_sum_ll(ncap, lscr);
+            block_sum2_ll(ncap, fsum, lscr);
             if (ncap > 0) {
-                for (int m = threadIdx.x; m < L; m += blockDim.x)
-                    if (__longlong_as_double((long long)keys[m]) > (double)N) nb[m] = N;
+                for (int m = threadIdx.x; m < L; m += blockDim.x) {
+                    const double w = uniform ? 1.0 : wgt[m];
+                    if (keys[m] != 0ull && (double)remaining * w / S > (double)N) nb[m] = N;
+                }
                 remaining -= (long long)N * ncap;
                 __syncthreads();
                 continue;
             }
-            // largest remainder among the candidates: rank the fractional
-            // parts (non-negative doubles order like their bit patterns; a
-            // candidate's key is its pattern + 1, others 0, so non-candidates
-            // rank below every candidate)
-            long long fsum = 0;
-            for (int m = threadIdx.x; m < L; m += blockDim.x) {
-                const double q = __longlong_as_double((long long)keys[m]);
-                unsigned long long key = 0ull;
-                if (q >= 0.0) {
-                    const double fl = floor(q);
-                    key = (unsigned long long)__double_as_longlong(q - fl) + 1ull;
-                    fsum += (long long)fl;
-                    nb[m] = (int)fl;       // floor; the remainder unit is added below
+            for (int m = threadIdx.x; m < L; m += blockDim.x)
+                if (keys[m] != 0ull) {   // floor; the remainder unit is added below
+                    const double w = uniform ? 1.0 : wgt[m];
+                    nb[m] = (int)floor((double)remaining * w / S);
                 }
-                keys[m] = key;
-            }
-            const long long R = remaining - block_sum_ll(fsum, lscr);
+            const long long R = remaining - fsum;
             for (int m = threadIdx.x; m < L; m += blockDim.x) {
                 const unsigned long long km = keys[m];
                 if (km == 0ull) continue;
@@ -357,22 +396,38 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     // scatter to frames, offsets, grids
     for (int m = threadIdx.x; m < L; m += blockDim.x) nf[lst[m]] = nb[m];
     __syncthreads();
-    int nloc[kPerThread];
-    int sum = 0;
+    // per frame: output rows, tensor-core operator rows (budgets padded to
+    // 16) and tensor-core units (column blocks of <= 256 tokens, each in
+    // groups of unit_tiles(round16(nc)) 128-channel tiles; the spatial kernel
+    // writes the unit records); one block scan gives all three offsets
+    const bool tc = c.path == WZ_PATH_TENSOR;
+    int nloc[kPerThread], ucnt[kPerThread];
+    int part[3] = {0, 0, 0};
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
         nloc[k] = (k < per && t < T) ? nf[t] : 0;
-        sum += nloc[k];
+        ucnt[k] = 0;
+        if (tc)
+            for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
+                const int nc = min(kColBlock, nloc[k] - j0);
+                ucnt[k] += (c.n_ct + unit_tiles((nc + 15) / 16 * 16) - 1) / unit_tiles((nc + 15) / 16 * 16);
+            }
+        part[0] += nloc[k];
+        part[1] += (nloc[k] + 15) & ~15;
+        part[2] += ucnt[k];
     }
-    int produced = 0;
-    int o = block_excl_scan(sum, iscr, &produced);
+    int pre[3], tot[3];
+    block_excl_scan3(part, iscr, pre, tot);
+    int o = pre[0], wo = pre[1], u = pre[2];
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
         if (k < per && t < T) {
             c.n[base + t] = nloc[k];
             c.off[base + t] = vp.row0 + o;
+            c.woff[base + t] = vp.w_row0 + wo;
+            if (tc) c.ustart[base + t] = u;
             const int h = grid_h(nloc[k], c.H, c.W);
             c.hw[2 * (base + t)] = h;
             c.hw[2 * (base + t) + 1] = h > 0 ? (nloc[k] + h - 1) / h : 0;
@@ -386,52 +441,15 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             }
         }
         o += nloc[k];
+        wo += (nloc[k] + 15) & ~15;
+        u += ucnt[k];
     }
     if (threadIdx.x == 0) {
-        c.prod[v] = produced;
-        if (c.out_count) c.out_count[v] = produced;
-    }
-    // first tensor-core operator row of each frame: budgets padded to 16
-    int s16 = 0;
-#pragma unroll
-    for (int k = 0; k < kPerThread; ++k) s16 += (nloc[k] + 15) & ~15;
-    int wtot = 0;
-    int wo = block_excl_scan(s16, iscr, &wtot);
-#pragma unroll
-    for (int k = 0; k < kPerThread; ++k) {
-        const int t = t0 + k;
-        if (k < per && t < T) c.woff[base + t] = vp.w_row0 + wo;
-        wo += (nloc[k] + 15) & ~15;
-    }
-    // tensor-core units: per frame, column blocks of <= 256 tokens; per
-    // block, groups of unit_tiles(round16(nc)) 128-channel tiles.  Here the
-    // count and the first unit of each frame; the spatial kernel writes the
-    // records.
-    if (c.path == WZ_PATH_TENSOR) {
-        int ucnt[kPerThread];
-        int us = 0;
-#pragma unroll
-        for (int k = 0; k < kPerThread; ++k) {
-            ucnt[k] = 0;
-            for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
-                const int nc = min(kColBlock, nloc[k] - j0);
-                const int ncp = (nc + 15) / 16 * 16;
-                const int cg = unit_tiles(ncp);
-                ucnt[k] += (c.n_ct + cg - 1) / cg;
-            }
-            us += ucnt[k];
-        }
-        int total = 0;
-        int u = block_excl_scan(us, iscr, &total);
-#pragma unroll
-        for (int k = 0; k < kPerThread; ++k) {
-            const int t = t0 + k;
-            if (k < per && t < T) c.ustart[base + t] = u;
-            u += ucnt[k];
-        }
-        if (threadIdx.x == 0) {
-            c.ucount[v] = min(total, c.max_units_v);
-            if (total > c.max_units_v) atomicOr(c.status, 2);
+        c.prod[v] = tot[0];
+        if (c.out_count) c.out_count[v] = tot[0];
+        if (tc) {
+            c.ucount[v] = min(tot[2], c.max_units_v);
+            if (tot[2] > c.max_units_v) atomicOr(c.status, 2);
         }
     }
 }

@@ -207,6 +207,37 @@ __device__ __forceinline__ long long block_sum_ll(long long v, long long *scratc
     return scratch[32];
 }
 
+// Two block-wide sums of long longs at once; `scratch` holds >= 66 values;
+// all threads receive both sums in place.
+__device__ __forceinline__ void block_sum2_ll(long long &a, long long &b, long long *scratch) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nw = (blockDim.x + 31) >> 5;
+    for (int o = 16; o > 0; o >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, o);
+        b += __shfl_xor_sync(0xffffffffu, b, o);
+    }
+    __syncthreads();
+    if (lane == 0) {
+        scratch[warp] = a;
+        scratch[33 + warp] = b;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        long long s = lane < nw ? scratch[lane] : 0, t = lane < nw ? scratch[33 + lane] : 0;
+        for (int o = 16; o > 0; o >>= 1) {
+            s += __shfl_xor_sync(0xffffffffu, s, o);
+            t += __shfl_xor_sync(0xffffffffu, t, o);
+        }
+        if (lane == 0) {
+            scratch[32] = s;
+            scratch[65] = t;
+        }
+    }
+    __syncthreads();
+    a = scratch[32];
+    b = scratch[65];
+}
+
 // ---- packed fp32 pairs (f32x2 instructions of sm_100-class GPUs) ----------
 
 typedef unsigned long long f2_t;
