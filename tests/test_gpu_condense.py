@@ -259,6 +259,26 @@ def test_batch_parity(wz):
         compare_condense(sub, ref, Xv.dtype)
 
 
+def test_config_serving_batch_sampled(wz):
+    """The serving batch at full size (32 videos x 64 frames, 13x13x3584 bf16,
+    Lq in [8, 128], ratios in {0.05, 0.1, 0.25}) in one call: every video's
+    budgets and index map bit-exact, the tokens of its first and last frame
+    with a budget."""
+    vids = [accepted_video(s, tries=4) for s in wl.batch_specs()]
+    X = torch.stack([v[1] for v in vids])
+    Qs = torch.cat([v[2] for v in vids])
+    out = wz.wz_condense_batch(X.cuda(), Qs.cuda(), [s.Lq for s, *_ in vids], [s.ratio for s, *_ in vids])
+    torch.cuda.synchronize()
+    offs = out["row_offsets"]
+    for v, (s, Xv, Qv, ref0) in enumerate(vids):
+        pos = np.nonzero(ref0["budgets"] > 0)[0]
+        frames = sorted({int(pos[0]), int(pos[-1])})
+        ref = oracle_run(Xv, Qv, s.ratio, token_frames=frames)
+        sub = {"budgets": out["budgets"][v], "count": out["count"][v:v + 1],
+               "index": out["index"][offs[v]:offs[v + 1]], "tokens": out["tokens"][offs[v]:offs[v + 1]]}
+        compare_condense(sub, ref, Xv.dtype, frames=frames)
+
+
 def test_relevance_entry_point(wz):
     X, Q, _ = wl.make_video(wl.VideoSpec(T=12, H=13, W=13, D=512, Lq=7, seed=8))
     ts, fs, fm = wz.wz_relevance(X.cuda(), Q.cuda(), frame_mean=True)
