@@ -389,6 +389,19 @@ WZ_API const char *wz_status_string(int status);
 /* Library version, 10000*major + 100*minor + patch. */
 WZ_API int wz_version(void);
 
+/*
+ * Self-test of the bounded waits that every pipelined kernel uses (TMA and
+ * tensor-core handoffs through shared-memory barriers): one block waits on a
+ * barrier that nothing completes, gives up after `timeout_ns` (globaltimer
+ * nanoseconds), records WZ_STATUS_WAIT_TIMEOUT in device_status[0] and
+ * exits, so the context stays usable.  device_status: [1] int32 device
+ * buffer, caller-owned, OR-ed into (not cleared).  Returns WZ_ERR_INVALID_ARG
+ * for a null status or a timeout of 0 or over one second, WZ_ERR_CUDA on a
+ * launch error, else WZ_OK (asynchronous on `stream`).
+ */
+#define WZ_STATUS_WAIT_TIMEOUT 0x100
+WZ_API int wz_selftest_bounded_wait(uint64_t timeout_ns, int32_t *device_status, wz_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

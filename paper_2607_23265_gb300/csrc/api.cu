@@ -10,6 +10,8 @@
 #include <cstring>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "wz_spatial.cuh"
 
 namespace wz {
@@ -24,6 +26,12 @@ constexpr size_t kAlign = 256;
 size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+// NVTX range around a host-side launch (a no-op unless a profiler listens).
+struct Nvtx {
+    explicit Nvtx(const char *name) { nvtxRangePushA(name); }
+    ~Nvtx() { nvtxRangePop(); }
+};
 
 // Sub-buffer offsets of one call's workspace.
 struct Layout {
@@ -348,15 +356,23 @@ int run_condense(const CondenseRequest &r) {
     auto mark = [&](int k) -> cudaError_t {
         return r.events ? cudaEventRecord((cudaEvent_t)r.events[k], r.stream) : cudaSuccess;
     };
+    Nvtx whole("wz::condense");
     WZ_CUDA(mark(2 * WZ_KERNEL_QUERY_POOL));
-    WZ_CUDA(launch_query_pool(c, par.data(), r.stream));
+    {
+        Nvtx n_("wz::query_pool");
+        WZ_CUDA(launch_query_pool(c, par.data(), r.stream));
+    }
     WZ_CUDA(mark(2 * WZ_KERNEL_QUERY_POOL + 1));
     WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE));
-    WZ_CUDA(launch_relevance_pass(c, r.stream));
+    {
+        Nvtx n_("wz::relevance_pass");
+        WZ_CUDA(launch_relevance_pass(c, r.stream));
+    }
     WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE + 1));
     if (c.relevance_mode == WZ_RELEVANCE_MAXSIM) {
         // the token x query-row cosines on the tensor cores, video by video
         // (the relevance pass left ||u|| in c.a)
+        Nvtx n_("wz::maxsim");
         for (int v = 0; v < r.V; ++v) {
             const int Lq = r.Lq[v], Lqp = (Lq + 15) / 16 * 16;
             const int64_t tok = (int64_t)s.T * s.N;
@@ -366,16 +382,26 @@ int run_condense(const CondenseRequest &r) {
         }
     }
     WZ_CUDA(mark(2 * WZ_KERNEL_FRAME_STATS));
-    WZ_CUDA(launch_frame_stats(c, r.stream));
+    {
+        Nvtx n_("wz::frame_stats");
+        WZ_CUDA(launch_frame_stats(c, r.stream));
+    }
     WZ_CUDA(mark(2 * WZ_KERNEL_FRAME_STATS + 1));
     WZ_CUDA(mark(2 * WZ_KERNEL_TEMPORAL));
-    WZ_CUDA(launch_temporal(c, r.stream));
+    {
+        Nvtx n_("wz::temporal");
+        WZ_CUDA(launch_temporal(c, r.stream));
+    }
     WZ_CUDA(mark(2 * WZ_KERNEL_TEMPORAL + 1));
     WZ_CUDA(mark(2 * WZ_KERNEL_SPATIAL));
-    WZ_CUDA(launch_spatial(c, r.stream));
+    {
+        Nvtx n_("wz::spatial");
+        WZ_CUDA(launch_spatial(c, r.stream));
+    }
     WZ_CUDA(mark(2 * WZ_KERNEL_SPATIAL + 1));
     WZ_CUDA(mark(2 * WZ_KERNEL_CONDENSE));
     if (rows > 0) {
+        Nvtx n_("wz::condense_tokens");
         if (c.path == WZ_PATH_TENSOR) WZ_CUDA(launch_condense_tc(c, r.stream));
         else WZ_CUDA(launch_condense_simt(c, r.stream));
     }

@@ -122,6 +122,7 @@ def _load():
         "wz_idwt2d": (i, [vp, vp, vp, vp, i, i, i, i, i, vp, vp]),
         "wz_status_string": (C.c_char_p, [i]),
         "wz_version": (i, []),
+        "wz_selftest_bounded_wait": (i, [C.c_uint64, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -411,6 +412,19 @@ def wz_idwt2d(LL, LH, HL, HH, H: int, W: int, wavelet: int = 4, stream=None):
 
 def wz_version() -> int:
     return int(_lib.wz_version())
+
+
+STATUS_WAIT_TIMEOUT = 0x100
+
+
+def wz_selftest_bounded_wait(timeout_ns: int, device_status: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Launch the bounded-wait self-test; returns the [1] int32 status tensor
+    (STATUS_WAIT_TIMEOUT set once the kernel has given up)."""
+    if device_status is None:
+        device_status = torch.zeros((1,), dtype=torch.int32, device="cuda")
+    _check(_lib.wz_selftest_bounded_wait(int(timeout_ns), device_status.data_ptr(),
+                                         _stream(stream, device_status.device)), "wz_selftest_bounded_wait")
+    return device_status
 
 
 def wz_project_workspace_size(B: int, C_: int) -> int:
