@@ -146,10 +146,28 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     // ---- per-frame tables ------------------------------------------------
     // the frame-independent tables (analysis matrices, supports), built once
     // per pass
-    for (int k = tid; k < L.tables; k += blockDim.x) reinterpret_cast<int *>(sm)[k] = reinterpret_cast<const int *>(c.stab)[k];
+    {   // 16-byte copies, two in flight per thread (the tables and the stab buffer are 16-byte aligned)
+        const int n4 = L.tables >> 2;
+        const int4 *src = reinterpret_cast<const int4 *>(c.stab);
+        int4 *dst = reinterpret_cast<int4 *>(sm);
+        const int bd = (int)blockDim.x;
+        for (int k = tid; k < n4; k += 2 * bd) {
+            const int4 x0 = src[k];
+            const bool two = k + bd < n4;
+            const int4 x1 = two ? src[k + bd] : x0;
+            dst[k] = x0;
+            if (two) dst[k + bd] = x1;
+        }
+    }
     // gate G of this frame (Eq. 6, Eq. 12), pooled by frame_stats
     const float *Gf = c.gate + f * (int64_t)c.gate_stride;
-    for (int k = tid; k < hp * wp; k += blockDim.x) G[k] = Gf[k];
+    for (int k = tid; k < hp * wp; k += 2 * blockDim.x) {
+        const float g0 = Gf[k];
+        const bool two = k + (int)blockDim.x < hp * wp;
+        const float g1 = two ? Gf[k + blockDim.x] : 0.f;
+        G[k] = g0;
+        if (two) G[k + blockDim.x] = g1;
+    }
     // bilinear columns through the synthesis: Q_v[q][b] and its support
     for (int k = tid; k < w * wp; k += blockDim.x) {
         const int q = k / wp, b = k % wp;

@@ -61,7 +61,19 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_ml_kernel(Ctx c, int 
     }
 
     // ---- per-frame tables ------------------------------------------------
-    for (int k = tid; k < T.copy; k += blockDim.x) si[k] = gi[k];
+    {   // 16-byte copies, two in flight per thread (T.copy is a multiple of 4 words)
+        const int n4 = T.copy >> 2;
+        const int4 *src = reinterpret_cast<const int4 *>(gi);
+        int4 *dst = reinterpret_cast<int4 *>(si);
+        const int bd = (int)blockDim.x;
+        for (int k = tid; k < n4; k += 2 * bd) {
+            const int4 x0 = src[k];
+            const bool two = k + bd < n4;
+            const int4 x1 = two ? src[k + bd] : x0;
+            dst[k] = x0;
+            if (two) dst[k + bd] = x1;
+        }
+    }
     const float *Gf = c.gate + f * (int64_t)c.gate_stride;
     for (int k = tid; k < c.gate_stride; k += blockDim.x) G[k] = Gf[k];
     // bilinear columns through each level's synthesis, and their supports
