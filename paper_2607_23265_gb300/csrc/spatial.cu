@@ -108,7 +108,7 @@ __device__ void plain_operator_rows(const Ctx &c, const SpatialSmem &L, float *s
     }
 }
 
-template <int HMAX, bool PLAIN>
+template <int WMAX, bool PLAIN>
 __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) {
     pdl_wait();
     pdl_trigger();
@@ -137,11 +137,11 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     float *AHl = sm + L.AHl, *AHh = sm + L.AHh, *AWl = sm + L.AWl, *AWh = sm + L.AWh;
     float *PAl = sm + L.PAl, *PAh = sm + L.PAh, *Yl = sm + L.Yl, *Yh = sm + L.Yh;
     float *Ql = sm + L.Ql, *Qh = sm + L.Qh, *red = sm + L.red;
-    int *blo = reinterpret_cast<int *>(sm + L.blo), *bhi = reinterpret_cast<int *>(sm + L.bhi);
+    const int *jlo = reinterpret_cast<const int *>(sm + L.jlo), *jhi = reinterpret_cast<const int *>(sm + L.jhi);
     int *qlo = reinterpret_cast<int *>(sm + L.qlo), *qhi = reinterpret_cast<int *>(sm + L.qhi);
-    int *irange = reinterpret_cast<int *>(red + 48);
     float *stg = sm + L.stage;
-    const int HP4 = L.HP4;
+    const int HP4 = L.HP4, WP4 = L.WP4;
+    (void)red;
 
     // ---- per-frame tables ------------------------------------------------
     // the frame-independent tables (analysis matrices, supports), built once
@@ -189,8 +189,9 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * c.K_pad;
     float *W32 = static_cast<float *>(c.Wop);
     const int K_pad = c.K_pad;
-    const int wsh = W <= 32 ? 5 : 6;
     const size_t kstride = (size_t)(c.w_rows >> 3) * 256;   // tile_index step of 32 columns
+    const int lane = tid & 31, warp = tid >> 5, nwarp = (int)(blockDim.x >> 5);
+    const int IH = (H + 31) >> 5;                            // 32-row slices of the map
     const int t = (int)(f % c.T);
 
     // ---- grid rows p = s0, s0 + S, ... ------------------------------------
@@ -204,10 +205,6 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
         synth_support(y0, y1, F, hp, alo, ahi);
         const int na = ahi - alo + 1;
         __syncthreads();   // previous row's Y / stage reads, the frame tables
-        if (tid == 0) {
-            irange[0] = HMAX;
-            irange[1] = -1;
-        }
         for (int k = tid; k < na * H; k += blockDim.x) {
             const int ai = alo + k / H, i = k % H;
             const float pl = (1.f - ly) * synth(c.rec_lo, F, y0, ai) + ly * synth(c.rec_lo, F, y1, ai);
@@ -216,8 +213,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
             PAh[k] = ph * AHh[ai * H + i];
         }
         __syncthreads();
-        // Y_v[b][i], rows padded to a multiple of 4 with zeros; [ilo, ihi] = rows it reaches
-        int my_lo = HMAX, my_hi = -1;
+        // Y_v[b][i], rows padded to a multiple of 4 with zeros
         for (int k = tid; k < wp * HP4; k += blockDim.x) {
             const int b = k / HP4, i = k % HP4;
             float yl = 0.f, yh = 0.f;
@@ -228,61 +224,54 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
                     yl += pl + ph * g;
                     yh += (pl + ph) * g;
                 }
-                if (yl != 0.f || yh != 0.f) {
-                    my_lo = min(my_lo, i);
-                    my_hi = max(my_hi, i);
-                }
             }
             Yl[k] = yl;
             Yh[k] = yh;
         }
-        for (int o = 16; o > 0; o >>= 1) {
-            my_lo = min(my_lo, __shfl_xor_sync(0xffffffffu, my_lo, o));
-            my_hi = max(my_hi, __shfl_xor_sync(0xffffffffu, my_hi, o));
-        }
-        if ((tid & 31) == 0 && my_hi >= 0) {
-            atomicMin(&irange[0], my_lo);
-            atomicMax(&irange[1], my_hi);
-        }
         __syncthreads();
-        const int i4lo = irange[0] >> 2, i4hi = irange[1] >> 2;   // empty when ihi < 0
         const int64_t row0 = (int64_t)c.off[f] + (int64_t)pi * w;                 // output row
         const int64_t wrow0 = bf ? (int64_t)c.woff[f] + (int64_t)pi * w : row0;   // operator row
-        // Rows are produced QB at a time: one thread per (output q, input
-        // column j) computes all H rows i in registers into a shared staging
-        // row; then the staged rows go out in 8-column groups (16-byte stores
-        // of the hi and lo halves, or of fp32).
+        // Rows are produced QB at a time.  One warp per (output token q,
+        // 32-row slice of the map), lane = input row i: per b of Q's support
+        // (uniform over the warp) the lane's coefficients Q_v[q,b] Y_v[b,i]
+        // times the analysis row A'_v[b,.] (a broadcast 16-byte read, only the
+        // column groups where the row is nonzero) accumulate all W columns j
+        // in registers; the lane then writes its row i of the staged row q.
+        // The staged rows go out in 8-column groups (16-byte stores of the hi
+        // and lo halves, or of fp32).
         for (int q0 = 0; q0 < nq; q0 += L.QB) {
             const int qn = min(L.QB, nq - q0);
-            // items (q, j): j is the lane within a stride of 32 or 64 columns
-            for (int item = tid; item < (qn << wsh); item += blockDim.x) {
-                const int ql_ = item >> wsh, j = item & ((1 << wsh) - 1);
-                if (j >= W) continue;
+            for (int item = warp; item < qn * IH; item += nwarp) {
+                const int ql_ = item / IH, i = (item - ql_ * IH) * 32 + lane;
                 const int q = q0 + ql_;
-                float acc[HMAX];
+                const bool live = i < H;
+                float acc[WMAX];
 #pragma unroll
-                for (int i = 0; i < HMAX; ++i) acc[i] = 0.f;
-                const int b1 = min(bhi[j], qhi[q]);
-                for (int b = max(blo[j], qlo[q]); b <= b1; ++b) {
-                    const float ql = Ql[q * wp + b] * AWl[b * W + j];
-                    const float qh = Qh[q * wp + b] * AWh[b * W + j];
-                    const float4 *yl = reinterpret_cast<const float4 *>(Yl + b * HP4);
-                    const float4 *yh = reinterpret_cast<const float4 *>(Yh + b * HP4);
+                for (int j = 0; j < WMAX; ++j) acc[j] = 0.f;
+                const int b1 = qhi[q];
+                for (int b = qlo[q]; b <= b1; ++b) {
+                    const float cl = live ? Ql[q * wp + b] * Yl[b * HP4 + i] : 0.f;
+                    const float ch = live ? Qh[q * wp + b] * Yh[b * HP4 + i] : 0.f;
+                    const int j4lo = jlo[b] >> 2, j4hi = jhi[b] >> 2;   // empty when jhi < 0
+                    const float4 *al = reinterpret_cast<const float4 *>(AWl + b * WP4);
+                    const float4 *ah = reinterpret_cast<const float4 *>(AWh + b * WP4);
 #pragma unroll
-                    for (int i4 = 0; i4 < HMAX / 4; ++i4) {
-                        if (i4 >= i4lo && i4 <= i4hi) {
-                            const float4 a4 = yl[i4], d4 = yh[i4];
-                            acc[4 * i4 + 0] = fmaf(a4.x, ql, fmaf(d4.x, qh, acc[4 * i4 + 0]));
-                            acc[4 * i4 + 1] = fmaf(a4.y, ql, fmaf(d4.y, qh, acc[4 * i4 + 1]));
-                            acc[4 * i4 + 2] = fmaf(a4.z, ql, fmaf(d4.z, qh, acc[4 * i4 + 2]));
-                            acc[4 * i4 + 3] = fmaf(a4.w, ql, fmaf(d4.w, qh, acc[4 * i4 + 3]));
+                    for (int j4 = 0; j4 < WMAX / 4; ++j4) {
+                        if (j4 >= j4lo && j4 <= j4hi) {
+                            const float4 a4 = al[j4], d4 = ah[j4];
+                            acc[4 * j4 + 0] = fmaf(cl, a4.x, fmaf(ch, d4.x, acc[4 * j4 + 0]));
+                            acc[4 * j4 + 1] = fmaf(cl, a4.y, fmaf(ch, d4.y, acc[4 * j4 + 1]));
+                            acc[4 * j4 + 2] = fmaf(cl, a4.z, fmaf(ch, d4.z, acc[4 * j4 + 2]));
+                            acc[4 * j4 + 3] = fmaf(cl, a4.w, fmaf(ch, d4.w, acc[4 * j4 + 3]));
                         }
                     }
                 }
-                float *srow = stg + ql_ * K_pad;
+                if (live) {
+                    float *srow = stg + ql_ * K_pad + i * W;
 #pragma unroll
-                for (int i = 0; i < HMAX; ++i)
-                    if (i < H) srow[i * W + j] = acc[i];
+                    for (int j = 0; j < WMAX; ++j)
+                        if (j < W) srow[j] = acc[j];
+                }
             }
             for (int k = tid; k < qn * (K_pad - N); k += blockDim.x)
                 stg[(k / (K_pad - N)) * K_pad + N + k % (K_pad - N)] = 0.f;
@@ -318,14 +307,14 @@ cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     if (c.spatial_mode == WZ_SPATIAL_WSM && c.wsm_levels > 1) return launch_spatial_ml(c, s);
     SpatialSmem L;
     L.init(c.H, c.W, c.hp, c.wp);
-    if ((L.Yl & 3) != 0 || (L.Yh & 3) != 0 || (L.stage & 3) != 0 || L.QB < 1) return cudaErrorMisalignedAddress;
+    if ((L.AWl & 3) != 0 || (L.AWh & 3) != 0 || (L.stage & 3) != 0 || L.QB < 1) return cudaErrorMisalignedAddress;
     const size_t smem = spatial_smem_bytes(c);
     const void *fn;
     const bool plain = c.spatial_mode != WZ_SPATIAL_WSM;
-    if (plain) fn = (const void *)spatial_kernel<4, true>;   // HMAX unused without the WSM
-    else if (c.H <= 16) fn = (const void *)spatial_kernel<16, false>;
-    else if (c.H <= 32) fn = (const void *)spatial_kernel<32, false>;
-    else if (c.H <= 64) fn = (const void *)spatial_kernel<64, false>;
+    if (plain) fn = (const void *)spatial_kernel<4, true>;   // WMAX unused without the WSM
+    else if (c.W <= 16) fn = (const void *)spatial_kernel<16, false>;
+    else if (c.W <= 32) fn = (const void *)spatial_kernel<32, false>;
+    else if (c.W <= 64) fn = (const void *)spatial_kernel<64, false>;
     else return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

@@ -13,9 +13,11 @@ namespace wz {
 constexpr int kStageFloats = 8 * 1024;   // staged operator rows (32 KB)
 
 struct SpatialSmem {
-    int N, hp, wp, H, W, HP4, K_pad, QB;
-    // float offsets; [0, tables) is the frame-independent part
-    int AHl, AHh, AWl, AWh, blo, bhi, tables;
+    int N, hp, wp, H, W, HP4, WP4, K_pad, QB;
+    // float offsets; [0, tables) is the frame-independent part.  The width
+    // analysis rows A'_v[b][.] are padded to WP4 columns (16-byte rows);
+    // jlo / jhi[b] are the first / last column where A'_L or A'_H is nonzero.
+    int AHl, AHh, AWl, AWh, jlo, jhi, tables;
     int G, PAl, PAh, Yl, Yh, Ql, Qh, red, qlo, qhi, M, stage, total;
     // Every table starts on a 16-byte boundary (float4 reads of Y, staged rows).
     __host__ __device__ void init(int H_, int W_, int hp_, int wp_) {
@@ -23,6 +25,7 @@ struct SpatialSmem {
         K_pad = (N + 31) & ~31;
         QB = kStageFloats / K_pad;                 // rows staged at a time (>= 2 for N <= 4096)
         HP4 = (H + 3) & ~3;
+        WP4 = (W + 3) & ~3;
         int o = 0;
         auto take = [&](int n) {
             const int at = o;
@@ -31,10 +34,10 @@ struct SpatialSmem {
         };
         AHl = take(hp * H);
         AHh = take(hp * H);
-        AWl = take(wp * W);
-        AWh = take(wp * W);
-        blo = take(W);
-        bhi = take(W);
+        AWl = take(wp * WP4);
+        AWh = take(wp * WP4);
+        jlo = take(wp);
+        jhi = take(wp);
         tables = o;
         G = take(hp * wp);
         PAl = take(hp * H);
@@ -174,7 +177,7 @@ inline size_t spatial_table_bytes(int H, int W, int F) {
 
 // Build the tables into c.stab (one CTA, any size).
 //   A[a][i] = sum_j dec[j] [ext(2a + 1 - j) == i]   (analysis along a side)
-//   blo/bhi[j] = first / last row b of A' with A'[b][j] != 0 (shared-memory
+//   jlo/jhi[b] = first / last column j with A'[b][j] != 0 (shared-memory
 //                atomics while A' is formed)
 __device__ inline void build_spatial_tables(const Ctx &c) {
     SpatialSmem L;
@@ -193,31 +196,32 @@ __device__ inline void build_spatial_tables(const Ctx &c) {
         tb[L.AHl + k] = sl;
         tb[L.AHh + k] = sh;
     }
-    __shared__ int s_blo[WZ_MAX_HW], s_bhi[WZ_MAX_HW];
-    for (int j = threadIdx.x; j < W; j += blockDim.x) {
-        s_blo[j] = wp;
-        s_bhi[j] = -1;
+    __shared__ int s_jlo[WZ_MAX_HW + kMaxTaps], s_jhi[WZ_MAX_HW + kMaxTaps];
+    for (int b = threadIdx.x; b < wp; b += blockDim.x) {
+        s_jlo[b] = L.WP4;
+        s_jhi[b] = -1;
     }
     __syncthreads();
-    for (int k = threadIdx.x; k < wp * W; k += blockDim.x) {
-        const int b = k / W, i = k % W;
+    for (int k = threadIdx.x; k < wp * L.WP4; k += blockDim.x) {
+        const int b = k / L.WP4, i = k % L.WP4;
         float sl = 0.f, sh = 0.f;
-        for (int j = 0; j < F; ++j)
-            if (ext_index(2 * b + 1 - j, W, c.mode) == i) {
-                sl += c.dec_lo[j];
-                sh += c.dec_hi[j];
-            }
+        if (i < W)
+            for (int j = 0; j < F; ++j)
+                if (ext_index(2 * b + 1 - j, W, c.mode) == i) {
+                    sl += c.dec_lo[j];
+                    sh += c.dec_hi[j];
+                }
         tb[L.AWl + k] = sl;
         tb[L.AWh + k] = sh;
         if (sl != 0.f || sh != 0.f) {
-            atomicMin(&s_blo[i], b);
-            atomicMax(&s_bhi[i], b);
+            atomicMin(&s_jlo[b], i);
+            atomicMax(&s_jhi[b], i);
         }
     }
     __syncthreads();
-    for (int j = threadIdx.x; j < W; j += blockDim.x) {
-        ti[L.blo + j] = s_blo[j];
-        ti[L.bhi + j] = s_bhi[j];
+    for (int b = threadIdx.x; b < wp; b += blockDim.x) {
+        ti[L.jlo + b] = s_jlo[b];
+        ti[L.jhi + b] = s_jhi[b];
     }
 }
 
