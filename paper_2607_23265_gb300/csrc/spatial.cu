@@ -21,6 +21,7 @@
 // them in shared memory and writes them as bf16 hi/lo pairs (tensor-core
 // path) or fp32 (CUDA-core path) in 16-byte groups, with the index map rows.
 // Trailing CTAs fill rows that cannot be produced with -1 / zeros.
+#include <algorithm>
 #include <cmath>
 
 #include "wz_spatial.cuh"
@@ -108,12 +109,11 @@ __device__ void plain_operator_rows(const Ctx &c, const SpatialSmem &L, float *s
     }
 }
 
-template <int WMAX, bool PLAIN>
-__global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) {
+// Ablation modes without the WSM: S CTAs per frame, grid rows p = s0, s0 + S, ...
+__global__ void __launch_bounds__(kSpatialThreads) spatial_plain_kernel(Ctx c, int S) {
     pdl_wait();
     pdl_trigger();
     extern __shared__ float sm[];
-    const int tid = threadIdx.x;
     const int64_t nblk_frames = (int64_t)c.V * c.T * S;
     if ((int64_t)blockIdx.x >= nblk_frames) {
         tail_rows(c, (int)(blockIdx.x - nblk_frames));
@@ -126,13 +126,28 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     const int h = c.hw[2 * f], w = c.hw[2 * f + 1];
     if (s0 >= h || s0 * w >= n) return;
     if (s0 == 0 && c.path == WZ_PATH_TENSOR) unit_records(c, f, n);
+    SpatialSmem L;
+    L.init(c.H, c.W, c.hp, c.wp);
+    plain_operator_rows(c, L, sm, f, s0, S, n, h, w);
+}
+
+// The WSM operator rows (single level), persistent: every CTA copies the
+// frame-independent tables once, then takes grid rows (frame f, row p) from
+// a global counter over the V*T*H candidates until none is left; a row
+// whose frame changes reloads the frame's gate and width rows.  Rows of
+// frames with a small budget cost as much as others, so the dynamic order
+// keeps the SMs evenly loaded.
+template <int WMAX>
+__global__ void __launch_bounds__(kSpatialThreads, WMAX <= 32 ? 4 : 2) spatial_wsm_kernel(Ctx c) {
+    pdl_wait();
+    pdl_trigger();
+    extern __shared__ float sm[];
+    __shared__ int s_item;
+    const int tid = threadIdx.x;
+    if ((int)blockIdx.x < kTailBlocks) tail_rows(c, (int)blockIdx.x);
     const int H = c.H, W = c.W, N = c.N, hp = c.hp, wp = c.wp, F = c.F;
     SpatialSmem L;
     L.init(H, W, hp, wp);
-    if constexpr (PLAIN) {   // ablation modes without the WSM
-        plain_operator_rows(c, L, sm, f, s0, S, n, h, w);
-        return;
-    }
     float *G = sm + L.G;
     float *AHl = sm + L.AHl, *AHh = sm + L.AHh, *AWl = sm + L.AWl, *AWh = sm + L.AWh;
     float *PAl = sm + L.PAl, *PAh = sm + L.PAh, *Yl = sm + L.Yl, *Yh = sm + L.Yh;
@@ -159,31 +174,6 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
             if (two) dst[k + bd] = x1;
         }
     }
-    // gate G of this frame (Eq. 6, Eq. 12), pooled by frame_stats
-    const float *Gf = c.gate + f * (int64_t)c.gate_stride;
-    for (int k = tid; k < hp * wp; k += 2 * blockDim.x) {
-        const float g0 = Gf[k];
-        const bool two = k + (int)blockDim.x < hp * wp;
-        const float g1 = two ? Gf[k + blockDim.x] : 0.f;
-        G[k] = g0;
-        if (two) G[k + blockDim.x] = g1;
-    }
-    // bilinear columns through the synthesis: Q_v[q][b] and its support
-    for (int k = tid; k < w * wp; k += blockDim.x) {
-        const int q = k / wp, b = k % wp;
-        int x0, x1;
-        float lx;
-        bilinear_src(q, W, w, x0, x1, lx);
-        Ql[k] = (1.f - lx) * synth(c.rec_lo, F, x0, b) + lx * synth(c.rec_lo, F, x1, b);
-        Qh[k] = (1.f - lx) * synth(c.rec_hi, F, x0, b) + lx * synth(c.rec_hi, F, x1, b);
-        if (b == 0) {
-            int l_, h_;
-            synth_support(x0, x1, F, wp, l_, h_);
-            qlo[q] = l_;
-            qhi[q] = h_;
-        }
-    }
-
     const bool bf = c.path == WZ_PATH_TENSOR;
     __nv_bfloat16 *Whi = static_cast<__nv_bfloat16 *>(c.Wop);
     __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * c.K_pad;
@@ -192,10 +182,50 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_kernel(Ctx c, int S) 
     const size_t kstride = (size_t)(c.w_rows >> 3) * 256;   // tile_index step of 32 columns
     const int lane = tid & 31, warp = tid >> 5, nwarp = (int)(blockDim.x >> 5);
     const int IH = (H + 31) >> 5;                            // 32-row slices of the map
-    const int t = (int)(f % c.T);
 
-    // ---- grid rows p = s0, s0 + S, ... ------------------------------------
-    for (int pi = s0; pi < h && pi * w < n; pi += S) {
+    const int64_t items = (int64_t)c.V * c.T * H;
+    int64_t cur_f = -1;
+    for (;;) {
+        __syncthreads();   // the previous row's reads of shared memory
+        if (tid == 0) s_item = atomicAdd(c.spatial_next, 1);
+        __syncthreads();
+        const int64_t item = s_item;
+        if (item >= items) break;
+        const int64_t f = item / H;
+        const int pi = (int)(item - f * H);
+        const int n = c.n[f];
+        if (n <= 0) continue;
+        const int h = c.hw[2 * f], w = c.hw[2 * f + 1];
+        if (pi >= h || pi * w >= n) continue;
+        if (pi == 0 && c.path == WZ_PATH_TENSOR) unit_records(c, f, n);
+        const int t = (int)(f % c.T);
+        if (f != cur_f) {
+            // gate G of this frame (Eq. 6, Eq. 12), pooled by frame_stats
+            const float *Gf = c.gate + f * (int64_t)c.gate_stride;
+            for (int k = tid; k < hp * wp; k += 2 * blockDim.x) {
+                const float g0 = Gf[k];
+                const bool two = k + (int)blockDim.x < hp * wp;
+                const float g1 = two ? Gf[k + blockDim.x] : 0.f;
+                G[k] = g0;
+                if (two) G[k + blockDim.x] = g1;
+            }
+            // bilinear columns through the synthesis: Q_v[q][b] and its support
+            for (int k = tid; k < w * wp; k += blockDim.x) {
+                const int q = k / wp, b = k % wp;
+                int x0, x1;
+                float lx;
+                bilinear_src(q, W, w, x0, x1, lx);
+                Ql[k] = (1.f - lx) * synth(c.rec_lo, F, x0, b) + lx * synth(c.rec_lo, F, x1, b);
+                Qh[k] = (1.f - lx) * synth(c.rec_hi, F, x0, b) + lx * synth(c.rec_hi, F, x1, b);
+                if (b == 0) {
+                    int l_, h_;
+                    synth_support(x0, x1, F, wp, l_, h_);
+                    qlo[q] = l_;
+                    qhi[q] = h_;
+                }
+            }
+            cur_f = f;
+        }
         const int nq = min(w, n - pi * w);
         // bilinear row through the synthesis: P_u[a] is nonzero for a in [alo, ahi]
         int y0, y1;
@@ -309,12 +339,12 @@ cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     L.init(c.H, c.W, c.hp, c.wp);
     if ((L.AWl & 3) != 0 || (L.AWh & 3) != 0 || (L.stage & 3) != 0 || L.QB < 1) return cudaErrorMisalignedAddress;
     const size_t smem = spatial_smem_bytes(c);
-    const void *fn;
     const bool plain = c.spatial_mode != WZ_SPATIAL_WSM;
-    if (plain) fn = (const void *)spatial_kernel<4, true>;   // WMAX unused without the WSM
-    else if (c.W <= 16) fn = (const void *)spatial_kernel<16, false>;
-    else if (c.W <= 32) fn = (const void *)spatial_kernel<32, false>;
-    else if (c.W <= 64) fn = (const void *)spatial_kernel<64, false>;
+    const void *fn;
+    if (plain) fn = (const void *)spatial_plain_kernel;
+    else if (c.W <= 16) fn = (const void *)spatial_wsm_kernel<16>;
+    else if (c.W <= 32) fn = (const void *)spatial_wsm_kernel<32>;
+    else if (c.W <= 64) fn = (const void *)spatial_wsm_kernel<64>;
     else return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -323,9 +353,17 @@ cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
     if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kSpatialThreads, smem)) != cudaSuccess)
         return e;
-    int S = spatial_split(c, sms * (per_sm > 0 ? per_sm : 1));
-    const unsigned blocks = (unsigned)((int64_t)c.V * c.T * S + kTailBlocks);
-    void *args[] = {const_cast<Ctx *>(&c), &S};
+    const int resident = sms * (per_sm > 0 ? per_sm : 1);
+    if (plain) {
+        int S = spatial_split(c, resident);
+        const unsigned blocks = (unsigned)((int64_t)c.V * c.T * S + kTailBlocks);
+        void *args[] = {const_cast<Ctx *>(&c), &S};
+        return launch_kernel(fn, dim3(blocks), dim3(kSpatialThreads), smem, s, args, c.pdl != 0);
+    }
+    // persistent: every resident CTA pulls grid rows; at least kTailBlocks
+    // CTAs so that the tail rows are covered
+    const unsigned blocks = (unsigned)std::max(resident, kTailBlocks);
+    void *args[] = {const_cast<Ctx *>(&c)};
     return launch_kernel(fn, dim3(blocks), dim3(kSpatialThreads), smem, s, args, c.pdl != 0);
 }
 

@@ -64,6 +64,7 @@ struct Ctx {
     void *Wop;            // operator: tensor path bf16 hi then lo in the tiled
                           // layout of tile_index(), CUDA-core path f32 [rows][K_pad]
     int *status;          // device status word (bounded waits)
+    int *spatial_next;    // next (frame, grid row) of the spatial operator kernel; zeroed by temporal
 
     void *out;            // [rows][D] dtype
     int *out_index;       // [rows][3]
