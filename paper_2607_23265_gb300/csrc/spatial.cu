@@ -80,13 +80,13 @@ __device__ void plain_operator_rows(const Ctx &c, const SpatialSmem &L, float *s
         for (int q0 = 0; q0 < nq; q0 += L.QB) {
             const int qn = min(L.QB, nq - q0);
             __syncthreads();   // M, and the previous batch's reads of the stage
-            for (int k = tid; k < qn * K_pad; k += blockDim.x) stg[k] = 0.f;
+            for (int k = tid; k < qn * L.KS; k += blockDim.x) stg[k] = 0.f;
             __syncthreads();
             for (int ql_ = tid; ql_ < qn; ql_ += blockDim.x) {
                 int x0, x1;
                 float lx;
                 bilinear_src(q0 + ql_, W, w, x0, x1, lx);
-                float *row = stg + ql_ * K_pad;
+                float *row = stg + ql_ * L.KS;
                 const int ys[2] = {y0, y1}, xs[2] = {x0, x1};
                 const float wy[2] = {1.f - ly, ly}, wx[2] = {1.f - lx, lx};
 #pragma unroll
@@ -98,7 +98,7 @@ __device__ void plain_operator_rows(const Ctx &c, const SpatialSmem &L, float *s
                     }
             }
             __syncthreads();
-            write_rows(stg, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
+            write_rows(stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
         }
         for (int q = tid; q < nq; q += blockDim.x) {
             int *o = c.out_index + (size_t)(row0 + q) * 3;
@@ -137,8 +137,8 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_plain_kernel(Ctx c, i
 // whose frame changes reloads the frame's gate and width rows.  Rows of
 // frames with a small budget cost as much as others, so the dynamic order
 // keeps the SMs evenly loaded.
-template <int WMAX>
-__global__ void __launch_bounds__(kSpatialThreads, WMAX <= 32 ? 4 : 2) spatial_wsm_kernel(Ctx c) {
+template <int BMAX>
+__global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c) {
     pdl_wait();
     pdl_trigger();
     extern __shared__ float sm[];
@@ -183,25 +183,27 @@ __global__ void __launch_bounds__(kSpatialThreads, WMAX <= 32 ? 4 : 2) spatial_w
     const int lane = tid & 31, warp = tid >> 5, nwarp = (int)(blockDim.x >> 5);
     const int IH = (H + 31) >> 5;                            // 32-row slices of the map
 
-    const int64_t items = (int64_t)c.V * c.T * H;
-    int64_t cur_f = -1;
+    // candidates (frame, grid row): f * H + p < V * T * H < 2^31, 32-bit
+    // index arithmetic throughout (no 64-bit divisions in the loop)
+    const int items = c.V * c.T * H;
+    int cur_f = -1;
     for (;;) {
         __syncthreads();   // the previous row's reads of shared memory
         if (tid == 0) s_item = atomicAdd(c.spatial_next, 1);
         __syncthreads();
-        const int64_t item = s_item;
+        const int item = s_item;
         if (item >= items) break;
-        const int64_t f = item / H;
-        const int pi = (int)(item - f * H);
+        const int f = item / H;
+        const int pi = item - f * H;
         const int n = c.n[f];
         if (n <= 0) continue;
         const int h = c.hw[2 * f], w = c.hw[2 * f + 1];
         if (pi >= h || pi * w >= n) continue;
         if (pi == 0 && c.path == WZ_PATH_TENSOR) unit_records(c, f, n);
-        const int t = (int)(f % c.T);
+        const int t = f % c.T;
         if (f != cur_f) {
             // gate G of this frame (Eq. 6, Eq. 12), pooled by frame_stats
-            const float *Gf = c.gate + f * (int64_t)c.gate_stride;
+            const float *Gf = c.gate + (int64_t)f * c.gate_stride;
             for (int k = tid; k < hp * wp; k += 2 * blockDim.x) {
                 const float g0 = Gf[k];
                 const bool two = k + (int)blockDim.x < hp * wp;
@@ -210,14 +212,15 @@ __global__ void __launch_bounds__(kSpatialThreads, WMAX <= 32 ? 4 : 2) spatial_w
                 if (two) G[k + blockDim.x] = g1;
             }
             // bilinear columns through the synthesis: Q_v[q][b] and its support
-            for (int k = tid; k < w * wp; k += blockDim.x) {
-                const int q = k / wp, b = k % wp;
+            for (int q = warp; q < w; q += nwarp) {   // warp per column q, lanes over b
                 int x0, x1;
                 float lx;
                 bilinear_src(q, W, w, x0, x1, lx);
-                Ql[k] = (1.f - lx) * synth(c.rec_lo, F, x0, b) + lx * synth(c.rec_lo, F, x1, b);
-                Qh[k] = (1.f - lx) * synth(c.rec_hi, F, x0, b) + lx * synth(c.rec_hi, F, x1, b);
-                if (b == 0) {
+                for (int b = lane; b < wp; b += 32) {
+                    Ql[q * wp + b] = (1.f - lx) * synth(c.rec_lo, F, x0, b) + lx * synth(c.rec_lo, F, x1, b);
+                    Qh[q * wp + b] = (1.f - lx) * synth(c.rec_hi, F, x0, b) + lx * synth(c.rec_hi, F, x1, b);
+                }
+                if (lane == 0) {
                     int l_, h_;
                     synth_support(x0, x1, F, wp, l_, h_);
                     qlo[q] = l_;
@@ -235,17 +238,20 @@ __global__ void __launch_bounds__(kSpatialThreads, WMAX <= 32 ? 4 : 2) spatial_w
         synth_support(y0, y1, F, hp, alo, ahi);
         const int na = ahi - alo + 1;
         __syncthreads();   // previous row's Y / stage reads, the frame tables
-        for (int k = tid; k < na * H; k += blockDim.x) {
-            const int ai = alo + k / H, i = k % H;
+        for (int u = warp; u < na; u += nwarp) {   // warp per coefficient row, lanes over i
+            const int ai = alo + u;
             const float pl = (1.f - ly) * synth(c.rec_lo, F, y0, ai) + ly * synth(c.rec_lo, F, y1, ai);
             const float ph = (1.f - ly) * synth(c.rec_hi, F, y0, ai) + ly * synth(c.rec_hi, F, y1, ai);
-            PAl[k] = pl * AHl[ai * H + i];
-            PAh[k] = ph * AHh[ai * H + i];
+            for (int i = lane; i < H; i += 32) {
+                PAl[u * H + i] = pl * AHl[ai * H + i];
+                PAh[u * H + i] = ph * AHh[ai * H + i];
+            }
         }
         __syncthreads();
         // Y_v[b][i], rows padded to a multiple of 4 with zeros
-        for (int k = tid; k < wp * HP4; k += blockDim.x) {
-            const int b = k / HP4, i = k % HP4;
+        for (int b = warp; b < wp; b += nwarp)   // warp per subband column b, lanes over i
+        for (int i = lane; i < HP4; i += 32) {
+            const int k = b * HP4 + i;
             float yl = 0.f, yh = 0.f;
             if (i < H) {
                 for (int u = 0; u < na; ++u) {
@@ -262,51 +268,63 @@ __global__ void __launch_bounds__(kSpatialThreads, WMAX <= 32 ? 4 : 2) spatial_w
         const int64_t row0 = (int64_t)c.off[f] + (int64_t)pi * w;                 // output row
         const int64_t wrow0 = bf ? (int64_t)c.woff[f] + (int64_t)pi * w : row0;   // operator row
         // Rows are produced QB at a time.  One warp per (output token q,
-        // 32-row slice of the map), lane = input row i: per b of Q's support
-        // (uniform over the warp) the lane's coefficients Q_v[q,b] Y_v[b,i]
-        // times the analysis row A'_v[b,.] (a broadcast 16-byte read, only the
-        // column groups where the row is nonzero) accumulate all W columns j
-        // in registers; the lane then writes its row i of the staged row q.
-        // The staged rows go out in 8-column groups (16-byte stores of the hi
-        // and lo halves, or of fp32).
+        // 32-row slice of the map), lane = input row i: the lane's
+        // coefficients c_v[b] = Q_v[q,b] Y_v[b,i] over the support of Q_v[q,.]
+        // (at most BMAX values, uniform over the warp) stay in registers; each
+        // 4-column group j of row i of the staged token q is then
+        // sum_b c_L[b] A'_L[b,j] + c_H[b] A'_H[b,j], with the analysis rows read
+        // as broadcast 16-byte words and only the groups the support reaches
+        // computed.  The staged rows go out in 8-column groups (write_rows).
         for (int q0 = 0; q0 < nq; q0 += L.QB) {
             const int qn = min(L.QB, nq - q0);
             for (int item = warp; item < qn * IH; item += nwarp) {
-                const int ql_ = item / IH, i = (item - ql_ * IH) * 32 + lane;
+                const int ql_ = IH == 1 ? item : item / IH, i = (item - ql_ * IH) * 32 + lane;
                 const int q = q0 + ql_;
                 const bool live = i < H;
-                float acc[WMAX];
+                const int b0 = qlo[q], nb = min(qhi[q] - b0 + 1, BMAX);
+                float cl[BMAX], ch[BMAX];
+                int jl = WP4, jh = -1;
 #pragma unroll
-                for (int j = 0; j < WMAX; ++j) acc[j] = 0.f;
-                const int b1 = qhi[q];
-                for (int b = qlo[q]; b <= b1; ++b) {
-                    const float cl = live ? Ql[q * wp + b] * Yl[b * HP4 + i] : 0.f;
-                    const float ch = live ? Qh[q * wp + b] * Yh[b * HP4 + i] : 0.f;
-                    const int j4lo = jlo[b] >> 2, j4hi = jhi[b] >> 2;   // empty when jhi < 0
-                    const float4 *al = reinterpret_cast<const float4 *>(AWl + b * WP4);
-                    const float4 *ah = reinterpret_cast<const float4 *>(AWh + b * WP4);
-#pragma unroll
-                    for (int j4 = 0; j4 < WMAX / 4; ++j4) {
-                        if (j4 >= j4lo && j4 <= j4hi) {
-                            const float4 a4 = al[j4], d4 = ah[j4];
-                            acc[4 * j4 + 0] = fmaf(cl, a4.x, fmaf(ch, d4.x, acc[4 * j4 + 0]));
-                            acc[4 * j4 + 1] = fmaf(cl, a4.y, fmaf(ch, d4.y, acc[4 * j4 + 1]));
-                            acc[4 * j4 + 2] = fmaf(cl, a4.z, fmaf(ch, d4.z, acc[4 * j4 + 2]));
-                            acc[4 * j4 + 3] = fmaf(cl, a4.w, fmaf(ch, d4.w, acc[4 * j4 + 3]));
-                        }
+                for (int bb = 0; bb < BMAX; ++bb) {
+                    const int b = b0 + bb;
+                    const bool on = bb < nb;
+                    cl[bb] = on && live ? Ql[q * wp + b] * Yl[b * HP4 + i] : 0.f;
+                    ch[bb] = on && live ? Qh[q * wp + b] * Yh[b * HP4 + i] : 0.f;
+                    if (on) {
+                        jl = min(jl, jlo[b]);
+                        jh = max(jh, jhi[b]);
                     }
                 }
-                if (live) {
-                    float *srow = stg + ql_ * K_pad + i * W;
+                float *srow = stg + ql_ * L.KS + i * W;
+                const int j4lo = jl >> 2, j4hi = jh >> 2;   // empty when jh < 0
+                for (int j4 = 0; 4 * j4 < W; ++j4) {
+                    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (j4 >= j4lo && j4 <= j4hi) {
 #pragma unroll
-                    for (int j = 0; j < WMAX; ++j)
-                        if (j < W) srow[j] = acc[j];
+                        for (int bb = 0; bb < BMAX; ++bb) {
+                            if (bb < nb) {
+                                const float4 a4 = reinterpret_cast<const float4 *>(AWl + (b0 + bb) * WP4)[j4];
+                                const float4 d4 = reinterpret_cast<const float4 *>(AWh + (b0 + bb) * WP4)[j4];
+                                acc.x = fmaf(cl[bb], a4.x, fmaf(ch[bb], d4.x, acc.x));
+                                acc.y = fmaf(cl[bb], a4.y, fmaf(ch[bb], d4.y, acc.y));
+                                acc.z = fmaf(cl[bb], a4.z, fmaf(ch[bb], d4.z, acc.z));
+                                acc.w = fmaf(cl[bb], a4.w, fmaf(ch[bb], d4.w, acc.w));
+                            }
+                        }
+                    }
+                    if (live) {
+                        const int j = 4 * j4;
+                        srow[j] = acc.x;
+                        if (j + 1 < W) srow[j + 1] = acc.y;
+                        if (j + 2 < W) srow[j + 2] = acc.z;
+                        if (j + 3 < W) srow[j + 3] = acc.w;
+                    }
                 }
             }
-            for (int k = tid; k < qn * (K_pad - N); k += blockDim.x)
-                stg[(k / (K_pad - N)) * K_pad + N + k % (K_pad - N)] = 0.f;
+            for (int ql_ = warp; ql_ < qn; ql_ += nwarp)   // padding columns [N, K_pad)
+                for (int j = N + lane; j < K_pad; j += 32) stg[ql_ * L.KS + j] = 0.f;
             __syncthreads();
-            write_rows(stg, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
+            write_rows(stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
             if (q0 + L.QB < nq) __syncthreads();
         }
         for (int q = tid; q < nq; q += blockDim.x) {
@@ -342,9 +360,10 @@ cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     const bool plain = c.spatial_mode != WZ_SPATIAL_WSM;
     const void *fn;
     if (plain) fn = (const void *)spatial_plain_kernel;
-    else if (c.W <= 16) fn = (const void *)spatial_wsm_kernel<16>;
-    else if (c.W <= 32) fn = (const void *)spatial_wsm_kernel<32>;
-    else if (c.W <= 64) fn = (const void *)spatial_wsm_kernel<64>;
+    // BMAX bounds the support of a bilinear column through the synthesis:
+    // at most (F - 1) / 2 + 2 coefficients
+    else if ((c.F - 1) / 2 + 2 <= 6) fn = (const void *)spatial_wsm_kernel<6>;
+    else if ((c.F - 1) / 2 + 2 <= 12) fn = (const void *)spatial_wsm_kernel<12>;
     else return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

@@ -198,15 +198,15 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_ml_kernel(Ctx c, int 
                         }
                     }
                 }
-                float *srow = stg + ql_ * K_pad;
+                float *srow = stg + ql_ * L.KS;
 #pragma unroll
                 for (int i = 0; i < HMAX; ++i)
                     if (i < H) srow[i * W + j] = acc[i];
             }
             for (int k = tid; k < qn * (K_pad - N); k += blockDim.x)
-                stg[(k / (K_pad - N)) * K_pad + N + k % (K_pad - N)] = 0.f;
+                stg[(k / (K_pad - N)) * L.KS + N + k % (K_pad - N)] = 0.f;
             __syncthreads();
-            write_rows(stg, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
+            write_rows(stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
             if (q0 + L.QB < nq) __syncthreads();
         }
         for (int q = tid; q < nq; q += blockDim.x) {

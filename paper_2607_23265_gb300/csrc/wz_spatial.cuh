@@ -13,7 +13,7 @@ namespace wz {
 constexpr int kStageFloats = 8 * 1024;   // staged operator rows (32 KB)
 
 struct SpatialSmem {
-    int N, hp, wp, H, W, HP4, WP4, K_pad, QB;
+    int N, hp, wp, H, W, HP4, WP4, K_pad, KS, QB;
     // float offsets; [0, tables) is the frame-independent part.  The width
     // analysis rows A'_v[b][.] are padded to WP4 columns (16-byte rows);
     // jlo / jhi[b] are the first / last column where A'_L or A'_H is nonzero.
@@ -23,7 +23,8 @@ struct SpatialSmem {
     __host__ __device__ void init(int H_, int W_, int hp_, int wp_) {
         H = H_; W = W_; hp = hp_; wp = wp_; N = H * W;
         K_pad = (N + 31) & ~31;
-        QB = kStageFloats / K_pad;                 // rows staged at a time (>= 2 for N <= 4096)
+        KS = K_pad + 4;                            // staged row stride (see write_rows)
+        QB = kStageFloats / KS;                    // rows staged at a time (>= 1 for N <= 4096)
         HP4 = (H + 3) & ~3;
         WP4 = (W + 3) & ~3;
         int o = 0;
@@ -50,7 +51,7 @@ struct SpatialSmem {
         qlo = take(W);
         qhi = take(W);
         M = take(N);                               // saliency map (ablation mode "saliency")
-        stage = take(QB * K_pad);
+        stage = take(QB * KS);
         total = o;
     }
 };
@@ -88,19 +89,28 @@ __device__ __forceinline__ void synth_support(int y0, int y1, int F, int na, int
     hi = min(na - 1, (y1 + F - 2) >> 1);
 }
 
-// Staged rows [0, qn) of a grid row go out in 8-column groups: bf16 hi and
-// lo halves at tile_index(r, 8 g, w_rows) (tensor path; r = r_first + row,
-// split into a row part and a column part) or fp32 rows (CUDA-core path).
-__device__ __forceinline__ void write_rows(const float *stg, int qn, int K_pad, int64_t r_first, bool bf,
+// Staged rows [0, qn) of a grid row (row stride ks floats) go out in
+// 8-column groups: bf16 hi and lo halves at tile_index(r, 8 g, w_rows)
+// (tensor path; r = r_first + row) or fp32 rows (CUDA-core path).  On the
+// tensor path a warp writes one 8-row group x 32-column chunk: lane = (column
+// quarter, row within the group), so its 32 16-byte stores fill one
+// contiguous 512-byte block of the tiled layout.  A stride ks = K_pad + 4
+// keeps the eight rows' shared-memory reads on distinct banks.
+__device__ __forceinline__ void write_rows(const float *stg, int ks, int qn, int K_pad, int64_t r_first, bool bf,
                                            __nv_bfloat16 *Whi, __nv_bfloat16 *Wlo, float *W32, size_t kstride) {
-    const int G8 = K_pad / 8;
-    int ql_ = (int)threadIdx.x / G8, g = (int)threadIdx.x % G8;
-    const int gstep = (int)blockDim.x % G8, qstep = (int)blockDim.x / G8;
-    for (; ql_ < qn;) {
-        const float4 v0 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g);
-        const float4 v1 = *reinterpret_cast<const float4 *>(stg + ql_ * K_pad + 8 * g + 4);
-        const int64_t r = r_first + ql_;
-        if (bf) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = (int)(blockDim.x >> 5);
+    if (bf) {
+        const int rr = lane & 7, qq = lane >> 3;
+        const int64_t rg0 = r_first >> 3, rg1 = (r_first + qn - 1) >> 3;
+        const int nrg = (int)(rg1 - rg0 + 1), nk = K_pad >> 5;
+        for (int it = warp; it < nrg * nk; it += nwarp) {
+            const int rgi = it / nk, g4 = it - rgi * nk;
+            const int64_t r = (rg0 + rgi) * 8 + rr;
+            const int ql_ = (int)(r - r_first);
+            if (ql_ < 0 || ql_ >= qn) continue;
+            const float *src = stg + ql_ * ks + 32 * g4 + 8 * qq;
+            const float4 v0 = *reinterpret_cast<const float4 *>(src);
+            const float4 v1 = *reinterpret_cast<const float4 *>(src + 4);
             const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
             uint32_t hw[4], lw[4];
 #pragma unroll
@@ -111,20 +121,18 @@ __device__ __forceinline__ void write_rows(const float *stg, int qn, int K_pad, 
                 hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
                 lw[e] = *reinterpret_cast<const uint32_t *>(&ll);
             }
-            const size_t ti = (size_t)(g >> 2) * kstride + (size_t)(r >> 3) * 256 + (size_t)(r & 7) * 8 +
-                              (size_t)(g & 3) * 64;
+            const size_t ti = (size_t)g4 * kstride + (size_t)(r >> 3) * 256 + (size_t)rr * 8 + (size_t)qq * 64;
             *reinterpret_cast<uint4 *>(Whi + ti) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
             *reinterpret_cast<uint4 *>(Wlo + ti) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-        } else {
-            float *dst = W32 + (size_t)r * K_pad + 8 * g;
-            *reinterpret_cast<float4 *>(dst) = v0;
-            *reinterpret_cast<float4 *>(dst + 4) = v1;
         }
-        g += gstep;
-        ql_ += qstep;
-        if (g >= G8) {
-            g -= G8;
-            ++ql_;
+    } else {
+        const int G8 = K_pad / 8;
+        for (int it = threadIdx.x; it < qn * G8; it += blockDim.x) {
+            const int ql_ = it / G8, g = it - ql_ * G8;
+            const float *src = stg + ql_ * ks + 8 * g;
+            float *dst = W32 + (size_t)(r_first + ql_) * K_pad + 8 * g;
+            *reinterpret_cast<float4 *>(dst) = *reinterpret_cast<const float4 *>(src);
+            *reinterpret_cast<float4 *>(dst + 4) = *reinterpret_cast<const float4 *>(src + 4);
         }
     }
 }
@@ -299,7 +307,7 @@ inline size_t ml_table_bytes(int H, int W, int F, int J) {
 
 // Shared memory of one multi-level spatial CTA.
 struct MLSmem {
-    int HP4, K_pad, QB;
+    int HP4, K_pad, KS, QB;
     int G;                                  // the frame's gates, levels 1..J (c.goff layout)
     int Ql[kMaxLevels], Qh[kMaxLevels];     // [w][w_l] (w <= W)
     int qlo[kMaxLevels], qhi[kMaxLevels];   // [W] int
@@ -309,7 +317,8 @@ struct MLSmem {
     __host__ __device__ void init(const MLTables &T) {
         const int H = T.H, W = T.W, N = H * W;
         K_pad = (N + 31) & ~31;
-        QB = kStageFloats / K_pad;
+        KS = K_pad + 4;                            // staged row stride (see write_rows)
+        QB = kStageFloats / KS;
         HP4 = (H + 3) & ~3;
         int o = T.copy;
         auto take = [&](int n) {
@@ -333,7 +342,7 @@ struct MLSmem {
         PAl = take(hmax * H);
         PAh = take(hmax * H);
         red = take(64);
-        stage = take(QB * K_pad);
+        stage = take(QB * KS);
         total = o;
     }
 };
