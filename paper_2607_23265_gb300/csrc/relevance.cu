@@ -409,16 +409,32 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
 // normalised a_{t,n} over the frame, average-pooled to the subband grid of
 // each DWT level (hp x wp for the first) and scaled by lambda.  `red` is >= 32
 // floats of shared scratch.
-__device__ void frame_gate(const Ctx &c, int64_t f, float *red) {
+constexpr int kGatePerThread = WZ_MAX_HW * WZ_MAX_HW / 512;   // a_{t,n} per thread of a 512-thread block
+
+// The frame's a_{t,n} (an external scorer's if given), this thread's share
+// k = threadIdx.x + 512 r, loaded into registers early so that the loads
+// overlap the frame statistics.
+__device__ __forceinline__ void gate_prefetch(const Ctx &c, int64_t f, float (&av)[kGatePerThread]) {
+    const float *a = (c.ext_a ? c.ext_a : c.a) + f * c.N;
+#pragma unroll
+    for (int r = 0; r < kGatePerThread; ++r) {
+        const int k = (int)threadIdx.x + 512 * r;
+        av[r] = k < c.N ? a[k] : 0.f;
+    }
+}
+
+__device__ void frame_gate(const Ctx &c, int64_t f, float *red, const float (&av)[kGatePerThread]) {
     __shared__ float M[WZ_MAX_HW * WZ_MAX_HW];
     const int N = c.N, H = c.H, W = c.W;
-    const float *a = (c.ext_a ? c.ext_a : c.a) + f * N;   // an external scorer's a_{t,n} if given
     float lo = INFINITY, hi = -INFINITY;
-    for (int k = threadIdx.x; k < N; k += blockDim.x) {
-        const float x = a[k];
-        M[k] = x;
-        lo = fminf(lo, x);
-        hi = fmaxf(hi, x);
+#pragma unroll
+    for (int r = 0; r < kGatePerThread; ++r) {
+        const int k = (int)threadIdx.x + 512 * r;
+        if (k < N) {
+            M[k] = av[r];
+            lo = fminf(lo, av[r]);
+            hi = fmaxf(hi, av[r]);
+        }
     }
     for (int o = 16; o > 0; o >>= 1) {
         lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
@@ -471,7 +487,10 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     __shared__ double wmax[16];
     extern __shared__ float4 sfs[];   // [D/4] frame sums (max-over-query scorer only)
     const bool maxsim = c.relevance_mode == WZ_RELEVANCE_MAXSIM;
+    const bool do_gate = c.gate && c.spatial_mode == WZ_SPATIAL_WSM;
     const int64_t f = blockIdx.x;
+    float av[kGatePerThread];
+    if (do_gate) gate_prefetch(c, f, av);
     const int t = (int)(f % c.T);
     const int v = (int)(f / c.T);
     const int64_t lo = f * c.N / c.L1;
@@ -485,13 +504,17 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f, p4 = 0.f;
     for (int i = threadIdx.x; i < nv; i += blockDim.x) {
         float4 sf = make_float4(0.f, 0.f, 0.f, 0.f), sp = sf;
-        for (int64_t cc = lo; cc <= hi; ++cc) {
+        for (int64_t cc = lo; cc <= hi; cc += 2) {   // two partial rows in flight, summed in order
             const float4 x = P[(size_t)(cc + f) * nv + i];
+            const float4 y = cc + 1 <= hi ? P[(size_t)(cc + 1 + f) * nv + i] : make_float4(0.f, 0.f, 0.f, 0.f);
             sf.x += x.x; sf.y += x.y; sf.z += x.z; sf.w += x.w;
+            if (cc + 1 <= hi) { sf.x += y.x; sf.y += y.y; sf.z += y.z; sf.w += y.w; }
         }
-        for (int64_t cc = lo2; cc <= hi2; ++cc) {
+        for (int64_t cc = lo2; cc <= hi2; cc += 2) {
             const float4 x = P[(size_t)(cc + g) * nv + i];
+            const float4 y = cc + 1 <= hi2 ? P[(size_t)(cc + 1 + g) * nv + i] : make_float4(0.f, 0.f, 0.f, 0.f);
             sp.x += x.x; sp.y += x.y; sp.z += x.z; sp.w += x.w;
+            if (cc + 1 <= hi2) { sp.x += y.x; sp.y += y.y; sp.z += y.z; sp.w += y.w; }
         }
         const float4 q = Qv[i];
         if (maxsim) sfs[i] = sf;
@@ -593,7 +616,7 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
         }
         if (c.frame_scores) c.frame_scores[f] = (float)r;
     }
-    if (c.gate && c.spatial_mode == WZ_SPATIAL_WSM) frame_gate(c, f, wsum[0]);
+    if (do_gate) frame_gate(c, f, wsum[0], av);
 }
 
 cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s) {
