@@ -53,6 +53,8 @@ def parse():
                    help="also time the projector P (Eq. 17) on the condensed tokens; 0 skips it")
     p.add_argument("--maxsim-steps", type=int, default=10,
                    help="also time the step with the max-over-query scorer; 0 skips it")
+    p.add_argument("--graph-steps", type=int, default=20,
+                   help="also time the step replayed from a captured CUDA graph; 0 skips it")
     p.add_argument("--variant-steps", type=int, default=5,
                    help="also time the wavelet, level, ablation and external-score variants; 0 skips them")
     return p.parse_args()
@@ -526,6 +528,34 @@ def run_ours(args, spec, world, rank, local):
     barrier()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.e2e_steps, world, dev)
 
+    # the same step captured once in a CUDA graph and replayed (launches of the
+    # six kernels submitted as one graph)
+    graph = None
+    if args.graph_steps > 0:
+        gs = torch.cuda.Stream(dev)
+        gs.wait_stream(stream)
+        with torch.cuda.stream(gs):
+            wz.wz_condense_ex(X, Q, spec.ratio, workspace=ws, out_tokens=tokens, out_index=index,
+                              device_status=status, path=args.path, stream=gs)
+        torch.cuda.synchronize(dev)
+        cg = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(cg, stream=gs):
+            wz.wz_condense_ex(X, Q, spec.ratio, workspace=ws, out_tokens=tokens, out_index=index,
+                              device_status=status, path=args.path, stream=gs)
+        for _ in range(3):
+            cg.replay()
+        barrier()
+        g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        for _ in range(args.graph_steps):
+            cg.replay()
+        g1.record(stream)
+        barrier()
+        gms = max_over_ranks(g0.elapsed_time(g1) / args.graph_steps, world, dev)
+        graph = {"ms_per_step": round(gms, 5), "value": job_value(T, world, gms), "unit": UNIT,
+                 "steps": args.graph_steps}
+        del cg
+
     projector = time_projector(wz, tokens, args.projector_steps, dev) if args.projector_steps > 0 else None
     maxsim = time_maxsim(wz, X, Q, spec.ratio, ws, status, args.maxsim_steps, dev) \
         if args.maxsim_steps > 0 and X.dtype == torch.bfloat16 and D % 64 == 0 else None
@@ -564,6 +594,7 @@ def run_ours(args, spec, world, rank, local):
             "clocks": clocks,
             "gpu_launches": len(KERNELS) * args.steps,
             "projector": projector,
+            "graph": graph,
             "maxsim": maxsim,
             "variants": variants,
         }
