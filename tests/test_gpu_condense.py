@@ -78,6 +78,8 @@ def _random_case(wz, T, H, W, D, Lq, ratio, seed=0, dtype="bf16", **kw):
     (33, 14, 14, 96, 5, 0.25),
     (600, 3, 4, 16, 2, 0.3),      # more frames than temporal threads: 2 frames per thread
     (4096, 2, 2, 8, 1, 0.4),      # longest video: 8 frames per thread, 4096-way ranking
+    (3, 4, 4, 32768, 2, 0.5),     # widest bf16 rows: 8 vectors per relevance thread, 256 channel tiles
+    (2, 3, 5, 12288, 3, 0.4),     # 4 vectors per relevance thread
 ])
 def test_shapes(wz, T, H, W, D, Lq, ratio):
     _random_case(wz, T, H, W, D, Lq, ratio, seed=T * 7 + H)
@@ -158,6 +160,12 @@ def test_external_scores(wz, which):
 
 def test_fp32_features(wz):
     _random_case(wz, 6, 14, 14, 96, 4, 0.25, seed=3, dtype="f32")
+
+
+@pytest.mark.parametrize("D", [16384, 4104])
+def test_fp32_wide_rows(wz, D):
+    # f32 rows up to the f32 limit (half of the bf16 one): 8 and 2 vectors per relevance thread
+    _random_case(wz, 3, 4, 4, D, 2, 0.5, seed=D, dtype="f32")
 
 
 def test_zero_budget(wz):
