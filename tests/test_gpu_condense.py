@@ -267,6 +267,26 @@ def test_batch_parity(wz):
         compare_condense(sub, ref, Xv.dtype)
 
 
+def test_batch_of_many_small_videos(wz):
+    """130 videos in one call (several hundred frames, more videos than the
+    prefix blocks of a warp): every video's budgets, index map and tokens."""
+    g = np.random.default_rng(9)
+    V, T, H, W, D = 130, 5, 5, 6, 64
+    Lqs = [int(x) for x in g.integers(1, 9, size=V)]
+    ratios = [float(x) for x in g.choice([0.1, 0.3, 0.7], size=V)]
+    vids = [accepted_random(T, H, W, D, lq, r, seed=5000 + 13 * v) for v, (lq, r) in enumerate(zip(Lqs, ratios))]
+    X = torch.stack([x for x, _ in vids])
+    Qs = torch.cat([q for _, q in vids])
+    out = wz.wz_condense_batch(X.cuda(), Qs.cuda(), Lqs, ratios)
+    torch.cuda.synchronize()
+    offs = out["row_offsets"]
+    for v, ((Xv, Qv), r) in enumerate(zip(vids, ratios)):
+        ref = oracle_run(Xv, Qv, r)
+        sub = {"budgets": out["budgets"][v], "count": out["count"][v:v + 1],
+               "index": out["index"][offs[v]:offs[v + 1]], "tokens": out["tokens"][offs[v]:offs[v + 1]]}
+        compare_condense(sub, ref, Xv.dtype)
+
+
 def test_config_serving_batch_sampled(wz):
     """The serving batch at full size (32 videos x 64 frames, 13x13x3584 bf16,
     Lq in [8, 128], ratios in {0.05, 0.1, 0.25}) in one call: every video's
