@@ -13,14 +13,19 @@
 //   W_m[(p,q),(i,j)] = sum_v sum_b Q_v[q,b] A'_v[b,j] Y_v[b,i],
 //   Y_v[b,i]         = sum_u sum_a P_u[p,a] A_u[a,i] g_uv[a,b].
 //
-// S CTAs per frame: each builds the frame's tables once (saliency map,
-// gate, analysis matrices, width rows Q_v) and then the rows of W_m for the
-// grid rows p = s, s + S, ... in fp32 (each thread owns one output token q
-// and input column j and sums only over the b where both Q_v[q, b] and
-// A'_v[b, j] are nonzero, and only over the rows i that Y_v reaches), stages
-// them in shared memory and writes them as bf16 hi/lo pairs (tensor-core
-// path) or fp32 (CUDA-core path) in 16-byte groups, with the index map rows.
-// Trailing CTAs fill rows that cannot be produced with -1 / zeros.
+// spatial_wsm_kernel is persistent: each CTA copies the frame-independent
+// tables (analysis matrices with their column supports) once and then pulls
+// (frame, grid row) candidates from a global counter; a new frame reloads
+// its gate and the width rows Q_v.  Per grid row: P_u A_u, then Y_v, then
+// one warp per output token q with lane = input row i, which keeps
+// c_v[b] = Q_v[q,b] Y_v[b,i] for the few b of the column's support in
+// registers and forms row i of the token's operator row four columns at a
+// time from broadcast reads of A'_v.  Rows are staged in shared memory and
+// leave as 512-byte coalesced warp stores of bf16 hi/lo halves in the tiled
+// operator layout (tensor-core path) or as fp32 rows (CUDA-core path), with
+// the index map rows.  The ablation modes without the WSM use
+// spatial_plain_kernel (S CTAs per frame).  CTAs with a low index also fill
+// the rows that cannot be produced (tau > 0) with -1 / zeros.
 #include <algorithm>
 #include <cmath>
 

@@ -6,11 +6,11 @@
 //   W_m[(p,q),(i,j)] = sum_l sum_v sum_b Q_v^l[q,b] AW_v^l[b,j] Y_v^l[b,i],
 //   Y_v^l[b,i]       = sum_u sum_a P_u^l[p,a] AH_u^l[a,i] g_uv^l[a,b],
 //
-// with g_LL = 1 only at the deepest level.  The CTA organisation follows the
-// single-level kernel: S CTAs per frame take the grid rows p = s0, s0 + S, ...;
-// per row every level's Y goes to shared memory, then each thread owns one
-// (output token q, input column j) and sums all levels into the H rows it
-// keeps in registers, over the b where both Q^l and AW^l are nonzero.
+// with g_LL = 1 only at the deepest level.  S CTAs per frame take the grid
+// rows p = s0, s0 + S, ...; per row every level's Y goes to shared memory,
+// then each thread owns one (output token q, input column j) and sums all
+// levels into the H rows it keeps in registers (HMAX >= H), over the b where
+// both Q^l and AW^l are nonzero.
 #include <cmath>
 
 #include "wz_spatial.cuh"
