@@ -93,6 +93,15 @@ def test_maxsim_with_ablation_and_simt(wz):
     compare_condense(out, ref, X.dtype)
 
 
+def test_maxsim_with_levels(wz):
+    kw = dict(wta_levels=2, wsm_levels=2, wsm_wavelet=2)
+    X, Q = accepted_random(8, 11, 12, 128, 9, 0.3, seed=17, relevance="maxsim", **kw)
+    ref = oracle_run(X, Q, 0.3, relevance="maxsim", **kw)
+    out = _run(wz, X, Q, 0.3, **kw)
+    compare_condense(out, ref, X.dtype)
+    _check_r(out, ref)
+
+
 def test_maxsim_batch(wz):
     # videos of 1, 20 and 128 query rows share one buffer of query rows in turn
     T, H, W, D = 16, 9, 9, 128
