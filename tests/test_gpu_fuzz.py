@@ -55,3 +55,34 @@ def test_fuzz_parity(wz, k):
     out = wz.wz_condense_ex(X.cuda(), Q.cuda(), ratio, **kw)
     torch.cuda.synchronize()
     compare_condense(out, ref, X.dtype)
+
+
+def draw_batch(k: int):
+    g = np.random.default_rng(9000 + k)
+    V = int(g.integers(2, 7))
+    T = int(g.choice([1, 3, 8, 20]))
+    H, W = int(g.integers(1, 20)), int(g.integers(1, 20))
+    relevance = str(g.choice(["mean", "maxsim"]))
+    D = int(g.choice([64, 128])) if relevance == "maxsim" else int(8 * g.integers(1, 30))
+    kw = dict(wta_wavelet=int(g.choice([1, 4])), wsm_wavelet=int(g.choice([1, 4, 44])),
+              temporal_mode=str(g.choice(["wta", "raw"])), spatial_mode=str(g.choice(["wsm", "saliency"])),
+              wta_levels=int(g.choice([1, 2])), wsm_levels=int(g.choice([1, 2])), relevance=relevance)
+    Lqs = [int(x) for x in g.integers(1, 12, size=V)]
+    ratios = [float(x) for x in g.choice([0.05, 0.2, 0.6], size=V)]
+    return V, T, H, W, D, kw, Lqs, ratios
+
+
+@pytest.mark.parametrize("k", range(12))
+def test_fuzz_batch_parity(wz, k):
+    V, T, H, W, D, kw, Lqs, ratios = draw_batch(k)
+    vids = [accepted_random(T, H, W, D, lq, r, seed=k * 1000 + v, **kw) for v, (lq, r) in enumerate(zip(Lqs, ratios))]
+    X = torch.stack([x for x, _ in vids])
+    Qs = torch.cat([q for _, q in vids])
+    out = wz.wz_condense_batch(X.cuda(), Qs.cuda(), Lqs, ratios, **kw)
+    torch.cuda.synchronize()
+    offs = out["row_offsets"]
+    for v, ((Xv, Qv), r) in enumerate(zip(vids, ratios)):
+        ref = oracle_run(Xv, Qv, r, **kw)
+        sub = {"budgets": out["budgets"][v], "count": out["count"][v:v + 1],
+               "index": out["index"][offs[v]:offs[v + 1]], "tokens": out["tokens"][offs[v]:offs[v + 1]]}
+        compare_condense(sub, ref, Xv.dtype)
