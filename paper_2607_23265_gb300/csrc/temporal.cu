@@ -109,7 +109,11 @@ __device__ __forceinline__ int grid_h(int n, int H, int W) {
 
 // Shared-memory arrays of one video, indexed by retained frame m (wgt,
 // keys, lst, nb) or by frame t (nf).
-__host__ __device__ inline size_t temporal_smem_offset_coef(int T) { return ((size_t)T * (8 + 8 + 4 + 4 + 4) + 7) & ~(size_t)7; }
+// keys start on a 16-byte boundary (the rank reads them two at a time)
+__host__ __device__ inline size_t temporal_smem_keys(int T) { return ((size_t)T * 8 + 15) & ~(size_t)15; }
+__host__ __device__ inline size_t temporal_smem_offset_coef(int T) {
+    return (temporal_smem_keys(T) + (size_t)T * (8 + 4 + 4 + 4) + 7) & ~(size_t)7;
+}
 // WTA coefficient arrays: the longest subband of any level (any filter).
 __host__ __device__ inline int temporal_coef_len(int T, int J) {
     const int k = (T + kMaxTaps - 1) / 2;
@@ -213,7 +217,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     const VideoPar vp = c.vpar[v];
     double *fr = c.fr + base * 4;          // r, delta, gamma, r~
     double *wgt = reinterpret_cast<double *>(tsm);                        // weight of retained frame m
-    unsigned long long *keys = reinterpret_cast<unsigned long long *>(wgt + T);   // quota / remainder key
+    unsigned long long *keys = reinterpret_cast<unsigned long long *>(tsm + temporal_smem_keys(T));   // remainder key
     int *lst = reinterpret_cast<int *>(keys + T);                         // retained frames
     int *nb = lst + T;                     // budget of retained frame m; -1 while active
     int *nf = nb + T;                      // budget of frame t
@@ -366,27 +370,23 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
                     nb[m] = (int)floor((double)remaining * w / S);
                 }
             const long long R = remaining - fsum;
+            const ulonglong2 *k2 = reinterpret_cast<const ulonglong2 *>(keys);
             for (int m = threadIdx.x; m < L; m += blockDim.x) {
                 const unsigned long long km = keys[m];
-                if (km == 0ull) continue;
-                // rank = #{k : key_k > key_m, or key_k == key_m and k < m}
-                int r0 = 0, r1 = 0, r2 = 0, r3 = 0;
-                int k = 0;
-                for (; k + 4 <= m; k += 4) {   // k < m: ties count
-                    r0 += keys[k] >= km;
-                    r1 += keys[k + 1] >= km;
-                    r2 += keys[k + 2] >= km;
-                    r3 += keys[k + 3] >= km;
+                // rank = #{k : key_k > key_m, or key_k == key_m and k < m}; the
+                // same loop in every lane: broadcast 16-byte reads of two keys
+                int r0 = 0, r1 = 0;
+#pragma unroll 4
+                for (int i = 0; i < (L >> 1); ++i) {
+                    const ulonglong2 p = k2[i];
+                    r0 += (p.x > km) | ((p.x == km) & (2 * i < m));
+                    r1 += (p.y > km) | ((p.y == km) & (2 * i + 1 < m));
                 }
-                for (; k < m; ++k) r0 += keys[k] >= km;
-                for (k = m + 1; k + 4 <= L; k += 4) {   // k > m: ties do not count
-                    r0 += keys[k] > km;
-                    r1 += keys[k + 1] > km;
-                    r2 += keys[k + 2] > km;
-                    r3 += keys[k + 3] > km;
+                if (L & 1) {
+                    const unsigned long long p = keys[L - 1];
+                    r0 += (p > km) | ((p == km) & (L - 1 < m));
                 }
-                for (; k < L; ++k) r0 += keys[k] > km;
-                if (r0 + r1 + r2 + r3 < R) nb[m] += 1;
+                if (km != 0ull && r0 + r1 < R) nb[m] += 1;
             }
             __syncthreads();
             break;
