@@ -400,6 +400,10 @@ WZ_API int wz_version(void);
  * launch error, else WZ_OK (asynchronous on `stream`).
  */
 #define WZ_STATUS_WAIT_TIMEOUT 0x100
+/* Set only by the bounds-checked build of the library (libwavezip_checked.so,
+ * compiled with WZ_CHECKED): a kernel computed an out-of-range index for a
+ * global write and skipped the write. */
+#define WZ_STATUS_BOUNDS 0x200
 WZ_API int wz_selftest_bounded_wait(uint64_t timeout_ns, int32_t *device_status, wz_stream_t stream);
 
 #ifdef __cplusplus

@@ -1,7 +1,10 @@
 """Build libwavezip.so in-tree with nvcc for sm_103a (no torch extension).
 
 Each CUDA source compiles in parallel to an object file under _build/, then
-one shared library is linked next to this file.  Run as
+one shared library is linked next to this file.  The checked variant
+(libwavezip_checked.so, objects under _build_checked/) is the same sources
+with WZ_CHECKED defined: the kernels' global writes test their index and
+record WZ_STATUS_BOUNDS instead of writing out of range.  Run as
 ``python -m paper_2607_23265_gb300.build`` or through ``__graft_entry__.build()``.
 """
 
@@ -17,6 +20,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libwavezip.so")
+BUILD_CHECKED = os.path.join(HERE, "_build_checked")
+LIB_CHECKED = os.path.join(HERE, "libwavezip_checked.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-I", os.path.join(HERE, "..", "include")]
@@ -33,9 +38,9 @@ def sources():
     return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cu"))
 
 
-def _compile(src: str, verbose: bool) -> str:
-    obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
-    cmd = [nvcc(), *ARCH, *FLAGS, "-c", src, "-o", obj]
+def _compile(src: str, verbose: bool, checked: bool = False) -> str:
+    obj = os.path.join(BUILD_CHECKED if checked else BUILD, os.path.basename(src)[:-3] + ".o")
+    cmd = [nvcc(), *ARCH, *FLAGS, *(["-DWZ_CHECKED"] if checked else []), "-c", src, "-o", obj]
     if verbose:
         cmd.insert(1, "-Xptxas=-v")
     res = subprocess.run(cmd, capture_output=True, text=True)
@@ -46,24 +51,35 @@ def _compile(src: str, verbose: bool) -> str:
     return obj
 
 
-def build(verbose: bool = False, force: bool = False) -> str:
-    """Compile every .cu under csrc/ and link libwavezip.so; returns its path."""
-    os.makedirs(BUILD, exist_ok=True)
+def build(verbose: bool = False, force: bool = False, checked: bool = False) -> str:
+    """Compile every .cu under csrc/ and link libwavezip.so (or, checked, the
+    bounds-checked libwavezip_checked.so); returns its path."""
+    out_dir, lib = (BUILD_CHECKED, LIB_CHECKED) if checked else (BUILD, LIB)
+    os.makedirs(out_dir, exist_ok=True)
     srcs = sources()
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cuh")]
     newest = max(os.path.getmtime(p) for p in srcs + headers + [os.path.join(HERE, "..", "include", "wavezip.h")])
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) > newest:
-        return LIB
+    if not force and os.path.exists(lib) and os.path.getmtime(lib) > newest:
+        return lib
     with cf.ThreadPoolExecutor(max_workers=min(len(srcs), os.cpu_count() or 4)) as pool:
-        objs = list(pool.map(lambda s: _compile(s, verbose), srcs))
-    tmp = LIB + ".tmp"
+        objs = list(pool.map(lambda s: _compile(s, verbose, checked), srcs))
+    tmp = lib + ".tmp"
     cmd = [nvcc(), *ARCH, "-shared", "-o", tmp, *objs, "-cudart", "shared"]
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
+
+
+def build_all(verbose: bool = False, force: bool = False) -> str:
+    """Both libraries, compiled side by side; returns the main library's path."""
+    with cf.ThreadPoolExecutor(max_workers=2) as pool:
+        main = pool.submit(build, verbose, force, False)
+        chk = pool.submit(build, verbose, force, True)
+        chk.result()
+        return main.result()
 
 
 if __name__ == "__main__":
-    print(build(verbose="-v" in sys.argv, force="-f" in sys.argv))
+    print(build_all(verbose="-v" in sys.argv, force="-f" in sys.argv))

@@ -54,7 +54,7 @@ __global__ void __launch_bounds__(256) condense_simt_kernel(Ctx c) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int r = r0 + ty * 4 + i;
-        if (r >= n) continue;
+        if (r >= n || !wz_in_range(c.status, (int64_t)orow + r < c.rows_total)) continue;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int ch = c0 + tx * 4 + j;

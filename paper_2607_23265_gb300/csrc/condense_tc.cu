@@ -348,7 +348,8 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
                     for (int r = 0; r < 4; ++r) {
                         const int t = r * 8 + (lane >> 2);
                         const int cc = (lane & 3) * 8;
-                        if (j0 + t < un.nc && ch0 + cc < c.D) {
+                        if (j0 + t < un.nc && ch0 + cc < c.D &&
+                            wz_in_range(c.status, (int64_t)(row0 + j0 + t) < c.rows_total)) {
                             const uint4 val = ptx::lds128(tr32 + (uint32_t)(t * 64 + cc * 2));
                             *reinterpret_cast<uint4 *>(out + (row0 + j0 + t) * rowb + (size_t)(ch0 + cc) * 2) = val;
                         }

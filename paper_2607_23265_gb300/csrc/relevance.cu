@@ -354,7 +354,8 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
         pos += n;
         wcount += nt;
         const bool frame_done = pos == c.N || tok >= end;
-        if (frame_done && !dead) {
+        if (frame_done && !dead &&
+            wz_in_range(c.status, (int64_t)blockIdx.x + (int64_t)f < (int64_t)c.G1 + (int64_t)c.V * c.T)) {
             // column partial of frame f from this CTA: slot blockIdx.x + f
             float *dst = c.part + ((size_t)blockIdx.x + (size_t)f) * c.D;
 #pragma unroll
@@ -389,6 +390,7 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
         if (tok >= end || wcount + CH > WIN || new_video) {
             consumer_sync();
             if (abort_flag) break;
+            if (!wz_in_range(c.status, wbase + wcount <= total)) wcount = 0;
             for (int t = threadIdx.x; t < wcount; t += NC) {
                 float dot = 0.f, nrm = 0.f;
                 for (int w = 0; w < nw; ++w) {
@@ -457,6 +459,7 @@ __device__ void frame_gate(const Ctx &c, int64_t f, float *red, const float (&av
     __syncthreads();
     for (int l = 1; l <= c.wsm_levels; ++l) {
         const int hp = c.lvl_h[l], wp = c.lvl_w[l];
+        if (!wz_in_range(c.status, c.goff[l - 1] + hp * wp <= c.gate_stride)) break;
         float *G = c.gate + f * (int64_t)c.gate_stride + c.goff[l - 1];
         for (int k = threadIdx.x; k < hp * wp; k += blockDim.x) {
             const int ai = k / wp, bj = k % wp;

@@ -103,9 +103,10 @@ __device__ void plain_operator_rows(const Ctx &c, const SpatialSmem &L, float *s
                     }
             }
             __syncthreads();
-            write_rows(stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
+            write_rows(c, stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
         }
         for (int q = tid; q < nq; q += blockDim.x) {
+            if (!wz_in_range(c.status, row0 + q < c.rows_total)) break;
             int *o = c.out_index + (size_t)(row0 + q) * 3;
             o[0] = t;
             o[1] = pi;
@@ -329,10 +330,11 @@ __global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c) 
             for (int ql_ = warp; ql_ < qn; ql_ += nwarp)   // padding columns [N, K_pad)
                 for (int j = N + lane; j < K_pad; j += 32) stg[ql_ * L.KS + j] = 0.f;
             __syncthreads();
-            write_rows(stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
+            write_rows(c, stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
             if (q0 + L.QB < nq) __syncthreads();
         }
         for (int q = tid; q < nq; q += blockDim.x) {
+            if (!wz_in_range(c.status, row0 + q < c.rows_total)) break;
             int *o = c.out_index + (size_t)(row0 + q) * 3;
             o[0] = t;
             o[1] = pi;

@@ -97,6 +97,20 @@ struct Ctx {
 
 // ---- device helpers -------------------------------------------------------
 
+// Index checks of the bounds-checked build (WZ_CHECKED): a write whose index
+// is out of range records WZ_STATUS_BOUNDS in the status word and is skipped.
+// In the normal build the check is a constant true and costs nothing.
+__device__ __forceinline__ bool wz_in_range(const int *status, bool ok) {
+#ifdef WZ_CHECKED
+    if (!ok) atomicOr(const_cast<int *>(status), WZ_STATUS_BOUNDS);
+    return ok;
+#else
+    (void)status;
+    (void)ok;
+    return true;
+#endif
+}
+
 // ---- programmatic dependent launch ---------------------------------------
 // Each kernel of the pass waits for the grid before it in the stream before it
 // touches global memory and then lets the next grid be scheduled, so launch

@@ -96,8 +96,10 @@ __device__ __forceinline__ void synth_support(int y0, int y1, int F, int na, int
 // quarter, row within the group), so its 32 16-byte stores fill one
 // contiguous 512-byte block of the tiled layout.  A stride ks = K_pad + 4
 // keeps the eight rows' shared-memory reads on distinct banks.
-__device__ __forceinline__ void write_rows(const float *stg, int ks, int qn, int K_pad, int64_t r_first, bool bf,
-                                           __nv_bfloat16 *Whi, __nv_bfloat16 *Wlo, float *W32, size_t kstride) {
+__device__ __forceinline__ void write_rows(const Ctx &c, const float *stg, int ks, int qn, int K_pad, int64_t r_first,
+                                           bool bf, __nv_bfloat16 *Whi, __nv_bfloat16 *Wlo, float *W32, size_t kstride) {
+    // operator rows that exist: w_rows (tensor path), rows_total (fp32 rows)
+    if (!wz_in_range(c.status, r_first + qn <= (bf ? c.w_rows : c.rows_total))) return;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = (int)(blockDim.x >> 5);
     if (bf) {
         const int rr = lane & 7, qq = lane >> 3;

@@ -9,6 +9,7 @@ implementation to fall back to, and importing fails if the library is absent.
 
 from __future__ import annotations
 
+import contextlib
 import ctypes as C
 import os
 
@@ -16,6 +17,7 @@ import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libwavezip.so")
+LIB_CHECKED_PATH = os.path.join(_HERE, "libwavezip_checked.so")   # bounds-checked build (WZ_CHECKED)
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_NO_MEMORY, ERR_WORKSPACE = 0, -1, -2, -3, -4, -5
 DTYPE_BF16, DTYPE_F32 = 0, 1
@@ -93,11 +95,11 @@ NUM_KERNELS = 6
 KERNEL_NAMES = ("query_pool", "relevance", "frame_stats", "temporal", "spatial", "condense")
 
 
-def _load():
-    if not os.path.exists(LIB_PATH):
-        raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2607_23265_gb300.build` "
+def _load(path: str = LIB_PATH):
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it with `python -m paper_2607_23265_gb300.build` "
                           "(the WaveZip path has no non-CUDA implementation)")
-    lib = C.CDLL(LIB_PATH)
+    lib = C.CDLL(path)
     vp, i, f, sz, i64 = C.c_void_p, C.c_int, C.c_float, C.c_size_t, C.c_int64
     sig = {
         "wz_budget_size": (i64, [i, i, i, f]),
@@ -415,6 +417,22 @@ def wz_version() -> int:
 
 
 STATUS_WAIT_TIMEOUT = 0x100
+STATUS_BOUNDS = 0x200
+
+
+@contextlib.contextmanager
+def checked_library():
+    """Route this module's calls to the bounds-checked build of the library
+    (libwavezip_checked.so) while the block runs: the same kernels, whose
+    global writes check their index and set STATUS_BOUNDS instead of writing
+    out of range."""
+    global _lib
+    saved = _lib
+    _lib = _load(LIB_CHECKED_PATH)
+    try:
+        yield
+    finally:
+        _lib = saved
 
 
 def wz_selftest_bounded_wait(timeout_ns: int, device_status: torch.Tensor | None = None, stream=None) -> torch.Tensor:
