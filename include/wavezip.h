@@ -61,7 +61,7 @@ typedef struct CUstream_st *wz_stream_t;
 /* Status codes. */
 #define WZ_OK               0
 #define WZ_ERR_INVALID_ARG  (-1) /* null pointer, bad size, bad enum          */
-#define WZ_ERR_UNSUPPORTED  (-2) /* valid but outside this build's limits     */
+#define WZ_ERR_UNSUPPORTED  (-2) /* valid but outside the library's limits   */
 #define WZ_ERR_CUDA         (-3) /* a CUDA runtime/driver call failed         */
 #define WZ_ERR_NO_MEMORY    (-4) /* cudaMallocAsync of the workspace failed   */
 #define WZ_ERR_WORKSPACE    (-5) /* caller's workspace smaller than required  */
@@ -119,7 +119,7 @@ typedef struct CUstream_st *wz_stream_t;
 #define WZ_WAVELET_DB4    4
 #define WZ_WAVELET_BIOR44 44
 
-/* Limits of this build (WZ_ERR_UNSUPPORTED beyond them). */
+/* Limits of the library (WZ_ERR_UNSUPPORTED beyond them). */
 #define WZ_MAX_HW      64    /* H, W <= 64                                  */
 #define WZ_MAX_T       4096  /* frames per video                            */
 #define WZ_MAX_VIDEOS  1024  /* videos per batch call                       */

@@ -700,7 +700,7 @@ const char *wz_status_string(int status) {
     switch (status) {
         case WZ_OK: return "ok";
         case WZ_ERR_INVALID_ARG: return "invalid argument";
-        case WZ_ERR_UNSUPPORTED: return "unsupported by this build";
+        case WZ_ERR_UNSUPPORTED: return "unsupported: beyond the library's limits";
         case WZ_ERR_CUDA: return "CUDA error";
         case WZ_ERR_NO_MEMORY: return "workspace allocation failed";
         case WZ_ERR_WORKSPACE: return "workspace too small";
