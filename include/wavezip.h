@@ -202,6 +202,20 @@ WZ_API size_t wz_condense_workspace_size(int T, int H, int W, int D, int dtype, 
 WZ_API int wz_condense_ex(const wz_condense_args *a);
 
 /*
+ * wz_condense_ex with the features, the query and the outputs in HOST memory
+ * (pinned for asynchronous copies; pageable works, with the copies staged by
+ * the driver): the call allocates device staging on `stream`
+ * (cudaMallocAsync), copies the inputs in, runs the pass, copies out_tokens,
+ * out_index and whichever of out_budgets / out_count / out_relevance are
+ * non-NULL back, and frees the staging, all ordered on `stream`.  The host
+ * buffers must stay valid until the stream reaches the end of the call.
+ * token_scores, frame_scores and kernel_events must be NULL (they are device
+ * inputs); workspace and device_status are ignored.  Returns WZ_ERR_NO_MEMORY
+ * when the staging cannot be allocated.
+ */
+WZ_API int wz_condense_host(const wz_condense_args *a);
+
+/*
  * Serving batch: V independent videos of equal T, H, W, D in one launch
  * sequence (the paper processes one video per request; a batch is V such
  * requests).  Per-video query lengths and keep ratios.

@@ -494,6 +494,61 @@ int wz_condense_ex(const wz_condense_args *a) {
     return run_condense(r);
 }
 
+int wz_condense_host(const wz_condense_args *a) {
+    if (!a || !a->features || !a->query || !a->out_tokens || !a->out_index) return WZ_ERR_INVALID_ARG;
+    if (a->token_scores || a->frame_scores || a->kernel_events) return WZ_ERR_INVALID_ARG;   // device-only inputs
+    int st = check_sizes(1, a->T, a->H, a->W, a->D, a->dtype);
+    if (st != WZ_OK) return st;
+    if (a->Lq < 1 || !valid_ratio(a->ratio)) return WZ_ERR_INVALID_ARG;
+    const int64_t B = budget(a->T, a->H * a->W, a->ratio);
+    const size_t esz = a->dtype == WZ_DTYPE_BF16 ? 2 : 4;
+    const size_t xb = (size_t)a->T * a->H * a->W * a->D * esz, qb = (size_t)a->Lq * a->D * esz;
+    const size_t tb = (size_t)B * a->D * esz, ib = (size_t)B * 3 * 4, bb = (size_t)a->T * 4, rb = (size_t)a->T * 16;
+    cudaStream_t s = (cudaStream_t)a->stream;
+    // device staging: features, query, the outputs, count and status, one allocation
+    size_t o = 0;
+    auto take = [&](size_t n) {
+        const size_t at = o;
+        o = align_up(o + n);
+        return at;
+    };
+    const size_t ox = take(xb), oq = take(qb), ot = take(tb), oi = take(ib), obu = take(bb), orl = take(rb),
+                 oc = take(16);
+    char *dev = nullptr;
+    if (cudaMallocAsync(reinterpret_cast<void **>(&dev), o, s) != cudaSuccess) {
+        cudaGetLastError();
+        return WZ_ERR_NO_MEMORY;
+    }
+    wz_condense_args d = *a;
+    d.features = dev + ox;
+    d.query = dev + oq;
+    d.out_tokens = dev + ot;
+    d.out_index = reinterpret_cast<int32_t *>(dev + oi);
+    d.out_budgets = a->out_budgets ? reinterpret_cast<int32_t *>(dev + obu) : nullptr;
+    d.out_relevance = a->out_relevance ? reinterpret_cast<float *>(dev + orl) : nullptr;
+    d.out_count = a->out_count ? reinterpret_cast<int32_t *>(dev + oc) : nullptr;
+    d.device_status = nullptr;
+    d.workspace = nullptr;   // staging and workspace both from the stream-ordered allocator
+    d.workspace_bytes = 0;
+    st = WZ_OK;
+    if (cudaMemcpyAsync(dev + ox, a->features, xb, cudaMemcpyHostToDevice, s) != cudaSuccess ||
+        cudaMemcpyAsync(dev + oq, a->query, qb, cudaMemcpyHostToDevice, s) != cudaSuccess)
+        st = WZ_ERR_CUDA;
+    if (st == WZ_OK) st = wz_condense_ex(&d);
+    if (st == WZ_OK) {
+        if (cudaMemcpyAsync(a->out_tokens, dev + ot, tb, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+            cudaMemcpyAsync(a->out_index, dev + oi, ib, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+            (a->out_budgets && cudaMemcpyAsync(a->out_budgets, dev + obu, bb, cudaMemcpyDeviceToHost, s) != cudaSuccess) ||
+            (a->out_relevance &&
+             cudaMemcpyAsync(a->out_relevance, dev + orl, rb, cudaMemcpyDeviceToHost, s) != cudaSuccess) ||
+            (a->out_count && cudaMemcpyAsync(a->out_count, dev + oc, 4, cudaMemcpyDeviceToHost, s) != cudaSuccess))
+            st = WZ_ERR_CUDA;
+    }
+    if (cudaFreeAsync(dev, s) != cudaSuccess && st == WZ_OK) st = WZ_ERR_CUDA;
+    if (st == WZ_ERR_CUDA) cudaGetLastError();
+    return st;
+}
+
 int wz_condense(const void *features, int T, int H, int W, int D, const void *query, int Lq,
                 float ratio, void *out_tokens, int32_t *out_index, wz_stream_t stream) {
     wz_condense_args a;

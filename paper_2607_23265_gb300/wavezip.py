@@ -107,6 +107,7 @@ def _load(path: str = LIB_PATH):
         "wz_condense_args_init": (None, [C.POINTER(CondenseArgs)]),
         "wz_condense_workspace_size": (sz, [i, i, i, i, i, f]),
         "wz_condense_ex": (i, [C.POINTER(CondenseArgs)]),
+        "wz_condense_host": (i, [C.POINTER(CondenseArgs)]),
         "wz_batch_args_init": (None, [C.POINTER(BatchArgs)]),
         "wz_batch_rows": (i64, [i, i, i, i, C.POINTER(C.c_float), C.POINTER(C.c_int64)]),
         "wz_batch_workspace_size": (sz, [i, i, i, i, i, i, C.POINTER(C.c_float)]),
@@ -254,6 +255,29 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
     a.stream = _stream(stream, dev)
     _check(_lib.wz_condense_ex(C.byref(a)), "wz_condense_ex")
     return {"tokens": tokens, "index": index, "budgets": budgets, "count": count, "relevance": rel}
+
+
+def wz_condense_host(features: torch.Tensor, query: torch.Tensor, ratio: float, out_tokens: torch.Tensor,
+                     out_index: torch.Tensor, *, lam: float = 1.5, tau: float = 0.0, wsm_wavelet: int = 4,
+                     wta_wavelet: int = 1, mode="symmetric", path="auto", relevance="mean", stream=None):
+    """wz_condense_host: features [T,H,W,D] and query [Lq,D] in (pinned) host memory, out_tokens [B,D]
+    and out_index [B,3] host tensors filled once the stream has run the call."""
+    for t, name in ((features, "features"), (query, "query"), (out_tokens, "out_tokens"), (out_index, "out_index")):
+        if t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous host tensor")
+    T, H, W, D = features.shape
+    a = CondenseArgs()
+    _lib.wz_condense_args_init(C.byref(a))
+    a.features, a.T, a.H, a.W, a.D = features.data_ptr(), T, H, W, D
+    a.dtype = _dtype_code(features)
+    a.query, a.Lq, a.ratio = query.data_ptr(), query.shape[0], ratio
+    a.lam, a.tau, a.wsm_wavelet, a.wta_wavelet = lam, tau, wsm_wavelet, wta_wavelet
+    a.mode = MODES[mode] if isinstance(mode, str) else int(mode)
+    a.path = PATHS[path] if isinstance(path, str) else int(path)
+    a.relevance_mode = _enum(RELEVANCE_MODES, relevance)
+    a.out_tokens, a.out_index = out_tokens.data_ptr(), out_index.data_ptr()
+    a.stream = _stream(stream, torch.device("cuda", torch.cuda.current_device()))
+    _check(_lib.wz_condense_host(C.byref(a)), "wz_condense_host")
 
 
 def wz_batch_rows(V, T, H, W, ratios):

@@ -336,3 +336,18 @@ def test_dwt_entry_points(wz, p, mode):
     Y = wz.wz_idwt2d(*bands, 13, 10, p)
     torch.cuda.synchronize()
     assert np.allclose(Y.cpu().numpy(), X.float().numpy(), atol=1e-4)
+
+
+def test_host_buffer_entry_point(wz):
+    """wz_condense_host on pinned host buffers equals the device call."""
+    X, Q = accepted_random(10, 13, 13, 128, 6, 0.2, seed=44)
+    B = wz.wz_budget_size(10, 13, 13, 0.2)
+    Xh, Qh = X.pin_memory(), Q.pin_memory()
+    tok = torch.empty((B, 128), dtype=torch.bfloat16).pin_memory()
+    idx = torch.empty((B, 3), dtype=torch.int32).pin_memory()
+    wz.wz_condense_host(Xh, Qh, 0.2, tok, idx)
+    torch.cuda.synchronize()
+    ref = run(wz, X, Q, 0.2)
+    assert torch.equal(tok, ref["tokens"].cpu()) and torch.equal(idx, ref["index"].cpu())
+    with pytest.raises(ValueError):
+        wz.wz_condense_host(X.cuda(), Qh, 0.2, tok, idx)
