@@ -103,7 +103,7 @@ __device__ void plain_operator_rows(const Ctx &c, const SpatialSmem &L, float *s
                     }
             }
             __syncthreads();
-            write_rows(c, stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
+            write_rows(c, stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride, 0, K_pad);
         }
         for (int q = tid; q < nq; q += blockDim.x) {
             if (!wz_in_range(c.status, row0 + q < c.rows_total)) break;
@@ -137,19 +137,68 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_plain_kernel(Ctx c, i
     plain_operator_rows(c, L, sm, f, s0, S, n, h, w);
 }
 
+// Grid rows of frame f that hold output tokens: p < h and p * w < n.
+__device__ __forceinline__ int frame_rows(const Ctx &c, int f) {
+    const int n = c.n[f];
+    if (n <= 0) return 0;
+    const int h = c.hw[2 * f], w = c.hw[2 * f + 1];
+    return min(h, (n + w - 1) / w);
+}
+
+// rowpre[f] = grid rows of the frames before f, rowpre[F] = all rows
+// (F <= kCompactFrames; block-wide scan, every thread a contiguous range).
+constexpr int kCompactFrames = 2048;
+__device__ void grid_row_prefix(const Ctx &c, int F, int *rowpre, int *wsum) {
+    constexpr int kPer = kCompactFrames / kSpatialThreads;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int per = (F + kSpatialThreads - 1) / kSpatialThreads;
+    const int f0 = tid * per;
+    int rows[kPer];
+    int sum = 0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+        rows[k] = (k < per && f0 + k < F) ? frame_rows(c, f0 + k) : 0;
+        sum += rows[k];
+    }
+    int incl = sum;
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    int run = incl - sum;
+    for (int w = 0; w < warp; ++w) run += wsum[w];
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+        if (k < per && f0 + k < F) rowpre[f0 + k] = run;
+        run += rows[k];
+    }
+    if (tid == 0) {
+        int tot = 0;
+        for (int w = 0; w < kSpatialThreads / 32; ++w) tot += wsum[w];
+        rowpre[F] = tot;
+    }
+}
+
 // The WSM operator rows (single level), persistent: every CTA copies the
 // frame-independent tables once, then takes grid rows (frame f, row p) from
-// a global counter over the V*T*H candidates until none is left; a row
-// whose frame changes reloads the frame's gate and width rows.  Rows of
-// frames with a small budget cost as much as others, so the dynamic order
-// keeps the SMs evenly loaded.
+// a global counter until none is left; a row whose frame changes reloads
+// the frame's gate and width rows.  Rows of frames with a small budget cost
+// as much as others, so the dynamic order keeps the SMs evenly loaded.  With
+// compact != 0 (at most kCompactFrames frames) every CTA first forms the
+// prefix of the frames' grid rows in shared memory and the counter runs over
+// the rows that exist; otherwise it runs over all V*T*H (frame, row) pairs.
 template <int BMAX>
-__global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c) {
+__global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c, int compact) {
     pdl_wait();
     pdl_trigger();
     extern __shared__ float sm[];
-    __shared__ int s_item;
+    __shared__ int s_item, s_f, s_wsum[kSpatialThreads / 32];
     const int tid = threadIdx.x;
+    // thread 0 claims the next row while the current one is formed, so the
+    // counter's round trip overlaps the work
+    int claimed = tid == 0 ? atomicAdd(c.spatial_next, 1) : 0;
     if ((int)blockIdx.x < kTailBlocks) tail_rows(c, (int)blockIdx.x);
     const int H = c.H, W = c.W, N = c.N, hp = c.hp, wp = c.wp, F = c.F;
     SpatialSmem L;
@@ -159,6 +208,8 @@ __global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c) 
     float *PAl = sm + L.PAl, *PAh = sm + L.PAh, *Yl = sm + L.Yl, *Yh = sm + L.Yh;
     float *Ql = sm + L.Ql, *Qh = sm + L.Qh, *red = sm + L.red;
     const int *jlo = reinterpret_cast<const int *>(sm + L.jlo), *jhi = reinterpret_cast<const int *>(sm + L.jhi);
+    const int *ilo = reinterpret_cast<const int *>(sm + L.ilo), *ihi = reinterpret_cast<const int *>(sm + L.ihi);
+    int *rowpre = reinterpret_cast<int *>(sm + L.total);   // compact: [V*T + 1]
     int *qlo = reinterpret_cast<int *>(sm + L.qlo), *qhi = reinterpret_cast<int *>(sm + L.qhi);
     float *stg = sm + L.stage;
     const int HP4 = L.HP4, WP4 = L.WP4;
@@ -191,16 +242,38 @@ __global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c) 
 
     // candidates (frame, grid row): f * H + p < V * T * H < 2^31, 32-bit
     // index arithmetic throughout (no 64-bit divisions in the loop)
-    const int items = c.V * c.T * H;
+    const int VT = c.V * c.T;
+    if (compact) {
+        grid_row_prefix(c, VT, rowpre, s_wsum);
+        __syncthreads();
+    }
+    const int items = compact ? rowpre[VT] : VT * H;
     int cur_f = -1;
     for (;;) {
         __syncthreads();   // the previous row's reads of shared memory
-        if (tid == 0) s_item = atomicAdd(c.spatial_next, 1);
+        if (tid == 0) {
+            const int it = claimed;
+            if (it < items) claimed = atomicAdd(c.spatial_next, 1);
+            int fi = 0;
+            if (compact && it < items) {
+                // the last frame whose first row is <= it (frames without
+                // rows share their successor's prefix)
+                int lo = 0, hi = VT - 1;
+                while (lo < hi) {
+                    const int mid = (lo + hi + 1) >> 1;
+                    if (rowpre[mid] <= it) lo = mid;
+                    else hi = mid - 1;
+                }
+                fi = lo;
+            }
+            s_item = it;
+            s_f = fi;
+        }
         __syncthreads();
         const int item = s_item;
         if (item >= items) break;
-        const int f = item / H;
-        const int pi = item - f * H;
+        const int f = compact ? s_f : item / H;
+        const int pi = compact ? item - rowpre[f] : item - f * H;
         const int n = c.n[f];
         if (n <= 0) continue;
         const int h = c.hw[2 * f], w = c.hw[2 * f + 1];
@@ -243,6 +316,11 @@ __global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c) 
         int alo, ahi;
         synth_support(y0, y1, F, hp, alo, ahi);
         const int na = ahi - alo + 1;
+        int zlo = H, zhi = -1;   // map rows the operator rows of this grid row reach
+        for (int a = alo; a <= ahi; ++a) {
+            zlo = min(zlo, ilo[a]);
+            zhi = max(zhi, ihi[a]);
+        }
         __syncthreads();   // previous row's Y / stage reads, the frame tables
         for (int u = warp; u < na; u += nwarp) {   // warp per coefficient row, lanes over i
             const int ai = alo + u;
@@ -254,83 +332,167 @@ __global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c) 
             }
         }
         __syncthreads();
-        // Y_v[b][i], rows padded to a multiple of 4 with zeros
-        for (int b = warp; b < wp; b += nwarp)   // warp per subband column b, lanes over i
-        for (int i = lane; i < HP4; i += 32) {
-            const int k = b * HP4 + i;
-            float yl = 0.f, yh = 0.f;
-            if (i < H) {
-                for (int u = 0; u < na; ++u) {
-                    const float g = G[(alo + u) * wp + b];
-                    const float pl = PAl[u * H + i], ph = PAh[u * H + i];
-                    yl += pl + ph * g;
-                    yh += (pl + ph) * g;
+        // Y_v[b][i], rows padded to a multiple of 4 with zeros; with at most
+        // 16 map rows reached (paired, below) only those rows, two columns b
+        // per warp
+        const int span = zhi - zlo + 1;
+        const bool paired = span <= 16 && H <= 32;
+        if (paired) {
+            const int r = lane & 15;
+            for (int b = 2 * warp + (lane >> 4); b < wp; b += 2 * nwarp) {
+                if (r < span) {
+                    const int i = zlo + r;
+                    float yl = 0.f, yh = 0.f;
+                    for (int u = 0; u < na; ++u) {
+                        const float g = G[(alo + u) * wp + b];
+                        const float pl = PAl[u * H + i], ph = PAh[u * H + i];
+                        yl += pl + ph * g;
+                        yh += (pl + ph) * g;
+                    }
+                    Yl[b * HP4 + i] = yl;
+                    Yh[b * HP4 + i] = yh;
                 }
             }
-            Yl[k] = yl;
-            Yh[k] = yh;
+        } else {
+            for (int b = warp; b < wp; b += nwarp)   // warp per subband column b, lanes over i
+            for (int i = lane; i < HP4; i += 32) {
+                const int k = b * HP4 + i;
+                float yl = 0.f, yh = 0.f;
+                if (i < H) {
+                    for (int u = 0; u < na; ++u) {
+                        const float g = G[(alo + u) * wp + b];
+                        const float pl = PAl[u * H + i], ph = PAh[u * H + i];
+                        yl += pl + ph * g;
+                        yh += (pl + ph) * g;
+                    }
+                }
+                Yl[k] = yl;
+                Yh[k] = yh;
+            }
         }
         __syncthreads();
         const int64_t row0 = (int64_t)c.off[f] + (int64_t)pi * w;                 // output row
         const int64_t wrow0 = bf ? (int64_t)c.woff[f] + (int64_t)pi * w : row0;   // operator row
-        // Rows are produced QB at a time.  One warp per (output token q,
-        // 32-row slice of the map), lane = input row i: the lane's
-        // coefficients c_v[b] = Q_v[q,b] Y_v[b,i] over the support of Q_v[q,.]
-        // (at most BMAX values, uniform over the warp) stay in registers; each
-        // 4-column group j of row i of the staged token q is then
+        // Rows are produced QB at a time.  The operator rows of this grid row
+        // reach the map rows [zlo, zhi] only (columns [zc_lo, zc_hi]); write_rows
+        // reads the staged columns [rc_lo, rc_hi) (the 32-column groups that
+        // meet them) and writes zeros elsewhere.  Lane = input row i: the
+        // lane's coefficients c_v[b] = Q_v[q,b] Y_v[b,i] over the support of
+        // Q_v[q,.] (at most BMAX values) stay in registers; each 4-column
+        // group j of row i of the staged token q is then
         // sum_b c_L[b] A'_L[b,j] + c_H[b] A'_H[b,j], with the analysis rows read
-        // as broadcast 16-byte words and only the groups the support reaches
-        // computed.  The staged rows go out in 8-column groups (write_rows).
+        // as 16-byte words and only the groups the support reaches computed.
+        // With at most 16 such rows a warp forms two tokens (a half-warp each,
+        // lanes over rows zlo + r), zeroing the read columns of their staged
+        // rows first; otherwise one warp per (token, 32-row slice of the map).
+        const int zc_lo = zlo * W, zc_hi = (zhi + 1) * W - 1;
+        const int rc_lo = span > 0 ? (zc_lo >> 5) << 5 : 0;
+        const int rc_hi = span > 0 ? min(K_pad, ((zc_hi >> 5) + 1) << 5) : 0;
         for (int q0 = 0; q0 < nq; q0 += L.QB) {
             const int qn = min(L.QB, nq - q0);
-            for (int item = warp; item < qn * IH; item += nwarp) {
-                const int ql_ = IH == 1 ? item : item / IH, i = (item - ql_ * IH) * 32 + lane;
-                const int q = q0 + ql_;
-                const bool live = i < H;
-                const int b0 = qlo[q], nb = min(qhi[q] - b0 + 1, BMAX);
-                float cl[BMAX], ch[BMAX];
-                int jl = WP4, jh = -1;
-#pragma unroll
-                for (int bb = 0; bb < BMAX; ++bb) {
-                    const int b = b0 + bb;
-                    const bool on = bb < nb;
-                    cl[bb] = on && live ? Ql[q * wp + b] * Yl[b * HP4 + i] : 0.f;
-                    ch[bb] = on && live ? Qh[q * wp + b] * Yh[b * HP4 + i] : 0.f;
-                    if (on) {
-                        jl = min(jl, jlo[b]);
-                        jh = max(jh, jhi[b]);
+            if (paired) {
+                const int half = lane >> 4, r = lane & 15;
+                for (int pr = warp; 2 * pr < qn; pr += nwarp) {
+                    const int ql_ = 2 * pr + half;
+                    const bool tok = ql_ < qn;
+                    if (tok) {
+                        float4 *z = reinterpret_cast<float4 *>(stg + ql_ * L.KS + rc_lo);
+                        for (int k = r; k < ((rc_hi - rc_lo) >> 2); k += 16) z[k] = make_float4(0.f, 0.f, 0.f, 0.f);
                     }
-                }
-                float *srow = stg + ql_ * L.KS + i * W;
-                const int j4lo = jl >> 2, j4hi = jh >> 2;   // empty when jh < 0
-                for (int j4 = 0; 4 * j4 < W; ++j4) {
-                    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                    if (j4 >= j4lo && j4 <= j4hi) {
+                    __syncwarp();
+                    const int q = q0 + (tok ? ql_ : 0);
+                    const bool live = tok && r < span;
+                    const int i = zlo + (live ? r : 0);
+                    const int b0 = qlo[q], nb = min(qhi[q] - b0 + 1, BMAX);
+                    float cl[BMAX], ch[BMAX];
+                    int jl = WP4, jh = -1;
 #pragma unroll
-                        for (int bb = 0; bb < BMAX; ++bb) {
-                            if (bb < nb) {
-                                const float4 a4 = reinterpret_cast<const float4 *>(AWl + (b0 + bb) * WP4)[j4];
-                                const float4 d4 = reinterpret_cast<const float4 *>(AWh + (b0 + bb) * WP4)[j4];
-                                acc.x = fmaf(cl[bb], a4.x, fmaf(ch[bb], d4.x, acc.x));
-                                acc.y = fmaf(cl[bb], a4.y, fmaf(ch[bb], d4.y, acc.y));
-                                acc.z = fmaf(cl[bb], a4.z, fmaf(ch[bb], d4.z, acc.z));
-                                acc.w = fmaf(cl[bb], a4.w, fmaf(ch[bb], d4.w, acc.w));
-                            }
+                    for (int bb = 0; bb < BMAX; ++bb) {
+                        const int b = b0 + bb;
+                        const bool on = bb < nb;
+                        cl[bb] = on && live ? Ql[q * wp + b] * Yl[b * HP4 + i] : 0.f;
+                        ch[bb] = on && live ? Qh[q * wp + b] * Yh[b * HP4 + i] : 0.f;
+                        if (on) {
+                            jl = min(jl, jlo[b]);
+                            jh = max(jh, jhi[b]);
                         }
                     }
-                    if (live) {
-                        const int j = 4 * j4;
-                        srow[j] = acc.x;
-                        if (j + 1 < W) srow[j + 1] = acc.y;
-                        if (j + 2 < W) srow[j + 2] = acc.z;
-                        if (j + 3 < W) srow[j + 3] = acc.w;
+                    float *srow = stg + ql_ * L.KS + i * W;
+                    const int j4lo = jl >> 2, j4hi = jh >> 2;   // empty when jh < 0
+                    for (int j4 = 0; 4 * j4 < W; ++j4) {
+                        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                        if (j4 >= j4lo && j4 <= j4hi) {
+#pragma unroll
+                            for (int bb = 0; bb < BMAX; ++bb) {
+                                if (bb < nb) {
+                                    const float4 a4 = reinterpret_cast<const float4 *>(AWl + (b0 + bb) * WP4)[j4];
+                                    const float4 d4 = reinterpret_cast<const float4 *>(AWh + (b0 + bb) * WP4)[j4];
+                                    acc.x = fmaf(cl[bb], a4.x, fmaf(ch[bb], d4.x, acc.x));
+                                    acc.y = fmaf(cl[bb], a4.y, fmaf(ch[bb], d4.y, acc.y));
+                                    acc.z = fmaf(cl[bb], a4.z, fmaf(ch[bb], d4.z, acc.z));
+                                    acc.w = fmaf(cl[bb], a4.w, fmaf(ch[bb], d4.w, acc.w));
+                                }
+                            }
+                        }
+                        if (live) {
+                            const int j = 4 * j4;
+                            srow[j] = acc.x;
+                            if (j + 1 < W) srow[j + 1] = acc.y;
+                            if (j + 2 < W) srow[j + 2] = acc.z;
+                            if (j + 3 < W) srow[j + 3] = acc.w;
+                        }
                     }
                 }
+            } else {
+                for (int item = warp; item < qn * IH; item += nwarp) {
+                    const int ql_ = IH == 1 ? item : item / IH, i = (item - ql_ * IH) * 32 + lane;
+                    const int q = q0 + ql_;
+                    const bool live = i < H;
+                    const int b0 = qlo[q], nb = min(qhi[q] - b0 + 1, BMAX);
+                    float cl[BMAX], ch[BMAX];
+                    int jl = WP4, jh = -1;
+#pragma unroll
+                    for (int bb = 0; bb < BMAX; ++bb) {
+                        const int b = b0 + bb;
+                        const bool on = bb < nb;
+                        cl[bb] = on && live ? Ql[q * wp + b] * Yl[b * HP4 + i] : 0.f;
+                        ch[bb] = on && live ? Qh[q * wp + b] * Yh[b * HP4 + i] : 0.f;
+                        if (on) {
+                            jl = min(jl, jlo[b]);
+                            jh = max(jh, jhi[b]);
+                        }
+                    }
+                    float *srow = stg + ql_ * L.KS + i * W;
+                    const int j4lo = jl >> 2, j4hi = jh >> 2;   // empty when jh < 0
+                    for (int j4 = 0; 4 * j4 < W; ++j4) {
+                        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                        if (j4 >= j4lo && j4 <= j4hi) {
+#pragma unroll
+                            for (int bb = 0; bb < BMAX; ++bb) {
+                                if (bb < nb) {
+                                    const float4 a4 = reinterpret_cast<const float4 *>(AWl + (b0 + bb) * WP4)[j4];
+                                    const float4 d4 = reinterpret_cast<const float4 *>(AWh + (b0 + bb) * WP4)[j4];
+                                    acc.x = fmaf(cl[bb], a4.x, fmaf(ch[bb], d4.x, acc.x));
+                                    acc.y = fmaf(cl[bb], a4.y, fmaf(ch[bb], d4.y, acc.y));
+                                    acc.z = fmaf(cl[bb], a4.z, fmaf(ch[bb], d4.z, acc.z));
+                                    acc.w = fmaf(cl[bb], a4.w, fmaf(ch[bb], d4.w, acc.w));
+                                }
+                            }
+                        }
+                        if (live) {
+                            const int j = 4 * j4;
+                            srow[j] = acc.x;
+                            if (j + 1 < W) srow[j + 1] = acc.y;
+                            if (j + 2 < W) srow[j + 2] = acc.z;
+                            if (j + 3 < W) srow[j + 3] = acc.w;
+                        }
+                    }
+                }
+                for (int ql_ = warp; ql_ < qn; ql_ += nwarp)   // padding columns [N, K_pad)
+                    for (int j = N + lane; j < K_pad; j += 32) stg[ql_ * L.KS + j] = 0.f;
             }
-            for (int ql_ = warp; ql_ < qn; ql_ += nwarp)   // padding columns [N, K_pad)
-                for (int j = N + lane; j < K_pad; j += 32) stg[ql_ * L.KS + j] = 0.f;
             __syncthreads();
-            write_rows(c, stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
+            write_rows(c, stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride, rc_lo, rc_hi - 1);
             if (q0 + L.QB < nq) __syncthreads();
         }
         for (int q = tid; q < nq; q += blockDim.x) {
@@ -347,6 +509,11 @@ size_t spatial_smem_bytes(const Ctx &c) {
     SpatialSmem L;
     L.init(c.H, c.W, c.hp, c.wp);
     return (size_t)L.total * sizeof(float);
+}
+
+// The WSM kernel's shared memory with the grid-row prefix of V*T frames.
+static size_t spatial_compact_smem_bytes(const Ctx &c) {
+    return (spatial_smem_bytes(c) + ((size_t)c.V * c.T + 1) * sizeof(int) + 15) & ~(size_t)15;
 }
 
 // CTAs per frame: about four waves over the SMs, at most one per grid row.
@@ -372,13 +539,20 @@ cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     else if ((c.F - 1) / 2 + 2 <= 6) fn = (const void *)spatial_wsm_kernel<6>;
     else if ((c.F - 1) / 2 + 2 <= 12) fn = (const void *)spatial_wsm_kernel<12>;
     else return cudaErrorInvalidValue;
-    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    // the compact row list when its prefix fits without costing a resident CTA
+    const size_t smem_c = spatial_compact_smem_bytes(c);
+    const size_t smem_max = plain || (int64_t)c.V * c.T > kCompactFrames ? smem : smem_c;
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max);
     if (e != cudaSuccess) return e;
-    int dev = 0, sms = 0, per_sm = 0;
+    int dev = 0, sms = 0, per_sm = 0, per_sm_c = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
     if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kSpatialThreads, smem)) != cudaSuccess)
         return e;
+    if (smem_max > smem &&
+        (e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_c, fn, kSpatialThreads, smem_c)) != cudaSuccess)
+        return e;
+    int compact = smem_max > smem && per_sm_c >= per_sm ? 1 : 0;
     const int resident = sms * (per_sm > 0 ? per_sm : 1);
     if (plain) {
         int S = spatial_split(c, resident);
@@ -389,8 +563,8 @@ cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     // persistent: every resident CTA pulls grid rows; at least kTailBlocks
     // CTAs so that the tail rows are covered
     const unsigned blocks = (unsigned)std::max(resident, kTailBlocks);
-    void *args[] = {const_cast<Ctx *>(&c)};
-    return launch_kernel(fn, dim3(blocks), dim3(kSpatialThreads), smem, s, args, c.pdl != 0);
+    void *args[] = {const_cast<Ctx *>(&c), &compact};
+    return launch_kernel(fn, dim3(blocks), dim3(kSpatialThreads), compact ? smem_c : smem, s, args, c.pdl != 0);
 }
 
 }  // namespace wz

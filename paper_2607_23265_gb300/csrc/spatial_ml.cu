@@ -206,7 +206,7 @@ __global__ void __launch_bounds__(kSpatialThreads) spatial_ml_kernel(Ctx c, int 
             for (int k = tid; k < qn * (K_pad - N); k += blockDim.x)
                 stg[(k / (K_pad - N)) * L.KS + N + k % (K_pad - N)] = 0.f;
             __syncthreads();
-            write_rows(c, stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride);
+            write_rows(c, stg, L.KS, qn, K_pad, (bf ? wrow0 : row0) + q0, bf, Whi, Wlo, W32, kstride, 0, K_pad);
             if (q0 + L.QB < nq) __syncthreads();
         }
         for (int q = tid; q < nq; q += blockDim.x) {

@@ -16,8 +16,9 @@ struct SpatialSmem {
     int N, hp, wp, H, W, HP4, WP4, K_pad, KS, QB;
     // float offsets; [0, tables) is the frame-independent part.  The width
     // analysis rows A'_v[b][.] are padded to WP4 columns (16-byte rows);
-    // jlo / jhi[b] are the first / last column where A'_L or A'_H is nonzero.
-    int AHl, AHh, AWl, AWh, jlo, jhi, tables;
+    // jlo / jhi[b] are the first / last column where A'_L or A'_H is nonzero,
+    // ilo / ihi[a] the first / last row where A_L or A_H is nonzero.
+    int AHl, AHh, AWl, AWh, jlo, jhi, ilo, ihi, tables;
     int G, PAl, PAh, Yl, Yh, Ql, Qh, red, qlo, qhi, M, stage, total;
     // Every table starts on a 16-byte boundary (float4 reads of Y, staged rows).
     __host__ __device__ void init(int H_, int W_, int hp_, int wp_) {
@@ -39,6 +40,8 @@ struct SpatialSmem {
         AWh = take(wp * WP4);
         jlo = take(wp);
         jhi = take(wp);
+        ilo = take(hp);
+        ihi = take(hp);
         tables = o;
         G = take(hp * wp);
         PAl = take(hp * H);
@@ -95,9 +98,12 @@ __device__ __forceinline__ void synth_support(int y0, int y1, int F, int na, int
 // tensor path a warp writes one 8-row group x 32-column chunk: lane = (column
 // quarter, row within the group), so its 32 16-byte stores fill one
 // contiguous 512-byte block of the tiled layout.  A stride ks = K_pad + 4
-// keeps the eight rows' shared-memory reads on distinct banks.
+// keeps the eight rows' shared-memory reads on distinct banks.  Columns
+// outside [zc_lo, zc_hi] are zero in every staged row: a column group that
+// holds only such columns is written as zeros without reading the stage.
 __device__ __forceinline__ void write_rows(const Ctx &c, const float *stg, int ks, int qn, int K_pad, int64_t r_first,
-                                           bool bf, __nv_bfloat16 *Whi, __nv_bfloat16 *Wlo, float *W32, size_t kstride) {
+                                           bool bf, __nv_bfloat16 *Whi, __nv_bfloat16 *Wlo, float *W32, size_t kstride,
+                                           int zc_lo, int zc_hi) {
     // operator rows that exist: w_rows (tensor path), rows_total (fp32 rows)
     if (!wz_in_range(c.status, r_first + qn <= (bf ? c.w_rows : c.rows_total))) return;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = (int)(blockDim.x >> 5);
@@ -110,18 +116,20 @@ __device__ __forceinline__ void write_rows(const Ctx &c, const float *stg, int k
             const int64_t r = (rg0 + rgi) * 8 + rr;
             const int ql_ = (int)(r - r_first);
             if (ql_ < 0 || ql_ >= qn) continue;
-            const float *src = stg + ql_ * ks + 32 * g4 + 8 * qq;
-            const float4 v0 = *reinterpret_cast<const float4 *>(src);
-            const float4 v1 = *reinterpret_cast<const float4 *>(src + 4);
-            const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-            uint32_t hw[4], lw[4];
+            uint32_t hw[4] = {0u, 0u, 0u, 0u}, lw[4] = {0u, 0u, 0u, 0u};
+            if (32 * g4 + 31 >= zc_lo && 32 * g4 <= zc_hi) {
+                const float *src = stg + ql_ * ks + 32 * g4 + 8 * qq;
+                const float4 v0 = *reinterpret_cast<const float4 *>(src);
+                const float4 v1 = *reinterpret_cast<const float4 *>(src + 4);
+                const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
-                const __nv_bfloat162 ll =
-                    __floats2bfloat162_rn(v[2 * e] - __low2float(hh), v[2 * e + 1] - __high2float(hh));
-                hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
-                lw[e] = *reinterpret_cast<const uint32_t *>(&ll);
+                for (int e = 0; e < 4; ++e) {
+                    const __nv_bfloat162 hh = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+                    const __nv_bfloat162 ll =
+                        __floats2bfloat162_rn(v[2 * e] - __low2float(hh), v[2 * e + 1] - __high2float(hh));
+                    hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
+                    lw[e] = *reinterpret_cast<const uint32_t *>(&ll);
+                }
             }
             const size_t ti = (size_t)g4 * kstride + (size_t)(r >> 3) * 256 + (size_t)rr * 8 + (size_t)qq * 64;
             *reinterpret_cast<uint4 *>(Whi + ti) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
@@ -131,10 +139,15 @@ __device__ __forceinline__ void write_rows(const Ctx &c, const float *stg, int k
         const int G8 = K_pad / 8;
         for (int it = threadIdx.x; it < qn * G8; it += blockDim.x) {
             const int ql_ = it / G8, g = it - ql_ * G8;
-            const float *src = stg + ql_ * ks + 8 * g;
             float *dst = W32 + (size_t)(r_first + ql_) * K_pad + 8 * g;
-            *reinterpret_cast<float4 *>(dst) = *reinterpret_cast<const float4 *>(src);
-            *reinterpret_cast<float4 *>(dst + 4) = *reinterpret_cast<const float4 *>(src + 4);
+            float4 v0 = make_float4(0.f, 0.f, 0.f, 0.f), v1 = v0;
+            if (8 * g + 7 >= zc_lo && 8 * g <= zc_hi) {
+                const float *src = stg + ql_ * ks + 8 * g;
+                v0 = *reinterpret_cast<const float4 *>(src);
+                v1 = *reinterpret_cast<const float4 *>(src + 4);
+            }
+            *reinterpret_cast<float4 *>(dst) = v0;
+            *reinterpret_cast<float4 *>(dst + 4) = v1;
         }
     }
 }
@@ -187,14 +200,26 @@ inline size_t spatial_table_bytes(int H, int W, int F) {
 
 // Build the tables into c.stab (one CTA, any size).
 //   A[a][i] = sum_j dec[j] [ext(2a + 1 - j) == i]   (analysis along a side)
-//   jlo/jhi[b] = first / last column j with A'[b][j] != 0 (shared-memory
-//                atomics while A' is formed)
+//   jlo/jhi[b] = first / last column j with A'[b][j] != 0, ilo/ihi[a] the
+//                same for the rows of A (shared-memory atomics while the
+//                matrices are formed)
 __device__ inline void build_spatial_tables(const Ctx &c) {
     SpatialSmem L;
     L.init(c.H, c.W, c.hp, c.wp);
     float *tb = c.stab;
     int *ti = reinterpret_cast<int *>(c.stab);
     const int H = c.H, W = c.W, hp = c.hp, wp = c.wp, F = c.F;
+    __shared__ int s_jlo[WZ_MAX_HW + kMaxTaps], s_jhi[WZ_MAX_HW + kMaxTaps];
+    __shared__ int s_ilo[WZ_MAX_HW + kMaxTaps], s_ihi[WZ_MAX_HW + kMaxTaps];
+    for (int b = threadIdx.x; b < wp; b += blockDim.x) {
+        s_jlo[b] = L.WP4;
+        s_jhi[b] = -1;
+    }
+    for (int a = threadIdx.x; a < hp; a += blockDim.x) {
+        s_ilo[a] = H;
+        s_ihi[a] = -1;
+    }
+    __syncthreads();
     for (int k = threadIdx.x; k < hp * H; k += blockDim.x) {
         const int a = k / H, i = k % H;
         float sl = 0.f, sh = 0.f;
@@ -205,13 +230,11 @@ __device__ inline void build_spatial_tables(const Ctx &c) {
             }
         tb[L.AHl + k] = sl;
         tb[L.AHh + k] = sh;
+        if (sl != 0.f || sh != 0.f) {
+            atomicMin(&s_ilo[a], i);
+            atomicMax(&s_ihi[a], i);
+        }
     }
-    __shared__ int s_jlo[WZ_MAX_HW + kMaxTaps], s_jhi[WZ_MAX_HW + kMaxTaps];
-    for (int b = threadIdx.x; b < wp; b += blockDim.x) {
-        s_jlo[b] = L.WP4;
-        s_jhi[b] = -1;
-    }
-    __syncthreads();
     for (int k = threadIdx.x; k < wp * L.WP4; k += blockDim.x) {
         const int b = k / L.WP4, i = k % L.WP4;
         float sl = 0.f, sh = 0.f;
@@ -232,6 +255,10 @@ __device__ inline void build_spatial_tables(const Ctx &c) {
     for (int b = threadIdx.x; b < wp; b += blockDim.x) {
         ti[L.jlo + b] = s_jlo[b];
         ti[L.jhi + b] = s_jhi[b];
+    }
+    for (int a = threadIdx.x; a < hp; a += blockDim.x) {
+        ti[L.ilo + a] = s_ilo[a];
+        ti[L.ihi + a] = s_ihi[a];
     }
 }
 
