@@ -75,7 +75,7 @@ struct TcMaps {
 };
 
 struct Unit {
-    int f, j0, ct0, nc, cg;
+    int f, j0, ct0, nc, cg, kclo, kchi;   // operator chunks [kclo, kchi] (the rest are zero)
 };
 
 __device__ __forceinline__ Unit decode_unit(const Ctx &c, const int *vprefix, int u) {
@@ -90,8 +90,10 @@ __device__ __forceinline__ Unit decode_unit(const Ctx &c, const int *vprefix, in
     r.f = q.x;
     r.j0 = q.y;
     r.ct0 = q.z;
-    r.nc = q.w & 0xffff;
-    r.cg = q.w >> 16;
+    r.nc = q.w & 0x1ff;
+    r.cg = (q.w >> 9) & 7;
+    r.kclo = (q.w >> 12) & 0xff;
+    r.kchi = (q.w >> 20) & 0xff;
     return r;
 }
 
@@ -100,12 +102,13 @@ __device__ __forceinline__ void fail(const Ctx &c, volatile int *abort_flag, int
     atomicOr(c.status, code);
 }
 
-// The MMAs of one unit: KC stages of kKC tokens, each two K = 16 steps over
+// The MMAs of one unit: stages kclo..kchi of kKC tokens, each two K = 16 steps over
 // CG channel tiles (hi|lo fused into one MMA, or hi and lo as two).  The
 // pattern is fixed at compile time and the stage descriptors are advanced by
 // a constant, so the issuing thread spends a few instructions per MMA.
 template <int CG, bool FUSED>
-__device__ __forceinline__ bool mma_unit(TcShared *S, uint8_t *ring, const Ctx &c, volatile int *abort_flag, int KC,
+__device__ __forceinline__ bool mma_unit(TcShared *S, uint8_t *ring, const Ctx &c, volatile int *abort_flag, int kclo,
+                                         int kchi,
                                          int &stage, uint32_t &phase, uint32_t dbase, int tcols, uint32_t idesc,
                                          int ncp) {
     const uint32_t ring32 = ptx::smem_u32(ring);
@@ -118,7 +121,7 @@ __device__ __forceinline__ bool mma_unit(TcShared *S, uint8_t *ring, const Ctx &
     uint32_t d[CG];
 #pragma unroll
     for (int ct = 0; ct < CG; ++ct) d[ct] = dbase + (uint32_t)(ct * tcols);
-    for (int kc = 0; kc < KC; ++kc) {
+    for (int kc = kclo; kc <= kchi; ++kc) {
         if (!ptx::mbar_wait(&S->full[stage], phase, kTimeoutNs)) {
             fail(c, abort_flag, 4);
             return false;
@@ -126,7 +129,7 @@ __device__ __forceinline__ bool mma_unit(TcShared *S, uint8_t *ring, const Ctx &
         ptx::tc_fence_after();
         const uint64_t so = (uint64_t)stage * kStageDesc;
         const uint64_t a0 = a_base + so, b0 = b_base + so;
-        const uint32_t acc = kc ? 1u : 0u;
+        const uint32_t acc = kc > kclo ? 1u : 0u;
 #pragma unroll
         for (int s = 0; s < 2; ++s) {
 #pragma unroll
@@ -212,8 +215,12 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
             const int ncp = (un.nc + 15) & ~15;
             const int64_t wrow0 = (int64_t)c.woff[un.f] + un.j0;     // multiple of 16
             const uint32_t bytes = (uint32_t)un.cg * 8192u + 2u * (uint32_t)ncp * 64u;
+            if (un.kclo > un.kchi || un.kchi >= KC) {   // not a record the spatial kernel writes
+                fail(c, abort_flag, 4);
+                break;
+            }
             bool ok = true;
-            for (int kc = 0; kc < KC; ++kc) {
+            for (int kc = un.kclo; kc <= un.kchi; ++kc) {
                 if (!ptx::mbar_wait(&S->empty[stage], phase ^ 1u, kTimeoutNs)) {
                     fail(c, abort_flag, 1);
                     ok = false;
@@ -261,19 +268,23 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
                 break;
             }
             ptx::tc_fence_after();
+            if (un.kclo > un.kchi || un.kchi >= KC) {
+                fail(c, abort_flag, 4);
+                break;
+            }
             const uint32_t idesc = ptx::idesc_bf16(128, fused ? 2 * ncp : ncp, true, false);
             const uint32_t dbase = tmem + (uint32_t)(b * kAccCols);
             bool ok = false;
             if (fused) {
                 switch (un.cg) {
-                    case 1: ok = mma_unit<1, true>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp); break;
-                    case 2: ok = mma_unit<2, true>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp); break;
-                    case 3: ok = mma_unit<3, true>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp); break;
-                    case 4: ok = mma_unit<4, true>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp); break;
+                    case 1: ok = mma_unit<1, true>(S, ring, c, abort_flag, un.kclo, un.kchi, stage, phase, dbase, tcols, idesc, ncp); break;
+                    case 2: ok = mma_unit<2, true>(S, ring, c, abort_flag, un.kclo, un.kchi, stage, phase, dbase, tcols, idesc, ncp); break;
+                    case 3: ok = mma_unit<3, true>(S, ring, c, abort_flag, un.kclo, un.kchi, stage, phase, dbase, tcols, idesc, ncp); break;
+                    case 4: ok = mma_unit<4, true>(S, ring, c, abort_flag, un.kclo, un.kchi, stage, phase, dbase, tcols, idesc, ncp); break;
                     default: fail(c, abort_flag, 4); break;
                 }
             } else if (un.cg == 1) {
-                ok = mma_unit<1, false>(S, ring, c, abort_flag, KC, stage, phase, dbase, tcols, idesc, ncp);
+                ok = mma_unit<1, false>(S, ring, c, abort_flag, un.kclo, un.kchi, stage, phase, dbase, tcols, idesc, ncp);
             } else {
                 fail(c, abort_flag, 4);
             }

@@ -278,7 +278,7 @@ __global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c, 
         if (n <= 0) continue;
         const int h = c.hw[2 * f], w = c.hw[2 * f + 1];
         if (pi >= h || pi * w >= n) continue;
-        if (pi == 0 && c.path == WZ_PATH_TENSOR) unit_records(c, f, n);
+        if (pi == 0 && c.path == WZ_PATH_TENSOR) unit_records(c, f, n, h, w, ilo, ihi);
         const int t = f % c.T;
         if (f != cur_f) {
             // gate G of this frame (Eq. 6, Eq. 12), pooled by frame_stats

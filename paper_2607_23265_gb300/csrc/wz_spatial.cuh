@@ -173,19 +173,46 @@ __device__ inline void tail_rows(const Ctx &c, int tb) {
 
 // The tensor-core work units of frame f (the temporal kernel placed them):
 // column blocks of <= 256 tokens, each in groups of unit_tiles(round16(nc))
-// 128-channel tiles.
-__device__ inline void unit_records(const Ctx &c, int64_t f, int n) {
+// 128-channel tiles.  A record is (f, j0, first tile, nc | tiles << 9 |
+// kc_lo << 12 | kc_hi << 20): the unit's operator rows are zero outside the
+// 32-column chunks [kc_lo, kc_hi] (K_pad <= 4096, so chunks fit 8 bits).
+// With the row supports ilo / ihi of the height analysis (single-level WSM;
+// h x w the frame's grid) that range is the chunks of the map rows the block's
+// grid rows reach, else every chunk.
+__device__ inline void unit_records(const Ctx &c, int64_t f, int n, int h = 0, int w = 0, const int *ilo = nullptr,
+                                    const int *ihi = nullptr) {
     const int v = (int)(f / c.T);
     int4 *units = c.units + (size_t)v * c.max_units_v;
     int u0 = c.ustart[f];
+    const int KC = c.K_pad >> 5;
     for (int j0 = 0; j0 < n; j0 += kColBlock) {
         const int nc = min(kColBlock, n - j0);
         const int cg = unit_tiles((nc + 15) / 16 * 16);
         const int cnt = (c.n_ct + cg - 1) / cg;
+        int klo = 0, khi = KC - 1;
+        if (ilo != nullptr && w > 0) {
+            int zlo = c.H, zhi = -1;
+            for (int p = j0 / w; p <= (j0 + nc - 1) / w && p < h; ++p) {
+                int y0, y1, alo, ahi;
+                float ly;
+                bilinear_src(p, c.H, h, y0, y1, ly);
+                synth_support(y0, y1, c.F, c.hp, alo, ahi);
+                for (int a = alo; a <= ahi; ++a) {
+                    zlo = min(zlo, ilo[a]);
+                    zhi = max(zhi, ihi[a]);
+                }
+            }
+            if (zhi >= zlo) {
+                klo = min(KC - 1, (zlo * c.W) >> 5);
+                khi = min(KC - 1, ((zhi + 1) * c.W - 1) >> 5);
+            } else {
+                klo = khi = 0;   // an all-zero block: one chunk of zeros
+            }
+        }
         for (int li = threadIdx.x; li < cnt; li += blockDim.x) {
             const int ct = li * cg;
             if (u0 + li < c.max_units_v)
-                units[u0 + li] = make_int4((int)f, j0, ct, nc | (min(cg, c.n_ct - ct) << 16));
+                units[u0 + li] = make_int4((int)f, j0, ct, nc | (min(cg, c.n_ct - ct) << 9) | (klo << 12) | (khi << 20));
         }
         u0 += cnt;
     }

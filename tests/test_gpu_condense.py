@@ -94,6 +94,23 @@ def test_options(wz, kw):
     _random_case(wz, 10, 13, 13, 128, 6, 0.2, seed=5, **kw)
 
 
+@pytest.mark.parametrize("T,H,W,D,ratio,kw", [
+    (3, 27, 27, 256, 0.8, {}),                       # ~583 tokens a frame: blocks of 256, 256, 71
+    (2, 40, 40, 64, 0.6, {}),                        # 960 tokens, a 40-row map: four blocks
+    (3, 27, 27, 128, 0.7, dict(mode="zero")),
+    (3, 27, 27, 128, 0.7, dict(mode="periodic")),    # supports wrap: every chunk
+    (3, 27, 27, 128, 0.7, dict(wsm_wavelet=44)),     # 10-tap supports
+    (3, 27, 27, 128, 0.7, dict(wsm_wavelet=1)),      # Haar: narrow supports
+    (3, 27, 27, 128, 0.7, dict(wsm_levels=2)),       # multi-level: every chunk
+    (2, 27, 27, 128, 0.8, dict(spatial_mode="saliency")),
+])
+def test_split_frames(wz, T, H, W, D, ratio, kw):
+    # frames of more than 256 tokens are condensed in blocks of 256 output
+    # tokens; a block's operator rows reach only part of the map, and the
+    # tensor-core units skip the 32-token chunks outside it
+    _random_case(wz, T, H, W, D, 4, ratio, seed=T * 31 + H, **kw)
+
+
 @pytest.mark.parametrize("kw", [dict(wta_levels=2), dict(wta_levels=3, wta_wavelet=2), dict(wta_levels=4, wta_wavelet=4),
                                 dict(wsm_levels=2), dict(wsm_levels=3, wsm_wavelet=1), dict(wsm_levels=2, wsm_wavelet=44),
                                 dict(wsm_levels=2, path="simt"), dict(wsm_levels=2, mode="zero"),
