@@ -25,28 +25,6 @@ constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
-// Frame order of the tensor-core unit list: position p holds frame
-// (p * S) mod T with S near T (1 - 1/phi) and coprime to T.  Budgets follow
-// the smoothed relevance, so neighbouring frames have similar budgets and a
-// unit's cost (operator bytes, MMA columns) grows with the budget; spreading
-// neighbours apart gives every wave of units over the SMs a mix of
-// tensor-heavy and feature-stream-bound units.
-int unit_frame_stride(int T) {
-    if (T <= 2) return 1;
-    int S = (int)(0.381966 * T + 0.5);
-    if (S < 1) S = 1;
-    auto gcd = [](int a, int b) {
-        while (b) {
-            const int t = a % b;
-            a = b;
-            b = t;
-        }
-        return a;
-    };
-    while (gcd(S, T) != 1) ++S;
-    return S;
-}
-
 bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
 // NVTX range around a host-side launch (a no-op unless a profiler listens).
@@ -213,7 +191,6 @@ void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.V = s.V; c.T = s.T; c.H = s.H; c.W = s.W; c.D = s.D; c.N = s.N; c.dtype = s.dtype;
     c.hp = s.hp; c.wp = s.wp; c.K_pad = s.K_pad; c.n_ct = s.n_ct;
     c.max_units_v = s.max_units_v; c.rows_total = s.rows_total; c.w_rows = s.w_rows;
-    c.ustride = unit_frame_stride(s.T);
     c.qbar32 = reinterpret_cast<float *>(ws + L.qbar32);
     c.qbar64 = reinterpret_cast<double *>(ws + L.qbar64);
     c.vpar = reinterpret_cast<VideoPar *>(ws + L.vpar);

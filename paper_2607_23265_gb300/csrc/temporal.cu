@@ -402,8 +402,6 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     // 16) and tensor-core units (column blocks of <= 256 tokens, each in
     // groups of unit_tiles(round16(nc)) 128-channel tiles; the spatial kernel
     // writes the unit records); one block scan gives all three offsets
-    // The unit list takes the frames in the order t_p = (p * ustride) mod T
-    // (position p = t0 + k of this thread): the third scan runs over positions.
     const bool tc = c.path == WZ_PATH_TENSOR;
     int nloc[kPerThread], ucnt[kPerThread];
     int part[3] = {0, 0, 0};
@@ -412,13 +410,11 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         const int t = t0 + k;
         nloc[k] = (k < per && t < T) ? nf[t] : 0;
         ucnt[k] = 0;
-        if (tc && k < per && t < T) {
-            const int np = nf[(int)(((long long)t * c.ustride) % T)];
-            for (int j0 = 0; j0 < np; j0 += kColBlock) {
-                const int nc = min(kColBlock, np - j0);
+        if (tc)
+            for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
+                const int nc = min(kColBlock, nloc[k] - j0);
                 ucnt[k] += (c.n_ct + unit_tiles((nc + 15) / 16 * 16) - 1) / unit_tiles((nc + 15) / 16 * 16);
             }
-        }
         part[0] += nloc[k];
         part[1] += (nloc[k] + 15) & ~15;
         part[2] += ucnt[k];
@@ -433,7 +429,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             c.n[base + t] = nloc[k];
             c.off[base + t] = vp.row0 + o;
             c.woff[base + t] = vp.w_row0 + wo;
-            if (tc) c.ustart[base + (int)(((long long)t * c.ustride) % T)] = u;
+            if (tc) c.ustart[base + t] = u;
             const int h = grid_h(nloc[k], c.H, c.W);
             c.hw[2 * (base + t)] = h;
             c.hw[2 * (base + t) + 1] = h > 0 ? (nloc[k] + h - 1) / h : 0;

@@ -35,7 +35,6 @@ struct Ctx {
     int G1;               // relevance CTAs actually launched
     int n_ct;             // 128-channel tiles
     int max_units_v;      // unit-list capacity per video
-    int ustride;          // unit-list frame order: position p holds frame (p * ustride) mod T
     int F;                // WSM filter taps
     int64_t L1;           // tokens per relevance CTA
     int64_t rows_total;   // sum of budgets over videos (output rows)

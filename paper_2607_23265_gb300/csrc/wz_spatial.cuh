@@ -191,16 +191,19 @@ __device__ inline void unit_records(const Ctx &c, int64_t f, int n, int h = 0, i
         const int cnt = (c.n_ct + cg - 1) / cg;
         int klo = 0, khi = KC - 1;
         if (ilo != nullptr && w > 0) {
+            // the analysis rows of grid rows p0..p1 lie in [alo(p0), ahi(p1)]
+            // (both ends grow with p): the union of their row supports
+            const int p0 = j0 / w, p1 = min(h - 1, (j0 + nc - 1) / w);
+            int y0, y1, alo, ahi, a0, a1;
+            float ly;
+            bilinear_src(p0, c.H, h, y0, y1, ly);
+            synth_support(y0, y1, c.F, c.hp, a0, ahi);
+            bilinear_src(p1, c.H, h, y0, y1, ly);
+            synth_support(y0, y1, c.F, c.hp, alo, a1);
             int zlo = c.H, zhi = -1;
-            for (int p = j0 / w; p <= (j0 + nc - 1) / w && p < h; ++p) {
-                int y0, y1, alo, ahi;
-                float ly;
-                bilinear_src(p, c.H, h, y0, y1, ly);
-                synth_support(y0, y1, c.F, c.hp, alo, ahi);
-                for (int a = alo; a <= ahi; ++a) {
-                    zlo = min(zlo, ilo[a]);
-                    zhi = max(zhi, ihi[a]);
-                }
+            for (int a = a0; a <= a1; ++a) {
+                zlo = min(zlo, ilo[a]);
+                zhi = max(zhi, ihi[a]);
             }
             if (zhi >= zlo) {
                 klo = min(KC - 1, (zlo * c.W) >> 5);
