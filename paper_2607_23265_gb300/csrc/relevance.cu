@@ -172,7 +172,10 @@ constexpr uint64_t kRelTimeoutNs = 2000000000ull;
 // together once per <= 64 tokens, so block barriers are rare.
 template <typename T, int VPT>
 __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kernel(Ctx c, int CH) {
-    pdl_wait();
+    // The producer streams only the features, which the kernels before this
+    // one do not write, so it starts before the wait for the previous grid
+    // (the query pooling) and fills the ring meanwhile; the consumers wait
+    // for it before they read u_q or write anything.
     pdl_trigger();
     constexpr int VEC = VecOf<T>::kElems;
     constexpr int GROUP = 8;                 // tokens per warp transpose-reduction
@@ -240,6 +243,7 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
     }
 
     // ---------------- consumers ----------------
+    pdl_wait();
     auto consumer_sync = [&]() { asm volatile("bar.sync 1, %0;" ::"r"(NC) : "memory"); };
     constexpr int NP = VEC / 2;                  // packed pairs per 16-byte vector
     constexpr int SHIFT = 1;                     // lane l holds reduced value l >> 1
