@@ -191,18 +191,22 @@ __device__ void grid_row_prefix(const Ctx &c, int F, int *rowpre, int *wsum) {
 // the rows that exist; otherwise it runs over all V*T*H (frame, row) pairs.
 template <int BMAX>
 __global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c, int compact) {
-    pdl_wait();
     pdl_trigger();
     extern __shared__ float sm[];
     __shared__ int s_item, s_f, s_wsum[kSpatialThreads / 32];
     const int tid = threadIdx.x;
+    const int H = c.H, W = c.W, N = c.N, hp = c.hp, wp = c.wp, F = c.F;
+    SpatialSmem L;
+    L.init(H, W, hp, wp);
+    // the frame-independent tables (analysis matrices, supports) come from the
+    // kernel parameters alone: formed before the wait for the temporal kernel,
+    // while it runs
+    build_spatial_tables_smem(c, L, sm);
+    pdl_wait();
     // thread 0 claims the next row while the current one is formed, so the
     // counter's round trip overlaps the work
     int claimed = tid == 0 ? atomicAdd(c.spatial_next, 1) : 0;
     if ((int)blockIdx.x < kTailBlocks) tail_rows(c, (int)blockIdx.x);
-    const int H = c.H, W = c.W, N = c.N, hp = c.hp, wp = c.wp, F = c.F;
-    SpatialSmem L;
-    L.init(H, W, hp, wp);
     float *G = sm + L.G;
     float *AHl = sm + L.AHl, *AHh = sm + L.AHh, *AWl = sm + L.AWl, *AWh = sm + L.AWh;
     float *PAl = sm + L.PAl, *PAh = sm + L.PAh, *Yl = sm + L.Yl, *Yh = sm + L.Yh;
@@ -215,22 +219,6 @@ __global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c, 
     const int HP4 = L.HP4, WP4 = L.WP4;
     (void)red;
 
-    // ---- per-frame tables ------------------------------------------------
-    // the frame-independent tables (analysis matrices, supports), built once
-    // per pass
-    {   // 16-byte copies, two in flight per thread (the tables and the stab buffer are 16-byte aligned)
-        const int n4 = L.tables >> 2;
-        const int4 *src = reinterpret_cast<const int4 *>(c.stab);
-        int4 *dst = reinterpret_cast<int4 *>(sm);
-        const int bd = (int)blockDim.x;
-        for (int k = tid; k < n4; k += 2 * bd) {
-            const int4 x0 = src[k];
-            const bool two = k + bd < n4;
-            const int4 x1 = two ? src[k + bd] : x0;
-            dst[k] = x0;
-            if (two) dst[k + bd] = x1;
-        }
-    }
     const bool bf = c.path == WZ_PATH_TENSOR;
     __nv_bfloat16 *Whi = static_cast<__nv_bfloat16 *>(c.Wop);
     __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * c.K_pad;

@@ -221,33 +221,23 @@ __device__ inline void unit_records(const Ctx &c, int64_t f, int n, int h = 0, i
     }
 }
 
-// Bytes of the frame-independent tables for an image of H x W and F taps.
-inline size_t spatial_table_bytes(int H, int W, int F) {
-    SpatialSmem L;
-    L.init(H, W, (H + F - 1) / 2, (W + F - 1) / 2);
-    return (size_t)L.tables * 4;
-}
-
-// Build the tables into c.stab (one CTA, any size).
+// The frame-independent tables, built by each spatial CTA into the head of
+// its own shared memory (tb) from the filter taps in the kernel parameters:
 //   A[a][i] = sum_j dec[j] [ext(2a + 1 - j) == i]   (analysis along a side)
 //   jlo/jhi[b] = first / last column j with A'[b][j] != 0, ilo/ihi[a] the
-//                same for the rows of A (shared-memory atomics while the
-//                matrices are formed)
-__device__ inline void build_spatial_tables(const Ctx &c) {
-    SpatialSmem L;
-    L.init(c.H, c.W, c.hp, c.wp);
-    float *tb = c.stab;
-    int *ti = reinterpret_cast<int *>(c.stab);
+//                same for the rows of A (shared-memory atomics on their slots
+//                while the matrices are formed)
+// Called by the whole block.
+__device__ inline void build_spatial_tables_smem(const Ctx &c, const SpatialSmem &L, float *tb) {
+    int *ti = reinterpret_cast<int *>(tb);
     const int H = c.H, W = c.W, hp = c.hp, wp = c.wp, F = c.F;
-    __shared__ int s_jlo[WZ_MAX_HW + kMaxTaps], s_jhi[WZ_MAX_HW + kMaxTaps];
-    __shared__ int s_ilo[WZ_MAX_HW + kMaxTaps], s_ihi[WZ_MAX_HW + kMaxTaps];
     for (int b = threadIdx.x; b < wp; b += blockDim.x) {
-        s_jlo[b] = L.WP4;
-        s_jhi[b] = -1;
+        ti[L.jlo + b] = L.WP4;
+        ti[L.jhi + b] = -1;
     }
     for (int a = threadIdx.x; a < hp; a += blockDim.x) {
-        s_ilo[a] = H;
-        s_ihi[a] = -1;
+        ti[L.ilo + a] = H;
+        ti[L.ihi + a] = -1;
     }
     __syncthreads();
     for (int k = threadIdx.x; k < hp * H; k += blockDim.x) {
@@ -261,8 +251,8 @@ __device__ inline void build_spatial_tables(const Ctx &c) {
         tb[L.AHl + k] = sl;
         tb[L.AHh + k] = sh;
         if (sl != 0.f || sh != 0.f) {
-            atomicMin(&s_ilo[a], i);
-            atomicMax(&s_ihi[a], i);
+            atomicMin(&ti[L.ilo + a], i);
+            atomicMax(&ti[L.ihi + a], i);
         }
     }
     for (int k = threadIdx.x; k < wp * L.WP4; k += blockDim.x) {
@@ -277,20 +267,20 @@ __device__ inline void build_spatial_tables(const Ctx &c) {
         tb[L.AWl + k] = sl;
         tb[L.AWh + k] = sh;
         if (sl != 0.f || sh != 0.f) {
-            atomicMin(&s_jlo[b], i);
-            atomicMax(&s_jhi[b], i);
+            atomicMin(&ti[L.jlo + b], i);
+            atomicMax(&ti[L.jhi + b], i);
         }
     }
     __syncthreads();
-    for (int b = threadIdx.x; b < wp; b += blockDim.x) {
-        ti[L.jlo + b] = s_jlo[b];
-        ti[L.jhi + b] = s_jhi[b];
-    }
-    for (int a = threadIdx.x; a < hp; a += blockDim.x) {
-        ti[L.ilo + a] = s_ilo[a];
-        ti[L.ihi + a] = s_ihi[a];
-    }
 }
+
+// Bytes of the frame-independent tables for an image of H x W and F taps.
+inline size_t spatial_table_bytes(int H, int W, int F) {
+    SpatialSmem L;
+    L.init(H, W, (H + F - 1) / 2, (W + F - 1) / 2);
+    return (size_t)L.tables * 4;
+}
+
 
 }  // namespace wz
 
