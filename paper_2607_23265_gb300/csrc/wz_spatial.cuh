@@ -225,51 +225,39 @@ __device__ inline void unit_records(const Ctx &c, int64_t f, int n, int h = 0, i
 // its own shared memory (tb) from the filter taps in the kernel parameters:
 //   A[a][i] = sum_j dec[j] [ext(2a + 1 - j) == i]   (analysis along a side)
 //   jlo/jhi[b] = first / last column j with A'[b][j] != 0, ilo/ihi[a] the
-//                same for the rows of A (shared-memory atomics on their slots
-//                while the matrices are formed)
-// Called by the whole block.
+//                same for the rows of A
+// Called by the whole block (hp + wp <= blockDim.x).
 __device__ inline void build_spatial_tables_smem(const Ctx &c, const SpatialSmem &L, float *tb) {
     int *ti = reinterpret_cast<int *>(tb);
     const int H = c.H, W = c.W, hp = c.hp, wp = c.wp, F = c.F;
-    for (int b = threadIdx.x; b < wp; b += blockDim.x) {
-        ti[L.jlo + b] = L.WP4;
-        ti[L.jhi + b] = -1;
-    }
-    for (int a = threadIdx.x; a < hp; a += blockDim.x) {
-        ti[L.ilo + a] = H;
-        ti[L.ihi + a] = -1;
-    }
-    __syncthreads();
-    for (int k = threadIdx.x; k < hp * H; k += blockDim.x) {
-        const int a = k / H, i = k % H;
-        float sl = 0.f, sh = 0.f;
-        for (int j = 0; j < F; ++j)
-            if (ext_index(2 * a + 1 - j, H, c.mode) == i) {
-                sl += c.dec_lo[j];
-                sh += c.dec_hi[j];
+    // one thread per analysis row: zero it, add tap j at ext(2a + 1 - j) for
+    // j = 0, 1, ... (each entry sums its taps in ascending order), then scan
+    // the row for its first and last nonzero column
+    const int r = threadIdx.x;
+    if (r < hp + wp) {
+        const bool hgt = r < hp;
+        const int a = hgt ? r : r - hp, n = hgt ? H : W, len = hgt ? H : L.WP4;
+        float *lo = tb + (hgt ? L.AHl + a * H : L.AWl + a * L.WP4);
+        float *hi = tb + (hgt ? L.AHh + a * H : L.AWh + a * L.WP4);
+        for (int i = 0; i < len; ++i) {
+            lo[i] = 0.f;
+            hi[i] = 0.f;
+        }
+        for (int j = 0; j < F; ++j) {
+            const int i = ext_index(2 * a + 1 - j, n, c.mode);   // -1: outside (zero extension)
+            if (i >= 0 && i < n) {
+                lo[i] += c.dec_lo[j];
+                hi[i] += c.dec_hi[j];
             }
-        tb[L.AHl + k] = sl;
-        tb[L.AHh + k] = sh;
-        if (sl != 0.f || sh != 0.f) {
-            atomicMin(&ti[L.ilo + a], i);
-            atomicMax(&ti[L.ihi + a], i);
         }
-    }
-    for (int k = threadIdx.x; k < wp * L.WP4; k += blockDim.x) {
-        const int b = k / L.WP4, i = k % L.WP4;
-        float sl = 0.f, sh = 0.f;
-        if (i < W)
-            for (int j = 0; j < F; ++j)
-                if (ext_index(2 * b + 1 - j, W, c.mode) == i) {
-                    sl += c.dec_lo[j];
-                    sh += c.dec_hi[j];
-                }
-        tb[L.AWl + k] = sl;
-        tb[L.AWh + k] = sh;
-        if (sl != 0.f || sh != 0.f) {
-            atomicMin(&ti[L.jlo + b], i);
-            atomicMax(&ti[L.jhi + b], i);
-        }
+        int first = hgt ? H : L.WP4, last = -1;
+        for (int i = 0; i < n; ++i)
+            if (lo[i] != 0.f || hi[i] != 0.f) {
+                first = min(first, i);
+                last = i;
+            }
+        ti[(hgt ? L.ilo : L.jlo) + a] = first;
+        ti[(hgt ? L.ihi : L.jhi) + a] = last;
     }
     __syncthreads();
 }
