@@ -14,7 +14,10 @@
 // W_m is fp32 split into bf16 hi + lo (two MMAs into one accumulator), so the
 // product keeps ~16 bits of W while X (exact in bf16) streams once.
 //
-// A unit of work is (frame, <= 256 output tokens, CG <= 4 channel tiles).
+// A unit of work is (frame, <= 256 output tokens, CG <= 4 channel tiles) over
+// the 32-token chunks [kclo, kchi] its operator rows reach (every chunk unless
+// a frame of more than 256 tokens is condensed in blocks); the rest of its
+// operator rows are zero and are neither loaded nor multiplied.
 // The cost of an MMA instruction hardly depends on N, so for N <= 128 the hi
 // and lo operator halves (adjacent in shared memory) form one MMA of N = 2N
 // whose accumulator holds the hi and lo products side by side; for larger N
