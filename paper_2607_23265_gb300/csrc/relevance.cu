@@ -591,37 +591,40 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
         wsum[warp][4] = p4;
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-        double vq = 0.0, vv = 0.0, vp = 0.0, qq = 0.0, pp = 0.0;
-        for (int w = 0; w < nw; ++w) {
-            vq += (double)wsum[w][0];
-            vv += (double)wsum[w][1];
-            vp += (double)wsum[w][2];
-            qq += (double)wsum[w][3];
-            pp += (double)wsum[w][4];
+    if (warp == 0) {
+        // lane k < 5 sums quantity k over the warps in order (one fp64 warp
+        // instruction per warp partial instead of five)
+        const int lane = threadIdx.x & 31;
+        double acc = 0.0;
+        if (lane < 5)
+            for (int w = 0; w < nw; ++w) acc += (double)wsum[w][lane];
+        const double vq = __shfl_sync(0xffffffffu, acc, 0), vv = __shfl_sync(0xffffffffu, acc, 1);
+        const double vp = __shfl_sync(0xffffffffu, acc, 2), qq = __shfl_sync(0xffffffffu, acc, 3);
+        const double pp = __shfl_sync(0xffffffffu, acc, 4);
+        if (lane == 0) {
+            const double qn = sqrt(qq);
+            double r = (vv > 0.0 && qn > 0.0) ? vq / (sqrt(vv) * qn) : 0.0;
+            if (maxsim) {
+                double best = -INFINITY;
+                for (int w = 0; w < nw; ++w) best = fmax(best, wmax[w]);
+                r = vv > 0.0 ? best / sqrt(vv) : 0.0;
+            }
+            if (c.ext_r) r = (double)c.ext_r[f];   // an external scorer's r_t
+            double d = 0.0;
+            if (t > 0) {
+                const double den = sqrt(vv * pp);
+                const double cs = den > 0.0 ? vp / den : 0.0;
+                d = fmin(2.0, fmax(0.0, 1.0 - cs)) + 0.0;   // + 0.0: never -0
+            }
+            c.fr[4 * f + 0] = r;
+            c.fr[4 * f + 1] = d;
+            if (c.drange) {   // non-negative doubles order like their bit patterns
+                const unsigned long long bits = (unsigned long long)__double_as_longlong(d);
+                atomicMin(&c.drange[2 * v], bits);
+                atomicMax(&c.drange[2 * v + 1], bits);
+            }
+            if (c.frame_scores) c.frame_scores[f] = (float)r;
         }
-        const double qn = sqrt(qq);
-        double r = (vv > 0.0 && qn > 0.0) ? vq / (sqrt(vv) * qn) : 0.0;
-        if (maxsim) {
-            double best = -INFINITY;
-            for (int w = 0; w < nw; ++w) best = fmax(best, wmax[w]);
-            r = vv > 0.0 ? best / sqrt(vv) : 0.0;
-        }
-        if (c.ext_r) r = (double)c.ext_r[f];   // an external scorer's r_t
-        double d = 0.0;
-        if (t > 0) {
-            const double den = sqrt(vv * pp);
-            const double cs = den > 0.0 ? vp / den : 0.0;
-            d = fmin(2.0, fmax(0.0, 1.0 - cs)) + 0.0;   // + 0.0: never -0
-        }
-        c.fr[4 * f + 0] = r;
-        c.fr[4 * f + 1] = d;
-        if (c.drange) {   // non-negative doubles order like their bit patterns
-            const unsigned long long bits = (unsigned long long)__double_as_longlong(d);
-            atomicMin(&c.drange[2 * v], bits);
-            atomicMax(&c.drange[2 * v + 1], bits);
-        }
-        if (c.frame_scores) c.frame_scores[f] = (float)r;
     }
     if (do_gate) frame_gate(c, f, wsum[0], av);
 }
