@@ -13,14 +13,16 @@
 //   W_m[(p,q),(i,j)] = sum_v sum_b Q_v[q,b] A'_v[b,j] Y_v[b,i],
 //   Y_v[b,i]         = sum_u sum_a P_u[p,a] A_u[a,i] g_uv[a,b].
 //
-// spatial_wsm_kernel is persistent: each CTA copies the frame-independent
-// tables (analysis matrices with their column supports) once and then pulls
-// (frame, grid row) candidates from a global counter; a new frame reloads
-// its gate and the width rows Q_v.  Per grid row: P_u A_u, then Y_v, then
-// one warp per output token q with lane = input row i, which keeps
-// c_v[b] = Q_v[q,b] Y_v[b,i] for the few b of the column's support in
-// registers and forms row i of the token's operator row four columns at a
-// time from broadcast reads of A'_v.  Rows are staged in shared memory and
+// spatial_wsm_kernel is persistent: each CTA forms the frame-independent
+// tables (analysis matrices with their row and column supports) once, before
+// it waits for the temporal kernel, and then pulls grid rows from a global
+// counter; a new frame reloads its gate and the width rows Q_v.  Per grid
+// row: P_u A_u, then Y_v over the map rows the row's operator rows reach,
+// then the tokens with lane = input row i (two tokens per warp when at most
+// 16 rows are reached), each lane keeping c_v[b] = Q_v[q,b] Y_v[b,i] for the
+// few b of the column's support in registers and forming row i of the
+// token's operator row four columns at a time from 16-byte reads of A'_v.
+// Rows are staged in shared memory and
 // leave as 512-byte coalesced warp stores of bf16 hi/lo halves in the tiled
 // operator layout (tensor-core path) or as fp32 rows (CUDA-core path), with
 // the index map rows.  The ablation modes without the WSM use

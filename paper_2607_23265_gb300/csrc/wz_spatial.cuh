@@ -1,9 +1,9 @@
 // Shared-memory layout of the spatial-operator CTA and the frame-independent
 // tables it starts from (Eq. 11-14): the db analysis matrices along height
-// and width with the boundary extension folded in, and the rows of the width
-// analysis that reach each column.  The tables depend only on (H, W, filter, extension); one CTA builds
-// them per pass into global memory with the same layout as the head of the
-// shared-memory block, so each spatial CTA copies them in one loop.
+// and width with the boundary extension folded in, and the first and last
+// nonzero entry of every analysis row.  The tables depend only on (H, W,
+// filter, extension), so each spatial CTA forms them from its kernel
+// parameters at the head of its shared-memory block.
 #pragma once
 
 #include "wz_internal.cuh"
