@@ -8,10 +8,18 @@ tokens, larger than L2, so no L2 flush is needed between steps), with the
 achieved HBM bandwidth of the dominant kernel against the measured peak.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--config NAME]
 
-Under torchrun every rank condenses its own independent video (replicas, weak
-scaling); the time is the max over ranks.  `--impl reference` times the CPU
-oracle on a bounded sample of the same workload instead.
+--config picks one of the five synthetic workloads (default: the 256-frame
+video); `serving32x64_13x13_bf16` condenses 32 videos in one wz_condense_batch
+launch sequence.  The input is the recipe's CPU draw (workload.py), the same
+tensor the parity tests compare.  Under torchrun every rank condenses its own
+independent inputs (replicas, weak scaling); the time is the max over ranks.
+`--impl reference` times the CPU oracle on the host cores instead, the whole
+workload per step.  The cpu_baseline leg runs the oracle on the very input the
+GPU condensed and reports, beside its time, whether the GPU's outputs of the
+timed step match it (budgets and index map bit-exact, tokens within the
+stated tolerance).
 """
 
 from __future__ import annotations
@@ -35,8 +43,9 @@ WORKLOAD = "video256_27x27_bf16"
 KERNELS = ("query_pool", "relevance", "frame_stats", "temporal", "spatial", "condense")
 KERNEL_SOURCES = {"query_pool": "relevance.cu", "relevance": "relevance.cu", "frame_stats": "relevance.cu",
                   "temporal": "temporal.cu", "spatial": "spatial.cu", "condense": "condense_tc.cu"}
-CPU_SAMPLE_FRAMES = 256         # oracle sample for the cpu_baseline leg: the whole 256-frame video (~15 s on one core)
-REF_SAMPLE_FRAMES = 16          # oracle sample per step of the reference arm
+L2_BYTES = 129 * 10**6          # GB300 L2
+L2_FLUSH_BYTES = 512 << 20
+BATCH_CPU_VIDEOS = 16           # cpu_baseline sample of the serving batch: its first 16 videos (~12 s on one core)
 
 
 def parse():
@@ -45,7 +54,9 @@ def parse():
     p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--config", default=WORKLOAD)
+    p.add_argument("--config", default=WORKLOAD,
+                   choices=["tiny_f32_16x14x14", "video64_13x13_bf16", "video128_16x16_objects",
+                            "video256_27x27_bf16", "serving32x64_13x13_bf16"])
     p.add_argument("--path", default="auto", choices=["auto", "tensor", "simt"])
     p.add_argument("--e2e-steps", type=int, default=5)
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -73,6 +84,35 @@ def replica_spec(spec, rank):
     return wl.VideoSpec(**{**spec.__dict__, "seed": spec.seed + 7919 * rank})
 
 
+class Workload:
+    """One benchmark workload: one video, or the serving batch of videos of
+    one shape (per-video Lq, ratio and seed)."""
+
+    def __init__(self, name, specs, batch):
+        self.name, self.specs, self.batch = name, specs, batch
+        s = specs[0]
+        self.T, self.H, self.W, self.D, self.dtype = s.T, s.H, s.W, s.D, s.dtype
+        self.frames = len(specs) * s.T
+
+
+def workload(name, rank=0):
+    import workload as wl
+    if name == wl.BATCH_NAME:
+        return Workload(name, [replica_spec(s, rank) for s in wl.batch_specs()], True)
+    return Workload(name, [replica_spec(wl.CONFIGS[name], rank)], False)
+
+
+def draw_inputs(w):
+    """Host tensors of the workload: features [T,H,W,D] (or [V,T,H,W,D]) and
+    the query rows [Lq,D] (or all videos' rows, [sum Lq, D])."""
+    import torch
+    import workload as wl
+    pairs = [wl.make_video(s)[:2] for s in w.specs]
+    if not w.batch:
+        return pairs[0]
+    return torch.stack([x for x, _ in pairs]), torch.cat([q for _, q in pairs])
+
+
 def max_over_ranks(x, world, device=None):
     """The slowest rank's value (the job time); a no-op on one rank."""
     if world == 1:
@@ -89,11 +129,23 @@ def job_value(frames_per_rank, world, ms):
     return frames_per_rank * world / (ms * 1e-3)
 
 
-def config_dict(spec, name):
-    return {"workload": name, "T": spec.T, "H": spec.H, "W": spec.W, "D": spec.D, "Lq": spec.Lq,
-            "ratio": spec.ratio, "features_dtype": spec.dtype, "seed": spec.seed,
-            "feature_bytes": spec.T * spec.H * spec.W * spec.D * (2 if spec.dtype == "bf16" else 4),
-            "l2": "inputs larger than L2 (no flush needed)", "parallelism": "replicas"}
+def config_dict(w):
+    s = w.specs[0]
+    esz = 2 if w.dtype == "bf16" else 4
+    fb = w.frames * w.H * w.W * w.D * esz
+    d = {"workload": w.name, "T": w.T, "H": w.H, "W": w.W, "D": w.D}
+    if w.batch:
+        d.update({"videos": len(w.specs), "Lq": [x.Lq for x in w.specs], "ratio": [x.ratio for x in w.specs],
+                  "seed": [x.seed for x in w.specs]})
+    else:
+        d.update({"Lq": s.Lq, "ratio": s.ratio, "seed": s.seed})
+    d.update({"features_dtype": w.dtype, "feature_bytes": fb,
+              "input": "the recipe's CPU draw (workload.py), the tensor the parity tests use",
+              "l2": ("inputs larger than L2 (no flush needed)" if fb > L2_BYTES else
+                     "inputs smaller than L2: L2 flushed (512 MB written) before each timed step, "
+                     "each step timed alone"),
+              "parallelism": "replicas"})
+    return d
 
 
 def measured_peak():
@@ -271,9 +323,9 @@ def source_hash(fname):
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(kernel):
-    """dram bytes per launch from the committed ncu summary, if the kernel's
-    source is unchanged since the capture; else None."""
+def recorded_traffic(kernel, workload_name):
+    """dram bytes per launch from the committed ncu summary of this workload,
+    if the kernel's source is unchanged since the capture; else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
@@ -281,6 +333,8 @@ def recorded_traffic(kernel):
     except (OSError, ValueError):
         return None
     if not rec or rec.get("source_sha256_16") != source_hash(KERNEL_SOURCES[kernel]):
+        return None
+    if rec.get("workload", WORKLOAD).split()[0] != workload_name:
         return None
     return rec.get("dram_bytes_per_launch")
 
@@ -327,131 +381,292 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(self.rows)}
 
 
-def cpu_baseline(spec, frames):
-    """Time the oracle, as it stands, on one host core: a `frames`-frame video
-    drawn with the same recipe.  Runs in a fresh interpreter pinned to one BLAS
-    thread."""
-    code = (
-        "import json,sys,time; sys.path.insert(0, %r)\n"
-        "import workload as wl, oracle as O\n"
-        "s = wl.VideoSpec(T=%d, H=%d, W=%d, D=%d, dtype=%r, Lq=%d, ratio=%r, ar=%r, cuts=%d, seed=%d)\n"
-        "X, Q, _ = wl.make_video(s)\n"
-        "x, q = X.double().numpy(), Q.double().numpy()\n"
-        "t = time.perf_counter(); O.condense(x, q, s.ratio); dt = time.perf_counter() - t\n"
-        "print(json.dumps({'seconds': dt, 'frames': s.T}))\n"
-    ) % (ROOT, frames, spec.H, spec.W, spec.D, spec.dtype, spec.Lq, spec.ratio, spec.ar,
-         max(1, spec.cuts * frames // spec.T), spec.seed)
-    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1",
-               CUDA_VISIBLE_DEVICES="")
-    res = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=900)
+# The parity tolerance of condensed tokens for bf16 inputs with fp32
+# accumulation: |gpu - oracle| <= 1e-3 + 2e-2 |oracle|, the oracle's value
+# rounded to the output dtype first.
+TOK_ATOL, TOK_RTOL = 1e-3, 2e-2
+
+_BASELINE_CODE = r"""
+import json, sys, time
+sys.path.insert(0, %(root)r)
+import numpy as np
+import oracle as O
+
+d = %(dir)r
+meta = json.load(open(d + "/meta.json"))
+bits = np.load(d + "/x.npy", mmap_mode="r")
+gpu = np.load(d + "/gpu.npz")
+Qs = [np.load(d + "/q%%d.npy" %% v) for v in range(meta["V"])]
+
+def f64(a):
+    a = np.asarray(a)
+    if a.dtype == np.uint16:
+        return (a.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return a.astype(np.float64)
+
+def bf16_round(x):     # round to nearest even bfloat16, as the output dtype
+    f = x.astype(np.float32).view(np.uint32).astype(np.uint64)
+    f = (f + 0x7FFF + ((f >> 16) & 1)) & 0xFFFF0000
+    return f.astype(np.uint32).view(np.float32).astype(np.float64)
+
+videos = meta["videos"]            # the bounded sample: these videos, whole
+secs, frames, res = 0.0, 0, {}
+for v in videos:
+    x = f64(bits[v] if meta["batch"] else bits)
+    t = time.perf_counter()
+    r = O.condense(x, Qs[v], meta["ratios"][v])
+    secs += time.perf_counter() - t
+    frames += x.shape[0]
+    res[v] = r
+# parity of the GPU's outputs of the timed step on the same input
+ok_b = ok_i = ok_t = True
+worst, maxerr, rows = 0.0, 0.0, 0
+for v in videos:
+    r = res[v]
+    a, b = meta["row_offsets"][v], meta["row_offsets"][v + 1]
+    ok_b &= bool(np.array_equal(gpu["budgets"][v].astype(np.int64), r["budgets"]))
+    ok_i &= bool(np.array_equal(gpu["index"][a:b].astype(np.int64), r["out_index"]))
+    ref = bf16_round(r["out_tokens"]) if meta["dtype"] == "bf16" else r["out_tokens"].astype(np.float32).astype(np.float64)
+    g = gpu["tokens"][a:b].astype(np.float64)
+    err = np.abs(g - ref)
+    bound = %(atol)r + %(rtol)r * np.abs(ref)
+    ok_t &= bool((err <= bound).all())
+    if err.size:
+        worst = max(worst, float((err / bound).max()))
+        maxerr = max(maxerr, float(err.max()))
+    rows += b - a
+print(json.dumps({"seconds": secs, "frames": frames, "parity": {
+    "videos": len(videos), "rows": int(rows), "budgets_equal": ok_b, "index_equal": ok_i,
+    "tokens_within_tolerance": ok_t, "max_abs_err": maxerr, "worst_err_over_bound": worst,
+    "tolerance": "|g - o| <= %(atol)r + %(rtol)r |o|"}}))
+"""
+
+_PARALLEL_CODE = r"""
+import json, os, sys, time
+sys.path.insert(0, %(root)r)
+import numpy as np
+from oracle.parallel import condense_parallel, condense_videos_parallel, spawn_pool
+
+d = %(dir)r
+meta = json.load(open(d + "/meta.json"))
+Qs = [np.load(d + "/q%%d.npy" %% v) for v in range(meta["V"])]
+n = os.cpu_count()
+pool = spawn_pool(n)
+try:
+    pool.map(abs, range(n))                     # workers up before the clock starts
+    if meta["batch"]:
+        t = time.perf_counter()
+        condense_videos_parallel(d + "/x.npy", Qs, meta["ratios"], pool)
+        dt = time.perf_counter() - t
+    else:
+        bits = np.load(d + "/x.npy")
+        t = time.perf_counter()
+        condense_parallel(bits, Qs[0], meta["ratios"][0], n, pool=pool)
+        dt = time.perf_counter() - t
+finally:
+    pool.terminate()
+print(json.dumps({"seconds": dt, "frames": meta["frames"], "cores": n}))
+"""
+
+
+def _oracle_env():
+    return dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1",
+                CUDA_VISIBLE_DEVICES="")
+
+
+def write_inputs(d, w, Xh, Qh, gpu=None):
+    """The step's host inputs (and optionally the GPU's outputs) for the
+    oracle legs, in directory d: x.npy (bf16 bit patterns or f32), q<v>.npy
+    (fp64), meta.json, gpu.npz."""
+    import numpy as np
+    import torch
+    x = Xh.view(torch.int16).numpy().view(np.uint16) if Xh.dtype == torch.bfloat16 else Xh.numpy()
+    np.save(os.path.join(d, "x.npy"), x)
+    q0 = 0
+    for v, s in enumerate(w.specs):
+        np.save(os.path.join(d, f"q{v}.npy"), Qh[q0:q0 + s.Lq].double().numpy())
+        q0 += s.Lq
+    rows = [0]
+    for s in w.specs:
+        rows.append(rows[-1] + int(round_half_away(s.ratio * s.T * s.H * s.W)))
+    meta = {"V": len(w.specs), "batch": w.batch, "dtype": w.dtype, "ratios": [s.ratio for s in w.specs],
+            "row_offsets": rows, "frames": w.frames, "videos": list(range(len(w.specs)))}
+    if gpu is not None:
+        tok, idx, bud = gpu
+        np.savez(os.path.join(d, "gpu.npz"), tokens=tok.float().numpy(), index=idx.numpy(),
+                 budgets=bud.reshape(len(w.specs), -1).numpy())
+    return meta
+
+
+def round_half_away(x):
+    import math
+    return math.floor(x + 0.5)
+
+
+def cpu_baseline(d, meta, w):
+    """The oracle, as it stands, on one host core, on the bench's own input
+    (the tensor the GPU condensed): the whole video, or for the serving batch
+    the first videos (a bounded sample, ~15 s).  Also checks the GPU's outputs
+    of the timed step against the oracle's on that sample."""
+    meta = dict(meta)
+    if w.batch:
+        meta["videos"] = list(range(BATCH_CPU_VIDEOS))
+    with open(os.path.join(d, "meta.json"), "w") as f:
+        json.dump(meta, f)
+    code = _BASELINE_CODE % {"root": ROOT, "dir": d, "atol": TOK_ATOL, "rtol": TOK_RTOL}
+    res = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=_oracle_env(),
+                         timeout=1200)
     if res.returncode != 0:
-        return {"value": None, "unit": UNIT, "cores": 1, "kind": "oracle", "error": res.stderr[-400:]}
+        return {"value": None, "unit": UNIT, "cores": 1, "kind": "oracle", "error": res.stderr[-400:]}, None
     r = json.loads(res.stdout.strip().splitlines()[-1])
-    return {"value": r["frames"] / r["seconds"], "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"first {frames} frames of the workload recipe ({spec.H}x{spec.W}x{spec.D} "
-                      f"{spec.dtype}, Lq={spec.Lq}, ratio={spec.ratio}) condensed by the fp64 oracle",
-            "seconds": r["seconds"]}
+    sample = (f"the whole {w.T}-frame video the GPU condensed ({w.H}x{w.W}x{w.D} {w.dtype}), fp64 oracle"
+              if not w.batch else
+              f"the first {BATCH_CPU_VIDEOS} of the {len(w.specs)} videos the GPU condensed "
+              f"({w.T} frames of {w.H}x{w.W}x{w.D} {w.dtype} each), fp64 oracle")
+    return ({"value": r["frames"] / r["seconds"], "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample,
+             "seconds": r["seconds"]}, r["parity"])
 
 
-def cpu_baseline_parallel(spec, frames):
-    """The oracle's per-frame steps spread over every host core (spawned
-    processes, frames sharing one block of shared memory), the coupling steps
-    in the parent: the second CPU baseline.  Same video as cpu_baseline."""
-    code = (
-        "import json,os,sys,time; sys.path.insert(0, %r)\n"
-        "import numpy as np, torch, workload as wl\n"
-        "from oracle.parallel import condense_parallel\n"
-        "s = wl.VideoSpec(T=%d, H=%d, W=%d, D=%d, dtype=%r, Lq=%d, ratio=%r, ar=%r, cuts=%d, seed=%d)\n"
-        "X, Q, _ = wl.make_video(s)\n"
-        "bits, q = X.view(torch.int16).numpy().view(np.uint16), Q.double().numpy()\n"
-        "n = os.cpu_count()\n"
-        "t = time.perf_counter(); condense_parallel(bits, q, s.ratio, n); dt = time.perf_counter() - t\n"
-        "print(json.dumps({'seconds': dt, 'frames': s.T, 'cores': n}))\n"
-    ) % (ROOT, frames, spec.H, spec.W, spec.D, spec.dtype, spec.Lq, spec.ratio, spec.ar,
-         max(1, spec.cuts * frames // spec.T), spec.seed)
-    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1",
-               CUDA_VISIBLE_DEVICES="")
-    if spec.dtype != "bf16":
+def cpu_baseline_parallel(d, meta, w):
+    """The second CPU baseline: the oracle's independent steps over a pool of
+    spawned processes, one per host core (frames of the video, or whole
+    videos of the batch), on the same input as cpu_baseline."""
+    if w.dtype != "bf16":
         return None
-    res = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=900)
+    with open(os.path.join(d, "meta.json"), "w") as f:
+        json.dump(meta, f)
+    code = _PARALLEL_CODE % {"root": ROOT, "dir": d}
+    res = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=_oracle_env(),
+                         timeout=1200)
     if res.returncode != 0:
-        return {"value": None, "unit": UNIT, "kind": "oracle, frames over a process pool", "error": res.stderr[-400:]}
+        return {"value": None, "unit": UNIT, "kind": "oracle over a process pool", "error": res.stderr[-400:]}
     r = json.loads(res.stdout.strip().splitlines()[-1])
+    what = "videos" if w.batch else "frames"
     return {"value": r["frames"] / r["seconds"], "unit": UNIT, "cores": r["cores"],
-            "kind": "oracle, per-frame steps over a process pool (one process per core)",
-            "sample": f"the same {frames}-frame video as cpu_baseline", "seconds": r["seconds"]}
+            "kind": f"oracle, {what} over a process pool (one process per core)",
+            "sample": f"the whole workload the GPU condensed ({w.frames} frames)", "seconds": r["seconds"]}
 
 
-def run_reference(args, spec, world, rank):
-    """The oracle, timed on the host cores, on a bounded sample per step."""
+def run_reference(args, w, world, rank):
+    """The oracle on the host cores, one whole workload per step: the frames
+    of the video (or the videos of the batch) spread over one spawned process
+    per core, as `oracle/parallel.py` drives it; the fp32 workload (16 small
+    frames) on one core."""
     if rank != 0:
         return
+    import tempfile
+
+    import numpy as np
     os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")
     import oracle as O
-    import workload as wl
-    frames = REF_SAMPLE_FRAMES
-    s = wl.VideoSpec(**{**spec.__dict__, "T": frames, "cuts": max(1, spec.cuts * frames // spec.T)})
-    X, Q, _ = wl.make_video(s)
-    x, q = X.double().numpy(), Q.double().numpy()
-    for _ in range(args.warmup):
-        O.condense(x, q, s.ratio)
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        O.condense(x, q, s.ratio)
-    dt = time.perf_counter() - t0
-    value = frames * args.steps / dt
-    sample = f"{frames}-frame video per step ({spec.H}x{spec.W}x{spec.D} {spec.dtype}, same recipe), fp64 oracle"
+    from oracle.parallel import condense_parallel, condense_videos_parallel, spawn_pool
+    Xh, Qh = draw_inputs(w)
+    n = os.cpu_count() or 1
+    Qs, q0 = [], 0
+    for s in w.specs:
+        Qs.append(Qh[q0:q0 + s.Lq].double().numpy())
+        q0 += s.Lq
+    with tempfile.TemporaryDirectory() as d:
+        pool = None
+        if w.dtype == "f32":
+            x = Xh.double().numpy()
+            cores, kind = 1, "oracle (one core)"
+
+            def step():
+                O.condense(x, Qs[0], w.specs[0].ratio)
+        else:
+            import torch
+            pool = spawn_pool(n)
+            pool.map(abs, range(n))
+            cores = n
+            bits = Xh.view(torch.int16).numpy().view(np.uint16)
+            if w.batch:
+                path = os.path.join(d, "x.npy")
+                np.save(path, bits)
+                kind = "oracle, videos over a process pool (one process per core)"
+
+                def step():
+                    condense_videos_parallel(path, Qs, [s.ratio for s in w.specs], pool)
+            else:
+                kind = "oracle, frames over a process pool (one process per core)"
+
+                def step():
+                    condense_parallel(bits, Qs[0], w.specs[0].ratio, n, pool=pool)
+        try:
+            for _ in range(args.warmup):
+                step()
+            t0 = time.perf_counter()
+            for _ in range(args.steps):
+                step()
+            dt = time.perf_counter() - t0
+        finally:
+            if pool is not None:
+                pool.terminate()
+    value = w.frames * args.steps / dt
+    sample = f"the whole workload per step ({w.frames} frames, the same recipe and seeds as the GPU arm)"
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * dt / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": config_dict(spec, args.config),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "data": "synthetic", "config": config_dict(w),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": kind, "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 
 
-def algorithmic_bytes(spec, budgets, B, K_pad):
-    """Bytes each kernel must move per launch (one video)."""
-    esz = 2 if spec.dtype == "bf16" else 4
-    N, D, T = spec.H * spec.W, spec.D, spec.T
+def algorithmic_bytes(w, budgets, rows):
+    """Bytes each kernel must move per launch (the whole workload).  budgets:
+    [V][T] per-frame token counts; rows: total condensed rows."""
+    esz = 2 if w.dtype == "bf16" else 4
+    N, D, T, V = w.H * w.W, w.D, w.T, len(w.specs)
+    K_pad = (N + 31) // 32 * 32
     active = int((budgets > 0).sum())
     return {
-        "relevance": T * N * D * esz + T * N * 4,
-        "condense": active * N * D * esz + B * D * esz + B * K_pad * 4,
+        "relevance": V * T * N * D * esz + V * T * N * 4,
+        "condense": active * N * D * esz + rows * D * esz + rows * K_pad * 4,
         # operator rows written (bf16 hi + lo) and the pooled gate of each
         # active frame read (db4: (H + 7) / 2 x (W + 7) / 2)
-        "spatial": B * K_pad * 4 + active * ((spec.H + 7) // 2) * ((spec.W + 7) // 2) * 4,
+        "spatial": rows * K_pad * 4 + active * ((w.H + 7) // 2) * ((w.W + 7) // 2) * 4,
         "frame_stats": None, "query_pool": None, "temporal": None,
     }
 
 
-def run_ours(args, spec, world, rank, local):
+def run_ours(args, w, world, rank, local):
+    import tempfile
+
     import torch
     import torch.distributed as dist
 
     import paper_2607_23265_gb300.build as build
     build.build()
     import paper_2607_23265_gb300.wavezip as wz
-    import workload as wl
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
-    X, Q, _ = wl.make_video(replica_spec(spec, rank), device=dev)
-    T, H, W, D = X.shape
-    B = wz.wz_budget_size(T, H, W, spec.ratio)
-    K_pad = (H * W + 31) // 32 * 32
-    ws = torch.empty((wz.wz_condense_workspace_size(T, H, W, D, wz._dtype_code(X), spec.ratio),),
-                     dtype=torch.uint8, device=dev)
+    Xh, Qh = draw_inputs(w)                       # host tensors (the recipe's CPU draw)
+    X, Q = Xh.to(dev), Qh.to(dev)
+    ratios = [s.ratio for s in w.specs]
+    Lqs = [s.Lq for s in w.specs]
+    if w.batch:
+        rows, _ = wz.wz_batch_rows(len(w.specs), w.T, w.H, w.W, ratios)
+        wsb = wz.wz_batch_workspace_size(len(w.specs), w.T, w.H, w.W, w.D, wz._dtype_code(X), ratios)
+    else:
+        rows = wz.wz_budget_size(w.T, w.H, w.W, ratios[0])
+        wsb = wz.wz_condense_workspace_size(w.T, w.H, w.W, w.D, wz._dtype_code(X), ratios[0])
+    ws = torch.empty((wsb,), dtype=torch.uint8, device=dev)
     status = torch.zeros((1,), dtype=torch.int32, device=dev)
-    tokens = torch.empty((B, D), dtype=X.dtype, device=dev)
-    index = torch.empty((B, 3), dtype=torch.int32, device=dev)
+    tokens = torch.empty((rows, w.D), dtype=X.dtype, device=dev)
+    index = torch.empty((rows, 3), dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
+    flush_l2 = X.numel() * X.element_size() <= L2_BYTES
 
     def step(events=None):
-        return wz.wz_condense_ex(X, Q, spec.ratio, workspace=ws, out_tokens=tokens, out_index=index,
+        if w.batch:
+            return wz.wz_condense_batch(X, Q, Lqs, ratios, workspace=ws, out_tokens=tokens, out_index=index,
+                                        device_status=status, path=args.path, kernel_events=events)
+        return wz.wz_condense_ex(X, Q, ratios[0], workspace=ws, out_tokens=tokens, out_index=index,
                                  device_status=status, path=args.path, kernel_events=events)
 
     def barrier():
@@ -475,14 +690,31 @@ def run_ours(args, spec, world, rank, local):
     time.sleep(0.4)
     barrier()
     # timed region: K plain steps (consecutive launches overlap through
-    # programmatic dependent launch)
+    # programmatic dependent launch).  Inputs smaller than L2 would stay in
+    # it from one step to the next, so for them every step is timed alone
+    # with L2 flushed (a 512 MB buffer written) before it.
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
-    t0.record(stream)
-    for k in range(args.steps):
-        res = step()
-    t1.record(stream)
-    barrier()
+    if flush_l2:
+        flush = torch.empty((L2_FLUSH_BYTES,), dtype=torch.uint8, device=dev)
+        marks = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                 for _ in range(args.steps)]
+        t0.record(stream)
+        for k in range(args.steps):
+            flush.zero_()
+            marks[k][0].record(stream)
+            res = step()
+            marks[k][1].record(stream)
+        t1.record(stream)
+        barrier()
+        step_ms = sum(a.elapsed_time(b) for a, b in marks) / args.steps
+    else:
+        t0.record(stream)
+        for k in range(args.steps):
+            res = step()
+        t1.record(stream)
+        barrier()
+        step_ms = t0.elapsed_time(t1) / args.steps
     # the same K steps again with an event pair around every kernel: the
     # per-kernel durations (an event between two launches removes their
     # overlap, so this pass is slower per step and reported separately)
@@ -494,23 +726,38 @@ def run_ours(args, spec, world, rank, local):
     t3.record(stream)
     barrier()
     clocks = sampler.stop()
-    ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world, dev)
+    ms = max_over_ranks(step_ms, world, dev)
     ms_instr = max_over_ranks(t2.elapsed_time(t3) / args.steps, world, dev)
     kern_ms = {name: statistics.mean(evs[k][2 * j].elapsed_time(evs[k][2 * j + 1]) for k in range(args.steps))
                for j, name in enumerate(KERNELS)}
     if int(status.item()) != 0:
         raise RuntimeError(f"device status {int(status.item())}: a bounded wait timed out")
     budgets = res["budgets"].cpu()
+    gpu_out = (tokens.cpu(), index.cpu(), budgets)
 
     # end to end through the public API: pinned host buffers in, results out
-    Xh = X.cpu().pin_memory()
-    Qh = Q.cpu().pin_memory()
-    tok_h = torch.empty((B, D), dtype=X.dtype).pin_memory()
-    idx_h = torch.empty((B, 3), dtype=torch.int32).pin_memory()
+    Xp = Xh.pin_memory()
+    Qp = Qh.pin_memory()
+    tok_h = torch.empty((rows, w.D), dtype=X.dtype).pin_memory()
+    idx_h = torch.empty((rows, 3), dtype=torch.int32).pin_memory()
+    if w.batch:
+        Xd = torch.empty_like(X)
+        Qd = torch.empty_like(Q)
 
-    def e2e_step():
-        # the C-ABI call on host buffers: copies in, the pass, copies out, all on the stream
-        wz.wz_condense_host(Xh, Qh, spec.ratio, tok_h, idx_h, path=args.path)
+        def e2e_step():
+            # copies in, the batch call, copies out, all on the stream
+            Xd.copy_(Xp, non_blocking=True)
+            Qd.copy_(Qp, non_blocking=True)
+            wz.wz_condense_batch(Xd, Qd, Lqs, ratios, workspace=ws, out_tokens=tokens, out_index=index,
+                                 device_status=status, path=args.path)
+            tok_h.copy_(tokens, non_blocking=True)
+            idx_h.copy_(index, non_blocking=True)
+        e2e_path = "pinned host -> device copies, wz_condense_batch, device -> pinned host copies on one stream"
+    else:
+        def e2e_step():
+            # the C-ABI call on host buffers: copies in, the pass, copies out, all on the stream
+            wz.wz_condense_host(Xp, Qp, ratios[0], tok_h, idx_h, path=args.path)
+        e2e_path = "wz_condense_host (C ABI, pinned host buffers)"
 
     e2e_step()
     barrier()
@@ -526,16 +773,16 @@ def run_ours(args, spec, world, rank, local):
     # the same step captured once in a CUDA graph and replayed (launches of the
     # six kernels submitted as one graph)
     graph = None
-    if args.graph_steps > 0:
+    if args.graph_steps > 0 and not w.batch:
         gs = torch.cuda.Stream(dev)
         gs.wait_stream(stream)
         with torch.cuda.stream(gs):
-            wz.wz_condense_ex(X, Q, spec.ratio, workspace=ws, out_tokens=tokens, out_index=index,
+            wz.wz_condense_ex(X, Q, ratios[0], workspace=ws, out_tokens=tokens, out_index=index,
                               device_status=status, path=args.path, stream=gs)
         torch.cuda.synchronize(dev)
         cg = torch.cuda.CUDAGraph()
         with torch.cuda.graph(cg, stream=gs):
-            wz.wz_condense_ex(X, Q, spec.ratio, workspace=ws, out_tokens=tokens, out_index=index,
+            wz.wz_condense_ex(X, Q, ratios[0], workspace=ws, out_tokens=tokens, out_index=index,
                               device_status=status, path=args.path, stream=gs)
         for _ in range(3):
             cg.replay()
@@ -547,43 +794,46 @@ def run_ours(args, spec, world, rank, local):
         g1.record(stream)
         barrier()
         gms = max_over_ranks(g0.elapsed_time(g1) / args.graph_steps, world, dev)
-        graph = {"ms_per_step": round(gms, 5), "value": job_value(T, world, gms), "unit": UNIT,
+        graph = {"ms_per_step": round(gms, 5), "value": job_value(w.frames, world, gms), "unit": UNIT,
                  "steps": args.graph_steps}
         del cg
 
-    projector = time_projector(wz, tokens, args.projector_steps, dev) if args.projector_steps > 0 else None
-    maxsim = time_maxsim(wz, X, Q, spec.ratio, ws, status, args.maxsim_steps, dev) \
-        if args.maxsim_steps > 0 and X.dtype == torch.bfloat16 and D % 64 == 0 else None
-    variants = time_variants(wz, X, Q, spec.ratio, ws, status, args.variant_steps, dev) \
-        if args.variant_steps > 0 else None
+    single_bf16 = not w.batch and X.dtype == torch.bfloat16
+    projector = time_projector(wz, tokens, args.projector_steps, dev) \
+        if args.projector_steps > 0 and single_bf16 and w.D % 64 == 0 else None
+    maxsim = time_maxsim(wz, X, Q, ratios[0], ws, status, args.maxsim_steps, dev) \
+        if args.maxsim_steps > 0 and single_bf16 and w.D % 64 == 0 else None
+    variants = time_variants(wz, X, Q, ratios[0], ws, status, args.variant_steps, dev) \
+        if args.variant_steps > 0 and not w.batch else None
 
     if rank == 0:
         peak, peak_kind = measured_peak()
-        ab = algorithmic_bytes(spec, budgets, B, K_pad)
+        ab = algorithmic_bytes(w, budgets.reshape(len(w.specs), -1), rows)
         dominant = max(KERNELS, key=lambda k: kern_ms[k])
         kern = {}
         for k in KERNELS:
             entry = {"ms": round(kern_ms[k], 5), "share": round(kern_ms[k] / sum(kern_ms.values()), 4)}
             if ab.get(k):
+                entry["bytes"] = ab[k]
                 entry["gb_s"] = round(ab[k] / (kern_ms[k] * 1e-3) / 1e9, 1)
+                entry["frac"] = round(ab[k] / (kern_ms[k] * 1e-3) / 1e9 / peak, 4)
             kern[k] = entry
         bytes_dom = ab.get(dominant)
         achieved = bytes_dom / (kern_ms[dominant] * 1e-3) / 1e9 if bytes_dom else None
-        frames = T * world
         out = {
-            "metric": METRIC, "value": job_value(T, world, ms), "unit": UNIT, "n_gpus": world,
+            "metric": METRIC, "value": job_value(w.frames, world, ms), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-            "data": "synthetic", "config": config_dict(spec, args.config),
-            "tokens_out_per_s": B * world / (ms * 1e-3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+            "data": "synthetic", "config": config_dict(w),
+            "tokens_out_per_s": rows * world / (ms * 1e-3),
             "roofline": {"bound": "hbm", "kernel": dominant, "achieved": achieved, "peak": peak,
                          "unit": "GB/s", "frac": achieved / peak if achieved else None,
-                         "traffic": recorded_traffic(dominant), "peak_source": peak_kind,
+                         "traffic": recorded_traffic(dominant, w.name), "peak_source": peak_kind,
                          "frac_of_8000": achieved / 8000.0 if achieved else None},
             "kernels": kern,
             "ms_per_step_with_kernel_events": ms_instr,
-            "active_frames": int((budgets > 0).sum()), "budget_B": B,
-            "e2e": {"value": job_value(T, world, e2e_ms), "unit": UNIT,
+            "active_frames": int((budgets > 0).sum()), "rows": rows,
+            "e2e": {"value": job_value(w.frames, world, e2e_ms), "unit": UNIT, "path": e2e_path,
                     "h2d_bytes_per_step": X.numel() * X.element_size() + Q.numel() * Q.element_size(),
                     "d2h_bytes_per_step": tokens.numel() * tokens.element_size() + index.numel() * 4},
             "clocks": clocks,
@@ -594,8 +844,10 @@ def run_ours(args, spec, world, rank, local):
             "variants": variants,
         }
         if world == 1 and not args.no_cpu_baseline:
-            out["cpu_baseline"] = cpu_baseline(spec, CPU_SAMPLE_FRAMES)
-            out["cpu_baseline_parallel"] = cpu_baseline_parallel(spec, CPU_SAMPLE_FRAMES)
+            with tempfile.TemporaryDirectory() as d:
+                meta = write_inputs(d, w, Xh, Qh, gpu_out)
+                out["cpu_baseline"], out["parity"] = cpu_baseline(d, meta, w)
+                out["cpu_baseline_parallel"] = cpu_baseline_parallel(d, meta, w)
         print(json.dumps(out))
     if world > 1:
         dist.destroy_process_group()
@@ -604,12 +856,11 @@ def run_ours(args, spec, world, rank, local):
 def main():
     args = parse()
     world, rank, local = dist_setup()
-    import workload as wl
-    spec = wl.CONFIGS[args.config]
+    w = workload(args.config, rank)
     if args.impl == "reference":
-        run_reference(args, spec, world, rank)
+        run_reference(args, w, world, rank)
     else:
-        run_ours(args, spec, world, rank, local)
+        run_ours(args, w, world, rank, local)
 
 
 if __name__ == "__main__":

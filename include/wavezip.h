@@ -275,11 +275,16 @@ WZ_API int wz_condense_batch(const wz_batch_args *a);
  * frame_scores [T] f32: r_t = cos(mean_n u_{t,n}, u_q).
  * frame_mean   [T][D] f32: the pooled feature v_bar_t (nullable).
  * workspace    >= wz_relevance_workspace_size() bytes, or NULL.
+ * device_status [1] int32, nullable: a bounded wait of the relevance pass
+ *              that gives up ORs a nonzero code into it (the caller zeroes
+ *              it; the bounds-checked build adds WZ_STATUS_BOUNDS); without
+ *              it the workspace's own word, zeroed on `stream`, takes the
+ *              code and the failure is not reported.
  */
 WZ_API int wz_relevance(const void *features, int T, int H, int W, int D, int dtype,
                  const void *query, int Lq, float *token_scores, float *frame_scores,
                  float *frame_mean, void *workspace, size_t workspace_bytes,
-                 wz_stream_t stream);
+                 int32_t *device_status, wz_stream_t stream);
 
 WZ_API size_t wz_relevance_workspace_size(int T, int H, int W, int D);
 
@@ -295,20 +300,30 @@ WZ_API size_t wz_relevance_workspace_size(int T, int H, int W, int D);
  * array of WZ_STATIC_SCRATCH_BYTES compiled into the library, which every GPU
  * that loads the library keeps until the process exits.
  *   - No cudaMalloc, cudaFree or other allocating call is made.
+ *   - The array used is the one of the current device: `stream` must belong
+ *     to the current device, and so must every pointer.
  *   - The first call on a device looks the array's device address up
  *     (cudaGetSymbolAddress) with that device current; make that first call
  *     before any stream capture.
  *   - Sizes whose sums do not fit the array return WZ_ERR_WORKSPACE before
- *     anything is enqueued (about (2*SMs + T) * D * 4 bytes are needed, e.g.
- *     up to T = 256 frames at D = 3584 on a GB300).
- *   - Every call shares the one array and keeps no state between calls
- *     (nothing in it must start at zero), so calls that overlap on the GPU
- *     (other streams, other host threads) race: serialise them.
+ *     anything is enqueued.  The sums take, each rounded up to 256 bytes,
+ *     12*D + 32 (query mean in f32 and f64, per-call parameters), (G1 + T)*D*4
+ *     (column partials), 32*T (per-frame statistics) and 16 (status word),
+ *     where G1 = min(2048, ceil(T*H*W/16), SMs x resident relevance CTAs per
+ *     SM) is the relevance grid (152 on a GB300 at D = 3584: about T <= 1000
+ *     frames fit at that width).
+ *   - device_status [1] int32, nullable: as for wz_relevance.  Without it the
+ *     array's own status word is zeroed on `stream` (cudaMemsetAsync) and
+ *     takes the bits, so a timed-out wait is not reported.
+ *   - Every call shares the one array; apart from that status word nothing
+ *     in it must start at zero and no state passes from one call to the next,
+ *     but calls that overlap on the GPU (other streams, other host threads)
+ *     race on it: serialise them.
  */
 #define WZ_STATIC_SCRATCH_BYTES (16u << 20)
 WZ_API int wz_relevance_static(const void *features, int T, int H, int W, int D, int dtype,
                                const void *query, int Lq, float *token_scores, float *frame_scores,
-                               float *frame_mean, wz_stream_t stream);
+                               float *frame_mean, int32_t *device_status, wz_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
 /* Projector P (Eq. 17): the condensed tokens through the model's MLP         */

@@ -620,12 +620,12 @@ size_t wz_relevance_workspace_size(int T, int H, int W, int D) {
 
 int wz_relevance(const void *features, int T, int H, int W, int D, int dtype, const void *query,
                  int Lq, float *token_scores, float *frame_scores, float *frame_mean,
-                 void *workspace, size_t workspace_bytes, wz_stream_t stream) {
+                 void *workspace, size_t workspace_bytes, int32_t *device_status, wz_stream_t stream) {
     int st = check_sizes(1, T, H, W, D, dtype);
     if (st != WZ_OK) return st;
     if (!features || !query || !token_scores || !frame_scores || Lq < 1) return WZ_ERR_INVALID_ARG;
     if (!aligned(features, 16) || !aligned(query, 16) || !aligned(token_scores, 4) ||
-        !aligned(frame_scores, 4) || (frame_mean && !aligned(frame_mean, 4)))
+        !aligned(frame_scores, 4) || (frame_mean && !aligned(frame_mean, 4)) || !aligned(device_status, 4))
         return WZ_ERR_INVALID_ARG;
     const Shape s = make_shape(1, T, H, W, D, dtype, 2, nullptr);
     const Layout L = make_layout(s, false, false);
@@ -647,6 +647,10 @@ int wz_relevance(const void *features, int T, int H, int W, int D, int dtype, co
     c.L1 = ((int64_t)T * s.N + c.G1 - 1) / c.G1;
     VideoPar par{0, Lq, 0, 0, 0};
     const cudaStream_t cs = (cudaStream_t)stream;
+    // a bounded wait that gives up reports to the caller's status word, else
+    // to the workspace's, which starts each call at zero
+    if (device_status) c.status = device_status;
+    else WZ_CUDA(cudaMemsetAsync(c.status, 0, sizeof(int), cs));
     WZ_CUDA(launch_query_pool(c, &par, cs));
     WZ_CUDA(launch_relevance_pass(c, cs));
     WZ_CUDA(launch_frame_stats(c, cs));

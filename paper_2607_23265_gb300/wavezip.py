@@ -112,9 +112,9 @@ def _load(path: str = LIB_PATH):
         "wz_batch_rows": (i64, [i, i, i, i, C.POINTER(C.c_float), C.POINTER(C.c_int64)]),
         "wz_batch_workspace_size": (sz, [i, i, i, i, i, i, C.POINTER(C.c_float)]),
         "wz_condense_batch": (i, [C.POINTER(BatchArgs)]),
-        "wz_relevance": (i, [vp, i, i, i, i, i, vp, i, vp, vp, vp, vp, sz, vp]),
+        "wz_relevance": (i, [vp, i, i, i, i, i, vp, i, vp, vp, vp, vp, sz, vp, vp]),
         "wz_relevance_workspace_size": (sz, [i, i, i, i]),
-        "wz_relevance_static": (i, [vp, i, i, i, i, i, vp, i, vp, vp, vp, vp]),
+        "wz_relevance_static": (i, [vp, i, i, i, i, i, vp, i, vp, vp, vp, vp, vp]),
         "wz_project_workspace_size": (sz, [i64, i]),
         "wz_project": (i, [C.POINTER(ProjectArgs)]),
         "wz_dwt_len": (i, [i, i]),
@@ -293,8 +293,9 @@ def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios,
                       tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
                       temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1, relevance="mean",
                       wta_levels: int = 1, wsm_levels: int = 1, workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
-                      stream=None):
-    """wz_condense_batch: features [V,T,H,W,D], queries [sum Lq, D]."""
+                      device_status: torch.Tensor | None = None, kernel_events=None, stream=None):
+    """wz_condense_batch: features [V,T,H,W,D], queries [sum Lq, D].  Options as
+    for wz_condense_ex; kernel_events brackets each kernel of the whole batch."""
     features = _cuda_contig(features, "features")
     queries = _cuda_contig(queries, "queries")
     V, T, H, W, D = features.shape
@@ -324,6 +325,10 @@ def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios,
     a.out_budgets, a.out_count, a.out_relevance = budgets.data_ptr(), count.data_ptr(), rel.data_ptr()
     if workspace is not None:
         a.workspace, a.workspace_bytes = workspace.data_ptr(), workspace.numel() * workspace.element_size()
+    a.device_status = _ptr(device_status)
+    if kernel_events is not None:
+        handles = (C.c_void_p * (2 * NUM_KERNELS))(*[e.cuda_event for e in kernel_events])
+        a.kernel_events = handles
     a.stream = _stream(stream, dev)
     _check(_lib.wz_condense_batch(C.byref(a)), "wz_condense_batch")
     return {"tokens": tokens, "index": index, "budgets": budgets, "count": count, "relevance": rel,
@@ -340,8 +345,10 @@ def wz_batch_workspace_size(V, T, H, W, D, dtype, ratios) -> int:
 # --------------------------------------------------------------------------
 
 def wz_relevance(features: torch.Tensor, query: torch.Tensor, *, frame_mean: bool = False,
-                 workspace: torch.Tensor | None = None, stream=None):
-    """(token_scores [T,H*W], frame_scores [T], frame_mean [T,D] or None)."""
+                 workspace: torch.Tensor | None = None, device_status: torch.Tensor | None = None, stream=None):
+    """(token_scores [T,H*W], frame_scores [T], frame_mean [T,D] or None).
+    device_status: optional [1] int32 word that a bounded wait which gives up
+    ORs a nonzero code into (the caller zeroes it)."""
     features = _cuda_contig(features, "features")
     query = _cuda_contig(query, "query")
     T, H, W, D = features.shape
@@ -352,23 +359,33 @@ def wz_relevance(features: torch.Tensor, query: torch.Tensor, *, frame_mean: boo
     wsp, wsb = (workspace.data_ptr(), workspace.numel() * workspace.element_size()) if workspace is not None else (None, 0)
     st = _lib.wz_relevance(features.data_ptr(), T, H, W, D, _dtype_code(features), query.data_ptr(),
                            query.shape[0], ts.data_ptr(), fs.data_ptr(), _ptr(fm), wsp, wsb,
-                           _stream(stream, dev))
+                           _ptr(device_status), _stream(stream, dev))
     _check(st, "wz_relevance")
     return ts, fs, fm
 
 
-def wz_relevance_static(features: torch.Tensor, query: torch.Tensor, *, frame_mean: bool = False, stream=None):
+def wz_relevance_static(features: torch.Tensor, query: torch.Tensor, *, frame_mean: bool = False,
+                        out=None, device_status: torch.Tensor | None = None, stream=None):
     """wz_relevance_static: the scores of wz_relevance without any device allocation
-    (its sums live in a fixed array inside the library; see include/wavezip.h)."""
+    (its sums live in a fixed array inside the library; see include/wavezip.h).
+    out: optional (token_scores, frame_scores, frame_mean or None) tensors to
+    write, so that the call itself allocates nothing on the torch side either.
+    The call runs with the features' device current (the library picks the
+    fixed array of the current device)."""
     features = _cuda_contig(features, "features")
     query = _cuda_contig(query, "query")
     T, H, W, D = features.shape
     dev = features.device
-    ts = torch.empty((T, H * W), dtype=torch.float32, device=dev)
-    fs = torch.empty((T,), dtype=torch.float32, device=dev)
-    fm = torch.empty((T, D), dtype=torch.float32, device=dev) if frame_mean else None
-    st = _lib.wz_relevance_static(features.data_ptr(), T, H, W, D, _dtype_code(features), query.data_ptr(),
-                                  query.shape[0], ts.data_ptr(), fs.data_ptr(), _ptr(fm), _stream(stream, dev))
+    if out is None:
+        ts = torch.empty((T, H * W), dtype=torch.float32, device=dev)
+        fs = torch.empty((T,), dtype=torch.float32, device=dev)
+        fm = torch.empty((T, D), dtype=torch.float32, device=dev) if frame_mean else None
+    else:
+        ts, fs, fm = out
+    with torch.cuda.device(dev):
+        st = _lib.wz_relevance_static(features.data_ptr(), T, H, W, D, _dtype_code(features), query.data_ptr(),
+                                      query.shape[0], ts.data_ptr(), fs.data_ptr(), _ptr(fm), _ptr(device_status),
+                                      _stream(stream, dev))
     _check(st, "wz_relevance_static")
     return ts, fs, fm
 

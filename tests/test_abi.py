@@ -131,8 +131,9 @@ def test_simple_entry_point_errors(wz):
     lib = wz._lib
     assert lib.wz_condense(None, 4, 5, 6, 16, P, 3, 0.5, P, P, None) == -1
     assert lib.wz_condense(P, 4, 5, 6, 10, P, 3, 0.5, P, P, None) == -2
-    assert lib.wz_relevance(P, 4, 5, 6, 16, 0, P, 0, P, P, None, None, 0, None) == -1
-    assert lib.wz_relevance(P, 4, 5, 6, 12, 0, P, 2, P, P, None, None, 0, None) == -2
+    assert lib.wz_relevance(P, 4, 5, 6, 16, 0, P, 0, P, P, None, None, 0, None, None) == -1
+    assert lib.wz_relevance(P, 4, 5, 6, 12, 0, P, 2, P, P, None, None, 0, None, None) == -2
+    assert lib.wz_relevance(P, 4, 5, 6, 16, 0, P, 2, P, P, None, None, 0, P + 2, None) == -1   # misaligned status
     assert lib.wz_dwt1d(None, 3, 8, 4, 0, P, P, None) == -1
     assert lib.wz_dwt1d(P, 3, 8, 4, 7, P, P, None) == -1
     assert lib.wz_idwt1d(P, P, 3, 0, 4, P, None) == -1

@@ -25,17 +25,67 @@ def wz():
     return m
 
 
-def test_static_scores_match_the_workspace_entry_point_twice(wz):
-    cases = [wl.VideoSpec(T=24, H=13, W=13, D=512, Lq=9, seed=31),
-             wl.VideoSpec(T=40, H=16, W=16, D=896, Lq=3, seed=32)]
+def _same(got, ref):
+    for g, r in zip(got, ref):
+        if r is None:
+            assert g is None
+        else:
+            assert np.allclose(g.cpu().double().numpy(), r.cpu().double().numpy(), atol=2e-6, rtol=0)
+
+
+@pytest.mark.parametrize("dtype,frame_mean", [("bf16", True), ("bf16", False), ("f32", True)])
+def test_static_scores_match_the_workspace_entry_point_twice(wz, dtype, frame_mean):
+    cases = [wl.VideoSpec(T=24, H=13, W=13, D=512, Lq=9, dtype=dtype, seed=31),
+             wl.VideoSpec(T=40, H=16, W=16, D=896, Lq=3, dtype=dtype, seed=32)]
     for spec in cases:                      # two calls in a row, different sizes
         X, Q, _ = wl.make_video(spec)
         Xc, Qc = X.cuda(), Q.cuda()
-        got = wz.wz_relevance_static(Xc, Qc, frame_mean=True)
-        ref = wz.wz_relevance(Xc, Qc, frame_mean=True)
+        got = wz.wz_relevance_static(Xc, Qc, frame_mean=frame_mean)
+        ref = wz.wz_relevance(Xc, Qc, frame_mean=frame_mean)
         torch.cuda.synchronize()
-        for g, r in zip(got, ref):
-            assert np.allclose(g.cpu().double().numpy(), r.cpu().double().numpy(), atol=2e-6, rtol=0)
+        _same(got, ref)
+
+
+def test_static_call_allocates_no_device_memory(wz):
+    X, Q, _ = wl.make_video(wl.VideoSpec(T=16, H=13, W=13, D=512, Lq=5, seed=33))
+    Xc, Qc = X.cuda(), Q.cuda()
+    out = (torch.empty((16, 169), device="cuda"), torch.empty((16,), device="cuda"),
+           torch.empty((16, 512), device="cuda"))
+    status = torch.zeros((1,), dtype=torch.int32, device="cuda")
+    wz.wz_relevance_static(Xc, Qc, out=out, device_status=status)   # loads the kernels, looks the array up
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(3):
+        wz.wz_relevance_static(Xc, Qc, out=out, device_status=status)
+        wz.wz_relevance_static(Xc, Qc, out=out)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert int(status.item()) == 0
+    _same(out, wz.wz_relevance(Xc, Qc, frame_mean=True))
+
+
+def test_static_status_word_and_checked_build(wz):
+    """Two calls report no failure in the caller's status word; the
+    bounds-checked build (index tests on every global write, its own fixed
+    array) sets no bit and gives the same scores, with or without a caller
+    status word."""
+    X, Q, _ = wl.make_video(wl.VideoSpec(T=20, H=13, W=13, D=512, Lq=4, seed=34))
+    Xc, Qc = X.cuda(), Q.cuda()
+    status = torch.zeros((1,), dtype=torch.int32, device="cuda")
+    first = wz.wz_relevance_static(Xc, Qc, frame_mean=True, device_status=status)
+    second = wz.wz_relevance_static(Xc, Qc, frame_mean=True, device_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    for x, y in zip(first, second):
+        assert torch.equal(x, y)
+    with wz.checked_library():
+        cst = torch.zeros((1,), dtype=torch.int32, device="cuda")
+        a = wz.wz_relevance_static(Xc, Qc, frame_mean=True, device_status=cst)
+        b = wz.wz_relevance_static(Xc, Qc, frame_mean=True)
+        torch.cuda.synchronize()
+    assert int(cst.item()) == 0
+    _same(a, first)
+    _same(b, first)
 
 
 def test_static_rejects_sizes_beyond_its_array(wz):
