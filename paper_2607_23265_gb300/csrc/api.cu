@@ -36,7 +36,7 @@ struct Nvtx {
 // Sub-buffer offsets of one call's workspace.
 struct Layout {
     size_t qbar32, qbar64, vpar, a, part, fr, list, n, off, woff, hw, prod,
-        units, ucount, ustart, stab, drange, gate, qnorm, qhl, status, snext, Wop, total;
+        units, ucount, ustart, stab, drange, gate, krange, qnorm, qhl, status, snext, Wop, total;
 };
 
 struct Shape {
@@ -74,6 +74,7 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.qnorm = take((size_t)s.V * WZ_MAX_LQ_MAXSIM * 4);
     L.qhl = take((size_t)2 * WZ_MAX_LQ_MAXSIM * s.D * 2);
     L.gate = with_operator ? take(VT * (size_t)gate_floats(s.H, s.W, kMaxTaps, kMaxLevels) * 4) : 0;
+    L.krange = with_operator ? take(VT * (size_t)((s.N + kColBlock - 1) / kColBlock) * (s.K_pad / 32) * 2) : 0;
     L.status = take(16);
     L.snext = take(16);
     L.Wop = with_operator ? take((size_t)std::max<int64_t>(s.rows_total, s.w_rows) * s.K_pad * 4) : 0;
@@ -214,6 +215,10 @@ void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.status = reinterpret_cast<int *>(ws + L.status);
     c.spatial_next = reinterpret_cast<int *>(ws + L.snext);
     if (L.Wop) c.Wop = ws + L.Wop;
+    if (L.krange) {
+        c.krange = reinterpret_cast<uint16_t *>(ws + L.krange);
+        c.krange_nblk = (s.N + kColBlock - 1) / kColBlock;
+    }
 }
 
 // Scratch either from the caller or from the stream-ordered allocator.

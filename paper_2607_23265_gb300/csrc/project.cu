@@ -220,6 +220,8 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
                     ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)c0, hi);
                     ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)(p.Lqp + c0), lo);
                     ptx::tmem_ld_wait();
+                    ptx::reg_fence16(hi);
+                    ptx::reg_fence16(lo);
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
                         if (c0 + j < p.Lq) best = fmaxf(best, __uint_as_float(hi[j]) + __uint_as_float(lo[j]));
@@ -234,6 +236,8 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
                 ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)c0, v0);
                 ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)c0 + 16, v1);
                 ptx::tmem_ld_wait();
+                ptx::reg_fence16(v0);
+                ptx::reg_fence16(v1);
                 float x[32];
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {

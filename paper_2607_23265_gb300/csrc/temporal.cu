@@ -200,10 +200,14 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     pdl_wait();
     pdl_trigger();
     if ((int)blockIdx.x == c.V) {
-        // the extra CTA: the spatial kernel's row counter and, with several
-        // WSM levels, the multi-level tables of the spatial operator (the
-        // single-level kernel forms its tables itself)
-        if (threadIdx.x == 0 && c.spatial_next) *c.spatial_next = 0;
+        // the extra CTA: the spatial kernel's row counter, the condensation's
+        // unit counter and, with several WSM levels, the multi-level tables
+        // of the spatial operator (the single-level kernel forms its tables
+        // itself)
+        if (threadIdx.x == 0 && c.spatial_next) {
+            c.spatial_next[0] = 0;
+            c.spatial_next[1] = 0;
+        }
         if (c.wsm_levels > 1) build_ml_tables(c);
         return;
     }

@@ -13,6 +13,7 @@ constexpr int kMaxTaps = 20;          // Daubechies order <= 10
 constexpr int kMaxLevels = WZ_MAX_LEVELS;   // decomposition levels of the WTA / WSM
 constexpr int kG1Max = 2048;          // relevance-pass CTAs (upper bound)
 constexpr int kColBlock = 256;        // output tokens per tensor-core unit
+constexpr int kUnitRanged = 1 << 28;  // unit record flag: per-chunk operator row ranges in Ctx::krange
 constexpr int kTileC = 128;           // channels per tensor-core M tile
 constexpr int kTmemCols = 512;        // tensor-memory columns of one condensation CTA
 
@@ -63,8 +64,12 @@ struct Ctx {
     float *gate;          // [V*T][hp*wp] gate G of each frame (Eq. 12)
     void *Wop;            // operator: tensor path bf16 hi then lo in the tiled
                           // layout of tile_index(), CUDA-core path f32 [rows][K_pad]
+    uint16_t *krange;     // [V*T][krange_nblk][K_pad/32] operator rows of a 256-token block that
+                          // reach a 32-token chunk: [16*(r & 0xff), 16*(r >> 8)) (tensor path)
+    int krange_nblk;      // blocks of 256 tokens per frame: ceil(H*W / 256)
     int *status;          // device status word (bounded waits)
-    int *spatial_next;    // next (frame, grid row) of the spatial operator kernel; zeroed by temporal
+    int *spatial_next;    // [0]: next (frame, grid row) of the spatial operator kernel, [1]: next
+                          // tensor-core unit of the condensation; both zeroed by temporal
 
     void *out;            // [rows][D] dtype
     int *out_index;       // [rows][3]
@@ -328,9 +333,16 @@ __host__ __device__ __forceinline__ int gate_floats(int H, int W, int F, int J) 
     return s;
 }
 
+// Tensor-core unit shape for a block of ncp (a multiple of 16, <= 256)
+// output tokens: the hi and lo operator halves form one MMA of N = 2 ncp for
+// ncp <= 64, else two MMAs of N = ncp; a unit spans as many 128-channel tiles
+// (at most 4) as the 512 accumulator columns of tensor memory hold, so each
+// operator tile in shared memory serves 2-4 channel tiles.
+__host__ __device__ __forceinline__ bool unit_fused(int ncp) { return ncp <= 64; }
+
 __host__ __device__ __forceinline__ int unit_tiles(int ncp) {
-    const int cols = ncp <= 128 ? 2 * ncp : ncp;
-    const int cg = 256 / cols;
+    const int cols = unit_fused(ncp) ? 2 * ncp : ncp;
+    const int cg = 512 / cols;
     return cg < 1 ? 1 : (cg > 4 ? 4 : cg);
 }
 

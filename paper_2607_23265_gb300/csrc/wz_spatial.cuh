@@ -173,12 +173,16 @@ __device__ inline void tail_rows(const Ctx &c, int tb) {
 
 // The tensor-core work units of frame f (the temporal kernel placed them):
 // column blocks of <= 256 tokens, each in groups of unit_tiles(round16(nc))
-// 128-channel tiles.  A record is (f, j0, first tile, nc | tiles << 9 |
-// kc_lo << 12 | kc_hi << 20): the unit's operator rows are zero outside the
-// 32-column chunks [kc_lo, kc_hi] (K_pad <= 4096, so chunks fit 8 bits).
-// With the row supports ilo / ihi of the height analysis (single-level WSM;
-// h x w the frame's grid) that range is the chunks of the map rows the block's
-// grid rows reach, else every chunk.
+// 128-channel tiles, as even as n_ct allows.  A record is (f, j0, first tile,
+// nc | tiles << 9 | kc_lo << 12 | kc_hi << 20 | ranged): the unit's operator
+// rows are zero outside the 32-column chunks [kc_lo, kc_hi] (K_pad <= 4096,
+// so chunks fit 8 bits).  With the row supports ilo / ihi of the height
+// analysis (single-level WSM; h x w the frame's grid) that range is the
+// chunks of the map rows the block's grid rows reach, else every chunk; and
+// for blocks of more than 64 tokens (two MMAs per step, see unit_fused) each
+// chunk also gets the rows of the block whose grid rows reach it (Ctx::krange,
+// flag kUnitRanged): the others are zero there, so the condensation neither
+// loads nor multiplies them.
 __device__ inline void unit_records(const Ctx &c, int64_t f, int n, int h = 0, int w = 0, const int *ilo = nullptr,
                                     const int *ihi = nullptr) {
     const int v = (int)(f / c.T);
@@ -212,10 +216,50 @@ __device__ inline void unit_records(const Ctx &c, int64_t f, int n, int h = 0, i
                 klo = khi = 0;   // an all-zero block: one chunk of zeros
             }
         }
+        const int ncp = (nc + 15) & ~15;
+        int ranged = 0;
+        if (ilo != nullptr && w > 0 && c.krange != nullptr && !unit_fused(ncp) && (j0 >> 8) < c.krange_nblk) {
+            // per chunk: the grid rows p of the block whose map rows [zl(p),
+            // zh(p)] meet the chunk's map rows, as 16-row operator ranges
+            ranged = kUnitRanged;
+            uint16_t *kr = c.krange + ((size_t)f * c.krange_nblk + (j0 >> 8)) * KC;
+            const int p0 = j0 / w, p1 = min(h - 1, (j0 + nc - 1) / w);
+            for (int kc = klo + (int)threadIdx.x; kc <= khi; kc += (int)blockDim.x) {
+                const int z0 = (kc * 32) / c.W, z1 = min(c.H - 1, (kc * 32 + 31) / c.W);
+                int pf = h, pl = -1;
+                for (int p = p0; p <= p1; ++p) {
+                    int y0, y1, a0, a1;
+                    float ly;
+                    bilinear_src(p, c.H, h, y0, y1, ly);
+                    synth_support(y0, y1, c.F, c.hp, a0, a1);
+                    int zl = c.H, zh = -1;
+                    for (int a = a0; a <= a1; ++a) {
+                        zl = min(zl, ilo[a]);
+                        zh = max(zh, ihi[a]);
+                    }
+                    if (zh >= z0 && zl <= z1) {
+                        pf = min(pf, p);
+                        pl = max(pl, p);
+                    }
+                }
+                int ja = 0, jb = 16;   // a chunk no row reaches: one group of zero rows
+                if (pl >= pf) {
+                    const int t0 = max(pf * w, j0) - j0, t1 = min((pl + 1) * w, j0 + nc) - j0;
+                    ja = (t0 >> 4) << 4;
+                    jb = min(ncp, (t1 + 15) & ~15);
+                    if (jb <= ja) {
+                        ja = 0;
+                        jb = 16;
+                    }
+                }
+                kr[kc] = (uint16_t)((ja >> 4) | ((jb >> 4) << 8));
+            }
+        }
         for (int li = threadIdx.x; li < cnt; li += blockDim.x) {
-            const int ct = li * cg;
+            // tiles of group li: [li * n_ct / cnt, (li + 1) * n_ct / cnt), sizes differing by at most one
+            const int ct = li * c.n_ct / cnt, ct1 = (li + 1) * c.n_ct / cnt;
             if (u0 + li < c.max_units_v)
-                units[u0 + li] = make_int4((int)f, j0, ct, nc | (min(cg, c.n_ct - ct) << 9) | (klo << 12) | (khi << 20));
+                units[u0 + li] = make_int4((int)f, j0, ct, nc | ((ct1 - ct) << 9) | (klo << 12) | (khi << 20) | ranged);
         }
         u0 += cnt;
     }
