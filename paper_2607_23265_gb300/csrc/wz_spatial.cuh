@@ -224,23 +224,34 @@ __device__ inline void unit_records(const Ctx &c, int64_t f, int n, int h = 0, i
             ranged = kUnitRanged;
             uint16_t *kr = c.krange + ((size_t)f * c.krange_nblk + (j0 >> 8)) * KC;
             const int p0 = j0 / w, p1 = min(h - 1, (j0 + nc - 1) / w);
-            for (int kc = klo + (int)threadIdx.x; kc <= khi; kc += (int)blockDim.x) {
-                const int z0 = (kc * 32) / c.W, z1 = min(c.H - 1, (kc * 32 + 31) / c.W);
-                int pf = h, pl = -1;
-                for (int p = p0; p <= p1; ++p) {
+            // a warp per chunk, a lane per grid row (p1 - p0 < 64): the rows
+            // that reach the chunk by ballot
+            const int lane = threadIdx.x & 31, nwarp = (int)(blockDim.x >> 5);
+            int zl[2], zh[2];
+#pragma unroll
+            for (int r = 0; r < 2; ++r) {
+                const int p = p0 + lane + 32 * r;
+                zl[r] = c.H;
+                zh[r] = -1;
+                if (p <= p1) {
                     int y0, y1, a0, a1;
                     float ly;
                     bilinear_src(p, c.H, h, y0, y1, ly);
                     synth_support(y0, y1, c.F, c.hp, a0, a1);
-                    int zl = c.H, zh = -1;
                     for (int a = a0; a <= a1; ++a) {
-                        zl = min(zl, ilo[a]);
-                        zh = max(zh, ihi[a]);
+                        zl[r] = min(zl[r], ilo[a]);
+                        zh[r] = max(zh[r], ihi[a]);
                     }
-                    if (zh >= z0 && zl <= z1) {
-                        pf = min(pf, p);
-                        pl = max(pl, p);
-                    }
+                }
+            }
+            for (int kc = klo + (int)(threadIdx.x >> 5); kc <= khi; kc += nwarp) {
+                const int z0 = (kc * 32) / c.W, z1 = min(c.H - 1, (kc * 32 + 31) / c.W);
+                const unsigned m0 = __ballot_sync(0xffffffffu, zh[0] >= z0 && zl[0] <= z1);
+                const unsigned m1 = __ballot_sync(0xffffffffu, zh[1] >= z0 && zl[1] <= z1);
+                int pf = h, pl = -1;
+                if (m0 | m1) {
+                    pf = p0 + (m0 ? __ffs(m0) - 1 : 32 + __ffs(m1) - 1);
+                    pl = p0 + (m1 ? 63 - __clz(m1) : 31 - __clz(m0));
                 }
                 int ja = 0, jb = 16;   // a chunk no row reaches: one group of zero rows
                 if (pl >= pf) {
@@ -252,7 +263,7 @@ __device__ inline void unit_records(const Ctx &c, int64_t f, int n, int h = 0, i
                         jb = 16;
                     }
                 }
-                kr[kc] = (uint16_t)((ja >> 4) | ((jb >> 4) << 8));
+                if (lane == 0) kr[kc] = (uint16_t)((ja >> 4) | ((jb >> 4) << 8));
             }
         }
         for (int li = threadIdx.x; li < cnt; li += blockDim.x) {
