@@ -370,13 +370,23 @@ int run_condense(const CondenseRequest &r) {
         WZ_CUDA(launch_query_pool(c, par.data(), r.stream));
     }
     WZ_CUDA(mark(2 * WZ_KERNEL_QUERY_POOL + 1));
-    WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE));
-    {
+    // max-over-query scorer of one video: one pass over the features computes
+    // the token norms, the channel sums and the token x query-row maxima
+    const int Lqp0 = (r.Lq[0] + 15) / 16 * 16;
+    const bool fused_maxsim = c.relevance_mode == WZ_RELEVANCE_MAXSIM && maxsim_pass_supported(c, Lqp0);
+    if (fused_maxsim) {
+        Nvtx n_("wz::maxsim_pass");
+        WZ_CUDA(launch_query_rows(c, 0, par[0].q_row0, r.Lq[0], Lqp0, r.stream));
+        WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE));
+        WZ_CUDA(launch_maxsim_pass(c, r.Lq[0], Lqp0, r.stream));
+        WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE + 1));
+    } else {
+        WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE));
         Nvtx n_("wz::relevance_pass");
         WZ_CUDA(launch_relevance_pass(c, r.stream));
+        WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE + 1));
     }
-    WZ_CUDA(mark(2 * WZ_KERNEL_RELEVANCE + 1));
-    if (c.relevance_mode == WZ_RELEVANCE_MAXSIM) {
+    if (c.relevance_mode == WZ_RELEVANCE_MAXSIM && !fused_maxsim) {
         // the token x query-row cosines on the tensor cores, video by video
         // (the relevance pass left ||u|| in c.a)
         Nvtx n_("wz::maxsim");

@@ -1,0 +1,474 @@
+// Max-over-query relevance in one pass over the features (the scorer of
+// reading R22 for a single video): the token x query-row cosines on the
+// 5th-generation tensor cores, and, from the same shared-memory tiles, each
+// token's norm and the per-frame channel sums that the frame statistics
+// (r_t, delta_t; Section 3.2.1, Eq. 7) need.
+//
+//   a_{t,n} = max_{j < Lq} <u_{t,n}, q_j / ||q_j||> / ||u_{t,n}||
+//
+// Token tiles of 128 rows (M) x K steps of 64 channels: A = the features,
+// K-major, one 2D TMA box {64, 128} with 128-byte swizzle; B = the unit
+// query rows as bf16 hi rows then lo rows (query_rows_kernel), N = 2 Lqp <=
+// 256, box {64, 2 Lqp}; fp32 accumulators in tensor memory, two buffers, so
+// the epilogue of a tile overlaps the main loop of the next.  CTA c covers
+// the tokens [c L1, (c+1) L1), exactly as the relevance pass does, and writes
+// its channel sums of every frame it touches into partial slot c + t, so
+// frame_stats_kernel reads them unchanged.
+//   warp 0       TMA producer (one thread)
+//   warp 1       TMEM allocation and the MMA issuer (one thread)
+//   warps 2-5    epilogue: tcgen05.ld (TMEM lane = token) -> max over the
+//                query rows of hi + lo -> / ||u|| -> a_{t,n}
+//   warps 6-9    channel sums and token norms: 8 channel pairs per warp, a
+//                lane per channel pair and quarter of the tile's rows (one
+//                warp per SM sub-partition; every element is read from
+//                shared memory once); the quarters combined by shuffles;
+//                the squares of a row's channels kept per lane over the
+//                tile's K steps and combined at the end of the tile; the sums of the
+//                frame open at the start of a tile and of the frame that
+//                starts inside it (frames have >= 128 tokens, so at most one
+//                starts inside a tile) accumulate in shared memory and are
+//                written to the frame's slot when the frame ends or the
+//                CTA's range does
+// Every mbarrier wait is bounded; on a timeout the kernel records a status
+// bit, drains what it issued, frees tensor memory and exits.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <cstring>
+
+#include "wz_internal.cuh"
+#include "wz_ptx.cuh"
+
+namespace wz {
+
+namespace {
+
+constexpr int kXM = 128, kXK = 64;
+constexpr int kXABytes = kXM * kXK * 2;             // 16 KB
+constexpr int kXMaxStages = 8;
+constexpr int kXThreads = 10 * 32;
+constexpr int kXAccCols = 256;
+constexpr uint64_t kXTimeoutNs = 2000000000ull;
+constexpr int kXReaders = 4;                        // channel-sum warps reading each stage
+
+struct XShared {
+    uint64_t full[kXMaxStages];
+    uint64_t empty[kXMaxStages];
+    uint64_t tfull[2], tempty[2];
+    uint64_t nfull[2], nempty[2];
+    uint64_t csync[2];
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort;
+    float norms[2][kXM];
+    float npart[2][4][kXM];   // per channel-sum warp: squares of its channels, per row
+};
+
+struct XMaps {
+    CUtensorMap a, b;
+};
+
+struct XArgs {
+    int stages, stage_stride;   // ring stages and bytes per stage (A then B)
+    int Lq, Lqp;
+    int acc_off;                // byte offset of the two channel-sum buffers (2 x D floats)
+    int shared_off;             // byte offset of XShared
+};
+
+__device__ __forceinline__ void xfail(const Ctx &c, volatile int *abort_flag, int code) {
+    *abort_flag = 1;
+    atomicOr(c.status, code);
+}
+
+// Token tile `it` of this CTA: first token and valid rows.
+__device__ __forceinline__ void xtile(const Ctx &c, int it, int64_t &base, int &nr) {
+    const int64_t total = (int64_t)c.T * c.N;
+    const int64_t beg = (int64_t)blockIdx.x * c.L1;
+    const int64_t end = min(total, beg + c.L1);
+    base = beg + (int64_t)it * kXM;
+    nr = (int)min((int64_t)kXM, end - base);
+}
+
+__device__ __forceinline__ int xtiles(const Ctx &c) {
+    const int64_t total = (int64_t)c.T * c.N;
+    const int64_t beg = (int64_t)blockIdx.x * c.L1;
+    const int64_t end = min(total, beg + c.L1);
+    return beg < end ? (int)((end - beg + kXM - 1) / kXM) : 0;
+}
+
+// The channel sums of this warp's 16 channels of every K step (acc), to the
+// partial slot of frame f, then acc cleared: lanes 0-15 one K step, lanes
+// 16-31 the next.
+__device__ __forceinline__ void xflush(const Ctx &c, float *acc, int64_t f, int ch_lo, int lane) {
+    float *dst = c.part + ((size_t)blockIdx.x + (size_t)f) * c.D;
+    for (int k0 = (lane >> 4) * kXK; k0 < c.D; k0 += 2 * kXK) {
+        const int ch = k0 + ch_lo + (lane & 15);
+        if (wz_in_range(c.status, (int64_t)blockIdx.x + f < (int64_t)c.G1 + c.T)) dst[ch] = acc[ch];
+        acc[ch] = 0.f;
+    }
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_constant__ XMaps maps, Ctx c, XArgs p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    float *acc_buf = reinterpret_cast<float *>(ring + p.acc_off);
+    XShared *S = reinterpret_cast<XShared *>(ring + p.shared_off);
+    volatile int *abort_flag = &S->abort;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < p.stages; ++s) {
+            ptx::mbar_init(&S->full[s], 1);
+            ptx::mbar_init(&S->empty[s], 1 + kXReaders);
+        }
+        for (int b = 0; b < 2; ++b) {
+            ptx::mbar_init(&S->tfull[b], 1);
+            ptx::mbar_init(&S->tempty[b], 4);
+            ptx::mbar_init(&S->nfull[b], 4);
+            ptx::mbar_init(&S->nempty[b], 4);
+            ptx::mbar_init(&S->csync[b], 4);
+        }
+        ptx::mbar_init(&S->drain, 1);
+        S->abort = 0;
+        ptx::fence_barrier_init();
+        ptx::fence_proxy_async_smem();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(&S->tmem_base, 2 * kXAccCols);
+        ptx::tmem_relinquish();
+    }
+    if (warp == 0 && lane == 0) {
+        ptx::prefetch_tmap(&maps.a);
+        ptx::prefetch_tmap(&maps.b);
+    }
+    // channel sums start at zero (shared memory only: before the wait)
+    for (int k = threadIdx.x; k < 2 * c.D; k += blockDim.x) acc_buf[k] = 0.f;
+    pdl_wait();   // the query rows come from the previous grid
+    pdl_trigger();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = S->tmem_base;
+    const int ntile = xtiles(c);
+    const int KS = c.D / kXK;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer ----------------
+        const uint64_t pol_a = ptx::policy_evict_first();
+        const uint64_t pol_b = ptx::policy_evict_last();
+        const uint32_t stage_bytes = (uint32_t)kXABytes + 2u * (uint32_t)p.Lqp * kXK * 2u;
+        int stage = 0;
+        uint32_t phase = 0;
+        int issued_parity[kXMaxStages];
+        for (int s = 0; s < kXMaxStages; ++s) issued_parity[s] = -1;
+        for (int it = 0; it < ntile && !*abort_flag; ++it) {
+            int64_t base;
+            int nr;
+            xtile(c, it, base, nr);
+            bool ok = true;
+            for (int ks = 0; ks < KS; ++ks) {
+                if (!ptx::mbar_wait(&S->empty[stage], phase ^ 1u, kXTimeoutNs)) {
+                    xfail(c, abort_flag, 16);
+                    ok = false;
+                    break;
+                }
+                uint8_t *st = ring + (size_t)stage * p.stage_stride;
+                ptx::mbar_arrive_expect_tx(&S->full[stage], stage_bytes);
+                ptx::tma_load_2d(st, &maps.a, &S->full[stage], ks * kXK, (int)base, pol_a);
+                ptx::tma_load_2d(st + kXABytes, &maps.b, &S->full[stage], ks * kXK, 0, pol_b);
+                issued_parity[stage] = (int)phase;
+                if (++stage == p.stages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok) break;
+        }
+        for (int s = 0; s < p.stages; ++s)
+            if (issued_parity[s] >= 0) ptx::mbar_wait(&S->full[s], (uint32_t)issued_parity[s], kXTimeoutNs);
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer ----------------
+        const uint32_t idesc = ptx::idesc_bf16(kXM, 2 * p.Lqp, false, false);   // both K-major
+        const uint32_t ring32 = ptx::smem_u32(ring);
+        const uint64_t a_base = ptx::smem_desc(ring32, 16, 1024, 2);              // 128-B swizzle
+        const uint64_t b_base = ptx::smem_desc(ring32 + kXABytes, 16, 1024, 2);
+        const uint64_t stage_desc = (uint64_t)(p.stage_stride >> 4);
+        int stage = 0;
+        uint32_t phase = 0;
+        for (int it = 0; it < ntile && !*abort_flag; ++it) {
+            const int b = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1);
+            if (!ptx::mbar_wait(&S->tempty[b], (use & 1u) ^ 1u, kXTimeoutNs)) {
+                xfail(c, abort_flag, 16);
+                break;
+            }
+            ptx::tc_fence_after();
+            const uint32_t d = tmem + (uint32_t)(b * kXAccCols);
+            bool ok = true;
+            for (int ks = 0; ks < KS; ++ks) {
+                if (!ptx::mbar_wait(&S->full[stage], phase, kXTimeoutNs)) {
+                    xfail(c, abort_flag, 16);
+                    ok = false;
+                    break;
+                }
+                ptx::tc_fence_after();
+                const uint64_t so = (uint64_t)stage * stage_desc;
+#pragma unroll
+                for (int k = 0; k < kXK / 16; ++k)   // K = 16 per MMA: 32 bytes along the swizzled row
+                    ptx::mma_bf16(d, a_base + so + (uint64_t)(2 * k), b_base + so + (uint64_t)(2 * k), idesc,
+                                  (ks | k) ? 1u : 0u);
+                ptx::mma_commit(&S->empty[stage]);
+                if (++stage == p.stages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok) break;
+            ptx::mma_commit(&S->tfull[b]);
+        }
+        ptx::mma_commit(&S->drain);
+        ptx::mbar_wait(&S->drain, 0, kXTimeoutNs);
+    } else if (warp >= 2 && warp < 6) {
+        // ---------------- epilogue: a_{t,n} ----------------
+        const int q = warp & 3;                      // TMEM lane quadrant: rows q*32 .. q*32+31
+        const int row = q * 32 + lane;
+        for (int it = 0; it < ntile && !*abort_flag; ++it) {
+            const int b = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1);
+            if (!ptx::mbar_wait(&S->tfull[b], use & 1u, kXTimeoutNs) ||
+                !ptx::mbar_wait(&S->nfull[b], use & 1u, kXTimeoutNs)) {
+                xfail(c, abort_flag, 32);
+                break;
+            }
+            ptx::tc_fence_after();
+            int64_t base;
+            int nr;
+            xtile(c, it, base, nr);
+            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * kXAccCols);
+            float best = -INFINITY;
+            for (int c0 = 0; c0 < p.Lqp; c0 += 16) {
+                uint32_t hi[16], lo[16];
+                ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)c0, hi);
+                ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)(p.Lqp + c0), lo);
+                ptx::tmem_ld_wait();
+                ptx::reg_fence16(hi);
+                ptx::reg_fence16(lo);
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    if (c0 + j < p.Lq) best = fmaxf(best, __uint_as_float(hi[j]) + __uint_as_float(lo[j]));
+            }
+            const float nrm = S->norms[b][row];
+            if (row < nr && wz_in_range(c.status, base + row < (int64_t)c.T * c.N))
+                c.a[base + row] = nrm > 0.f ? best / nrm : 0.f;
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                ptx::mbar_arrive(&S->tempty[b]);
+                ptx::mbar_arrive(&S->nempty[b]);
+            }
+        }
+    } else if (warp >= 6) {
+        // ---------------- per-frame channel sums ----------------
+        // lane: channel pair p2 of this warp's 16 channels of a K step, and
+        // the quarter of the tile's rows it sums (each quarter walks its rows
+        // from a different start, which keeps the quarters on different banks)
+        const int wsel = warp - 6;
+        const int p2 = lane & 7, rq = lane >> 3;
+        const int cw = wsel * 16 + 2 * p2;              // channels cw, cw + 1 of the K step
+        const uint32_t coff = (uint32_t)((cw * 2) & 15);
+        const int chunk = (cw * 2) >> 4;
+        float *acc_open = acc_buf, *acc_next = acc_buf + c.D;
+        int64_t open_f = ntile > 0 ? ((int64_t)blockIdx.x * c.L1) / c.N : 0;
+        bool open_has = false;
+        int stage = 0;
+        uint32_t phase = 0;
+        for (int it = 0; it < ntile && !*abort_flag; ++it) {
+            int64_t base;
+            int nr;
+            xtile(c, it, base, nr);
+            // a frame starts inside the tile at row rb (frames have >= 128 tokens)
+            const int to_end = (int)((int64_t)c.N - base % c.N);
+            const int rb = to_end < nr ? to_end : nr;
+            float sq[32];   // squares of this lane's two channels, row 32 rq + ((i + 2 rq) & 31)
+#pragma unroll
+            for (int i = 0; i < 32; ++i) sq[i] = 0.f;
+            bool ok = true;
+            for (int ks = 0; ks < KS; ++ks) {
+                if (!ptx::mbar_wait(&S->full[stage], phase, kXTimeoutNs)) {
+                    xfail(c, abort_flag, 32);
+                    ok = false;
+                    break;
+                }
+                const uint32_t st32 = ptx::smem_u32(ring + (size_t)stage * p.stage_stride);
+                float s0x = 0.f, s0y = 0.f, s1x = 0.f, s1y = 0.f;
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const int r = 32 * rq + ((i + 2 * rq) & 31);
+                    uint32_t wv;
+                    asm volatile("ld.shared.b32 %0, [%1];"
+                                 : "=r"(wv)
+                                 : "r"(st32 + (uint32_t)(r * 128 + ((chunk ^ (r & 7)) << 4)) + coff));
+                    const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
+                    sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
+                    if (r < rb) {
+                        s0x += x;
+                        s0y += y;
+                    } else if (r < nr) {
+                        s1x += x;
+                        s1y += y;
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&S->empty[stage]);
+#pragma unroll
+                for (int o = 8; o < 32; o <<= 1) {   // the four row quarters, in a fixed order
+                    s0x += __shfl_xor_sync(0xffffffffu, s0x, o);
+                    s0y += __shfl_xor_sync(0xffffffffu, s0y, o);
+                    s1x += __shfl_xor_sync(0xffffffffu, s1x, o);
+                    s1y += __shfl_xor_sync(0xffffffffu, s1y, o);
+                }
+                if (rq == 0) {
+                    const int ch = ks * kXK + cw;
+                    acc_open[ch] += s0x;
+                    acc_open[ch + 1] += s0y;
+                    if (rb < nr) {
+                        acc_next[ch] += s1x;
+                        acc_next[ch + 1] += s1y;
+                    }
+                }
+                if (++stage == p.stages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok) break;
+            // token norms: this warp's squares summed over its 8 channel pairs,
+            // then the four warps' partials in a fixed order
+            const int b = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                float v = sq[i];
+                v += __shfl_xor_sync(0xffffffffu, v, 1);
+                v += __shfl_xor_sync(0xffffffffu, v, 2);
+                v += __shfl_xor_sync(0xffffffffu, v, 4);
+                if (p2 == 0) S->npart[b][wsel][32 * rq + ((i + 2 * rq) & 31)] = v;
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&S->csync[b]);
+            if (!ptx::mbar_wait(&S->csync[b], use & 1u, kXTimeoutNs) ||
+                !ptx::mbar_wait(&S->nempty[b], (use & 1u) ^ 1u, kXTimeoutNs)) {
+                xfail(c, abort_flag, 32);
+                break;
+            }
+            {
+                const int row = 32 * wsel + lane;
+                const float t2 = ((S->npart[b][0][row] + S->npart[b][1][row]) + S->npart[b][2][row]) + S->npart[b][3][row];
+                S->norms[b][row] = sqrtf(t2);
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&S->nfull[b]);
+            __syncwarp();
+            open_has = true;
+            if (rb < nr) {   // the open frame ended inside the tile
+                xflush(c, acc_open, open_f, wsel * 16, lane);
+                float *t = acc_open;
+                acc_open = acc_next;
+                acc_next = t;
+                ++open_f;
+            }
+            if ((base + nr) % c.N == 0) {   // and the frame open now ends with the tile
+                __syncwarp();
+                xflush(c, acc_open, open_f, wsel * 16, lane);
+                ++open_f;
+                open_has = false;
+            }
+            __syncwarp();
+        }
+        if (open_has && !*abort_flag) xflush(c, acc_open, open_f, wsel * 16, lane);   // the CTA's share of it
+    }
+    __syncthreads();
+    if (warp == 1) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, 2 * kXAccCols);
+    }
+}
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 maxsim_encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    }
+    return fn;
+}
+
+bool xencode(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap *m, const void *base, int64_t rows, int cols,
+             int box_rows) {
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+    cuuint32_t box[2] = {(cuuint32_t)kXK, (cuuint32_t)box_rows};
+    cuuint32_t es[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct XLayout {
+    int stages, stride, acc_off, shared_off;
+    size_t smem;
+};
+
+XLayout xlayout(int D, int Lqp) {
+    XLayout L{};
+    L.stride = (kXABytes + 2 * Lqp * kXK * 2 + 1023) / 1024 * 1024;
+    const size_t fixed = 1024 + (size_t)2 * D * 4 + (sizeof(XShared) + 127) / 128 * 128;
+    const size_t cap = 227 * 1024;
+    L.stages = fixed < cap ? (int)((cap - fixed) / (size_t)L.stride) : 0;
+    if (L.stages > kXMaxStages) L.stages = kXMaxStages;
+    L.acc_off = L.stages * L.stride;
+    L.shared_off = L.acc_off + 2 * D * 4;
+    L.smem = 1024 + (size_t)L.shared_off + sizeof(XShared);
+    return L;
+}
+
+}  // namespace
+
+// The fused pass applies to one video with frames of at least 128 tokens,
+// D a multiple of 64 up to 4096 and at most 128 query rows (Lqp <= 128).
+bool maxsim_pass_supported(const Ctx &c, int Lqp) {
+    if (c.V != 1 || c.N < kXM || c.D % kXK != 0 || c.D > 4096 || c.dtype != WZ_DTYPE_BF16) return false;
+    if (Lqp < 16 || Lqp > 128 || Lqp % 16 != 0) return false;
+    return xlayout(c.D, Lqp).stages >= 2;
+}
+
+cudaError_t launch_maxsim_pass(const Ctx &c, int Lq, int Lqp, cudaStream_t s) {
+    if (!maxsim_pass_supported(c, Lqp) || Lq < 1 || Lq > Lqp) return cudaErrorInvalidValue;
+    auto enc = maxsim_encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    XMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    if (!xencode(enc, &maps.a, c.X, (int64_t)c.T * c.N, c.D, kXM) || !xencode(enc, &maps.b, c.qhl, 2 * Lqp, c.D, 2 * Lqp))
+        return cudaErrorInvalidValue;
+    const XLayout L = xlayout(c.D, Lqp);
+    XArgs p{};
+    p.stages = L.stages;
+    p.stage_stride = L.stride;
+    p.Lq = Lq;
+    p.Lqp = Lqp;
+    p.acc_off = L.acc_off;
+    p.shared_off = L.shared_off;
+    cudaError_t e = cudaFuncSetAttribute(maxsim_pass_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem);
+    if (e != cudaSuccess) return e;
+    void *args[] = {&maps, const_cast<Ctx *>(&c), &p};
+    return launch_kernel((const void *)maxsim_pass_kernel, dim3(c.G1), dim3(kXThreads), L.smem, s, args, c.pdl != 0);
+}
+
+}  // namespace wz

@@ -357,6 +357,11 @@ cudaError_t launch_spatial_ml(const Ctx &c, cudaStream_t s);
 size_t spatial_ml_smem_bytes(int H, int W, int F, int J);   // 0 if the layout does not fit
 cudaError_t launch_project_gemm(const void *A, int M, int K, const void *B, int N, const float *bias, void *out,
                                 bool gelu, int *status, bool pdl, cudaStream_t s);
+// Max-over-query relevance of one video in one pass over the features
+// (maxsim.cu): token norms, channel-sum partials and a_{t,n}, in place of the
+// relevance pass and the max-over-query GEMM.
+bool maxsim_pass_supported(const Ctx &c, int Lqp);
+cudaError_t launch_maxsim_pass(const Ctx &c, int Lq, int Lqp, cudaStream_t s);
 cudaError_t launch_maxsim_gemm(const void *X, int M, int K, const void *QHL, int Lq, int Lqp, float *a, int *status,
                                bool pdl, cudaStream_t s);
 cudaError_t launch_query_rows(const Ctx &c, int v, int q_row0, int Lq, int Lqp, cudaStream_t s);
