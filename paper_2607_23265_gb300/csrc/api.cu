@@ -36,7 +36,7 @@ struct Nvtx {
 // Sub-buffer offsets of one call's workspace.
 struct Layout {
     size_t qbar32, qbar64, vpar, a, part, fr, list, n, off, woff, hw, prod,
-        units, ucount, ustart, stab, drange, gate, krange, qnorm, qhl, status, snext, Wop, total;
+        units, ucount, ustart, ustartB, stab, drange, gate, krange, qnorm, qhl, status, snext, Wop, total;
 };
 
 struct Shape {
@@ -68,6 +68,7 @@ Layout make_layout(const Shape &s, bool with_a, bool with_operator) {
     L.units = take((size_t)s.V * s.max_units_v * 16);
     L.ucount = take((size_t)s.V * 4);
     L.ustart = take(VT * 4);
+    L.ustartB = take(VT * 4);
     L.stab = take(std::max(spatial_table_bytes(s.H, s.W, kMaxTaps),            // any wavelet,
                            ml_table_bytes(s.H, s.W, kMaxTaps, kMaxLevels)));   // any level count
     L.drange = take((size_t)s.V * 16);
@@ -207,6 +208,7 @@ void bind(Ctx &c, const Shape &s, const Layout &L, char *ws) {
     c.units = reinterpret_cast<int4 *>(ws + L.units);
     c.ucount = reinterpret_cast<int *>(ws + L.ucount);
     c.ustart = reinterpret_cast<int *>(ws + L.ustart);
+    c.ustartB = reinterpret_cast<int *>(ws + L.ustartB);
     c.stab = reinterpret_cast<float *>(ws + L.stab);
     c.drange = reinterpret_cast<unsigned long long *>(ws + L.drange);
     c.qnorm = reinterpret_cast<float *>(ws + L.qnorm);

@@ -53,13 +53,16 @@ __device__ int block_excl_scan(int x, int *ws, int *total) {
 
 // Three exclusive block scans at once (same barriers as one); ws holds
 // >= 3 * 33 ints.  Returns the exclusive prefixes and the totals.
-__device__ void block_excl_scan3(const int (&x)[3], int *ws, int (&excl)[3], int (&total)[3]) {
+template <int K>
+__device__ void block_excl_scan(const int (&x)[K], int *ws, int (&excl)[K], int (&total)[K]) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nw = blockDim.x >> 5;
-    int incl[3] = {x[0], x[1], x[2]};
+    int incl[K];
+#pragma unroll
+    for (int k = 0; k < K; ++k) incl[k] = x[k];
     for (int o = 1; o < 32; o <<= 1) {
 #pragma unroll
-        for (int k = 0; k < 3; ++k) {
+        for (int k = 0; k < K; ++k) {
             const int y = __shfl_up_sync(0xffffffffu, incl[k], o);
             if (lane >= o) incl[k] += y;
         }
@@ -67,12 +70,12 @@ __device__ void block_excl_scan3(const int (&x)[3], int *ws, int (&excl)[3], int
     __syncthreads();
     if (lane == 31) {
 #pragma unroll
-        for (int k = 0; k < 3; ++k) ws[33 * k + warp] = incl[k];
+        for (int k = 0; k < K; ++k) ws[33 * k + warp] = incl[k];
     }
     __syncthreads();
     if (warp == 0) {
 #pragma unroll
-        for (int k = 0; k < 3; ++k) {
+        for (int k = 0; k < K; ++k) {
             const int w = lane < nw ? ws[33 * k + lane] : 0;
             int wi = w;
             for (int o = 1; o < 32; o <<= 1) {
@@ -86,7 +89,7 @@ __device__ void block_excl_scan3(const int (&x)[3], int *ws, int (&excl)[3], int
     }
     __syncthreads();
 #pragma unroll
-    for (int k = 0; k < 3; ++k) {
+    for (int k = 0; k < K; ++k) {
         excl[k] = ws[33 * k + warp] + incl[k] - x[k];
         total[k] = ws[33 * k + 32];
     }
@@ -214,7 +217,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     extern __shared__ __align__(16) unsigned char tsm[];
     __shared__ double dscr[64];
     __shared__ long long lscr[66];
-    __shared__ int iscr[3 * 33];
+    __shared__ int iscr[4 * 33];
     const int v = blockIdx.x;
     const int T = c.T;
     const int64_t base = (int64_t)v * T;
@@ -405,27 +408,35 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     // per frame: output rows, tensor-core operator rows (budgets padded to
     // 16) and tensor-core units (column blocks of <= 256 tokens, each in
     // groups of unit_tiles(round16(nc)) 128-channel tiles; the spatial kernel
-    // writes the unit records); one block scan gives all three offsets
+    // writes the unit records); one block scan gives all the offsets.  The
+    // units of every frame's first block come first in the video's list, the
+    // units of later blocks (frames over 256 tokens; their operator rows
+    // reach only part of the map, so they are the short ones) after them:
+    // the condensation claims units in list order, and short units last keep
+    // its tail short.
     const bool tc = c.path == WZ_PATH_TENSOR;
-    int nloc[kPerThread], ucnt[kPerThread];
-    int part[3] = {0, 0, 0};
+    int nloc[kPerThread], ucnt[kPerThread], ucntB[kPerThread];
+    int part[4] = {0, 0, 0, 0};
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
         nloc[k] = (k < per && t < T) ? nf[t] : 0;
         ucnt[k] = 0;
+        ucntB[k] = 0;
         if (tc)
             for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
                 const int nc = min(kColBlock, nloc[k] - j0);
-                ucnt[k] += (c.n_ct + unit_tiles((nc + 15) / 16 * 16) - 1) / unit_tiles((nc + 15) / 16 * 16);
+                const int cg = unit_tiles((nc + 15) / 16 * 16);
+                (j0 == 0 ? ucnt[k] : ucntB[k]) += (c.n_ct + cg - 1) / cg;
             }
         part[0] += nloc[k];
         part[1] += (nloc[k] + 15) & ~15;
         part[2] += ucnt[k];
+        part[3] += ucntB[k];
     }
-    int pre[3], tot[3];
-    block_excl_scan3(part, iscr, pre, tot);
-    int o = pre[0], wo = pre[1], u = pre[2];
+    int pre[4], tot[4];
+    block_excl_scan<4>(part, iscr, pre, tot);
+    int o = pre[0], wo = pre[1], u = pre[2], uB = tot[2] + pre[3];
 #pragma unroll
     for (int k = 0; k < kPerThread; ++k) {
         const int t = t0 + k;
@@ -433,7 +444,10 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             c.n[base + t] = nloc[k];
             c.off[base + t] = vp.row0 + o;
             c.woff[base + t] = vp.w_row0 + wo;
-            if (tc) c.ustart[base + t] = u;
+            if (tc) {
+                c.ustart[base + t] = u;
+                c.ustartB[base + t] = uB;
+            }
             const int h = grid_h(nloc[k], c.H, c.W);
             c.hw[2 * (base + t)] = h;
             c.hw[2 * (base + t) + 1] = h > 0 ? (nloc[k] + h - 1) / h : 0;
@@ -449,13 +463,14 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         o += nloc[k];
         wo += (nloc[k] + 15) & ~15;
         u += ucnt[k];
+        uB += ucntB[k];
     }
     if (threadIdx.x == 0) {
         c.prod[v] = tot[0];
         if (c.out_count) c.out_count[v] = tot[0];
         if (tc) {
-            c.ucount[v] = min(tot[2], c.max_units_v);
-            if (tot[2] > c.max_units_v) atomicOr(c.status, 2);
+            c.ucount[v] = min(tot[2] + tot[3], c.max_units_v);
+            if (tot[2] + tot[3] > c.max_units_v) atomicOr(c.status, 2);
         }
     }
 }

@@ -58,7 +58,8 @@ struct Ctx {
     int *prod;            // [V] produced rows
     int4 *units;          // [V][max_units_v] tensor-core work units
     int *ucount;          // [V]
-    int *ustart;          // [V*T] first unit of each frame in its video's list
+    int *ustart;          // [V*T] first unit of each frame's first block in its video's list
+    int *ustartB;         // [V*T] first unit of the frame's later blocks (after every first block)
     float *stab;          // frame-independent tables of the spatial operator
     unsigned long long *drange;   // [V][2] min / max of delta_t as bit patterns (delta >= +0)
     float *gate;          // [V*T][hp*wp] gate G of each frame (Eq. 12)

@@ -171,7 +171,8 @@ __device__ inline void tail_rows(const Ctx &c, int tb) {
     }
 }
 
-// The tensor-core work units of frame f (the temporal kernel placed them):
+// The tensor-core work units of frame f (the temporal kernel placed them: the
+// first block's units at ustart[f], the later blocks' at ustartB[f]):
 // column blocks of <= 256 tokens, each in groups of unit_tiles(round16(nc))
 // 128-channel tiles, as even as n_ct allows.  A record is (f, j0, first tile,
 // nc | tiles << 9 | kc_lo << 12 | kc_hi << 20 | ranged): the unit's operator
@@ -190,6 +191,7 @@ __device__ inline void unit_records(const Ctx &c, int64_t f, int n, int h = 0, i
     int u0 = c.ustart[f];
     const int KC = c.K_pad >> 5;
     for (int j0 = 0; j0 < n; j0 += kColBlock) {
+        if (j0 == kColBlock) u0 = c.ustartB[f];   // later blocks: the second part of the list
         const int nc = min(kColBlock, n - j0);
         const int cg = unit_tiles((nc + 15) / 16 * 16);
         const int cnt = (c.n_ct + cg - 1) / cg;
