@@ -147,42 +147,6 @@ __device__ __forceinline__ int frame_rows(const Ctx &c, int f) {
     return min(h, (n + w - 1) / w);
 }
 
-// rowpre[f] = grid rows of the frames before f, rowpre[F] = all rows
-// (F <= kCompactFrames; block-wide scan, every thread a contiguous range).
-constexpr int kCompactFrames = 2048;
-__device__ void grid_row_prefix(const Ctx &c, int F, int *rowpre, int *wsum) {
-    constexpr int kPer = kCompactFrames / kSpatialThreads;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int per = (F + kSpatialThreads - 1) / kSpatialThreads;
-    const int f0 = tid * per;
-    int rows[kPer];
-    int sum = 0;
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-        rows[k] = (k < per && f0 + k < F) ? frame_rows(c, f0 + k) : 0;
-        sum += rows[k];
-    }
-    int incl = sum;
-    for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-    }
-    if (lane == 31) wsum[warp] = incl;
-    __syncthreads();
-    int run = incl - sum;
-    for (int w = 0; w < warp; ++w) run += wsum[w];
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-        if (k < per && f0 + k < F) rowpre[f0 + k] = run;
-        run += rows[k];
-    }
-    if (tid == 0) {
-        int tot = 0;
-        for (int w = 0; w < kSpatialThreads / 32; ++w) tot += wsum[w];
-        rowpre[F] = tot;
-    }
-}
-
 // The WSM operator rows (single level), persistent: every CTA copies the
 // frame-independent tables once, then takes grid rows (frame f, row p) from
 // a global counter until none is left; a row whose frame changes reloads
@@ -234,7 +198,7 @@ __global__ void __launch_bounds__(kSpatialThreads, 4) spatial_wsm_kernel(Ctx c, 
     // index arithmetic throughout (no 64-bit divisions in the loop)
     const int VT = c.V * c.T;
     if (compact) {
-        grid_row_prefix(c, VT, rowpre, s_wsum);
+        frame_prefix(VT, rowpre, s_wsum, [&](int fr) { return frame_rows(c, fr); });
         __syncthreads();
     }
     const int items = compact ? rowpre[VT] : VT * H;
@@ -517,6 +481,10 @@ int spatial_split(const Ctx &c, int resident) {
 
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s) {
     if (c.spatial_mode == WZ_SPATIAL_WSM && c.wsm_levels > 1) return launch_spatial_ml(c, s);
+    // tensor path: the 16-row kernel where it applies
+    bool launched = false;
+    const cudaError_t et = launch_spatial_tc(c, s, &launched);
+    if (launched || et != cudaSuccess) return et;
     SpatialSmem L;
     L.init(c.H, c.W, c.hp, c.wp);
     if ((L.AWl & 3) != 0 || (L.AWh & 3) != 0 || (L.stage & 3) != 0 || L.QB < 1) return cudaErrorMisalignedAddress;

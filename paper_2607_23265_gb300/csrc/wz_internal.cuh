@@ -354,6 +354,7 @@ cudaError_t launch_relevance_pass(const Ctx &c, cudaStream_t s);
 cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s);
 cudaError_t launch_temporal(const Ctx &c, cudaStream_t s);
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s);
+cudaError_t launch_spatial_tc(const Ctx &c, cudaStream_t s, bool *launched);
 cudaError_t launch_spatial_ml(const Ctx &c, cudaStream_t s);
 size_t spatial_ml_smem_bytes(int H, int W, int F, int J);   // 0 if the layout does not fit
 cudaError_t launch_project_gemm(const void *A, int M, int K, const void *B, int N, const float *bias, void *out,

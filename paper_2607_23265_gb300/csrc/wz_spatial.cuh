@@ -154,6 +154,44 @@ __device__ __forceinline__ void write_rows(const Ctx &c, const float *stg, int k
 
 constexpr int kSpatialThreads = 256;
 constexpr int kTailBlocks = 64;
+constexpr int kCompactFrames = 2048;   // frames whose work prefix a spatial CTA keeps in shared memory
+
+// pre[f] = sum of count(f') over the frames f' < f, pre[F] = the total
+// (F <= kCompactFrames; a block-wide scan, every thread a contiguous range of
+// frames).  The caller synchronises the block before reading pre.
+template <class Count>
+__device__ void frame_prefix(int F, int *pre, int *wsum, Count count) {
+    constexpr int kPer = kCompactFrames / kSpatialThreads;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int per = (F + kSpatialThreads - 1) / kSpatialThreads;
+    const int f0 = tid * per;
+    int cnt[kPer];
+    int sum = 0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+        cnt[k] = (k < per && f0 + k < F) ? count(f0 + k) : 0;
+        sum += cnt[k];
+    }
+    int incl = sum;
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    int run = incl - sum;
+    for (int w = 0; w < warp; ++w) run += wsum[w];
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+        if (k < per && f0 + k < F) pre[f0 + k] = run;
+        run += cnt[k];
+    }
+    if (tid == 0) {
+        int tot = 0;
+        for (int w = 0; w < kSpatialThreads / 32; ++w) tot += wsum[w];
+        pre[F] = tot;
+    }
+}
 
 // Rows past the produced count (tau > 0): index -1, zero tokens.  Tail CTA
 // tb of kTailBlocks.
