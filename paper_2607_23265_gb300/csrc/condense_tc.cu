@@ -545,9 +545,8 @@ condense_tc_kernel(const __grid_constant__ TcMaps maps, Ctx c) {
     }
 }
 
-namespace {
-
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+// cuTensorMapEncodeTiled from the driver (resolved once; null when missing).
+PFN_cuTensorMapEncodeTiled_v12000 tmap_encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (!fn) {
         void *p = nullptr;
@@ -560,12 +559,10 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-}  // namespace
-
 bool tensor_path_available() { return true; }
 
 cudaError_t launch_condense_tc(const Ctx &c, cudaStream_t s) {
-    auto enc = encode_fn();
+    auto enc = tmap_encode_fn();
     if (!enc) return cudaErrorNotSupported;
     if (c.dtype != WZ_DTYPE_BF16 || c.rows_total < 1) return cudaErrorInvalidValue;
     TcMaps maps;

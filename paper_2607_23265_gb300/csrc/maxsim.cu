@@ -397,19 +397,6 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
 
 namespace {
 
-PFN_cuTensorMapEncodeTiled_v12000 maxsim_encode_fn() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (!fn) {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-    }
-    return fn;
-}
-
 bool xencode(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap *m, const void *base, int64_t rows, int cols,
              int box_rows) {
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
@@ -451,7 +438,7 @@ bool maxsim_pass_supported(const Ctx &c, int Lqp) {
 
 cudaError_t launch_maxsim_pass(const Ctx &c, int Lq, int Lqp, cudaStream_t s) {
     if (!maxsim_pass_supported(c, Lqp) || Lq < 1 || Lq > Lqp) return cudaErrorInvalidValue;
-    auto enc = maxsim_encode_fn();
+    auto enc = tmap_encode_fn();
     if (!enc) return cudaErrorNotSupported;
     XMaps maps;
     memset(&maps, 0, sizeof(maps));

@@ -285,19 +285,6 @@ project_gemm_kernel(const __grid_constant__ PMaps maps, PArgs p) {
 
 namespace {
 
-PFN_cuTensorMapEncodeTiled_v12000 project_encode_fn() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (!fn) {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-    }
-    return fn;
-}
-
 bool encode_2d(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap *m, const void *base, int rows, int cols,
                int box_rows) {
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
@@ -316,7 +303,7 @@ bool encode_2d(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap *m, const void
 cudaError_t launch_project_gemm(const void *A, int M, int K, const void *B, int N, const float *bias, void *out,
                                 bool gelu, int *status, bool pdl, cudaStream_t s) {
     if (M < 1) return cudaSuccess;
-    auto enc = project_encode_fn();
+    auto enc = tmap_encode_fn();
     if (!enc) return cudaErrorNotSupported;
     PMaps maps;
     memset(&maps, 0, sizeof(maps));
@@ -347,7 +334,7 @@ cudaError_t launch_maxsim_gemm(const void *X, int M, int K, const void *QHL, int
                                bool pdl, cudaStream_t s) {
     if (M < 1) return cudaSuccess;
     if (Lq < 1 || Lqp % 16 != 0 || Lq > Lqp || 2 * Lqp > kPN || K % kPK != 0) return cudaErrorInvalidValue;
-    auto enc = project_encode_fn();
+    auto enc = tmap_encode_fn();
     if (!enc) return cudaErrorNotSupported;
     PMaps maps;
     memset(&maps, 0, sizeof(maps));

@@ -11,8 +11,9 @@
 // (budgets padded to 16), so a work item is one 16-row group of one frame and
 // owns its rows outright: the CTA forms the group in shared memory directly
 // in the tiled bf16 hi / lo layout of tile_index() (one 1 KB block per
-// 32-column chunk and half) and sends each block to global memory with one
-// bulk copy, zeros included.  Thread (t, s) of the 256 takes operator row t
+// 32-column chunk and half) and sends the whole group, zeros included, to
+// global memory with one 4D tensor store (256 elements x 2 row groups x
+// chunks x halves).  Thread (t, s) of the 256 takes operator row t
 // of the group (token j = 16 g + t, grid cell (p, q)) and the map rows
 // i = zlo + s, zlo + s + 16, ... that the row reaches: it forms the
 // coefficients c_v[b] = Q_v[q,b] Y_v[b,i] for the few b of the column's
@@ -33,11 +34,13 @@ namespace wz {
 namespace {
 
 constexpr int kTcRows = 16;                       // operator rows per work item
+constexpr int kGateRegs = 4;                      // gate entries per thread held in registers
 constexpr int kTcChunkBytes = kTcRows * 32 * 2;   // 16 rows x 32 columns of one bf16 half: 1 KB
 
 // Float offsets of the CTA's shared memory after the frame-independent tables.
 struct TcSmem {
     int gpre;    // [VT + 1] int: 16-row groups of the frames before f
+    int fdat;    // [VT][3] int: n | h << 13 | w << 20, off, woff of frame f
     int G;       // [hp][wp]: the item's frame gate
     int P;       // [16][2][BMAX]: P_L, P_H of row t's grid row at a = a0(t) + k
     int Q;       // [16][2][BMAX]: Q_L, Q_H of row t's grid column at b = b0(t) + k
@@ -53,6 +56,7 @@ struct TcSmem {
             return at;
         };
         gpre = take(VT + 1, 4);
+        fdat = take(3 * VT, 4);
         G = take(L.hp * L.wp, 4);
         P = take(kTcRows * 2 * bmax, 4);
         Q = take(kTcRows * 2 * bmax, 4);
@@ -65,24 +69,51 @@ struct TcSmem {
 // Per-row ints of TcSmem::tok.
 enum { kTokA0 = 0, kTokNA, kTokB0, kTokNB, kTokZlo, kTokSpan, kTokJ4 };
 
-// Operator entry (row t of the group, column k) as bf16 hi and lo halves in
-// the staged tiled layout: chunk k / 32, then the 8-row group, then the
-// 8-column quarter, then row and column within the 8 x 8 core matrix.
-__device__ __forceinline__ void stage_put(__nv_bfloat16 *hi, int lo_off, int t, int k, float x) {
-    const int e = (k >> 5) * 512 + (t >> 3) * 256 + ((k >> 3) & 3) * 64 + (t & 7) * 8 + (k & 7);
+// Operator entries (row t of the group, columns k ...) as bf16 hi and lo
+// halves in the staged tiled layout: chunk k / 32, then the 8-row group, then
+// the 8-column quarter, then row and column within the 8 x 8 core matrix.
+__device__ __forceinline__ int stage_elem(int t, int k) {
+    return (k >> 5) * 512 + (t >> 3) * 256 + ((k >> 3) & 3) * 64 + (t & 7) * 8 + (k & 7);
+}
+__device__ __forceinline__ void stage_put1(__nv_bfloat16 *hi, int lo_off, int t, int k, float x) {
+    const int e = stage_elem(t, k);
     const __nv_bfloat16 h = __float2bfloat16_rn(x);
     hi[e] = h;
     hi[lo_off + e] = __float2bfloat16_rn(x - __bfloat162float(h));
+}
+// Columns k, k + 1 with k even: one quarter, one 32-bit store per half.
+__device__ __forceinline__ void stage_put2(__nv_bfloat16 *hi, int lo_off, int t, int k, float x, float y) {
+    const int e = stage_elem(t, k);
+    const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+    const float2 hf = __bfloat1622float2(h);
+    *reinterpret_cast<__nv_bfloat162 *>(hi + e) = h;
+    *reinterpret_cast<__nv_bfloat162 *>(hi + lo_off + e) = __floats2bfloat162_rn(x - hf.x, y - hf.y);
+}
+// Columns k .. k + n - 1 (1 <= n <= 4) from v.x ...
+__device__ __forceinline__ void stage_put4(__nv_bfloat16 *hi, int lo_off, int t, int k, float4 v, int n) {
+    if ((k & 1) == 0) {
+        if (n >= 2) stage_put2(hi, lo_off, t, k, v.x, v.y);
+        else stage_put1(hi, lo_off, t, k, v.x);
+        if (n == 4) stage_put2(hi, lo_off, t, k + 2, v.z, v.w);
+        else if (n == 3) stage_put1(hi, lo_off, t, k + 2, v.z);
+    } else {
+        stage_put1(hi, lo_off, t, k, v.x);
+        if (n >= 3) stage_put2(hi, lo_off, t, k + 1, v.y, v.z);
+        else if (n == 2) stage_put1(hi, lo_off, t, k + 1, v.y);
+        if (n == 4) stage_put1(hi, lo_off, t, k + 3, v.w);
+    }
 }
 
 }  // namespace
 
 template <int BMAX>
-__global__ void __launch_bounds__(kSpatialThreads, BMAX <= 6 ? 3 : 2) spatial_wsm_tc_kernel(Ctx c) {
+__global__ void __launch_bounds__(kSpatialThreads, BMAX <= 6 ? 3 : 2)
+    spatial_wsm_tc_kernel(const __grid_constant__ CUtensorMap wmap, Ctx c) {
     pdl_trigger();
-    extern __shared__ __align__(16) float sm[];
+    extern __shared__ __align__(128) float sm[];
     __shared__ int s_item, s_f, s_wsum[kSpatialThreads / 32];
-    const int tid = threadIdx.x, lane = tid & 31;
+    const int tid = threadIdx.x;
+    if (tid == 0) ptx::prefetch_tmap(&wmap);
     const int H = c.H, W = c.W, hp = c.hp, wp = c.wp, F = c.F, VT = c.V * c.T;
     SpatialSmem L;
     L.init(H, W, hp, wp);
@@ -95,8 +126,16 @@ __global__ void __launch_bounds__(kSpatialThreads, BMAX <= 6 ? 3 : 2) spatial_ws
     // thread 0 claims the next group while the current one is formed
     int claimed = tid == 0 ? atomicAdd(c.spatial_next, 1) : 0;
     if ((int)blockIdx.x < kTailBlocks) tail_rows(c, (int)blockIdx.x);
-    int *gpre = reinterpret_cast<int *>(sm + S.gpre);
-    frame_prefix(VT, gpre, s_wsum, [&](int f) { return (max(c.n[f], 0) + kTcRows - 1) / kTcRows; });
+    int *gpre = reinterpret_cast<int *>(sm + S.gpre), *fdat = reinterpret_cast<int *>(sm + S.fdat);
+    // the prefix of the frames' group counts; the frames' budgets, grids and
+    // row offsets stay in shared memory (n <= 4096, h, w <= 64)
+    frame_prefix(VT, gpre, s_wsum, [&](int f) {
+        const int n = max(c.n[f], 0);
+        fdat[3 * f] = n | (c.hw[2 * f] << 13) | (c.hw[2 * f + 1] << 20);
+        fdat[3 * f + 1] = c.off[f];
+        fdat[3 * f + 2] = c.woff[f];
+        return (n + kTcRows - 1) / kTcRows;
+    });
     __syncthreads();
     const int items = gpre[VT];
 
@@ -110,15 +149,17 @@ __global__ void __launch_bounds__(kSpatialThreads, BMAX <= 6 ? 3 : 2) spatial_ws
     const int KC = L.K_pad >> 5, WP4 = L.WP4;
     const int lo_off = KC * 512;                           // elements from a hi entry to its lo entry
     const int stage_words = KC * kTcChunkBytes * 2 / 16;   // uint4 words of the stage
-    __nv_bfloat16 *Whi = static_cast<__nv_bfloat16 *>(c.Wop);
-    __nv_bfloat16 *Wlo = Whi + (size_t)c.w_rows * L.K_pad;
     const int t = tid >> 4, s = tid & 15;   // operator row of the group, slot of the row's work
+
+    // the frames' tensor-core unit records, frame f by CTA f mod gridDim.x
+    // (before the groups: the counter balances the CTAs afterwards)
+    for (int f = blockIdx.x; f < VT; f += gridDim.x) {
+        const int nhw = fdat[3 * f], n = nhw & 8191;
+        if (n > 0) unit_records(c, f, n, (nhw >> 13) & 127, nhw >> 20, ilo, ihi);
+    }
 
     for (;;) {
         __syncthreads();   // the previous group's reads of shared memory
-        // warp 0 issued the previous group's bulk stores: their reads of the
-        // stage have finished before the stage is cleared
-        if (tid < 32) ptx::bulk_wait_read();
         if (tid == 0) {
             const int it = claimed;
             if (it < items) claimed = atomicAdd(c.spatial_next, 1);
@@ -141,16 +182,16 @@ __global__ void __launch_bounds__(kSpatialThreads, BMAX <= 6 ? 3 : 2) spatial_ws
         const int item = s_item;
         if (item >= items) break;
         const int f = s_f, g = item - gpre[f];
-        const int n = c.n[f], h = c.hw[2 * f], w = c.hw[2 * f + 1];
-        if (g == 0) unit_records(c, f, n, h, w, ilo, ihi);
-        {
-            uint4 *z = reinterpret_cast<uint4 *>(stg);
-            for (int k = tid; k < stage_words; k += blockDim.x) z[k] = make_uint4(0u, 0u, 0u, 0u);
-        }
-        {
-            // gate G of the frame (Eq. 6, Eq. 12), pooled by frame_stats
-            const float *Gf = c.gate + (int64_t)f * c.gate_stride;
-            for (int k = tid; k < hp * wp; k += blockDim.x) G[k] = Gf[k];
+        const int nhw = fdat[3 * f], n = nhw & 8191, h = (nhw >> 13) & 127, w = nhw >> 20;
+        // gate G of the frame (Eq. 6, Eq. 12), pooled by frame_stats: loaded
+        // into registers here, stored to shared memory after the row setup
+        const float *Gf = c.gate + (int64_t)f * c.gate_stride;
+        const int ng = hp * wp;
+        float gr[kGateRegs];
+#pragma unroll
+        for (int r = 0; r < kGateRegs; ++r) {
+            const int k = tid + r * kSpatialThreads;
+            gr[r] = k < ng ? Gf[k] : 0.f;
         }
         {
             // row t: token j of the frame, grid cell (p, q); the bilinear row
@@ -192,7 +233,7 @@ __global__ void __launch_bounds__(kSpatialThreads, BMAX <= 6 ? 3 : 2) spatial_ws
                 T[kTokZlo] = zlo;
                 T[kTokSpan] = valid && jh >= 0 ? max(0, zhi - zlo + 1) : 0;
                 T[kTokJ4] = jh >= 0 ? (jl >> 2) | ((jh >> 2) << 16) : 0;
-                const int64_t row = (int64_t)c.off[f] + j;
+                const int64_t row = (int64_t)fdat[3 * f + 1] + j;
                 if (valid && wz_in_range(c.status, row < c.rows_total)) {
                     int *o = c.out_index + (size_t)row * 3;
                     o[0] = f % c.T;
@@ -200,6 +241,21 @@ __global__ void __launch_bounds__(kSpatialThreads, BMAX <= 6 ? 3 : 2) spatial_ws
                     o[2] = q;
                 }
             }
+        }
+#pragma unroll
+        for (int r = 0; r < kGateRegs; ++r) {
+            const int k = tid + r * kSpatialThreads;
+            if (k < ng) G[k] = gr[r];
+        }
+        for (int k = tid + kGateRegs * kSpatialThreads; k < ng; k += kSpatialThreads) G[k] = Gf[k];
+        // thread 0 issued the previous group's store: its reads of the stage
+        // have finished (waited for here, after the loads above) before the
+        // stage is cleared
+        if (tid == 0) ptx::bulk_wait_read();
+        __syncthreads();
+        {
+            uint4 *z = reinterpret_cast<uint4 *>(stg);
+            for (int k = tid; k < stage_words; k += blockDim.x) z[k] = make_uint4(0u, 0u, 0u, 0u);
         }
         __syncthreads();   // the stage is clear; G, P, Q and the row data are in place
         {
@@ -249,30 +305,22 @@ __global__ void __launch_bounds__(kSpatialThreads, BMAX <= 6 ? 3 : 2) spatial_ws
                             acc.w = fmaf(cl[bb], a4.w, fmaf(ch[bb], d4.w, acc.w));
                         }
                     }
-                    const int k = i * W + 4 * j4;
-                    stage_put(shi, lo_off, t, k, acc.x);
-                    if (4 * j4 + 1 < W) stage_put(shi, lo_off, t, k + 1, acc.y);
-                    if (4 * j4 + 2 < W) stage_put(shi, lo_off, t, k + 2, acc.z);
-                    if (4 * j4 + 3 < W) stage_put(shi, lo_off, t, k + 3, acc.w);
+                    stage_put4(shi, lo_off, t, i * W + 4 * j4, acc, min(4, W - 4 * j4));
                 }
             }
         }
-        // the stage goes out as 2 * KC bulk copies of 1 KB (hi chunks, then lo)
+        // the stage goes out as one tensor store: row groups r0 / 8 and
+        // r0 / 8 + 1 of every chunk, hi and lo
         ptx::fence_proxy_async_smem();
         __syncthreads();
-        if (tid < 32) {
-            const int64_t r0 = (int64_t)c.woff[f] + kTcRows * g;
-            if (wz_in_range(c.status, r0 + kTcRows <= c.w_rows))
-                for (int k = lane; k < 2 * KC; k += 32) {
-                    const int kc = k < KC ? k : k - KC;
-                    __nv_bfloat16 *dst = (k < KC ? Whi : Wlo) + tile_index(r0, 32 * kc, c.w_rows);
-                    ptx::bulk_store(dst, stg + (size_t)k * kTcChunkBytes, kTcChunkBytes);
-                }
+        if (tid == 0) {
+            const int64_t r0 = (int64_t)fdat[3 * f + 2] + kTcRows * g;
+            if (wz_in_range(c.status, r0 + kTcRows <= c.w_rows)) ptx::tma_store_4d(&wmap, stg, 0, (int)(r0 >> 3), 0, 0);
             ptx::bulk_commit();
         }
     }
     // the operator rows are in global memory before the CTA ends
-    if (tid < 32) ptx::bulk_wait();
+    if (tid == 0) ptx::bulk_wait();
 }
 
 // Dynamic shared memory of spatial_wsm_tc_kernel (bytes).
@@ -304,7 +352,22 @@ cudaError_t launch_spatial_tc(const Ctx &c, cudaStream_t s, bool *launched) {
         return cudaSuccess;
     }
     const size_t smem = spatial_tc_smem_bytes(c, bm);
-    if (smem > (size_t)100 * 1024) return cudaSuccess;
+    const int KC = (c.H * c.W + 31) / 32;
+    auto enc = tmap_encode_fn();
+    if (smem > (size_t)100 * 1024 || KC > 256 || !enc) return cudaSuccess;
+    // the tiled operator as [half][chunk][8-row group][256 elements]
+    CUtensorMap wmap;
+    {
+        const cuuint64_t groups = (cuuint64_t)(c.w_rows >> 3);
+        cuuint64_t dims[4] = {256, groups, (cuuint64_t)KC, 2};
+        cuuint64_t strides[3] = {512, groups * 512, (cuuint64_t)c.w_rows * (cuuint64_t)(32 * KC) * 2};
+        cuuint32_t box[4] = {256, 2, (cuuint32_t)KC, 2};
+        cuuint32_t es[4] = {1, 1, 1, 1};
+        if (enc(&wmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, c.Wop, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaSuccess;
+    }
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     int dev = 0, sms = 0, per_sm = 0;
@@ -316,7 +379,7 @@ cudaError_t launch_spatial_tc(const Ctx &c, cudaStream_t s, bool *launched) {
     // persistent: every resident CTA pulls groups; at least kTailBlocks CTAs
     // so that the tail rows are covered
     const unsigned blocks = (unsigned)std::max(sms * per_sm, kTailBlocks);
-    void *args[] = {const_cast<Ctx *>(&c)};
+    void *args[] = {&wmap, const_cast<Ctx *>(&c)};
     *launched = true;
     return launch_kernel(fn, dim3(blocks), dim3(kSpatialThreads), smem, s, args, c.pdl != 0);
 }

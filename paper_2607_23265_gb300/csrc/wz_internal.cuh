@@ -1,6 +1,8 @@
 // Internal declarations of the WaveZip CUDA library (not part of the C ABI).
 #pragma once
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -355,6 +357,8 @@ cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s);
 cudaError_t launch_temporal(const Ctx &c, cudaStream_t s);
 cudaError_t launch_spatial(const Ctx &c, cudaStream_t s);
 cudaError_t launch_spatial_tc(const Ctx &c, cudaStream_t s, bool *launched);
+// cuTensorMapEncodeTiled from the driver (resolved once; null when missing).
+PFN_cuTensorMapEncodeTiled_v12000 tmap_encode_fn();
 cudaError_t launch_spatial_ml(const Ctx &c, cudaStream_t s);
 size_t spatial_ml_smem_bytes(int H, int W, int F, int J);   // 0 if the layout does not fit
 cudaError_t launch_project_gemm(const void *A, int M, int K, const void *B, int N, const float *bias, void *out,
