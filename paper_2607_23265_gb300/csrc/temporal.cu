@@ -114,9 +114,11 @@ __device__ __forceinline__ int grid_h(int n, int H, int W) {
 // keys, lst, nb) or by frame t (nf).
 // keys start on a 16-byte boundary (the rank reads them two at a time)
 __host__ __device__ inline size_t temporal_smem_keys(int T) { return ((size_t)T * 8 + 15) & ~(size_t)15; }
-__host__ __device__ inline size_t temporal_smem_offset_coef(int T) {
+// the quotas of the current round (double, indexed by m) follow nf
+__host__ __device__ inline size_t temporal_smem_quota(int T) {
     return (temporal_smem_keys(T) + (size_t)T * (8 + 4 + 4 + 4) + 7) & ~(size_t)7;
 }
+__host__ __device__ inline size_t temporal_smem_offset_coef(int T) { return temporal_smem_quota(T) + (size_t)T * 8; }
 // WTA coefficient arrays: the longest subband of any level (any filter).
 __host__ __device__ inline int temporal_coef_len(int T, int J) {
     const int k = (T + kMaxTaps - 1) / 2;
@@ -228,6 +230,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     int *lst = reinterpret_cast<int *>(keys + T);                         // retained frames
     int *nb = lst + T;                     // budget of retained frame m; -1 while active
     int *nf = nb + T;                      // budget of frame t
+    double *qv = reinterpret_cast<double *>(tsm + temporal_smem_quota(T));   // quota of retained frame m
     const int J = c.wta_levels;
     const int KH = temporal_coef_len(T, J);
     double *A0 = reinterpret_cast<double *>(tsm + temporal_smem_offset_coef(T));   // WTA approximation
@@ -252,8 +255,16 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         keep[k] = 0;
         if (k < per && t < T) {
             const double d = fr[4 * t + 1];
-            fr[4 * t + 2] = hi > lo ? (d - lo) / (hi - lo) : 0.0;
+            const double gm = hi > lo ? (d - lo) / (hi - lo) : 0.0;
+            fr[4 * t + 2] = gm;
             fr[4 * t + 3] = NAN;
+            if (c.out_rel) {   // r~ follows with the WTA (NaN: filtered)
+                float *orl = c.out_rel + (base + t) * 4;
+                orl[0] = (float)fr[4 * t];
+                orl[1] = (float)d;
+                orl[2] = (float)gm;
+                orl[3] = NAN;
+            }
             keep[k] = (t == 0 || d >= tau) ? 1 : 0;
             cnt += keep[k];
             nf[t] = 0;
@@ -302,6 +313,7 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         }
         const int t = lst[m];
         fr[4 * t + 3] = rt;
+        if (c.out_rel) c.out_rel[(base + t) * 4 + 3] = (float)rt;
         const double wv = c.temporal_mode == WZ_TEMPORAL_WTA ? rt
                           : c.temporal_mode == WZ_TEMPORAL_RAW ? fr[4 * t] : 1.0;
         wgt[m] = fmax(wv, 0.0);
@@ -358,42 +370,48 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
                     ncap += (q > (double)N);
                     fsum += (long long)fl;
                     key = (unsigned long long)__double_as_longlong(q - fl) + 1ull;
+                    qv[m] = q;
                 }
                 keys[m] = key;
             }
             block_sum2_ll(ncap, fsum, lscr);
             if (ncap > 0) {
-                for (int m = threadIdx.x; m < L; m += blockDim.x) {
-                    const double w = uniform ? 1.0 : wgt[m];
-                    if (keys[m] != 0ull && (double)remaining * w / S > (double)N) nb[m] = N;
-                }
+                for (int m = threadIdx.x; m < L; m += blockDim.x)
+                    if (keys[m] != 0ull && qv[m] > (double)N) nb[m] = N;
                 remaining -= (long long)N * ncap;
                 __syncthreads();
                 continue;
             }
-            for (int m = threadIdx.x; m < L; m += blockDim.x)
-                if (keys[m] != 0ull) {   // floor; the remainder unit is added below
-                    const double w = uniform ? 1.0 : wgt[m];
-                    nb[m] = (int)floor((double)remaining * w / S);
-                }
             const long long R = remaining - fsum;
             const ulonglong2 *k2 = reinterpret_cast<const ulonglong2 *>(keys);
-            for (int m = threadIdx.x; m < L; m += blockDim.x) {
-                const unsigned long long km = keys[m];
-                // rank = #{k : key_k > key_m, or key_k == key_m and k < m}; the
-                // same loop in every lane: broadcast 16-byte reads of two keys
+            // rank = #{k : key_k > key_m, or key_k == key_m and k < m}, counted
+            // by gs lanes per frame (the largest power of two <= 32 with
+            // gs * L <= threads), each over every gs-th pair of keys with
+            // broadcast 16-byte reads, summed by shuffles; the floor and the
+            // remainder unit together
+            int gs = 1;
+            while (gs < 32 && 2 * gs * L <= (int)blockDim.x) gs <<= 1;
+            const int sl = threadIdx.x & (gs - 1);
+            for (int b0 = 0; b0 < L * gs; b0 += blockDim.x) {
+                const int m = (b0 + (int)threadIdx.x) / gs;
+                const bool on = m < L;
+                const unsigned long long km = on ? keys[m] : 0ull;
                 int r0 = 0, r1 = 0;
+                if (on) {
 #pragma unroll 4
-                for (int i = 0; i < (L >> 1); ++i) {
-                    const ulonglong2 p = k2[i];
-                    r0 += (p.x > km) | ((p.x == km) & (2 * i < m));
-                    r1 += (p.y > km) | ((p.y == km) & (2 * i + 1 < m));
+                    for (int i = sl; i < (L >> 1); i += gs) {
+                        const ulonglong2 p = k2[i];
+                        r0 += (p.x > km) | ((p.x == km) & (2 * i < m));
+                        r1 += (p.y > km) | ((p.y == km) & (2 * i + 1 < m));
+                    }
+                    if ((L & 1) && sl == 0) {
+                        const unsigned long long p = keys[L - 1];
+                        r0 += (p > km) | ((p == km) & (L - 1 < m));
+                    }
                 }
-                if (L & 1) {
-                    const unsigned long long p = keys[L - 1];
-                    r0 += (p > km) | ((p == km) & (L - 1 < m));
-                }
-                if (km != 0ull && r0 + r1 < R) nb[m] += 1;
+                int r = r0 + r1;
+                for (int o = 1; o < gs; o <<= 1) r += __shfl_xor_sync(0xffffffffu, r, o);
+                if (on && sl == 0 && km != 0ull) nb[m] = (int)floor(qv[m]) + (r < R ? 1 : 0);
             }
             __syncthreads();
             break;
@@ -426,8 +444,9 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
         if (tc)
             for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
                 const int nc = min(kColBlock, nloc[k] - j0);
-                const int cg = unit_tiles((nc + 15) / 16 * 16);
-                (j0 == 0 ? ucnt[k] : ucntB[k]) += (c.n_ct + cg - 1) / cg;
+                const int cg = unit_tiles((nc + 15) / 16 * 16), add = (c.n_ct + cg - 1) / cg;
+                if (j0 == 0) ucnt[k] += add;
+                else ucntB[k] += add;
             }
         part[0] += nloc[k];
         part[1] += (nloc[k] + 15) & ~15;
@@ -452,13 +471,6 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
             c.hw[2 * (base + t)] = h;
             c.hw[2 * (base + t) + 1] = h > 0 ? (nloc[k] + h - 1) / h : 0;
             if (c.out_budgets) c.out_budgets[base + t] = nloc[k];
-            if (c.out_rel) {
-                float *orl = c.out_rel + (base + t) * 4;
-                orl[0] = (float)fr[4 * t];
-                orl[1] = (float)fr[4 * t + 1];
-                orl[2] = (float)fr[4 * t + 2];
-                orl[3] = (float)fr[4 * t + 3];
-            }
         }
         o += nloc[k];
         wo += (nloc[k] + 15) & ~15;
