@@ -42,7 +42,7 @@ UNIT = "frames/s"
 WORKLOAD = "video256_27x27_bf16"
 KERNELS = ("query_pool", "relevance", "frame_stats", "temporal", "spatial", "condense")
 KERNEL_SOURCES = {"query_pool": "relevance.cu", "relevance": "relevance.cu", "frame_stats": "relevance.cu",
-                  "temporal": "temporal.cu", "spatial": "spatial.cu", "condense": "condense_tc.cu"}
+                  "temporal": "temporal.cu", "spatial": "spatial_tc.cu", "condense": "condense_tc.cu"}
 L2_BYTES = 129 * 10**6          # GB300 L2
 L2_FLUSH_BYTES = 512 << 20
 BATCH_CPU_VIDEOS = 16           # cpu_baseline sample of the serving batch: its first 16 videos (~12 s on one core)

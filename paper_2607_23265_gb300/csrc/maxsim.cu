@@ -7,10 +7,13 @@
 //   a_{t,n} = max_{j < Lq} <u_{t,n}, q_j / ||q_j||> / ||u_{t,n}||
 //
 // Token tiles of 128 rows (M) x K steps of 64 channels: A = the features,
-// K-major, one 2D TMA box {64, 128} with 128-byte swizzle; B = the unit
-// query rows as bf16 hi rows then lo rows (query_rows_kernel), N = 2 Lqp <=
-// 256, box {64, 2 Lqp}; fp32 accumulators in tensor memory, two buffers, so
-// the epilogue of a tile overlaps the main loop of the next.  CTA c covers
+// K-major with 128-byte swizzle; B = the unit query rows as bf16 hi rows then
+// lo rows (query_rows_kernel), N = 2 Lqp <= 256.  A ring stage holds G
+// consecutive K steps of both, each loaded by one 3D TMA box ({64, 128, G}
+// and {64, 2 Lqp, G}): a token row arrives as G * 128 contiguous bytes per
+// load, not 128, which keeps HBM reads efficient.  fp32 accumulators in
+// tensor memory, two buffers, so the epilogue of a tile overlaps the main
+// loop of the next.  CTA c covers
 // the tokens [c L1, (c+1) L1), exactly as the relevance pass does, and writes
 // its channel sums of every frame it touches into partial slot c + t, so
 // frame_stats_kernel reads them unchanged.
@@ -46,6 +49,8 @@ namespace {
 constexpr int kXM = 128, kXK = 64;
 constexpr int kXABytes = kXM * kXK * 2;             // 16 KB
 constexpr int kXMaxStages = 8;
+constexpr int kXGroups = 4;                         // K steps per ring stage (at most)
+constexpr int kXMinStages = 2;
 constexpr int kXThreads = 10 * 32;
 constexpr int kXAccCols = 256;
 constexpr uint64_t kXTimeoutNs = 2000000000ull;
@@ -69,7 +74,8 @@ struct XMaps {
 };
 
 struct XArgs {
-    int stages, stage_stride;   // ring stages and bytes per stage (A then B)
+    int stages, stage_stride;   // ring stages and bytes per stage (G A tiles, then G B tiles)
+    int G;                      // K steps per stage
     int Lq, Lqp;
     int acc_off;                // byte offset of the two channel-sum buffers (2 x D floats)
     int shared_off;             // byte offset of XShared
@@ -157,7 +163,8 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
         // ---------------- TMA producer ----------------
         const uint64_t pol_a = ptx::policy_evict_first();
         const uint64_t pol_b = ptx::policy_evict_last();
-        const uint32_t stage_bytes = (uint32_t)kXABytes + 2u * (uint32_t)p.Lqp * kXK * 2u;
+        const uint32_t b_bytes = 2u * (uint32_t)p.Lqp * kXK * 2u;
+        const uint32_t stage_bytes = (uint32_t)p.G * ((uint32_t)kXABytes + b_bytes);
         int stage = 0;
         uint32_t phase = 0;
         int issued_parity[kXMaxStages];
@@ -167,7 +174,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             int nr;
             xtile(c, it, base, nr);
             bool ok = true;
-            for (int ks = 0; ks < KS; ++ks) {
+            for (int ks = 0; ks < KS; ks += p.G) {
                 if (!ptx::mbar_wait(&S->empty[stage], phase ^ 1u, kXTimeoutNs)) {
                     xfail(c, abort_flag, 16);
                     ok = false;
@@ -175,8 +182,8 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                 }
                 uint8_t *st = ring + (size_t)stage * p.stage_stride;
                 ptx::mbar_arrive_expect_tx(&S->full[stage], stage_bytes);
-                ptx::tma_load_2d(st, &maps.a, &S->full[stage], ks * kXK, (int)base, pol_a);
-                ptx::tma_load_2d(st + kXABytes, &maps.b, &S->full[stage], ks * kXK, 0, pol_b);
+                ptx::tma_load_3d(st, &maps.a, &S->full[stage], 0, (int)base, ks, pol_a);
+                ptx::tma_load_3d(st + p.G * kXABytes, &maps.b, &S->full[stage], 0, 0, ks, pol_b);
                 issued_parity[stage] = (int)phase;
                 if (++stage == p.stages) {
                     stage = 0;
@@ -192,7 +199,8 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
         const uint32_t idesc = ptx::idesc_bf16(kXM, 2 * p.Lqp, false, false);   // both K-major
         const uint32_t ring32 = ptx::smem_u32(ring);
         const uint64_t a_base = ptx::smem_desc(ring32, 16, 1024, 2);              // 128-B swizzle
-        const uint64_t b_base = ptx::smem_desc(ring32 + kXABytes, 16, 1024, 2);
+        const uint64_t b_base = ptx::smem_desc(ring32 + (uint32_t)(p.G * kXABytes), 16, 1024, 2);
+        const uint64_t b_sub = (uint64_t)((2 * p.Lqp * kXK * 2) >> 4);   // one K step of B
         const uint64_t stage_desc = (uint64_t)(p.stage_stride >> 4);
         int stage = 0;
         uint32_t phase = 0;
@@ -206,7 +214,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             ptx::tc_fence_after();
             const uint32_t d = tmem + (uint32_t)(b * kXAccCols);
             bool ok = true;
-            for (int ks = 0; ks < KS; ++ks) {
+            for (int ks = 0; ks < KS; ks += p.G) {
                 if (!ptx::mbar_wait(&S->full[stage], phase, kXTimeoutNs)) {
                     xfail(c, abort_flag, 16);
                     ok = false;
@@ -214,10 +222,13 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                 }
                 ptx::tc_fence_after();
                 const uint64_t so = (uint64_t)stage * stage_desc;
+                for (int g = 0; g < p.G; ++g) {
+                    const uint64_t ao = so + (uint64_t)g * (kXABytes >> 4), bo = so + (uint64_t)g * b_sub;
 #pragma unroll
-                for (int k = 0; k < kXK / 16; ++k)   // K = 16 per MMA: 32 bytes along the swizzled row
-                    ptx::mma_bf16(d, a_base + so + (uint64_t)(2 * k), b_base + so + (uint64_t)(2 * k), idesc,
-                                  (ks | k) ? 1u : 0u);
+                    for (int k = 0; k < kXK / 16; ++k)   // K = 16 per MMA: 32 bytes along the swizzled row
+                        ptx::mma_bf16(d, a_base + ao + (uint64_t)(2 * k), b_base + bo + (uint64_t)(2 * k), idesc,
+                                      (ks | g | k) ? 1u : 0u);
+                }
                 ptx::mma_commit(&S->empty[stage]);
                 if (++stage == p.stages) {
                     stage = 0;
@@ -294,47 +305,52 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
 #pragma unroll
             for (int i = 0; i < 32; ++i) sq[i] = 0.f;
             bool ok = true;
-            for (int ks = 0; ks < KS; ++ks) {
+            for (int ks = 0; ks < KS; ks += p.G) {
                 if (!ptx::mbar_wait(&S->full[stage], phase, kXTimeoutNs)) {
                     xfail(c, abort_flag, 32);
                     ok = false;
                     break;
                 }
-                const uint32_t st32 = ptx::smem_u32(ring + (size_t)stage * p.stage_stride);
-                float s0x = 0.f, s0y = 0.f, s1x = 0.f, s1y = 0.f;
+                const uint32_t st0 = ptx::smem_u32(ring + (size_t)stage * p.stage_stride);
+                for (int g = 0; g < p.G; ++g) {
+                    const uint32_t st32 = st0 + (uint32_t)(g * kXABytes);
+                    float s0x = 0.f, s0y = 0.f, s1x = 0.f, s1y = 0.f;
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int r = 32 * rq + ((i + 2 * rq) & 31);
-                    uint32_t wv;
-                    asm volatile("ld.shared.b32 %0, [%1];"
-                                 : "=r"(wv)
-                                 : "r"(st32 + (uint32_t)(r * 128 + ((chunk ^ (r & 7)) << 4)) + coff));
-                    const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
-                    sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
-                    if (r < rb) {
-                        s0x += x;
-                        s0y += y;
-                    } else if (r < nr) {
-                        s1x += x;
-                        s1y += y;
+                    for (int i = 0; i < 32; ++i) {
+                        const int r = 32 * rq + ((i + 2 * rq) & 31);
+                        uint32_t wv;
+                        asm volatile("ld.shared.b32 %0, [%1];"
+                                     : "=r"(wv)
+                                     : "r"(st32 + (uint32_t)(r * 128 + ((chunk ^ (r & 7)) << 4)) + coff));
+                        const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
+                        sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
+                        if (r < rb) {
+                            s0x += x;
+                            s0y += y;
+                        } else if (r < nr) {
+                            s1x += x;
+                            s1y += y;
+                        }
                     }
-                }
-                __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(&S->empty[stage]);
+                    if (g == p.G - 1) {   // the stage's last K step is in registers: hand the stage back
+                        __syncwarp();
+                        if (lane == 0) ptx::mbar_arrive(&S->empty[stage]);
+                    }
 #pragma unroll
-                for (int o = 8; o < 32; o <<= 1) {   // the four row quarters, in a fixed order
-                    s0x += __shfl_xor_sync(0xffffffffu, s0x, o);
-                    s0y += __shfl_xor_sync(0xffffffffu, s0y, o);
-                    s1x += __shfl_xor_sync(0xffffffffu, s1x, o);
-                    s1y += __shfl_xor_sync(0xffffffffu, s1y, o);
-                }
-                if (rq == 0) {
-                    const int ch = ks * kXK + cw;
-                    acc_open[ch] += s0x;
-                    acc_open[ch + 1] += s0y;
-                    if (rb < nr) {
-                        acc_next[ch] += s1x;
-                        acc_next[ch + 1] += s1y;
+                    for (int o = 8; o < 32; o <<= 1) {   // the four row quarters, in a fixed order
+                        s0x += __shfl_xor_sync(0xffffffffu, s0x, o);
+                        s0y += __shfl_xor_sync(0xffffffffu, s0y, o);
+                        s1x += __shfl_xor_sync(0xffffffffu, s1x, o);
+                        s1y += __shfl_xor_sync(0xffffffffu, s1y, o);
+                    }
+                    if (rq == 0) {
+                        const int ch = (ks + g) * kXK + cw;
+                        acc_open[ch] += s0x;
+                        acc_open[ch + 1] += s0y;
+                        if (rb < nr) {
+                            acc_next[ch] += s1x;
+                            acc_next[ch + 1] += s1y;
+                        }
                     }
                 }
                 if (++stage == p.stages) {
@@ -397,28 +413,37 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
 
 namespace {
 
+// [rows][cols] bf16 as {64 channels, rows, cols / 64 K steps}: box {64,
+// box_rows, G}, i.e. G consecutive K-step tiles of box_rows rows.
 bool xencode(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap *m, const void *base, int64_t rows, int cols,
-             int box_rows) {
-    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
-    cuuint32_t box[2] = {(cuuint32_t)kXK, (cuuint32_t)box_rows};
-    cuuint32_t es[2] = {1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
+             int box_rows, int G) {
+    cuuint64_t dims[3] = {(cuuint64_t)kXK, (cuuint64_t)rows, (cuuint64_t)(cols / kXK)};
+    cuuint64_t strides[2] = {(cuuint64_t)cols * 2, (cuuint64_t)kXK * 2};
+    cuuint32_t box[3] = {(cuuint32_t)kXK, (cuuint32_t)box_rows, (cuuint32_t)G};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 struct XLayout {
-    int stages, stride, acc_off, shared_off;
+    int stages, stride, G, acc_off, shared_off;
     size_t smem;
 };
 
+// K steps per stage: the most of kXGroups (dividing the D / 64 K steps)
+// that still leaves kXMinStages stages.
 XLayout xlayout(int D, int Lqp) {
     XLayout L{};
-    L.stride = (kXABytes + 2 * Lqp * kXK * 2 + 1023) / 1024 * 1024;
     const size_t fixed = 1024 + (size_t)2 * D * 4 + (sizeof(XShared) + 127) / 128 * 128;
     const size_t cap = 227 * 1024;
-    L.stages = fixed < cap ? (int)((cap - fixed) / (size_t)L.stride) : 0;
+    for (int G = kXGroups; G >= 1; --G) {
+        if ((D / kXK) % G != 0) continue;
+        L.G = G;
+        L.stride = G * (kXABytes + 2 * Lqp * kXK * 2);   // multiples of 1 KB (2 Lqp % 16 == 0)
+        L.stages = fixed < cap ? (int)((cap - fixed) / (size_t)L.stride) : 0;
+        if (L.stages >= kXMinStages) break;
+    }
     if (L.stages > kXMaxStages) L.stages = kXMaxStages;
     L.acc_off = L.stages * L.stride;
     L.shared_off = L.acc_off + 2 * D * 4;
@@ -442,12 +467,14 @@ cudaError_t launch_maxsim_pass(const Ctx &c, int Lq, int Lqp, cudaStream_t s) {
     if (!enc) return cudaErrorNotSupported;
     XMaps maps;
     memset(&maps, 0, sizeof(maps));
-    if (!xencode(enc, &maps.a, c.X, (int64_t)c.T * c.N, c.D, kXM) || !xencode(enc, &maps.b, c.qhl, 2 * Lqp, c.D, 2 * Lqp))
-        return cudaErrorInvalidValue;
     const XLayout L = xlayout(c.D, Lqp);
+    if (!xencode(enc, &maps.a, c.X, (int64_t)c.T * c.N, c.D, kXM, L.G) ||
+        !xencode(enc, &maps.b, c.qhl, 2 * Lqp, c.D, 2 * Lqp, L.G))
+        return cudaErrorInvalidValue;
     XArgs p{};
     p.stages = L.stages;
     p.stage_stride = L.stride;
+    p.G = L.G;
     p.Lq = Lq;
     p.Lqp = Lqp;
     p.acc_off = L.acc_off;
