@@ -8,16 +8,18 @@
 //
 // Token tiles of 128 rows (M) x K steps of 64 channels: A = the features,
 // K-major with 128-byte swizzle; B = the unit query rows as bf16 hi rows then
-// lo rows (query_rows_kernel), N = 2 Lqp <= 256.  A ring stage holds G
-// consecutive K steps of both, each loaded by one 3D TMA box ({64, 128, G}
-// and {64, 2 Lqp, G}): a token row arrives as G * 128 contiguous bytes per
-// load, not 128, which keeps HBM reads efficient.  fp32 accumulators in
-// tensor memory, two buffers, so the epilogue of a tile overlaps the main
-// loop of the next.  CTA c covers
-// the tokens [c L1, (c+1) L1), exactly as the relevance pass does, and writes
-// its channel sums of every frame it touches into partial slot c + t, so
-// frame_stats_kernel reads them unchanged.
-//   warp 0       TMA producer (one thread)
+// lo rows (query_rows_kernel), N = 2 Lqp <= 256.  A stage holds G
+// consecutive K steps, loaded by one 3D TMA box ({64, 128, G} for the
+// features, {64, 2 Lqp, G} for the query rows): a token row arrives as G * 128
+// contiguous bytes per load, not 128, which keeps HBM reads efficient.  The
+// features and the query rows have rings of their own, so the query rows
+// (read from L2 for every tile) take two stages and the rest of shared memory
+// keeps feature reads in flight.  fp32 accumulators in tensor memory, two
+// buffers, so the epilogue of a tile overlaps the main loop of the next.
+// CTA c covers the tokens [c L1, (c+1) L1), exactly as the relevance pass
+// does, and writes its channel sums of every frame it touches into partial
+// slot c + t, so frame_stats_kernel reads them unchanged.
+//   warp 0       TMA producer of the features (one thread)
 //   warp 1       TMEM allocation and the MMA issuer (one thread)
 //   warps 2-5    epilogue: tcgen05.ld (TMEM lane = token) -> max over the
 //                query rows of hi + lo -> / ||u|| -> a_{t,n}
@@ -32,6 +34,7 @@
 //                starts inside a tile) accumulate in shared memory and are
 //                written to the frame's slot when the frame ends or the
 //                CTA's range does
+//   warp 10      TMA producer of the query rows (one thread)
 // Every mbarrier wait is bounded; on a timeout the kernel records a status
 // bit, drains what it issued, frees tensor memory and exits.
 #include <cuda.h>
@@ -51,14 +54,17 @@ constexpr int kXABytes = kXM * kXK * 2;             // 16 KB
 constexpr int kXMaxStages = 8;
 constexpr int kXGroups = 4;                         // K steps per ring stage (at most)
 constexpr int kXMinStages = 2;
-constexpr int kXThreads = 10 * 32;
+constexpr int kXThreads = 11 * 32;
+constexpr int kXBStages = 2;                        // query-row stages (their own ring)
 constexpr int kXAccCols = 256;
 constexpr uint64_t kXTimeoutNs = 2000000000ull;
 constexpr int kXReaders = 4;                        // channel-sum warps reading each stage
 
 struct XShared {
-    uint64_t full[kXMaxStages];
+    uint64_t full[kXMaxStages];    // feature ring
     uint64_t empty[kXMaxStages];
+    uint64_t bfull[kXBStages];     // query-row ring
+    uint64_t bempty[kXBStages];
     uint64_t tfull[2], tempty[2];
     uint64_t nfull[2], nempty[2];
     uint64_t csync[2];
@@ -74,7 +80,8 @@ struct XMaps {
 };
 
 struct XArgs {
-    int stages, stage_stride;   // ring stages and bytes per stage (G A tiles, then G B tiles)
+    int stages, stage_stride;   // feature ring: stages and bytes per stage (G A tiles)
+    int b_off, b_stride;        // query-row ring (kXBStages stages of G B tiles): byte offset, bytes per stage
     int G;                      // K steps per stage
     int Lq, Lqp;
     int acc_off;                // byte offset of the two channel-sum buffers (2 x D floats)
@@ -129,6 +136,10 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             ptx::mbar_init(&S->full[s], 1);
             ptx::mbar_init(&S->empty[s], 1 + kXReaders);
         }
+        for (int s = 0; s < kXBStages; ++s) {
+            ptx::mbar_init(&S->bfull[s], 1);
+            ptx::mbar_init(&S->bempty[s], 1);
+        }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(&S->tfull[b], 1);
             ptx::mbar_init(&S->tempty[b], 4);
@@ -160,11 +171,9 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
     const int KS = c.D / kXK;
 
     if (warp == 0 && lane == 0) {
-        // ---------------- TMA producer ----------------
+        // ---------------- TMA producer: features ----------------
         const uint64_t pol_a = ptx::policy_evict_first();
-        const uint64_t pol_b = ptx::policy_evict_last();
-        const uint32_t b_bytes = 2u * (uint32_t)p.Lqp * kXK * 2u;
-        const uint32_t stage_bytes = (uint32_t)p.G * ((uint32_t)kXABytes + b_bytes);
+        const uint32_t stage_bytes = (uint32_t)p.G * (uint32_t)kXABytes;
         int stage = 0;
         uint32_t phase = 0;
         int issued_parity[kXMaxStages];
@@ -183,7 +192,6 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                 uint8_t *st = ring + (size_t)stage * p.stage_stride;
                 ptx::mbar_arrive_expect_tx(&S->full[stage], stage_bytes);
                 ptx::tma_load_3d(st, &maps.a, &S->full[stage], 0, (int)base, ks, pol_a);
-                ptx::tma_load_3d(st + p.G * kXABytes, &maps.b, &S->full[stage], 0, 0, ks, pol_b);
                 issued_parity[stage] = (int)phase;
                 if (++stage == p.stages) {
                     stage = 0;
@@ -194,16 +202,45 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
         }
         for (int s = 0; s < p.stages; ++s)
             if (issued_parity[s] >= 0) ptx::mbar_wait(&S->full[s], (uint32_t)issued_parity[s], kXTimeoutNs);
+    } else if (warp == 10 && lane == 0) {
+        // ---------------- TMA producer: query rows (from L2), K step by K step ----------------
+        const uint64_t pol_b = ptx::policy_evict_last();
+        const uint32_t stage_bytes = (uint32_t)p.G * 2u * (uint32_t)p.Lqp * kXK * 2u;
+        int stage = 0;
+        uint32_t phase = 0;
+        int issued_parity[kXBStages];
+        for (int s = 0; s < kXBStages; ++s) issued_parity[s] = -1;
+        for (int it = 0; it < ntile && !*abort_flag; ++it) {
+            bool ok = true;
+            for (int ks = 0; ks < KS; ks += p.G) {
+                if (!ptx::mbar_wait(&S->bempty[stage], phase ^ 1u, kXTimeoutNs)) {
+                    xfail(c, abort_flag, 16);
+                    ok = false;
+                    break;
+                }
+                ptx::mbar_arrive_expect_tx(&S->bfull[stage], stage_bytes);
+                ptx::tma_load_3d(ring + p.b_off + (size_t)stage * p.b_stride, &maps.b, &S->bfull[stage], 0, 0, ks,
+                                 pol_b);
+                issued_parity[stage] = (int)phase;
+                if (++stage == kXBStages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok) break;
+        }
+        for (int s = 0; s < kXBStages; ++s)
+            if (issued_parity[s] >= 0) ptx::mbar_wait(&S->bfull[s], (uint32_t)issued_parity[s], kXTimeoutNs);
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer ----------------
         const uint32_t idesc = ptx::idesc_bf16(kXM, 2 * p.Lqp, false, false);   // both K-major
         const uint32_t ring32 = ptx::smem_u32(ring);
         const uint64_t a_base = ptx::smem_desc(ring32, 16, 1024, 2);              // 128-B swizzle
-        const uint64_t b_base = ptx::smem_desc(ring32 + (uint32_t)(p.G * kXABytes), 16, 1024, 2);
+        const uint64_t b_base = ptx::smem_desc(ring32 + (uint32_t)p.b_off, 16, 1024, 2);
         const uint64_t b_sub = (uint64_t)((2 * p.Lqp * kXK * 2) >> 4);   // one K step of B
-        const uint64_t stage_desc = (uint64_t)(p.stage_stride >> 4);
-        int stage = 0;
-        uint32_t phase = 0;
+        const uint64_t stage_desc = (uint64_t)(p.stage_stride >> 4), bstage_desc = (uint64_t)(p.b_stride >> 4);
+        int stage = 0, bstage = 0;
+        uint32_t phase = 0, bphase = 0;
         for (int it = 0; it < ntile && !*abort_flag; ++it) {
             const int b = it & 1;
             const uint32_t use = (uint32_t)(it >> 1);
@@ -215,24 +252,30 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             const uint32_t d = tmem + (uint32_t)(b * kXAccCols);
             bool ok = true;
             for (int ks = 0; ks < KS; ks += p.G) {
-                if (!ptx::mbar_wait(&S->full[stage], phase, kXTimeoutNs)) {
+                if (!ptx::mbar_wait(&S->full[stage], phase, kXTimeoutNs) ||
+                    !ptx::mbar_wait(&S->bfull[bstage], bphase, kXTimeoutNs)) {
                     xfail(c, abort_flag, 16);
                     ok = false;
                     break;
                 }
                 ptx::tc_fence_after();
-                const uint64_t so = (uint64_t)stage * stage_desc;
+                const uint64_t so = (uint64_t)stage * stage_desc, sbo = (uint64_t)bstage * bstage_desc;
                 for (int g = 0; g < p.G; ++g) {
-                    const uint64_t ao = so + (uint64_t)g * (kXABytes >> 4), bo = so + (uint64_t)g * b_sub;
+                    const uint64_t ao = so + (uint64_t)g * (kXABytes >> 4), bo = sbo + (uint64_t)g * b_sub;
 #pragma unroll
                     for (int k = 0; k < kXK / 16; ++k)   // K = 16 per MMA: 32 bytes along the swizzled row
                         ptx::mma_bf16(d, a_base + ao + (uint64_t)(2 * k), b_base + bo + (uint64_t)(2 * k), idesc,
                                       (ks | g | k) ? 1u : 0u);
                 }
                 ptx::mma_commit(&S->empty[stage]);
+                ptx::mma_commit(&S->bempty[bstage]);
                 if (++stage == p.stages) {
                     stage = 0;
                     phase ^= 1u;
+                }
+                if (++bstage == kXBStages) {
+                    bstage = 0;
+                    bphase ^= 1u;
                 }
             }
             if (!ok) break;
@@ -279,16 +322,22 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                 ptx::mbar_arrive(&S->nempty[b]);
             }
         }
-    } else if (warp >= 6) {
+    } else if (warp >= 6 && warp < 10) {
         // ---------------- per-frame channel sums ----------------
         // lane: channel pair p2 of this warp's 16 channels of a K step, and
-        // the quarter of the tile's rows it sums (each quarter walks its rows
-        // from a different start, which keeps the quarters on different banks)
+        // the quarter rq of the tile's rows it sums.  Its i-th row is
+        // 32 rq + (i ^ 2 rq) (each quarter walks its rows in another order,
+        // which keeps the quarters on different banks); with the 128-byte
+        // swizzle (16-byte chunk k of row r at r * 128 + ((k ^ (r & 7)) << 4))
+        // that row's word sits at lane_off + (xo(i) ^ xl), xo(i) a constant
+        // of the unrolled loop and xl one of the lane
         const int wsel = warp - 6;
         const int p2 = lane & 7, rq = lane >> 3;
         const int cw = wsel * 16 + 2 * p2;              // channels cw, cw + 1 of the K step
         const uint32_t coff = (uint32_t)((cw * 2) & 15);
         const int chunk = (cw * 2) >> 4;
+        const uint32_t lane_off = (uint32_t)(rq * 4096) + coff;
+        const uint32_t xl = ((uint32_t)rq << 8) | ((uint32_t)(chunk ^ (2 * rq)) << 4);
         float *acc_open = acc_buf, *acc_next = acc_buf + c.D;
         int64_t open_f = ntile > 0 ? ((int64_t)blockIdx.x * c.L1) / c.N : 0;
         bool open_has = false;
@@ -301,7 +350,8 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             // a frame starts inside the tile at row rb (frames have >= 128 tokens)
             const int to_end = (int)((int64_t)c.N - base % c.N);
             const int rb = to_end < nr ? to_end : nr;
-            float sq[32];   // squares of this lane's two channels, row 32 rq + ((i + 2 rq) & 31)
+            float sq[32];   // squares of this lane's two channels, row 32 rq + (i ^ 2 rq)
+            const bool whole = rb == kXM;   // every row of the tile in the open frame
 #pragma unroll
             for (int i = 0; i < 32; ++i) sq[i] = 0.f;
             bool ok = true;
@@ -313,23 +363,35 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                 }
                 const uint32_t st0 = ptx::smem_u32(ring + (size_t)stage * p.stage_stride);
                 for (int g = 0; g < p.G; ++g) {
-                    const uint32_t st32 = st0 + (uint32_t)(g * kXABytes);
+                    const uint32_t lb = st0 + (uint32_t)(g * kXABytes) + lane_off;
                     float s0x = 0.f, s0y = 0.f, s1x = 0.f, s1y = 0.f;
+                    if (whole) {
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const int r = 32 * rq + ((i + 2 * rq) & 31);
-                        uint32_t wv;
-                        asm volatile("ld.shared.b32 %0, [%1];"
-                                     : "=r"(wv)
-                                     : "r"(st32 + (uint32_t)(r * 128 + ((chunk ^ (r & 7)) << 4)) + coff));
-                        const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
-                        sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
-                        if (r < rb) {
+                        for (int i = 0; i < 32; ++i) {
+                            const uint32_t xo = ((uint32_t)i << 7) | ((uint32_t)(i & 7) << 4);
+                            uint32_t wv;
+                            asm volatile("ld.shared.b32 %0, [%1];" : "=r"(wv) : "r"(lb + (xo ^ xl)));
+                            const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
+                            sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
                             s0x += x;
                             s0y += y;
-                        } else if (r < nr) {
-                            s1x += x;
-                            s1y += y;
+                        }
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const int r = 32 * rq + (i ^ (2 * rq));
+                            const uint32_t xo = ((uint32_t)i << 7) | ((uint32_t)(i & 7) << 4);
+                            uint32_t wv;
+                            asm volatile("ld.shared.b32 %0, [%1];" : "=r"(wv) : "r"(lb + (xo ^ xl)));
+                            const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
+                            sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
+                            if (r < rb) {
+                                s0x += x;
+                                s0y += y;
+                            } else if (r < nr) {
+                                s1x += x;
+                                s1y += y;
+                            }
                         }
                     }
                     if (g == p.G - 1) {   // the stage's last K step is in registers: hand the stage back
@@ -369,7 +431,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                 v += __shfl_xor_sync(0xffffffffu, v, 1);
                 v += __shfl_xor_sync(0xffffffffu, v, 2);
                 v += __shfl_xor_sync(0xffffffffu, v, 4);
-                if (p2 == 0) S->npart[b][wsel][32 * rq + ((i + 2 * rq) & 31)] = v;
+                if (p2 == 0) S->npart[b][wsel][32 * rq + (i ^ (2 * rq))] = v;
             }
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&S->csync[b]);
@@ -427,12 +489,13 @@ bool xencode(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap *m, const void *
 }
 
 struct XLayout {
-    int stages, stride, G, acc_off, shared_off;
+    int stages, stride, G, b_off, b_stride, acc_off, shared_off;
     size_t smem;
 };
 
 // K steps per stage: the most of kXGroups (dividing the D / 64 K steps)
-// that still leaves kXMinStages stages.
+// that leaves kXMinStages feature stages beside the kXBStages query-row
+// stages.
 XLayout xlayout(int D, int Lqp) {
     XLayout L{};
     const size_t fixed = 1024 + (size_t)2 * D * 4 + (sizeof(XShared) + 127) / 128 * 128;
@@ -440,12 +503,15 @@ XLayout xlayout(int D, int Lqp) {
     for (int G = kXGroups; G >= 1; --G) {
         if ((D / kXK) % G != 0) continue;
         L.G = G;
-        L.stride = G * (kXABytes + 2 * Lqp * kXK * 2);   // multiples of 1 KB (2 Lqp % 16 == 0)
-        L.stages = fixed < cap ? (int)((cap - fixed) / (size_t)L.stride) : 0;
+        L.stride = G * kXABytes;
+        L.b_stride = G * 2 * Lqp * kXK * 2;   // multiples of 1 KB (2 Lqp % 16 == 0)
+        const size_t used = fixed + (size_t)kXBStages * L.b_stride;
+        L.stages = used < cap ? (int)((cap - used) / (size_t)L.stride) : 0;
         if (L.stages >= kXMinStages) break;
     }
     if (L.stages > kXMaxStages) L.stages = kXMaxStages;
-    L.acc_off = L.stages * L.stride;
+    L.b_off = L.stages * L.stride;
+    L.acc_off = L.b_off + kXBStages * L.b_stride;
     L.shared_off = L.acc_off + 2 * D * 4;
     L.smem = 1024 + (size_t)L.shared_off + sizeof(XShared);
     return L;
@@ -474,6 +540,8 @@ cudaError_t launch_maxsim_pass(const Ctx &c, int Lq, int Lqp, cudaStream_t s) {
     XArgs p{};
     p.stages = L.stages;
     p.stage_stride = L.stride;
+    p.b_off = L.b_off;
+    p.b_stride = L.b_stride;
     p.G = L.G;
     p.Lq = Lq;
     p.Lqp = Lqp;
