@@ -21,19 +21,19 @@
 // slot c + t, so frame_stats_kernel reads them unchanged.
 //   warp 0       TMA producer of the features (one thread)
 //   warp 1       TMEM allocation and the MMA issuer (one thread)
-//   warps 2-5    epilogue: tcgen05.ld (TMEM lane = token) -> max over the
-//                query rows of hi + lo -> / ||u|| -> a_{t,n}
-//   warps 6-9    channel sums and token norms: 8 channel pairs per warp, a
-//                lane per channel pair and quarter of the tile's rows (one
-//                warp per SM sub-partition; every element is read from
-//                shared memory once); the quarters combined by shuffles;
-//                the squares of a row's channels kept per lane over the
-//                tile's K steps and combined at the end of the tile; the sums of the
+//   warps 2-9    channel sums and token norms: 4 channel pairs per warp, a
+//                lane per channel pair and eighth of the tile's rows (two
+//                warps per SM sub-partition; every element is read from
+//                shared memory once); the eighths combined by shuffles; the
+//                squares of a row's channels kept per lane over the tile's K
+//                steps and combined at the end of the tile; the sums of the
 //                frame open at the start of a tile and of the frame that
 //                starts inside it (frames have >= 128 tokens, so at most one
 //                starts inside a tile) accumulate in shared memory and are
 //                written to the frame's slot when the frame ends or the
-//                CTA's range does
+//                CTA's range does.  After each tile warps 2-5 also form
+//                a_{t,n} for the rows of their tensor-memory lane quadrant:
+//                tcgen05.ld -> max over the query rows of hi + lo -> / ||u||
 //   warp 10      TMA producer of the query rows (one thread)
 // Every mbarrier wait is bounded; on a timeout the kernel records a status
 // bit, drains what it issued, frees tensor memory and exits.
@@ -58,7 +58,7 @@ constexpr int kXThreads = 11 * 32;
 constexpr int kXBStages = 2;                        // query-row stages (their own ring)
 constexpr int kXAccCols = 256;
 constexpr uint64_t kXTimeoutNs = 2000000000ull;
-constexpr int kXReaders = 4;                        // channel-sum warps reading each stage
+constexpr int kXReaders = 8;                        // channel-sum warps reading each stage
 
 struct XShared {
     uint64_t full[kXMaxStages];    // feature ring
@@ -66,13 +66,11 @@ struct XShared {
     uint64_t bfull[kXBStages];     // query-row ring
     uint64_t bempty[kXBStages];
     uint64_t tfull[2], tempty[2];
-    uint64_t nfull[2], nempty[2];
     uint64_t csync[2];
     uint64_t drain;
     uint32_t tmem_base;
     int abort;
-    float norms[2][kXM];
-    float npart[2][4][kXM];   // per channel-sum warp: squares of its channels, per row
+    float npart[2][kXReaders][kXM];   // per channel-sum warp: squares of its channels, per row
 };
 
 struct XMaps {
@@ -109,13 +107,13 @@ __device__ __forceinline__ int xtiles(const Ctx &c) {
     return beg < end ? (int)((end - beg + kXM - 1) / kXM) : 0;
 }
 
-// The channel sums of this warp's 16 channels of every K step (acc), to the
-// partial slot of frame f, then acc cleared: lanes 0-15 one K step, lanes
-// 16-31 the next.
+// The channel sums of this warp's 8 channels of every K step (acc), to the
+// partial slot of frame f, then acc cleared: lane group lane / 8 takes every
+// fourth K step.
 __device__ __forceinline__ void xflush(const Ctx &c, float *acc, int64_t f, int ch_lo, int lane) {
     float *dst = c.part + ((size_t)blockIdx.x + (size_t)f) * c.D;
-    for (int k0 = (lane >> 4) * kXK; k0 < c.D; k0 += 2 * kXK) {
-        const int ch = k0 + ch_lo + (lane & 15);
+    for (int k0 = (lane >> 3) * kXK; k0 < c.D; k0 += 4 * kXK) {
+        const int ch = k0 + ch_lo + (lane & 7);
         if (wz_in_range(c.status, (int64_t)blockIdx.x + f < (int64_t)c.G1 + c.T)) dst[ch] = acc[ch];
         acc[ch] = 0.f;
     }
@@ -143,9 +141,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(&S->tfull[b], 1);
             ptx::mbar_init(&S->tempty[b], 4);
-            ptx::mbar_init(&S->nfull[b], 4);
-            ptx::mbar_init(&S->nempty[b], 4);
-            ptx::mbar_init(&S->csync[b], 4);
+            ptx::mbar_init(&S->csync[b], kXReaders);
         }
         ptx::mbar_init(&S->drain, 1);
         S->abort = 0;
@@ -283,61 +279,22 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
         }
         ptx::mma_commit(&S->drain);
         ptx::mbar_wait(&S->drain, 0, kXTimeoutNs);
-    } else if (warp >= 2 && warp < 6) {
-        // ---------------- epilogue: a_{t,n} ----------------
-        const int q = warp & 3;                      // TMEM lane quadrant: rows q*32 .. q*32+31
-        const int row = q * 32 + lane;
-        for (int it = 0; it < ntile && !*abort_flag; ++it) {
-            const int b = it & 1;
-            const uint32_t use = (uint32_t)(it >> 1);
-            if (!ptx::mbar_wait(&S->tfull[b], use & 1u, kXTimeoutNs) ||
-                !ptx::mbar_wait(&S->nfull[b], use & 1u, kXTimeoutNs)) {
-                xfail(c, abort_flag, 32);
-                break;
-            }
-            ptx::tc_fence_after();
-            int64_t base;
-            int nr;
-            xtile(c, it, base, nr);
-            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * kXAccCols);
-            float best = -INFINITY;
-            for (int c0 = 0; c0 < p.Lqp; c0 += 16) {
-                uint32_t hi[16], lo[16];
-                ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)c0, hi);
-                ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)(p.Lqp + c0), lo);
-                ptx::tmem_ld_wait();
-                ptx::reg_fence16(hi);
-                ptx::reg_fence16(lo);
-#pragma unroll
-                for (int j = 0; j < 16; ++j)
-                    if (c0 + j < p.Lq) best = fmaxf(best, __uint_as_float(hi[j]) + __uint_as_float(lo[j]));
-            }
-            const float nrm = S->norms[b][row];
-            if (row < nr && wz_in_range(c.status, base + row < (int64_t)c.T * c.N))
-                c.a[base + row] = nrm > 0.f ? best / nrm : 0.f;
-            ptx::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) {
-                ptx::mbar_arrive(&S->tempty[b]);
-                ptx::mbar_arrive(&S->nempty[b]);
-            }
-        }
-    } else if (warp >= 6 && warp < 10) {
-        // ---------------- per-frame channel sums ----------------
-        // lane: channel pair p2 of this warp's 16 channels of a K step, and
-        // the quarter rq of the tile's rows it sums.  Its i-th row is
-        // 32 rq + (i ^ 2 rq) (each quarter walks its rows in another order,
-        // which keeps the quarters on different banks); with the 128-byte
-        // swizzle (16-byte chunk k of row r at r * 128 + ((k ^ (r & 7)) << 4))
-        // that row's word sits at lane_off + (xo(i) ^ xl), xo(i) a constant
-        // of the unrolled loop and xl one of the lane
-        const int wsel = warp - 6;
-        const int p2 = lane & 7, rq = lane >> 3;
-        const int cw = wsel * 16 + 2 * p2;              // channels cw, cw + 1 of the K step
-        const uint32_t coff = (uint32_t)((cw * 2) & 15);
-        const int chunk = (cw * 2) >> 4;
-        const uint32_t lane_off = (uint32_t)(rq * 4096) + coff;
-        const uint32_t xl = ((uint32_t)rq << 8) | ((uint32_t)(chunk ^ (2 * rq)) << 4);
+    } else if (warp >= 2 && warp < 10) {
+        // ---------------- channel sums and token norms (warps 2-9), a_{t,n} (warps 2-5) ----------------
+        // lane: channel pair p4 of this warp's 8 channels of a K step, and the
+        // eighth re of the tile's rows it sums.  Its i-th row is 16 re + (i ^ re)
+        // (each eighth walks its rows in another order, which keeps the eighths
+        // on different banks); with the 128-byte swizzle (16-byte chunk k of
+        // row r at r * 128 + ((k ^ (r & 7)) << 4)) that row's word sits at
+        // lane_off + (xo(i) ^ xl), xo(i) a constant of the unrolled loop and xl
+        // one of the lane.  Warps 2-5 then take the tile's a_{t,n} for the rows
+        // of their tensor-memory lane quadrant.
+        const int wsel = warp - 2;
+        const bool epi = warp < 6;
+        const int p4 = lane & 3, re = lane >> 2;
+        const int cw = wsel * 8 + 2 * p4;               // channels cw, cw + 1 of the K step
+        const uint32_t lane_off = (uint32_t)(re * 2048) + (uint32_t)(4 * p4);
+        const uint32_t xl = ((uint32_t)re << 7) | ((uint32_t)(wsel ^ re) << 4);
         float *acc_open = acc_buf, *acc_next = acc_buf + c.D;
         int64_t open_f = ntile > 0 ? ((int64_t)blockIdx.x * c.L1) / c.N : 0;
         bool open_has = false;
@@ -350,10 +307,10 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             // a frame starts inside the tile at row rb (frames have >= 128 tokens)
             const int to_end = (int)((int64_t)c.N - base % c.N);
             const int rb = to_end < nr ? to_end : nr;
-            float sq[32];   // squares of this lane's two channels, row 32 rq + (i ^ 2 rq)
             const bool whole = rb == kXM;   // every row of the tile in the open frame
+            float sq[16];                   // squares of this lane's two channels, row 16 re + (i ^ re)
 #pragma unroll
-            for (int i = 0; i < 32; ++i) sq[i] = 0.f;
+            for (int i = 0; i < 16; ++i) sq[i] = 0.f;
             bool ok = true;
             for (int ks = 0; ks < KS; ks += p.G) {
                 if (!ptx::mbar_wait(&S->full[stage], phase, kXTimeoutNs)) {
@@ -367,7 +324,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                     float s0x = 0.f, s0y = 0.f, s1x = 0.f, s1y = 0.f;
                     if (whole) {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
+                        for (int i = 0; i < 16; ++i) {
                             const uint32_t xo = ((uint32_t)i << 7) | ((uint32_t)(i & 7) << 4);
                             uint32_t wv;
                             asm volatile("ld.shared.b32 %0, [%1];" : "=r"(wv) : "r"(lb + (xo ^ xl)));
@@ -378,8 +335,8 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                         }
                     } else {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const int r = 32 * rq + (i ^ (2 * rq));
+                        for (int i = 0; i < 16; ++i) {
+                            const int r = 16 * re + (i ^ re);
                             const uint32_t xo = ((uint32_t)i << 7) | ((uint32_t)(i & 7) << 4);
                             uint32_t wv;
                             asm volatile("ld.shared.b32 %0, [%1];" : "=r"(wv) : "r"(lb + (xo ^ xl)));
@@ -399,13 +356,13 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                         if (lane == 0) ptx::mbar_arrive(&S->empty[stage]);
                     }
 #pragma unroll
-                    for (int o = 8; o < 32; o <<= 1) {   // the four row quarters, in a fixed order
+                    for (int o = 4; o < 32; o <<= 1) {   // the eight row eighths, in a fixed order
                         s0x += __shfl_xor_sync(0xffffffffu, s0x, o);
                         s0y += __shfl_xor_sync(0xffffffffu, s0y, o);
                         s1x += __shfl_xor_sync(0xffffffffu, s1x, o);
                         s1y += __shfl_xor_sync(0xffffffffu, s1y, o);
                     }
-                    if (rq == 0) {
+                    if (re == 0) {
                         const int ch = (ks + g) * kXK + cw;
                         acc_open[ch] += s0x;
                         acc_open[ch + 1] += s0y;
@@ -421,36 +378,22 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                 }
             }
             if (!ok) break;
-            // token norms: this warp's squares summed over its 8 channel pairs,
-            // then the four warps' partials in a fixed order
+            // token norms: this warp's squares summed over its 4 channel pairs,
+            // one partial per warp and row
             const int b = it & 1;
             const uint32_t use = (uint32_t)(it >> 1);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
+            for (int i = 0; i < 16; ++i) {
                 float v = sq[i];
                 v += __shfl_xor_sync(0xffffffffu, v, 1);
                 v += __shfl_xor_sync(0xffffffffu, v, 2);
-                v += __shfl_xor_sync(0xffffffffu, v, 4);
-                if (p2 == 0) S->npart[b][wsel][32 * rq + (i ^ (2 * rq))] = v;
+                if (p4 == 0) S->npart[b][wsel][16 * re + (i ^ re)] = v;
             }
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&S->csync[b]);
-            if (!ptx::mbar_wait(&S->csync[b], use & 1u, kXTimeoutNs) ||
-                !ptx::mbar_wait(&S->nempty[b], (use & 1u) ^ 1u, kXTimeoutNs)) {
-                xfail(c, abort_flag, 32);
-                break;
-            }
-            {
-                const int row = 32 * wsel + lane;
-                const float t2 = ((S->npart[b][0][row] + S->npart[b][1][row]) + S->npart[b][2][row]) + S->npart[b][3][row];
-                S->norms[b][row] = sqrtf(t2);
-            }
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&S->nfull[b]);
-            __syncwarp();
             open_has = true;
             if (rb < nr) {   // the open frame ended inside the tile
-                xflush(c, acc_open, open_f, wsel * 16, lane);
+                xflush(c, acc_open, open_f, wsel * 8, lane);
                 float *t = acc_open;
                 acc_open = acc_next;
                 acc_next = t;
@@ -458,13 +401,48 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             }
             if ((base + nr) % c.N == 0) {   // and the frame open now ends with the tile
                 __syncwarp();
-                xflush(c, acc_open, open_f, wsel * 16, lane);
+                xflush(c, acc_open, open_f, wsel * 8, lane);
                 ++open_f;
                 open_has = false;
             }
             __syncwarp();
+            if (epi) {
+                // a_{t,n} of the rows of this warp's lane quadrant: the eight
+                // warps' partial squares in a fixed order, then the max over
+                // the query rows of hi + lo from tensor memory
+                if (!ptx::mbar_wait(&S->csync[b], use & 1u, kXTimeoutNs) ||
+                    !ptx::mbar_wait(&S->tfull[b], use & 1u, kXTimeoutNs)) {
+                    xfail(c, abort_flag, 32);
+                    break;
+                }
+                ptx::tc_fence_after();
+                const int q = warp & 3;                  // TMEM lane quadrant: rows q*32 .. q*32+31
+                const int row = q * 32 + lane;
+                float t2 = 0.f;
+#pragma unroll
+                for (int w = 0; w < kXReaders; ++w) t2 += S->npart[b][w][row];
+                const float nrm = sqrtf(t2);
+                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * kXAccCols);
+                float best = -INFINITY;
+                for (int c0 = 0; c0 < p.Lqp; c0 += 16) {
+                    uint32_t hi[16], lo[16];
+                    ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)c0, hi);
+                    ptx::tmem_ld_32x32b_x16(tbase + (uint32_t)(p.Lqp + c0), lo);
+                    ptx::tmem_ld_wait();
+                    ptx::reg_fence16(hi);
+                    ptx::reg_fence16(lo);
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                        if (c0 + j < p.Lq) best = fmaxf(best, __uint_as_float(hi[j]) + __uint_as_float(lo[j]));
+                }
+                if (row < nr && wz_in_range(c.status, base + row < (int64_t)c.T * c.N))
+                    c.a[base + row] = nrm > 0.f ? best / nrm : 0.f;
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&S->tempty[b]);
+            }
         }
-        if (open_has && !*abort_flag) xflush(c, acc_open, open_f, wsel * 16, lane);   // the CTA's share of it
+        if (open_has && !*abort_flag) xflush(c, acc_open, open_f, wsel * 8, lane);   // the CTA's share of it
     }
     __syncthreads();
     if (warp == 1) {
