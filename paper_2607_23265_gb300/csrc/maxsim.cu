@@ -80,7 +80,6 @@ struct XMaps {
 struct XArgs {
     int stages, stage_stride;   // feature ring: stages and bytes per stage (G A tiles)
     int b_off, b_stride;        // query-row ring (kXBStages stages of G B tiles): byte offset, bytes per stage
-    int G;                      // K steps per stage
     int Lq, Lqp;
     int acc_off;                // byte offset of the two channel-sum buffers (2 x D floats)
     int shared_off;             // byte offset of XShared
@@ -121,9 +120,11 @@ __device__ __forceinline__ void xflush(const Ctx &c, float *acc, int64_t f, int 
 
 }  // namespace
 
+template <int G>   // K steps per ring stage
 __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_constant__ XMaps maps, Ctx c, XArgs p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const size_t ring_off = (size_t)(ring - smem_raw);
     float *acc_buf = reinterpret_cast<float *>(ring + p.acc_off);
     XShared *S = reinterpret_cast<XShared *>(ring + p.shared_off);
     volatile int *abort_flag = &S->abort;
@@ -169,7 +170,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
     if (warp == 0 && lane == 0) {
         // ---------------- TMA producer: features ----------------
         const uint64_t pol_a = ptx::policy_evict_first();
-        const uint32_t stage_bytes = (uint32_t)p.G * (uint32_t)kXABytes;
+        const uint32_t stage_bytes = (uint32_t)G * (uint32_t)kXABytes;
         int stage = 0;
         uint32_t phase = 0;
         int issued_parity[kXMaxStages];
@@ -179,7 +180,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             int nr;
             xtile(c, it, base, nr);
             bool ok = true;
-            for (int ks = 0; ks < KS; ks += p.G) {
+            for (int ks = 0; ks < KS; ks += G) {
                 if (!ptx::mbar_wait(&S->empty[stage], phase ^ 1u, kXTimeoutNs)) {
                     xfail(c, abort_flag, 16);
                     ok = false;
@@ -201,14 +202,14 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
     } else if (warp == 10 && lane == 0) {
         // ---------------- TMA producer: query rows (from L2), K step by K step ----------------
         const uint64_t pol_b = ptx::policy_evict_last();
-        const uint32_t stage_bytes = (uint32_t)p.G * 2u * (uint32_t)p.Lqp * kXK * 2u;
+        const uint32_t stage_bytes = (uint32_t)G * 2u * (uint32_t)p.Lqp * kXK * 2u;
         int stage = 0;
         uint32_t phase = 0;
         int issued_parity[kXBStages];
         for (int s = 0; s < kXBStages; ++s) issued_parity[s] = -1;
         for (int it = 0; it < ntile && !*abort_flag; ++it) {
             bool ok = true;
-            for (int ks = 0; ks < KS; ks += p.G) {
+            for (int ks = 0; ks < KS; ks += G) {
                 if (!ptx::mbar_wait(&S->bempty[stage], phase ^ 1u, kXTimeoutNs)) {
                     xfail(c, abort_flag, 16);
                     ok = false;
@@ -247,7 +248,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             ptx::tc_fence_after();
             const uint32_t d = tmem + (uint32_t)(b * kXAccCols);
             bool ok = true;
-            for (int ks = 0; ks < KS; ks += p.G) {
+            for (int ks = 0; ks < KS; ks += G) {
                 if (!ptx::mbar_wait(&S->full[stage], phase, kXTimeoutNs) ||
                     !ptx::mbar_wait(&S->bfull[bstage], bphase, kXTimeoutNs)) {
                     xfail(c, abort_flag, 16);
@@ -256,7 +257,8 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                 }
                 ptx::tc_fence_after();
                 const uint64_t so = (uint64_t)stage * stage_desc, sbo = (uint64_t)bstage * bstage_desc;
-                for (int g = 0; g < p.G; ++g) {
+#pragma unroll
+                for (int g = 0; g < G; ++g) {
                     const uint64_t ao = so + (uint64_t)g * (kXABytes >> 4), bo = sbo + (uint64_t)g * b_sub;
 #pragma unroll
                     for (int k = 0; k < kXK / 16; ++k)   // K = 16 per MMA: 32 bytes along the swizzled row
@@ -312,34 +314,43 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
 #pragma unroll
             for (int i = 0; i < 16; ++i) sq[i] = 0.f;
             bool ok = true;
-            for (int ks = 0; ks < KS; ks += p.G) {
+            for (int ks = 0; ks < KS; ks += G) {
                 if (!ptx::mbar_wait(&S->full[stage], phase, kXTimeoutNs)) {
                     xfail(c, abort_flag, 32);
                     ok = false;
                     break;
                 }
-                const uint32_t st0 = ptx::smem_u32(ring + (size_t)stage * p.stage_stride);
-                for (int g = 0; g < p.G; ++g) {
-                    const uint32_t lb = st0 + (uint32_t)(g * kXABytes) + lane_off;
+                // (indexed from the shared array itself: shared-memory loads)
+                const uint8_t *st0 = smem_raw + ring_off + (size_t)stage * p.stage_stride;
+#pragma unroll
+                for (int g = 0; g < G; ++g) {
+                    const uint8_t *lb = st0 + g * kXABytes + lane_off;
                     float s0x = 0.f, s0y = 0.f, s1x = 0.f, s1y = 0.f;
                     if (whole) {
+                        // even and odd rows in two sums each (shorter dependent chains)
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
                             const uint32_t xo = ((uint32_t)i << 7) | ((uint32_t)(i & 7) << 4);
-                            uint32_t wv;
-                            asm volatile("ld.shared.b32 %0, [%1];" : "=r"(wv) : "r"(lb + (xo ^ xl)));
+                            const uint32_t wv = *reinterpret_cast<const uint32_t *>(lb + (xo ^ xl));
                             const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
                             sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
-                            s0x += x;
-                            s0y += y;
+                            if (i & 1) {
+                                s1x += x;
+                                s1y += y;
+                            } else {
+                                s0x += x;
+                                s0y += y;
+                            }
                         }
+                        s0x += s1x;
+                        s0y += s1y;
+                        s1x = s1y = 0.f;
                     } else {
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
                             const int r = 16 * re + (i ^ re);
                             const uint32_t xo = ((uint32_t)i << 7) | ((uint32_t)(i & 7) << 4);
-                            uint32_t wv;
-                            asm volatile("ld.shared.b32 %0, [%1];" : "=r"(wv) : "r"(lb + (xo ^ xl)));
+                            const uint32_t wv = *reinterpret_cast<const uint32_t *>(lb + (xo ^ xl));
                             const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
                             sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
                             if (r < rb) {
@@ -351,7 +362,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                             }
                         }
                     }
-                    if (g == p.G - 1) {   // the stage's last K step is in registers: hand the stage back
+                    if (g == G - 1) {   // the stage's last K step is in registers: hand the stage back
                         __syncwarp();
                         if (lane == 0) ptx::mbar_arrive(&S->empty[stage]);
                     }
@@ -478,7 +489,7 @@ XLayout xlayout(int D, int Lqp) {
     XLayout L{};
     const size_t fixed = 1024 + (size_t)2 * D * 4 + (sizeof(XShared) + 127) / 128 * 128;
     const size_t cap = 227 * 1024;
-    for (int G = kXGroups; G >= 1; --G) {
+    for (int G = kXGroups; G >= 1; G >>= 1) {
         if ((D / kXK) % G != 0) continue;
         L.G = G;
         L.stride = G * kXABytes;
@@ -520,15 +531,17 @@ cudaError_t launch_maxsim_pass(const Ctx &c, int Lq, int Lqp, cudaStream_t s) {
     p.stage_stride = L.stride;
     p.b_off = L.b_off;
     p.b_stride = L.b_stride;
-    p.G = L.G;
     p.Lq = Lq;
     p.Lqp = Lqp;
     p.acc_off = L.acc_off;
     p.shared_off = L.shared_off;
-    cudaError_t e = cudaFuncSetAttribute(maxsim_pass_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem);
+    const void *fn = L.G == 4 ? (const void *)maxsim_pass_kernel<4>
+                     : L.G == 2 ? (const void *)maxsim_pass_kernel<2>
+                                : (const void *)maxsim_pass_kernel<1>;
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem);
     if (e != cudaSuccess) return e;
     void *args[] = {&maps, const_cast<Ctx *>(&c), &p};
-    return launch_kernel((const void *)maxsim_pass_kernel, dim3(c.G1), dim3(kXThreads), L.smem, s, args, c.pdl != 0);
+    return launch_kernel(fn, dim3(c.G1), dim3(kXThreads), L.smem, s, args, c.pdl != 0);
 }
 
 }  // namespace wz
