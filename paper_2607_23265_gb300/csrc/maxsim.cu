@@ -22,9 +22,9 @@
 //   warp 0       TMA producer of the features (one thread)
 //   warp 1       TMEM allocation and the MMA issuer (one thread)
 //   warps 2-9    channel sums and token norms: 4 channel pairs per warp, a
-//                lane per channel pair and eighth of the tile's rows (two
-//                warps per SM sub-partition; every element is read from
-//                shared memory once); the eighths combined by shuffles; the
+//                lane per channel pair and class of the tile's rows mod 8
+//                (two warps per SM sub-partition; every element is read from
+//                shared memory once); the classes combined by shuffles; the
 //                squares of a row's channels kept per lane over the tile's K
 //                steps and combined at the end of the tile; the sums of the
 //                frame open at the start of a tile and of the frame that
@@ -284,19 +284,17 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
     } else if (warp >= 2 && warp < 10) {
         // ---------------- channel sums and token norms (warps 2-9), a_{t,n} (warps 2-5) ----------------
         // lane: channel pair p4 of this warp's 8 channels of a K step, and the
-        // eighth re of the tile's rows it sums.  Its i-th row is 16 re + (i ^ re)
-        // (each eighth walks its rows in another order, which keeps the eighths
-        // on different banks); with the 128-byte swizzle (16-byte chunk k of
-        // row r at r * 128 + ((k ^ (r & 7)) << 4)) that row's word sits at
-        // lane_off + (xo(i) ^ xl), xo(i) a constant of the unrolled loop and xl
-        // one of the lane.  Warps 2-5 then take the tile's a_{t,n} for the rows
-        // of their tensor-memory lane quadrant.
+        // rows r = 8 i + re (i < 16) of the tile it sums.  With the 128-byte
+        // swizzle (16-byte chunk k of row r at r * 128 + ((k ^ (r & 7)) << 4))
+        // every one of those rows has r & 7 = re, so the lane's words sit at
+        // lane_off + 1024 i (the eight values of re put the 32 lanes on 32
+        // banks).  Warps 2-5 then take the tile's a_{t,n} for the rows of
+        // their tensor-memory lane quadrant.
         const int wsel = warp - 2;
         const bool epi = warp < 6;
         const int p4 = lane & 3, re = lane >> 2;
         const int cw = wsel * 8 + 2 * p4;               // channels cw, cw + 1 of the K step
-        const uint32_t lane_off = (uint32_t)(re * 2048) + (uint32_t)(4 * p4);
-        const uint32_t xl = ((uint32_t)re << 7) | ((uint32_t)(wsel ^ re) << 4);
+        const uint32_t lane_off = (uint32_t)(re * 128) + ((uint32_t)(wsel ^ re) << 4) + (uint32_t)(4 * p4);
         float *acc_open = acc_buf, *acc_next = acc_buf + c.D;
         int64_t open_f = ntile > 0 ? ((int64_t)blockIdx.x * c.L1) / c.N : 0;
         bool open_has = false;
@@ -310,7 +308,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
             const int to_end = (int)((int64_t)c.N - base % c.N);
             const int rb = to_end < nr ? to_end : nr;
             const bool whole = rb == kXM;   // every row of the tile in the open frame
-            float sq[16];                   // squares of this lane's two channels, row 16 re + (i ^ re)
+            float sq[16];                   // squares of this lane's two channels, row 8 i + re
 #pragma unroll
             for (int i = 0; i < 16; ++i) sq[i] = 0.f;
             bool ok = true;
@@ -330,8 +328,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                         // even and odd rows in two sums each (shorter dependent chains)
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
-                            const uint32_t xo = ((uint32_t)i << 7) | ((uint32_t)(i & 7) << 4);
-                            const uint32_t wv = *reinterpret_cast<const uint32_t *>(lb + (xo ^ xl));
+                            const uint32_t wv = *reinterpret_cast<const uint32_t *>(lb + 1024 * i);
                             const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
                             sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
                             if (i & 1) {
@@ -348,9 +345,8 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                     } else {
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
-                            const int r = 16 * re + (i ^ re);
-                            const uint32_t xo = ((uint32_t)i << 7) | ((uint32_t)(i & 7) << 4);
-                            const uint32_t wv = *reinterpret_cast<const uint32_t *>(lb + (xo ^ xl));
+                            const int r = 8 * i + re;
+                            const uint32_t wv = *reinterpret_cast<const uint32_t *>(lb + 1024 * i);
                             const float x = __uint_as_float(wv << 16), y = __uint_as_float(wv & 0xffff0000u);
                             sq[i] = fmaf(x, x, fmaf(y, y, sq[i]));
                             if (r < rb) {
@@ -367,7 +363,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                         if (lane == 0) ptx::mbar_arrive(&S->empty[stage]);
                     }
 #pragma unroll
-                    for (int o = 4; o < 32; o <<= 1) {   // the eight row eighths, in a fixed order
+                    for (int o = 4; o < 32; o <<= 1) {   // the eight row classes, in a fixed order
                         s0x += __shfl_xor_sync(0xffffffffu, s0x, o);
                         s0y += __shfl_xor_sync(0xffffffffu, s0y, o);
                         s1x += __shfl_xor_sync(0xffffffffu, s1x, o);
@@ -398,7 +394,7 @@ __global__ void __launch_bounds__(kXThreads, 1) maxsim_pass_kernel(const __grid_
                 float v = sq[i];
                 v += __shfl_xor_sync(0xffffffffu, v, 1);
                 v += __shfl_xor_sync(0xffffffffu, v, 2);
-                if (p4 == 0) S->npart[b][wsel][16 * re + (i ^ re)] = v;
+                if (p4 == 0) S->npart[b][wsel][8 * i + re] = v;
             }
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&S->csync[b]);
