@@ -477,6 +477,56 @@ __device__ void frame_gate(const Ctx &c, int64_t f, float *red, const float (&av
     }
 }
 
+// The gate of frame f (as frame_gate) formed by threads 256..511 of
+// frame_stats_kernel (t0 = threadIdx.x - 256, named barrier 2) while threads
+// 0..255 form the frame statistics: the two chains overlap.
+__device__ void gate_half(const Ctx &c, int64_t f, int t0) {
+    __shared__ float M2[WZ_MAX_HW * WZ_MAX_HW];
+    __shared__ float red2[16];
+    auto sync = [] { asm volatile("bar.sync 2, 256;" ::: "memory"); };
+    const int N = c.N, H = c.H, W = c.W, lane = t0 & 31, w = t0 >> 5;
+    const float *a = (c.ext_a ? c.ext_a : c.a) + f * N;
+    float lo = INFINITY, hi = -INFINITY;
+    for (int k = t0; k < N; k += 256) {
+        const float x = a[k];
+        M2[k] = x;
+        lo = fminf(lo, x);
+        hi = fmaxf(hi, x);
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    if (lane == 0) {
+        red2[w] = lo;
+        red2[8 + w] = hi;
+    }
+    sync();
+    lo = INFINITY;
+    hi = -INFINITY;
+    for (int k = 0; k < 8; ++k) {
+        lo = fminf(lo, red2[k]);
+        hi = fmaxf(hi, red2[8 + k]);
+    }
+    const float rng = hi - lo;
+    for (int k = t0; k < N; k += 256) M2[k] = rng > 0.f ? (M2[k] - lo) / rng : 0.f;
+    sync();
+    for (int l = 1; l <= c.wsm_levels; ++l) {
+        const int hp = c.lvl_h[l], wp = c.lvl_w[l];
+        if (!wz_in_range(c.status, c.goff[l - 1] + hp * wp <= c.gate_stride)) break;
+        float *G = c.gate + f * (int64_t)c.gate_stride + c.goff[l - 1];
+        for (int k = t0; k < hp * wp; k += 256) {
+            const int ai = k / wp, bj = k % wp;
+            const int r0 = (ai * H) / hp, r1 = ((ai + 1) * H + hp - 1) / hp;
+            const int c0 = (bj * W) / wp, c1 = ((bj + 1) * W + wp - 1) / wp;
+            float s = 0.f;
+            for (int y = r0; y < r1; ++y)
+                for (int x = c0; x < c1; ++x) s += M2[y * W + x];
+            G[k] = c.lambda * (s / (float)((r1 - r0) * (c1 - c0)));
+        }
+    }
+}
+
 // One block per frame: the frame sums (fixed list of CTA partials) for all
 // channels, read as 16-byte vectors; fp32 products summed over each thread's
 // channels and across each warp, the warp totals in fp64; then
@@ -496,8 +546,17 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     const bool maxsim = c.relevance_mode == WZ_RELEVANCE_MAXSIM;
     const bool do_gate = c.gate && c.spatial_mode == WZ_SPATIAL_WSM;
     const int64_t f = blockIdx.x;
+    // with the mean scorer, threads 256..511 form the gate while 0..255 form
+    // the statistics; the max-over-query scorer takes every warp for its
+    // query rows and forms the gate after them
+    const bool split = !maxsim && do_gate;
+    if (split && threadIdx.x >= 256) {
+        gate_half(c, f, (int)threadIdx.x - 256);
+        return;
+    }
+    const int nst = split ? 256 : (int)blockDim.x;   // threads forming the statistics
     float av[kGatePerThread];
-    if (do_gate) gate_prefetch(c, f, av);
+    if (do_gate && !split) gate_prefetch(c, f, av);
     const int t = (int)(f % c.T);
     const int v = (int)(f / c.T);
     const int64_t lo = f * c.N / c.L1;
@@ -509,7 +568,7 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     const float4 *P = reinterpret_cast<const float4 *>(c.part);
     const float4 *Qv = reinterpret_cast<const float4 *>(c.qbar32 + (size_t)v * c.D);
     float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f, p4 = 0.f;
-    for (int i = threadIdx.x; i < nv; i += blockDim.x) {
+    for (int i = threadIdx.x; i < nv; i += nst) {
         float4 sf = make_float4(0.f, 0.f, 0.f, 0.f), sp = sf;
         for (int64_t cc = lo; cc <= hi; cc += 2) {   // two partial rows in flight, summed in order
             const float4 x = P[(size_t)(cc + f) * nv + i];
@@ -545,7 +604,7 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
         p3 += __shfl_xor_sync(0xffffffffu, p3, o);
         p4 += __shfl_xor_sync(0xffffffffu, p4, o);
     }
-    const int warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    const int warp = threadIdx.x >> 5, nw = nst >> 5;
     if (maxsim) {
         __syncthreads();   // sfs complete
         const int lane = threadIdx.x & 31;
@@ -590,7 +649,8 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
         wsum[warp][3] = p3;
         wsum[warp][4] = p4;
     }
-    __syncthreads();
+    if (split) asm volatile("bar.sync 1, 256;" ::: "memory");   // the statistics' warps only
+    else __syncthreads();
     if (warp == 0) {
         // lane k < 5 sums quantity k over the warps in order (one fp64 warp
         // instruction per warp partial instead of five)
@@ -626,7 +686,7 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
             if (c.frame_scores) c.frame_scores[f] = (float)r;
         }
     }
-    if (do_gate) frame_gate(c, f, wsum[0], av);
+    if (do_gate && !split) frame_gate(c, f, wsum[0], av);
 }
 
 cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s) {
