@@ -433,49 +433,52 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     // the condensation claims units in list order, and short units last keep
     // its tail short.
     const bool tc = c.path == WZ_PATH_TENSOR;
-    int nloc[kPerThread], ucnt[kPerThread], ucntB[kPerThread];
-    int part[4] = {0, 0, 0, 0};
-#pragma unroll
-    for (int k = 0; k < kPerThread; ++k) {
-        const int t = t0 + k;
-        nloc[k] = (k < per && t < T) ? nf[t] : 0;
-        ucnt[k] = 0;
-        ucntB[k] = 0;
+    // units of frame t's first block (ua) and of its later blocks (ub)
+    auto frame_units = [&](int n, int &ua, int &ub) {
+        ua = ub = 0;
         if (tc)
-            for (int j0 = 0; j0 < nloc[k]; j0 += kColBlock) {
-                const int nc = min(kColBlock, nloc[k] - j0);
+            for (int j0 = 0; j0 < n; j0 += kColBlock) {
+                const int nc = min(kColBlock, n - j0);
                 const int cg = unit_tiles((nc + 15) / 16 * 16), add = (c.n_ct + cg - 1) / cg;
-                if (j0 == 0) ucnt[k] += add;
-                else ucntB[k] += add;
+                if (j0 == 0) ua += add;
+                else ub += add;
             }
-        part[0] += nloc[k];
-        part[1] += (nloc[k] + 15) & ~15;
-        part[2] += ucnt[k];
-        part[3] += ucntB[k];
+    };
+    // this thread's frames t0 .. t0 + per - 1 (their budgets re-read from
+    // shared memory: no per-thread arrays)
+    const int t1 = min(T, t0 + per);
+    int part[4] = {0, 0, 0, 0};
+    for (int t = t0; t < t1; ++t) {
+        const int n = nf[t];
+        int ua, ub;
+        frame_units(n, ua, ub);
+        part[0] += n;
+        part[1] += (n + 15) & ~15;
+        part[2] += ua;
+        part[3] += ub;
     }
     int pre[4], tot[4];
     block_excl_scan<4>(part, iscr, pre, tot);
     int o = pre[0], wo = pre[1], u = pre[2], uB = tot[2] + pre[3];
-#pragma unroll
-    for (int k = 0; k < kPerThread; ++k) {
-        const int t = t0 + k;
-        if (k < per && t < T) {
-            c.n[base + t] = nloc[k];
-            c.off[base + t] = vp.row0 + o;
-            c.woff[base + t] = vp.w_row0 + wo;
-            if (tc) {
-                c.ustart[base + t] = u;
-                c.ustartB[base + t] = uB;
-            }
-            const int h = grid_h(nloc[k], c.H, c.W);
-            c.hw[2 * (base + t)] = h;
-            c.hw[2 * (base + t) + 1] = h > 0 ? (nloc[k] + h - 1) / h : 0;
-            if (c.out_budgets) c.out_budgets[base + t] = nloc[k];
+    for (int t = t0; t < t1; ++t) {
+        const int n = nf[t];
+        int ua, ub;
+        frame_units(n, ua, ub);
+        c.n[base + t] = n;
+        c.off[base + t] = vp.row0 + o;
+        c.woff[base + t] = vp.w_row0 + wo;
+        if (tc) {
+            c.ustart[base + t] = u;
+            c.ustartB[base + t] = uB;
         }
-        o += nloc[k];
-        wo += (nloc[k] + 15) & ~15;
-        u += ucnt[k];
-        uB += ucntB[k];
+        const int h = grid_h(n, c.H, c.W);
+        c.hw[2 * (base + t)] = h;
+        c.hw[2 * (base + t) + 1] = h > 0 ? (n + h - 1) / h : 0;
+        if (c.out_budgets) c.out_budgets[base + t] = n;
+        o += n;
+        wo += (n + 15) & ~15;
+        u += ua;
+        uB += ub;
     }
     if (threadIdx.x == 0) {
         c.prod[v] = tot[0];
