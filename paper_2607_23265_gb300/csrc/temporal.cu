@@ -96,8 +96,6 @@ __device__ void block_excl_scan(const int (&x)[K], int *ws, int (&excl)[K], int 
     __syncthreads();
 }
 
-// Frames per thread for the scans (T <= 4096 with 256 threads).
-constexpr int kPerThread = WZ_MAX_T / kTemporalThreads;
 
 // h = min(H, ceil(sqrt(n H / W))): a float estimate corrected to the exact
 // smallest h >= 1 with h^2 W >= n H in integers.
@@ -138,7 +136,8 @@ __host__ __device__ inline size_t temporal_smem_bytes(int T, int J) {
 }
 
 // Threads of the CTA: one frame per thread up to 512 frames, at most
-// kPerThread frames per thread beyond (fp64 work scales with the warps).
+// WZ_MAX_T / kTemporalThreads frames per thread beyond (fp64 work scales with
+// the warps).
 inline int temporal_threads(int T) { return T <= 512 ? (T < 32 ? 32 : (T + 31) / 32 * 32) : 512; }
 
 // WTA levels 2..J (J > 1): level 1 left its approximation in A0, its gate in
@@ -244,37 +243,33 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
     const double hi = __longlong_as_double((long long)c.drange[2 * v + 1]);
     // gamma_t and the retained set (frame 1 always kept)
     const double tau = (double)c.tau;
-    // each thread owns `per` consecutive frames (per <= kPerThread)
+    // each thread owns `per` consecutive frames t0 .. t1 - 1;
+    // nf[t] holds the frame's keep flag until the retained list is written
     const int per = (T + (int)blockDim.x - 1) / (int)blockDim.x;
-    int keep[kPerThread];
+    const int t0 = threadIdx.x * per, t1 = min(T, t0 + per);
     int cnt = 0;
-    const int t0 = threadIdx.x * per;
-#pragma unroll
-    for (int k = 0; k < kPerThread; ++k) {
-        const int t = t0 + k;
-        keep[k] = 0;
-        if (k < per && t < T) {
-            const double d = fr[4 * t + 1];
-            const double gm = hi > lo ? (d - lo) / (hi - lo) : 0.0;
-            fr[4 * t + 2] = gm;
-            fr[4 * t + 3] = NAN;
-            if (c.out_rel) {   // r~ follows with the WTA (NaN: filtered)
-                float *orl = c.out_rel + (base + t) * 4;
-                orl[0] = (float)fr[4 * t];
-                orl[1] = (float)d;
-                orl[2] = (float)gm;
-                orl[3] = NAN;
-            }
-            keep[k] = (t == 0 || d >= tau) ? 1 : 0;
-            cnt += keep[k];
-            nf[t] = 0;
+    for (int t = t0; t < t1; ++t) {
+        const double d = fr[4 * t + 1];
+        const double gm = hi > lo ? (d - lo) / (hi - lo) : 0.0;
+        fr[4 * t + 2] = gm;
+        fr[4 * t + 3] = NAN;
+        if (c.out_rel) {   // r~ follows with the WTA (NaN: filtered)
+            float *orl = c.out_rel + (base + t) * 4;
+            orl[0] = (float)fr[4 * t];
+            orl[1] = (float)d;
+            orl[2] = (float)gm;
+            orl[3] = NAN;
         }
+        const int kp = (t == 0 || d >= tau) ? 1 : 0;
+        nf[t] = kp;
+        cnt += kp;
     }
     int L = 0;
     int pos = block_excl_scan(cnt, iscr, &L);
-#pragma unroll
-    for (int k = 0; k < kPerThread; ++k)
-        if (k < per && keep[k]) lst[pos++] = t0 + k;
+    for (int t = t0; t < t1; ++t) {
+        if (nf[t]) lst[pos++] = t;
+        nf[t] = 0;
+    }
     __syncthreads();
 
     // WTA (Eq. 8-10): DWT of r over the retained sequence with the WTA
@@ -444,9 +439,8 @@ __global__ void __launch_bounds__(kTemporalThreads) temporal_kernel(Ctx c) {
                 else ub += add;
             }
     };
-    // this thread's frames t0 .. t0 + per - 1 (their budgets re-read from
-    // shared memory: no per-thread arrays)
-    const int t1 = min(T, t0 + per);
+    // this thread's frames t0 .. t1 - 1 (their budgets re-read from shared
+    // memory: no per-thread arrays)
     int part[4] = {0, 0, 0, 0};
     for (int t = t0; t < t1; ++t) {
         const int n = nf[t];
