@@ -429,8 +429,7 @@ __device__ __forceinline__ void gate_prefetch(const Ctx &c, int64_t f, float (&a
     }
 }
 
-__device__ void frame_gate(const Ctx &c, int64_t f, float *red, const float (&av)[kGatePerThread]) {
-    __shared__ float M[WZ_MAX_HW * WZ_MAX_HW];
+__device__ void frame_gate(const Ctx &c, int64_t f, float *red, const float (&av)[kGatePerThread], float *M) {
     const int N = c.N, H = c.H, W = c.W;
     float lo = INFINITY, hi = -INFINITY;
 #pragma unroll
@@ -477,17 +476,17 @@ __device__ void frame_gate(const Ctx &c, int64_t f, float *red, const float (&av
     }
 }
 
-// The gate of frame f (as frame_gate) formed by threads 256..511 of
-// frame_stats_kernel (t0 = threadIdx.x - 256, named barrier 2) while threads
-// 0..255 form the frame statistics: the two chains overlap.
-__device__ void gate_half(const Ctx &c, int64_t f, int t0) {
-    __shared__ float M2[WZ_MAX_HW * WZ_MAX_HW];
-    __shared__ float red2[16];
-    auto sync = [] { asm volatile("bar.sync 2, 256;" ::: "memory"); };
-    const int N = c.N, H = c.H, W = c.W, lane = t0 & 31, w = t0 >> 5;
+// The gate of frame f (as frame_gate) formed by the upper half of
+// frame_stats_kernel's threads (t0 = threadIdx.x - nth, named barrier 2 over
+// nth threads) while the lower half forms the frame statistics: the two
+// chains overlap.
+__device__ void gate_half(const Ctx &c, int64_t f, int t0, int nth, float *M2) {
+    __shared__ float red2[32];
+    auto sync = [nth] { asm volatile("bar.sync 2, %0;" ::"r"(nth) : "memory"); };
+    const int N = c.N, H = c.H, W = c.W, lane = t0 & 31, w = t0 >> 5, nw = nth >> 5;
     const float *a = (c.ext_a ? c.ext_a : c.a) + f * N;
     float lo = INFINITY, hi = -INFINITY;
-    for (int k = t0; k < N; k += 256) {
+    for (int k = t0; k < N; k += nth) {
         const float x = a[k];
         M2[k] = x;
         lo = fminf(lo, x);
@@ -499,23 +498,23 @@ __device__ void gate_half(const Ctx &c, int64_t f, int t0) {
     }
     if (lane == 0) {
         red2[w] = lo;
-        red2[8 + w] = hi;
+        red2[16 + w] = hi;
     }
     sync();
     lo = INFINITY;
     hi = -INFINITY;
-    for (int k = 0; k < 8; ++k) {
+    for (int k = 0; k < nw; ++k) {
         lo = fminf(lo, red2[k]);
-        hi = fmaxf(hi, red2[8 + k]);
+        hi = fmaxf(hi, red2[16 + k]);
     }
     const float rng = hi - lo;
-    for (int k = t0; k < N; k += 256) M2[k] = rng > 0.f ? (M2[k] - lo) / rng : 0.f;
+    for (int k = t0; k < N; k += nth) M2[k] = rng > 0.f ? (M2[k] - lo) / rng : 0.f;
     sync();
     for (int l = 1; l <= c.wsm_levels; ++l) {
         const int hp = c.lvl_h[l], wp = c.lvl_w[l];
         if (!wz_in_range(c.status, c.goff[l - 1] + hp * wp <= c.gate_stride)) break;
         float *G = c.gate + f * (int64_t)c.gate_stride + c.goff[l - 1];
-        for (int k = t0; k < hp * wp; k += 256) {
+        for (int k = t0; k < hp * wp; k += nth) {
             const int ai = k / wp, bj = k % wp;
             const int r0 = (ai * H) / hp, r1 = ((ai + 1) * H + hp - 1) / hp;
             const int c0 = (bj * W) / wp, c1 = ((bj + 1) * W + wp - 1) / wp;
@@ -542,19 +541,21 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
     pdl_trigger();
     __shared__ float wsum[16][5];
     __shared__ double wmax[16];
+    __shared__ float gate_map[WZ_MAX_HW * WZ_MAX_HW];   // the frame's saliency map (either gate form)
     extern __shared__ float4 sfs[];   // [D/4] frame sums (max-over-query scorer only)
     const bool maxsim = c.relevance_mode == WZ_RELEVANCE_MAXSIM;
     const bool do_gate = c.gate && c.spatial_mode == WZ_SPATIAL_WSM;
     const int64_t f = blockIdx.x;
-    // with the mean scorer, threads 256..511 form the gate while 0..255 form
-    // the statistics; the max-over-query scorer takes every warp for its
-    // query rows and forms the gate after them
+    // with the mean scorer, the upper half of the threads forms the gate
+    // while the lower half forms the statistics; the max-over-query scorer
+    // takes every warp for its query rows and forms the gate after them
     const bool split = !maxsim && do_gate;
-    if (split && threadIdx.x >= 256) {
-        gate_half(c, f, (int)threadIdx.x - 256);
+    const int half = (int)blockDim.x / 2;
+    if (split && (int)threadIdx.x >= half) {
+        gate_half(c, f, (int)threadIdx.x - half, half, gate_map);
         return;
     }
-    const int nst = split ? 256 : (int)blockDim.x;   // threads forming the statistics
+    const int nst = split ? half : (int)blockDim.x;   // threads forming the statistics
     float av[kGatePerThread];
     if (do_gate && !split) gate_prefetch(c, f, av);
     const int t = (int)(f % c.T);
@@ -649,7 +650,7 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
         wsum[warp][3] = p3;
         wsum[warp][4] = p4;
     }
-    if (split) asm volatile("bar.sync 1, 256;" ::: "memory");   // the statistics' warps only
+    if (split) asm volatile("bar.sync 1, %0;" ::"r"(half) : "memory");   // the statistics' warps only
     else __syncthreads();
     if (warp == 0) {
         // lane k < 5 sums quantity k over the warps in order (one fp64 warp
@@ -686,7 +687,7 @@ __global__ void __launch_bounds__(512) frame_stats_kernel(Ctx c) {
             if (c.frame_scores) c.frame_scores[f] = (float)r;
         }
     }
-    if (do_gate && !split) frame_gate(c, f, wsum[0], av);
+    if (do_gate && !split) frame_gate(c, f, wsum[0], av, gate_map);
 }
 
 cudaError_t launch_query_pool(const Ctx &c, const VideoPar *hpar, cudaStream_t s) {
@@ -777,7 +778,16 @@ cudaError_t launch_frame_stats(const Ctx &c, cudaStream_t s) {
             cudaFuncSetAttribute((const void *)frame_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
     }
-    return launch_kernel((const void *)frame_stats_kernel, dim3(c.V * c.T), dim3(512), smem, s, args, c.pdl != 0);
+    // 512 threads a frame (4 CTAs per SM); with the mean scorer's split form
+    // and more frames than one wave of those, 256 (twice the CTAs in flight)
+    const bool split = c.relevance_mode != WZ_RELEVANCE_MAXSIM && c.gate && c.spatial_mode == WZ_SPATIAL_WSM;
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const int threads = split && (int64_t)c.V * c.T > 4 * (int64_t)sms ? 256 : 512;
+    return launch_kernel((const void *)frame_stats_kernel, dim3(c.V * c.T), dim3(threads), smem, s, args,
+                         c.pdl != 0);
 }
 
 cudaError_t launch_query_rows(const Ctx &c, int v, int q_row0, int Lq, int Lqp, cudaStream_t s) {
