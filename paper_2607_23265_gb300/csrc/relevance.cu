@@ -180,7 +180,7 @@ __global__ void __launch_bounds__(kRelMaxConsumers + 32, 1) relevance_pass_kerne
     constexpr int VEC = VecOf<T>::kElems;
     constexpr int GROUP = 8;                 // tokens per warp transpose-reduction
     constexpr int NV = 2 * GROUP;            // GROUP dots + GROUP squared norms
-    constexpr int WIN = 64;                  // tokens per cross-warp reduction
+    constexpr int WIN = 128;                 // tokens per cross-warp reduction
     constexpr int NWMAX = kRelMaxConsumers / 32;
     extern __shared__ __align__(128) uint8_t rsm[];
     __shared__ float wpart[2][NWMAX][2][WIN];
