@@ -198,7 +198,18 @@ WZ_API void wz_condense_args_init(wz_condense_args *a);
 /* Workspace bytes that wz_condense_ex needs for these sizes. */
 WZ_API size_t wz_condense_workspace_size(int T, int H, int W, int D, int dtype, float ratio);
 
-/* Condense one video (arguments above).  Returns a WZ_* status. */
+/*
+ * Condense one video (arguments above).  Returns a WZ_* status.
+ * Replay cache: when `workspace` is given, `kernel_events` is NULL and
+ * `stream` is not being captured, an argument set (every pointer, size and
+ * option, on the current device) seen for the second time has its launch
+ * sequence captured into a CUDA graph (on a private stream; that call pays
+ * the capture and instantiation on the host), and that call and every later
+ * one with identical arguments launch the graph into `stream`; the first call
+ * with an argument set launches the kernels one by one.  The inputs are read when
+ * the graph runs, so new contents in the same buffers are condensed anew.
+ * Otherwise the kernels are launched one by one.  See wz_graph_cache.
+ */
 WZ_API int wz_condense_ex(const wz_condense_args *a);
 
 /*
@@ -263,7 +274,20 @@ WZ_API int64_t wz_batch_rows(int V, int T, int H, int W, const float *ratio, int
 
 WZ_API size_t wz_batch_workspace_size(int V, int T, int H, int W, int D, int dtype, const float *ratio);
 
+/* The serving batch (arguments above; same replay cache as wz_condense_ex). */
 WZ_API int wz_condense_batch(const wz_batch_args *a);
+
+/*
+ * Replay cache of wz_condense_ex / wz_condense_batch: the number of argument
+ * sets whose executable graphs are kept (least recently used dropped first;
+ * default 8).  capacity >= 0 sets it (0 disables the cache and frees every
+ * kept graph; a graph still running is freed when it completes); a negative
+ * capacity only queries.  stats: HOST int64[3], nullable, filled after the
+ * change with {graphs kept, replays, captures} (the last two count since the
+ * library was loaded).  Returns the capacity in force before the call.
+ * Thread-safe; host only.
+ */
+WZ_API int wz_graph_cache(int capacity, int64_t *stats);
 
 /* ------------------------------------------------------------------------ */
 /* Cross-Modal Scorer, similarity branch (Section 3.2.1)                     */

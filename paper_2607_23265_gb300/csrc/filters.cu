@@ -10,6 +10,7 @@
 // coefficient list of (z+1)^p prod (z - z_i), normalised to sum sqrt(2).
 #include <cmath>
 #include <complex>
+#include <mutex>
 #include <vector>
 
 #include "wz_internal.cuh"
@@ -170,9 +171,33 @@ int wavelet_taps(int wavelet) {
     return 0;
 }
 
+// Each bank is derived once and kept: the derivation runs in long double,
+// which hosts with a 128-bit long double emulate in software, and every
+// condensation call sets up two banks.
 bool wavelet_bank(int wavelet, double *dec_lo, double *dec_hi, double *rec_lo, double *rec_hi) {
-    if (wavelet == WZ_WAVELET_BIOR44) return bior44(dec_lo, dec_hi, rec_lo, rec_hi);
-    return daubechies(wavelet, dec_lo, dec_hi, rec_lo, rec_hi);
+    struct Bank {
+        bool done = false, ok = false;
+        double f[4][kMaxTaps] = {};
+    };
+    static std::mutex mu;
+    static Bank banks[WZ_WAVELET_BIOR44 + 1];
+    if (wavelet < 1 || wavelet > WZ_WAVELET_BIOR44) return false;
+    Bank &b = banks[wavelet];
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (!b.done) {
+            b.ok = wavelet == WZ_WAVELET_BIOR44 ? bior44(b.f[0], b.f[1], b.f[2], b.f[3])
+                                                : daubechies(wavelet, b.f[0], b.f[1], b.f[2], b.f[3]);
+            b.done = true;
+        }
+    }
+    if (!b.ok) return false;
+    double *out[4] = {dec_lo, dec_hi, rec_lo, rec_hi};
+    const int F = wavelet_taps(wavelet);
+    for (int j = 0; j < 4; ++j)
+        if (out[j])
+            for (int k = 0; k < F; ++k) out[j][k] = b.f[j][k];
+    return true;
 }
 
 }  // namespace wz

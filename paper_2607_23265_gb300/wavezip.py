@@ -125,6 +125,7 @@ def _load(path: str = LIB_PATH):
         "wz_idwt2d": (i, [vp, vp, vp, vp, i, i, i, i, i, vp, vp]),
         "wz_status_string": (C.c_char_p, [i]),
         "wz_version": (i, []),
+        "wz_graph_cache": (i, [i, C.POINTER(C.c_int64)]),
         "wz_selftest_bounded_wait": (i, [C.c_uint64, vp, vp]),
     }
     for name, (res, args) in sig.items():
@@ -198,11 +199,21 @@ def wz_condense(features: torch.Tensor, query: torch.Tensor, ratio: float, strea
     return tokens, index
 
 
+def _out(t, shape, dtype, dev, name):
+    """A caller-given output tensor (checked) or a new one."""
+    if t is None:
+        return torch.empty(shape, dtype=dtype, device=dev)
+    if tuple(t.shape) != tuple(shape) or t.dtype != dtype or t.device != dev or not t.is_contiguous():
+        raise ValueError(f"{name}: expected a contiguous {dtype} tensor of shape {tuple(shape)} on {dev}")
+    return t
+
+
 def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *, lam: float = 1.5,
                    tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
                    temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1,
                    token_scores: torch.Tensor | None = None, frame_scores: torch.Tensor | None = None,
                    relevance="mean", wta_levels: int = 1, wsm_levels: int = 1, workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
+                   out_budgets=None, out_count=None, out_relevance=None,
                    device_status: torch.Tensor | None = None, kernel_events=None, stream=None):
     """wz_condense_ex.  Returns a dict with tokens, index, budgets, count and relevance.
 
@@ -213,7 +224,9 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
     relevance: "mean" (the mean query row) or "maxsim" (maximum cosine over
     the query rows; bf16 features, D % 64 == 0, at most 128 query rows).
     wta_levels / wsm_levels: decomposition levels of the two wavelet modules
-    (1..4; the DWT cascades on the approximation band)."""
+    (1..4; the DWT cascades on the approximation band).
+    out_*: optional preallocated outputs; with a workspace and the same
+    buffers on every call, repeated calls replay one captured CUDA graph."""
     features = _cuda_contig(features, "features")
     query = _cuda_contig(query, "query")
     T, H, W, D = features.shape
@@ -223,9 +236,9 @@ def wz_condense_ex(features: torch.Tensor, query: torch.Tensor, ratio: float, *,
         raise WaveZipError(ERR_INVALID_ARG, "wz_condense_ex")
     tokens = out_tokens if out_tokens is not None else torch.empty((B, D), dtype=features.dtype, device=dev)
     index = out_index if out_index is not None else torch.empty((B, 3), dtype=torch.int32, device=dev)
-    budgets = torch.empty((T,), dtype=torch.int32, device=dev)
-    count = torch.empty((1,), dtype=torch.int32, device=dev)
-    rel = torch.empty((T, 4), dtype=torch.float32, device=dev)
+    budgets = _out(out_budgets, (T,), torch.int32, dev, "out_budgets")
+    count = _out(out_count, (1,), torch.int32, dev, "out_count")
+    rel = _out(out_relevance, (T, 4), torch.float32, dev, "out_relevance")
     a = CondenseArgs()
     _lib.wz_condense_args_init(C.byref(a))
     a.features, a.T, a.H, a.W, a.D = features.data_ptr(), T, H, W, D
@@ -293,6 +306,7 @@ def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios,
                       tau: float = 0.0, wsm_wavelet: int = 4, mode="symmetric", path="auto",
                       temporal_mode="wta", spatial_mode="wsm", wta_wavelet: int = 1, relevance="mean",
                       wta_levels: int = 1, wsm_levels: int = 1, workspace: torch.Tensor | None = None, out_tokens=None, out_index=None,
+                      out_budgets=None, out_count=None, out_relevance=None,
                       device_status: torch.Tensor | None = None, kernel_events=None, stream=None):
     """wz_condense_batch: features [V,T,H,W,D], queries [sum Lq, D].  Options as
     for wz_condense_ex; kernel_events brackets each kernel of the whole batch."""
@@ -303,9 +317,9 @@ def wz_condense_batch(features: torch.Tensor, queries: torch.Tensor, Lq, ratios,
     rows, offs = wz_batch_rows(V, T, H, W, ratios)
     tokens = out_tokens if out_tokens is not None else torch.empty((rows, D), dtype=features.dtype, device=dev)
     index = out_index if out_index is not None else torch.empty((rows, 3), dtype=torch.int32, device=dev)
-    budgets = torch.empty((V, T), dtype=torch.int32, device=dev)
-    count = torch.empty((V,), dtype=torch.int32, device=dev)
-    rel = torch.empty((V, T, 4), dtype=torch.float32, device=dev)
+    budgets = _out(out_budgets, (V, T), torch.int32, dev, "out_budgets")
+    count = _out(out_count, (V,), torch.int32, dev, "out_count")
+    rel = _out(out_relevance, (V, T, 4), torch.float32, dev, "out_relevance")
     lq = (C.c_int32 * V)(*[int(x) for x in Lq])
     rt = (C.c_float * V)(*[float(x) for x in ratios])
     ro = (C.c_int64 * (V + 1))()
@@ -455,6 +469,15 @@ def wz_idwt2d(LL, LH, HL, HH, H: int, W: int, wavelet: int = 4, stream=None):
 
 def wz_version() -> int:
     return int(_lib.wz_version())
+
+
+def wz_graph_cache(capacity: int = -1) -> dict:
+    """Set the replay cache's capacity (0 disables it; negative only
+    queries).  Returns the capacity in force before the call and the cache's
+    counters after it: graphs kept, replays and captures."""
+    st = (C.c_int64 * 3)()
+    prev = int(_lib.wz_graph_cache(int(capacity), st))
+    return {"previous_capacity": prev, "kept": int(st[0]), "replays": int(st[1]), "captures": int(st[2])}
 
 
 STATUS_WAIT_TIMEOUT = 0x100
