@@ -169,3 +169,30 @@ def test_workspace_sizes_are_host_only(wz):
     assert wz.wz_condense_workspace_size(4, 4, 4, 12, 0, 0.5) == 0
     assert wz.wz_relevance_workspace_size(64, 13, 13, 3584) > 0
     assert wz.wz_batch_workspace_size(2, 64, 13, 13, 3584, 0, [0.1, 0.25]) > n1 / 100
+
+
+def test_graph_cache_capacity_is_host_only(wz):
+    """The replay cache's capacity and counters: set, query and restore
+    without a GPU (an empty cache makes no CUDA call)."""
+    st = wz.wz_graph_cache(-1)
+    prev = st["previous_capacity"]
+    assert prev >= 0 and st["kept"] == 0 and st["replays"] == 0 and st["captures"] == 0
+    try:
+        assert wz.wz_graph_cache(3)["previous_capacity"] == prev
+        assert wz.wz_graph_cache(-5)["previous_capacity"] == 3     # negative: query only
+        assert wz.wz_graph_cache(0)["previous_capacity"] == 3
+        assert wz.wz_graph_cache(-1) == {"previous_capacity": 0, "kept": 0, "replays": 0, "captures": 0}
+    finally:
+        wz.wz_graph_cache(prev)
+    assert wz.wz_graph_cache(-1)["previous_capacity"] == prev
+
+
+def test_cached_path_checks_arguments_first(wz):
+    """A call that would use the replay cache (caller workspace, no events)
+    is rejected by the same argument checks, before any CUDA call."""
+    for over, code in [(dict(D=12), -2), (dict(ratio=0.0), -1), (dict(workspace_bytes=16), -5)]:
+        a = _args(wz, workspace=5 * P, workspace_bytes=1 << 30)
+        for k, v in over.items():
+            setattr(a, k, v)
+        assert wz._lib.wz_condense_ex(C.byref(a)) == code
+    assert wz.wz_graph_cache(-1)["kept"] == 0
