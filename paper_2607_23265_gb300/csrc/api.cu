@@ -497,8 +497,11 @@ int run_condense_cached(const CondenseRequest &r) {
     int dev = 0;
     WZ_CUDA(cudaGetDevice(&dev));
     const std::string key = request_key(r, dev);
-    std::lock_guard<std::mutex> lock(g_graph_mu);
-    if (g_graph_capacity <= 0) return run_condense(r);
+    std::unique_lock<std::mutex> lock(g_graph_mu);
+    if (g_graph_capacity <= 0) {
+        lock.unlock();
+        return run_condense(r);
+    }
     for (auto it = g_graphs.begin(); it != g_graphs.end(); ++it) {
         if (it->key != key) continue;
         g_graphs.splice(g_graphs.begin(), g_graphs, it);
@@ -510,6 +513,7 @@ int run_condense_cached(const CondenseRequest &r) {
     if (seen == g_seen.end()) {
         g_seen.push_front(key);
         trim_graphs(g_graph_capacity);
+        lock.unlock();   // direct launches need no cache state
         return run_condense(r);
     }
     g_seen.erase(seen);
